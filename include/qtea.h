@@ -1,0 +1,138 @@
+/*
+ * qtea.h: C ABI of the GB300 (sm_103a) QTEA decode GEMV library.
+ *
+ * The operation is the inference-time product of the QTEA paper ("Ternary LLMs with
+ * Sparse Residual Salient Weight and By-Column Optimization"):
+ *
+ *   y[m][o] = alpha[o] * sum_j T[o][j] * v[j] * x[m][j]                 (Sec. 3.5, Eq. 10)
+ *           + sum_{c < s} [pos(o/4, c) == o % 4] * R[o/4][c] * x[m][S_c]  (Sec. 3.5, Eq. 11)
+ *
+ * i.e. y = x * W^T with the dequantized weight of Sec. 3.3, Eq. 4 (W^ = v_j * alpha_o * T_oj,
+ * the bias beta being zero) plus the column-semi-sparse residual of Sec. 3.2 / Sec. 3.5: in
+ * each salient column S_c, every group of four consecutive output rows holds exactly one
+ * residual value and its 2-bit position inside the group (1:4 sparsity along the rows).
+ * One scale per output row is supported (group size = K); per-group alpha/beta is not.
+ *
+ * Conventions for every entry point:
+ *   - fp16 tensors are IEEE 754 binary16 bit patterns passed as uint16_t.
+ *   - All tensor pointers are DEVICE pointers owned by the caller, except the packed
+ *     ternary weights, which the library owns inside a qtea_layout.
+ *   - Arrays are dense and row-major. 16-byte alignment is required where stated.
+ *   - Entry points return a qtea_status. Nothing is printed, no exception crosses the
+ *     ABI, and there is no CPU fallback: without a usable GPU every call that computes
+ *     fails with QTEA_ERR_CUDA.
+ *   - `stream` is a cudaStream_t (0 = legacy default stream).
+ */
+#ifndef QTEA_H_
+#define QTEA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* qtea_stream_t; /* identical to cudaStream_t */
+typedef struct qtea_layout qtea_layout;    /* opaque, library-owned packed ternary weights */
+
+typedef enum qtea_status {
+  QTEA_OK = 0,
+  QTEA_ERR_INVALID_ARG = 1, /* null pointer, negative or inconsistent size, misalignment */
+  QTEA_ERR_BAD_CODES = 2,   /* a ternary code outside {-1, 0, +1} */
+  QTEA_ERR_UNSUPPORTED = 3, /* a valid request this build does not implement */
+  QTEA_ERR_CUDA = 4,        /* a CUDA runtime error (no device, launch failure, ...) */
+  QTEA_ERR_ALLOC = 5,       /* device memory allocation failed */
+  QTEA_ERR_TIMEOUT = 6      /* a bounded wait inside a kernel gave up (see qtea_device_status) */
+} qtea_status;
+
+typedef enum qtea_format {
+  QTEA_FMT_2BIT = 0, /* 4 codes per byte; the only format qtea_gemv consumes */
+  QTEA_FMT_BASE3 = 1 /* 5 codes per byte, 26 bytes per 128 columns (Sec. 3.5); not implemented */
+} qtea_format;
+
+/* Largest batch (rows of x) one qtea_gemv call accepts. */
+#define QTEA_MAX_M 16
+
+/*
+ * Pack ternary codes into the library's 2-bit layout (Sec. 3.1, Eq. 2 gives T; the layout is
+ * this library's own, chosen for 16-byte coalesced loads).
+ *
+ *   ternary_codes  device int8 [N][K], values -1, 0, +1 (read only; may be freed afterwards)
+ *   N, K           output rows and input columns, N >= 0, K >= 0
+ *   group_size     must equal K (one alpha per row); anything else -> QTEA_ERR_UNSUPPORTED
+ *   n_salient      number of salient columns s the layout will be used with, s >= 0;
+ *                  if s > 0, N must be a multiple of 4 (groups of four rows)
+ *   format         QTEA_FMT_2BIT (QTEA_FMT_BASE3 -> QTEA_ERR_UNSUPPORTED)
+ *   out            receives the new layout on success, NULL on failure
+ *
+ * Packed layout (2-bit): K_pad = K rounded up to a multiple of 64. Row r occupies bytes
+ * [r*K_pad/4, (r+1)*K_pad/4); column k sits in byte r*K_pad/4 + k/4 at bits 2*(k%4) and
+ * 2*(k%4)+1 (least significant first) as the code T+1; columns k >= K hold code 1.
+ *
+ * The call validates every code on the device and synchronizes `stream` once to read the
+ * result; invalid codes give QTEA_ERR_BAD_CODES and no layout. It allocates the packed
+ * bytes and the split-K workspace of qtea_gemv (both freed by qtea_free).
+ */
+int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, int n_salient, int format,
+                     qtea_stream_t stream, qtea_layout** out);
+
+/*
+ * y = x * W^T for the layout's N x K ternary weights plus the 1:4 salient residual
+ * (Eq. 10 and Eq. 11 with beta = 0 and one alpha per row).
+ *
+ *   x              device fp16 [M][K], activations
+ *   packed_ternary layout from qtea_pack_layout
+ *   row_scale      device fp16 [N], alpha_o (one scale per output row)
+ *   col_scale      device fp16 [K], v_j, the column-wise rescale factors (Sec. 3.3, Eq. 4)
+ *   salient_idx    device int32 [s], strictly ascending column indices, each in [0, K)
+ *   residual_vals  device fp16 [N/4][s]: R of group q (rows 4q..4q+3) in salient column c
+ *   residual_idx   device uint8 [N/4][ceil(s/4)]: 2-bit position of that value in its
+ *                  group; entry (q, c) at bits 2*(c%4) of byte q*ceil(s/4) + c/4
+ *   y              device fp32 [M][N], overwritten
+ *   M              batch, 1 <= M <= QTEA_MAX_M
+ *   stream         CUDA stream; the call is asynchronous and allocates nothing
+ *
+ * s is the layout's n_salient; with s = 0 the three residual pointers may be NULL.
+ * Alignment: x, row_scale, col_scale and y must be 4-byte aligned. The salient indices are
+ * not validated on the device: out-of-order or duplicate indices give an unspecified y
+ * (each listed column's residual is still added once), indices outside [0, K) are
+ * clamped into range and never read out of bounds.
+ * Calls that share a layout must be ordered on one stream: the layout holds the split-K
+ * workspace. Results are bitwise reproducible for a given (layout, inputs, device).
+ * Numerics: the ternary sum is accumulated exactly in integers over 512-column blocks,
+ * with v*x represented in 24-bit fixed point relative to the block's largest |v*x|; block
+ * sums, alpha and the residual are combined in fp32.
+ */
+int qtea_gemv(const uint16_t* x, const qtea_layout* packed_ternary, const uint16_t* row_scale,
+              const uint16_t* col_scale, const int32_t* salient_idx, const uint16_t* residual_vals,
+              const uint8_t* residual_idx, float* y, int M, qtea_stream_t stream);
+
+/* Release a layout and its device memory. NULL is ignored. The caller orders it after the
+ * last qtea_gemv that uses the layout has completed; it synchronizes nothing itself. */
+void qtea_free(qtea_layout* layout);
+
+/* Static English description of a status code. Never NULL. */
+const char* qtea_status_string(int status);
+
+/* Read-only description of a layout (all sizes in elements unless named *_bytes). */
+typedef struct qtea_layout_desc {
+  int N, K, K_pad, group_size, n_salient, format;
+  size_t packed_bytes;      /* size of the packed ternary weights */
+  const void* packed_data;  /* device pointer to the packed ternary weights */
+} qtea_layout_desc;
+
+int qtea_layout_describe(const qtea_layout* layout, qtea_layout_desc* out);
+
+/*
+ * Status written by the kernels of this layout: QTEA_OK, or QTEA_ERR_TIMEOUT if a bounded
+ * wait inside a kernel gave up (the kernel then skipped its remaining work and y is
+ * unspecified). Synchronizes `stream`, reads the flag and clears it.
+ */
+int qtea_device_status(const qtea_layout* layout, qtea_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QTEA_H_ */

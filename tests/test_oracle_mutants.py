@@ -1,0 +1,125 @@
+"""Planted mistakes: each mutant of the oracle must fail at least one pin.
+
+A copy of the oracle's C source gets one plausible error (a dropped term, a wrong sign,
+index or bit order), is compiled into a temporary library, and is run through a compact
+version of the pins in test_oracle.py. The real oracle must pass all of them; every
+mutant must fail at least one, which shows the pins can see that kind of mistake.
+"""
+import os
+import subprocess
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+F16 = np.float16
+SRC = os.path.join(os.path.dirname(oracle.__file__), "qtea_oracle.c")
+
+
+def f(bits):
+    return np.asarray(bits, dtype=np.uint16).view(F16).astype(np.float64)
+
+
+def dense(p, beta=None, g=None):
+    N, K = p.T.shape
+    g = K if g is None else g
+    G = -(-K // g)
+    cols = np.arange(K) // g
+    a = f(p.alpha).reshape(N, G)[:, cols]
+    b = 0 if beta is None else f(beta).reshape(N, G)[:, cols]
+    W = a * f(p.v)[None] * p.T + b
+    pos = synth.residual_positions(p.residual_idx, p.s)
+    for q in range(N // 4 if p.s else 0):
+        for c in range(p.s):
+            W[4 * q + pos[q, c], p.salient_idx[c]] += f(p.residual_vals)[q, c]
+    return W
+
+
+def pin_failures(lib):
+    """Names of the pins this oracle build fails."""
+    fails = []
+
+    def check(name, ok):
+        if not ok:
+            fails.append(name)
+
+    # binary16 decoding of every pattern
+    bits = np.arange(65536, dtype=np.uint32)
+    ref = bits.astype(np.uint16).view(F16).astype(np.float64)
+    got = np.array([lib.qo_half_to_double(int(b)) for b in bits])
+    fin = np.isfinite(ref)
+    check("half", np.array_equal(got[fin], ref[fin]))
+    # brute force, one scale per row
+    for (N, K, s, M) in [(8, 64, 8, 2), (64, 256, 8, 1)]:
+        p = synth.make_problem("m", N, K, M, s, seed=N + K + s)
+        try:
+            y, b = oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx, lib=lib)
+        except oracle.OracleError:
+            check("dense", False)
+            continue
+        W = dense(p)
+        x = f(p.x)
+        check("dense", np.allclose(y, x @ W.T, rtol=1e-12, atol=1e-12))
+        check("bound", np.allclose(b, np.abs(x[:, None, :] * W[None]).sum(-1), rtol=1e-12, atol=0))
+    # brute force, group scales with bias (Eq. 10 in full)
+    p = synth.make_problem("m", 8, 256, 2, 4, seed=77)
+    p.alpha = synth.uniform_f16(1, 2, (8, 2), 0.01, 0.05)
+    beta = synth.normal_f16(1, 9, (8, 2), 0.0, 0.01)
+    y, _ = oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx,
+                       beta=beta, group_size=128, lib=lib)
+    check("groups", np.allclose(y, f(p.x) @ dense(p, beta, 128).T, rtol=1e-12, atol=1e-13))
+    # packing: known bytes and round trip
+    T = np.zeros((1, 64), np.int8)
+    T[0, :4] = [1, -1, 1, 0]
+    check("pack2", int(oracle.pack(T, "2bit", lib=lib)[0]) == (2 | 0 << 2 | 2 << 4 | 1 << 6))
+    T = np.zeros((1, 128), np.int8)
+    T[0, :5] = [1, -1, 0, 0, 0]
+    check("pack3", int(oracle.pack(T, "base3", lib=lib)[0]) == 119)
+    # LUT symmetry and single-digit entries
+    xs = np.array([0.3, -1.25, 2.0, 0.125, -0.5])
+    lut = oracle.lut5(xs, lib=lib)
+    check("lut", np.array_equal(lut, -lut[::-1]) and all(lut[121 + 3 ** d] == xs[d] for d in range(5)))
+    return fails
+
+
+MUTANTS = {
+    "drop_residual_term": [("acc += qo_half_to_double(residual_vals", "acc += 0.0 * qo_half_to_double(residual_vals")],
+    "wrong_residual_row": [("== o % 4)\n          acc +=", "== (o + 1) % 4)\n          acc +=")],
+    "ternary_sign_flip": [("tvx += (double)T[", "tvx -= (double)T[")],
+    "rescale_index_shift": [("qo_half_to_double(v[j]) * xj", "qo_half_to_double(v[(j + 1) % K]) * xj")],
+    "bias_times_rescaled_x": [("sx += xj;", "sx += xj * qo_half_to_double(v[j]);")],
+    "alpha_first_group_only": [("double a = qo_half_to_double(alpha[(size_t)o * G + g]);\n        double b = beta ? qo_half_to_double(beta[(size_t)o * G + g]) : 0.0;\n        acc +=",
+                                "double a = qo_half_to_double(alpha[(size_t)o * G]);\n        double b = beta ? qo_half_to_double(beta[(size_t)o * G + g]) : 0.0;\n        acc +=")],
+    "transposed_codes": [("tvx += (double)T[(size_t)o * K + j]", "tvx += (double)T[((size_t)j * N + o) % ((size_t)N * K)]")],
+    "bound_without_abs_w": [("fabs(qo_half_to_double(xm[j]) * w_row[j])", "fabs(qo_half_to_double(xm[j])) * w_row[j]")],
+    "pack_msb_first": [("(uint8_t)(code << (2 * (k % 4)))", "(uint8_t)(code << (6 - 2 * (k % 4)))")],
+    "half_exponent_bias": [("expo - 25", "expo - 24")],
+    "half_subnormal_scale": [("ldexp((double)frac, -24)", "ldexp((double)frac, -23)")],
+    "base3_digit_order": [("int value = 0, weight = 1;", "int value = 0, weight = 81;"), ("weight *= 3;", "weight /= 3;")],
+    "lut_digit_offset": [("(double)(rest % 3 - 1) * xs[d]", "(double)(rest % 3) * xs[d]")],
+}
+
+
+@pytest.fixture(scope="module")
+def mutant_dir(tmp_path_factory):
+    return tmp_path_factory.mktemp("oracle_mutants")
+
+
+def test_real_oracle_passes_every_pin():
+    assert pin_failures(oracle.load()) == []
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, mutant_dir):
+    src = open(SRC).read()
+    for old, new in MUTANTS[name]:
+        assert old in src, f"mutation anchor for {name} not found"
+        src = src.replace(old, new)
+    c_path = mutant_dir / f"{name}.c"
+    so_path = mutant_dir / f"{name}.so"
+    c_path.write_text(src)
+    subprocess.check_call(["gcc", "-O2", "-std=c99", "-fPIC", "-shared", "-o", str(so_path), str(c_path), "-lm"])
+    lib = oracle.load(str(so_path))
+    assert pin_failures(lib), f"mutant {name} passed every pin"
