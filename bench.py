@@ -1,0 +1,477 @@
+#!/usr/bin/env python3
+"""Benchmark of the batch-1 QTEA ternary + 1:4 residual GEMV on GB300.
+
+Workload: the seven linear layers of one Llama3-8B decoder layer (q/k/v/o/gate/up/down, out x in
+= 4096x4096, 1024x4096, 1024x4096, 4096x4096, 14336x4096, 14336x4096, 4096x14336) at batch M = 1,
+with synthetic weights drawn like the paper's models would be stored (ternary codes
+P(-1,0,+1) = (0.3,0.4,0.3), alpha ~ U(0.01,0.05), v ~ U(0.8,1.2), 3% salient columns, residual
+~ N(0,0.02), x ~ N(0,1)). `--layers` independent layers are resident in HBM and the steps
+rotate through them, so every step reads weights that are not in L2.
+
+A step = the seven GEMVs of one layer. value = algorithmic bytes moved per step (packed ternary
+codes, alpha, v, salient indices, residual values and positions, x, y) x steps / device time.
+Prints one JSON line (rank 0).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "µs/call and achieved HBM GB/s (% of GB300 peak) for batch-1 ternary+1:4 GEMV"
+WORKLOAD = "llama3_8b_layer_gemvs_m1"
+CONFIG_ID = 1
+
+
+def algorithmic_bytes(N, K, s, M=1):
+    K_pad = -(-K // 64) * 64
+    return (N * K_pad // 4 + 2 * N + 2 * K + 4 * s + 2 * (N // 4) * s + (N // 4) * ((s + 3) // 4)
+            + 2 * M * K + 4 * M * N)
+
+
+def profiled_traffic():
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source still
+    matches the one that was profiled (else None)."""
+    import hashlib
+    prof = os.path.join(ROOT, "profiles", "qtea_gemv_m1_llama3_8b_layer.md")
+    src = os.path.join(ROOT, "paper_2609_00224_gb300", "csrc", "qtea_gemv_m1.cu")
+    try:
+        text = open(prof).read()
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        fields = dict(l.split(":", 1) for l in text.splitlines() if l.startswith(("kernel_source_sha256_16:",
+                                                                                   "traffic_bytes_per_launch:")))
+        if fields.get("kernel_source_sha256_16", "").strip() != sha:
+            return None
+        return int(fields["traffic_bytes_per_launch"].strip())
+    except Exception:
+        return None
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during the timed region."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        mhz, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                mhz.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not mhz:
+            return None
+        return {"sm_mhz": statistics.median(mhz), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(mhz)}
+
+
+class ExternalEvents:
+    """Records a CUDA event as an event-record node while a stream is being captured
+    (cuEventRecordWithFlags with CU_EVENT_RECORD_EXTERNAL), so graph replays time each launch."""
+
+    def __init__(self):
+        import ctypes
+        self.ok = False
+        try:
+            self.cu = ctypes.CDLL("libcuda.so.1")
+            self.cu.cuEventRecordWithFlags.restype = ctypes.c_int
+            self.cu.cuEventRecordWithFlags.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint]
+            self.ok = True
+        except Exception:
+            self.ok = False
+
+    def record(self, event, stream):
+        rc = self.cu.cuEventRecordWithFlags(event.cuda_event, stream.cuda_stream, 1)
+        if rc != 0:
+            raise RuntimeError(f"cuEventRecordWithFlags failed with {rc}")
+
+
+# ---------------------------------------------------------------------------- workload
+
+def make_layer(layer, torch, qt, synth, keep_host=False):
+    """Generate one layer's seven problems, pack them on the device, keep device operands."""
+    out = []
+    for mi, (name, N, K) in enumerate(synth.config_shapes(CONFIG_ID)):
+        p = synth.config_problem(CONFIG_ID, mi, layer=layer)
+        f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
+        T = torch.from_numpy(p.T).cuda()
+        lay = qt.qtea_pack_layout(T, n_salient=p.s)
+        del T
+        g = dict(name=name, N=N, K=K, s=p.s, layout=lay, x=f16(p.x), alpha=f16(p.alpha.reshape(-1)), v=f16(p.v),
+                 sal=torch.from_numpy(p.salient_idx).cuda(), rv=f16(p.residual_vals),
+                 ri=torch.from_numpy(p.residual_idx).cuda(), y=torch.empty((1, N), dtype=torch.float32, device="cuda"),
+                 bytes=algorithmic_bytes(N, K, p.s))
+        if keep_host:
+            g["host"] = p
+        out.append(g)
+    return out
+
+
+def run_step(qt, layer, stream):
+    for g in layer:
+        qt.qtea_gemv(g["x"], g["layout"], g["alpha"], g["v"], g["sal"], g["rv"], g["ri"], y=g["y"], stream=stream)
+
+
+def oracle_sample_seconds(problems, rows_stride, budget_s):
+    """Time the oracle (as it stands, 1 thread) over sampled rows of the given problems."""
+    import oracle
+    done_bytes, t_total, n_rows_total = 0.0, 0.0, 0
+    i = 0
+    while t_total < budget_s and i < len(problems) * 100:
+        p = problems[i % len(problems)]
+        rows = np.arange(i // len(problems) % rows_stride, p.N, rows_stride, dtype=np.int32)
+        t0 = time.perf_counter()
+        oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx, rows=rows,
+                    want_bound=False)
+        t_total += time.perf_counter() - t0
+        done_bytes += algorithmic_bytes(p.N, p.K, p.s) * len(rows) / p.N
+        n_rows_total += len(rows)
+        i += 1
+    return done_bytes, t_total, n_rows_total
+
+
+# ---------------------------------------------------------------------------- arms
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def reference_arm(args):
+    """The oracle, as it stands, on the host cores: each step a bounded sample of the workload."""
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return 0
+    import oracle
+    import synth
+    oracle.build()
+    synth.build()
+    problems = [synth.config_problem(CONFIG_ID, mi, layer=0) for mi in range(7)]
+    rows_stride = 64  # every 64th output row of each of the 7 GEMVs per step
+    for _ in range(args.warmup):
+        oracle_sample_seconds(problems[1:2], rows_stride * 4, 0.0)
+    tot_b, tot_t, tot_rows = 0.0, 0.0, 0
+    for step in range(args.steps):
+        for p in problems:
+            rows = np.arange(step % rows_stride, p.N, rows_stride, dtype=np.int32)
+            t0 = time.perf_counter()
+            oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx, rows=rows,
+                        want_bound=False)
+            tot_t += time.perf_counter() - t0
+            tot_b += algorithmic_bytes(p.N, p.K, p.s) * len(rows) / p.N
+            tot_rows += len(rows)
+    value = tot_b / tot_t / 1e9
+    sample = (f"each step: every {rows_stride}th output row of the 7 Llama3-8B layer GEMVs "
+              f"({tot_rows // max(args.steps, 1)} rows/step), fp64 oracle, 1 thread")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / max(args.steps, 1),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "M": 1, "note": "bounded row sample per step"},
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def qtea_arm(args):
+    import torch
+    import synth
+    import paper_2609_00224_gb300 as qt
+
+    world, rank, local = dist_setup()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    qt.load()
+    warmup = max(args.warmup, 3)
+    stream = torch.cuda.Stream()
+    t_gen = time.perf_counter()
+    layers = [make_layer(l, torch, qt, synth, keep_host=(l == 0 and rank == 0 and not args.no_cpu_baseline))
+              for l in range(args.layers)]
+    for L in layers:
+        for g in L:
+            g["layout"].set_activation_precision(args.act_bits)
+    torch.cuda.synchronize()
+    t_gen = time.perf_counter() - t_gen
+    resident = sum(g["layout"].describe()["packed_bytes"] for L in layers for g in L)
+    step_bytes = [sum(g["bytes"] for g in L) for L in layers]
+    l2 = torch.cuda.get_device_properties(local).L2_cache_size
+    launches_per_step = 7
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    # ---- CUDA graphs: the warm-up steps and the K timed steps are each captured once; the timed
+    #      graph records an event before and after every launch (event-record nodes), so the
+    #      per-launch durations come from the timed region itself
+    ext = ExternalEvents()
+    n_ev = args.steps * launches_per_step
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_ev)]
+    for a_, b_ in ev:  # materialise the event handles before capture
+        a_.record(stream)
+        b_.record(stream)
+    torch.cuda.synchronize()
+
+    group_args = [[dict(x=g["x"], layout=g["layout"], row_scale=g["alpha"], col_scale=g["v"], salient_idx=g["sal"],
+                        residual_vals=g["rv"], residual_idx=g["ri"], y=g["y"]) for g in L] for L in layers]
+
+    def capture(steps, with_events, grouped=True):
+        """One step = the 7 GEMVs of one layer: one grouped launch, or 7 single launches."""
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=stream):
+            k = 0
+            for st in range(steps):
+                li = st % len(layers)
+                if grouped:
+                    if with_events:
+                        ext.record(ev[k][0], stream)
+                    qt.qtea_gemv_grouped(group_args[li], stream=stream)
+                    if with_events:
+                        ext.record(ev[k][1], stream)
+                    k += 1
+                    continue
+                for gm in layers[li]:
+                    if with_events:
+                        ext.record(ev[k][0], stream)
+                    qt.qtea_gemv(gm["x"], gm["layout"], gm["alpha"], gm["v"], gm["sal"], gm["rv"], gm["ri"],
+                                 y=gm["y"], stream=stream)
+                    if with_events:
+                        ext.record(ev[k][1], stream)
+                    k += 1
+        return gr
+
+    g_warm = capture(warmup, False)
+    g_timed = capture(args.steps, ext.ok)
+    with torch.cuda.stream(stream):
+        g_warm.replay()
+    barrier()
+
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    barrier()
+    with torch.cuda.stream(stream):
+        t_start.record(stream)
+        g_timed.replay()
+        t_end.record(stream)
+    barrier()
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    durs = [a_.elapsed_time(b_) for a_, b_ in ev[:args.steps]] if ext.ok else None
+    status = max(qt.qtea_device_status(g["layout"]) for L in layers for g in L)
+    if status:
+        raise RuntimeError(f"device status {status} after the timed region")
+    if world > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    bytes_all = sum(step_bytes[st % len(layers)] for st in range(args.steps)) * world
+    value = bytes_all / (total_ms * 1e-3) / 1e9
+
+    # roofline of the GEMV kernel: the only kernel of the timed region, one grouped launch per step
+    if durs is None:  # no event-record nodes: fall back to the region average
+        durs = [total_ms / args.steps] * args.steps
+    kern_bytes = sum(step_bytes[st % len(layers)] for st in range(args.steps))
+    achieved = kern_bytes / (sum(durs) * 1e-3) / 1e9
+    peak, peak_src = load_peaks()
+
+    # ---- per-GEMV latency: the same steps with one launch per GEMV, each launch timed
+    per_shape = {}
+    if ext.ok and not args.no_per_shape:
+        g_single = capture(args.steps, True, grouped=False)
+        with torch.cuda.stream(stream):
+            g_single.replay()
+        barrier()
+        sd = [a_.elapsed_time(b_) for a_, b_ in ev]
+        for j, gm in enumerate(layers[0]):
+            d = [sd[st * launches_per_step + j] * 1e3 for st in range(args.steps)]
+            med = statistics.median(d)
+            N, K, bts = gm["N"], gm["K"], gm["bytes"]
+            per_shape[gm["name"]] = {"N": N, "K": K, "s": gm["s"], "us_per_call": round(med, 3),
+                                     "gbs": round(bts / (med * 1e-6) / 1e9, 1),
+                                     "eff_bits_per_weight": round(8 * (bts - 2 * K - 4 * N) / (N * K), 3)}
+        del g_single
+
+    # ---- the other activation precision, same steps (reported beside the headline mode)
+    alt = {}
+    other = 16 if args.act_bits == 24 else 24
+    for L in layers:
+        for g in L:
+            g["layout"].set_activation_precision(other)
+    g_alt = capture(args.steps, False)
+    with torch.cuda.stream(stream):
+        g_alt.replay()
+    barrier()
+    ea, eb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        ea.record(stream)
+        g_alt.replay()
+        eb.record(stream)
+    barrier()
+    alt_ms = ea.elapsed_time(eb)
+    alt[f"act{other}"] = {"value": round(kern_bytes / (alt_ms * 1e-3) / 1e9, 1), "unit": "GB/s",
+                          "ms_per_step": round(alt_ms / args.steps, 5)}
+    for L in layers:
+        for g in L:
+            g["layout"].set_activation_precision(args.act_bits)
+    del g_alt
+
+    # ---- end to end through the public API with host buffers (pinned), copies inside the region
+    e2e = None
+    if not args.no_e2e:
+        L0 = layers
+        hx = [[g["x"].cpu().pin_memory() for g in L] for L in L0]
+        hy = [[torch.empty((1, g["N"]), dtype=torch.float32).pin_memory() for g in L] for L in L0]
+        h2d = sum(2 * g["K"] for g in L0[0])
+        d2h = sum(4 * g["N"] for g in L0[0])
+        with torch.cuda.stream(stream):
+            for i in range(warmup):
+                L = L0[i % len(L0)]
+                for j, g in enumerate(L):
+                    g["x"].copy_(hx[i % len(L0)][j], non_blocking=True)
+                    qt.qtea_gemv(g["x"], g["layout"], g["alpha"], g["v"], g["sal"], g["rv"], g["ri"], y=g["y"],
+                                 stream=stream)
+                    hy[i % len(L0)][j].copy_(g["y"], non_blocking=True)
+        barrier()
+        ge = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(ge, stream=stream):
+            for st in range(args.steps):
+                li = st % len(L0)
+                for j, g in enumerate(L0[li]):
+                    g["x"].copy_(hx[li][j], non_blocking=True)
+                qt.qtea_gemv_grouped(group_args[li], stream=stream)
+                for j, g in enumerate(L0[li]):
+                    hy[li][j].copy_(g["y"], non_blocking=True)
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            ge.replay()
+            e1.record(stream)
+        barrier()
+        e2e_ms = e0.elapsed_time(e1)
+        if world > 1:
+            t = torch.tensor([e2e_ms], device="cuda")
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e = {"value": round(bytes_all / (e2e_ms * 1e-3) / 1e9, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
+               "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms / args.steps, 5)}
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        probs = [g["host"] for g in layers[0]]
+        b, t, rows = oracle_sample_seconds(probs, 16, args.cpu_seconds)
+        cpu = {"value": round(b / t / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
+               "sample": f"{rows} output rows (every 16th row, cycling over the 7 layer-0 GEMVs) for "
+                         f"{t:.1f} s, fp64, 1 thread"}
+
+    traffic = profiled_traffic()
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": round(value, 1), "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+            "warmup": warmup, "ms_per_step": round(total_ms / args.steps, 5), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None,
+            "dtype": f"i32 dp4a (2-bit codes x {args.act_bits}-bit fixed-point v*x) + fp32",
+            "data": "synthetic",
+            "config": {"workload": WORKLOAD, "M": 1, "shapes": [[g["name"], g["N"], g["K"], g["s"]] for g in layers[0]],
+                       "layers_resident": args.layers, "resident_weight_bytes": resident, "l2_bytes": l2,
+                       "l2": "inputs larger than L2: steps rotate over the resident layers",
+                       "parallelism": "replicas" if world > 1 else "single"},
+            "us_per_call": per_shape,
+            "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                         "frac": round(achieved / peak, 4), "peak_source": peak_src, "traffic": traffic,
+                         "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
+                         "us_per_launch": round(1e3 * sum(durs) / args.steps, 3)},
+            "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
+            "setup_s": round(t_gen, 1),
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["qtea", "reference"], default="qtea")
+    ap.add_argument("--layers", type=int, default=16)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-per-shape", action="store_true")
+    ap.add_argument("--act-bits", type=int, choices=[16, 24], default=24,
+                    help="activation precision of the timed region (24 = exact default, 16 = fast mode)")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        return reference_arm(args)
+    return qtea_arm(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -94,19 +94,46 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
  *   stream         CUDA stream; the call is asynchronous and allocates nothing
  *
  * s is the layout's n_salient; with s = 0 the three residual pointers may be NULL.
- * Alignment: x, row_scale, col_scale and y must be 4-byte aligned. The salient indices are
+ * Alignment: fp16 arrays 2 bytes, salient_idx and y 4 bytes. The salient indices are
  * not validated on the device: out-of-order or duplicate indices give an unspecified y
  * (each listed column's residual is still added once), indices outside [0, K) are
  * clamped into range and never read out of bounds.
  * Calls that share a layout must be ordered on one stream: the layout holds the split-K
- * workspace. Results are bitwise reproducible for a given (layout, inputs, device).
+ * workspace. Results are bitwise reproducible for a given (layout, inputs, device); a grouped
+ * call (qtea_gemv_grouped) is reproducible for the same group, but its rounding may differ
+ * from separate calls because the split of work over the CTAs differs.
  * Numerics: the ternary sum is accumulated exactly in integers over 512-column blocks,
- * with v*x represented in 24-bit fixed point relative to the block's largest |v*x|; block
- * sums, alpha and the residual are combined in fp32.
+ * with v*x represented in fixed point relative to the block's largest |v*x| (24-bit unless
+ * qtea_set_activation_precision selects 16-bit); block sums, alpha and the residual are
+ * combined in fp32.
  */
 int qtea_gemv(const uint16_t* x, const qtea_layout* packed_ternary, const uint16_t* row_scale,
               const uint16_t* col_scale, const int32_t* salient_idx, const uint16_t* residual_vals,
               const uint8_t* residual_idx, float* y, int M, qtea_stream_t stream);
+
+/* One GEMV of a grouped call: the arguments of qtea_gemv except M and the stream. */
+typedef struct qtea_gemv_problem {
+  const uint16_t* x;
+  const qtea_layout* packed_ternary;
+  const uint16_t* row_scale;
+  const uint16_t* col_scale;
+  const int32_t* salient_idx;
+  const uint16_t* residual_vals;
+  const uint8_t* residual_idx;
+  float* y;
+} qtea_gemv_problem;
+
+/*
+ * Several independent GEMVs with the same batch M, as if qtea_gemv were called for each in
+ * order, but with M = 1 problems sharing launches: up to 8 problems whose activation staging
+ * fits shared memory run in one persistent kernel, which removes per-launch ramp-up and tail
+ * time when the problems are small (e.g. the q/k/v/o/gate/up/down GEMVs of one decoder layer).
+ * Every problem is validated before anything is launched; a failing check returns its status
+ * and launches nothing. No two problems may write overlapping y, and problems must not share
+ * a layout. QTEA_ERR_TIMEOUT from a grouped launch is recorded in the layout of the first
+ * problem of that launch (qtea_device_status). The call is asynchronous on `stream`.
+ */
+int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, qtea_stream_t stream);
 
 /* Release a layout and its device memory. NULL is ignored. The caller orders it after the
  * last qtea_gemv that uses the layout has completed; it synchronizes nothing itself. */
@@ -120,9 +147,27 @@ typedef struct qtea_layout_desc {
   int N, K, K_pad, group_size, n_salient, format;
   size_t packed_bytes;      /* size of the packed ternary weights */
   const void* packed_data;  /* device pointer to the packed ternary weights */
+  int batch1_kernel;        /* 1 if M = 1 calls run the TMA stream-K batch-1 kernel, 0 if they
+                               fall back to the general kernel (e.g. no tensor-map support) */
 } qtea_layout_desc;
 
 int qtea_layout_describe(const qtea_layout* layout, qtea_layout_desc* out);
+
+/* Copy the layout's packed ternary bytes (qtea_layout_desc.packed_bytes of them) to the
+ * caller's device buffer `dst`, asynchronously on `stream`. `bytes` must equal packed_bytes. */
+int qtea_layout_copy_packed(const qtea_layout* layout, void* dst, size_t bytes, qtea_stream_t stream);
+
+/*
+ * Activation precision of batch-1 (M = 1) calls on this layout. The ternary sum is always
+ * accumulated exactly in integers over 512-column blocks; what changes is how finely v*x is
+ * represented in fixed point relative to the block's largest |v*x|:
+ *   bits = 24 (default): 24-bit, three byte planes per column.
+ *   bits = 16: 16-bit (two byte planes, a third fewer dot-product instructions per weight)
+ *              for every block whose largest |v*x| is at most 8 times the block's root mean
+ *              square; blocks with outliers, and layouts with K < 1024, keep 24 bits.
+ * Returns QTEA_ERR_INVALID_ARG for other values. Batch sizes M > 1 are not affected.
+ */
+int qtea_set_activation_precision(qtea_layout* layout, int bits);
 
 /*
  * Status written by the kernels of this layout: QTEA_OK, or QTEA_ERR_TIMEOUT if a bounded

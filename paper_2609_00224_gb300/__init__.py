@@ -1,0 +1,238 @@
+"""Python binding of the QTEA GB300 GEMV library (``libqtea.so``, C ABI in ``include/qtea.h``).
+
+The functions here have the C entry points' names and only marshal arguments: they check
+dtypes and shapes of torch CUDA tensors, pass raw device pointers and the current CUDA
+stream, and raise ``QteaError`` on a non-zero status. Every step of the computation runs in
+the library's kernels; there is no fallback: if the library cannot be built or loaded, or
+no GPU is present, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+from . import build as _build
+
+QTEA_OK = 0
+QTEA_ERR_INVALID_ARG = 1
+QTEA_ERR_BAD_CODES = 2
+QTEA_ERR_UNSUPPORTED = 3
+QTEA_ERR_CUDA = 4
+QTEA_ERR_ALLOC = 5
+QTEA_ERR_TIMEOUT = 6
+QTEA_FMT_2BIT = 0
+QTEA_FMT_BASE3 = 1
+QTEA_MAX_M = 16
+
+_lib = None
+
+
+class QteaError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+        self.status = status
+
+
+class _Problem(ctypes.Structure):
+    _fields_ = [("x", ctypes.c_void_p), ("packed_ternary", ctypes.c_void_p), ("row_scale", ctypes.c_void_p),
+                ("col_scale", ctypes.c_void_p), ("salient_idx", ctypes.c_void_p), ("residual_vals", ctypes.c_void_p),
+                ("residual_idx", ctypes.c_void_p), ("y", ctypes.c_void_p)]
+
+
+class _LayoutDesc(ctypes.Structure):
+    _fields_ = [("N", ctypes.c_int), ("K", ctypes.c_int), ("K_pad", ctypes.c_int), ("group_size", ctypes.c_int),
+                ("n_salient", ctypes.c_int), ("format", ctypes.c_int), ("packed_bytes", ctypes.c_size_t),
+                ("packed_data", ctypes.c_void_p), ("batch1_kernel", ctypes.c_int)]
+
+
+def library_path() -> str:
+    return _build.LIB_PATH
+
+
+def load(build_if_missing: bool = True):
+    """Load libqtea.so (compiling it first if it is missing or stale)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.build() if build_if_missing else _build.LIB_PATH
+    if not os.path.exists(path):
+        raise RuntimeError(f"QTEA CUDA library not found at {path}; run paper_2609_00224_gb300/build.py")
+    lib = ctypes.CDLL(path)
+    P, i32 = ctypes.c_void_p, ctypes.c_int
+    lib.qtea_pack_layout.restype = i32
+    lib.qtea_pack_layout.argtypes = [P, i32, i32, i32, i32, i32, P, ctypes.POINTER(P)]
+    lib.qtea_gemv.restype = i32
+    lib.qtea_gemv.argtypes = [P, P, P, P, P, P, P, P, i32, P]
+    lib.qtea_free.restype = None
+    lib.qtea_free.argtypes = [P]
+    lib.qtea_status_string.restype = ctypes.c_char_p
+    lib.qtea_status_string.argtypes = [i32]
+    lib.qtea_layout_describe.restype = i32
+    lib.qtea_layout_describe.argtypes = [P, ctypes.POINTER(_LayoutDesc)]
+    lib.qtea_device_status.restype = i32
+    lib.qtea_device_status.argtypes = [P, P]
+    lib.qtea_gemv_grouped.restype = i32
+    lib.qtea_gemv_grouped.argtypes = [P, i32, i32, P]
+    lib.qtea_set_activation_precision.restype = i32
+    lib.qtea_set_activation_precision.argtypes = [P, i32]
+    lib.qtea_layout_copy_packed.restype = i32
+    lib.qtea_layout_copy_packed.argtypes = [P, P, ctypes.c_size_t, P]
+    _lib = lib
+    return lib
+
+
+def status_string(status: int) -> str:
+    return load().qtea_status_string(int(status)).decode()
+
+
+def _stream(stream) -> Optional[int]:
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _ptr(t, dtypes, name, shape=None):
+    import torch
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype not in dtypes:
+        raise TypeError(f"{name} has dtype {t.dtype}, expected one of {dtypes}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+    return t.data_ptr()
+
+
+def _f16_types():
+    import torch
+    return (torch.float16, torch.int16) + ((torch.uint16,) if hasattr(torch, "uint16") else ())
+
+
+class Layout:
+    """Owner of a qtea_layout handle (packed ternary weights + split-K workspace)."""
+
+    def __init__(self, handle: int, N: int, K: int, n_salient: int):
+        self._h = ctypes.c_void_p(handle)
+        self.N, self.K, self.n_salient = N, K, n_salient
+
+    @property
+    def handle(self):
+        if not self._h:
+            raise ValueError("layout was freed")
+        return self._h
+
+    def describe(self) -> dict:
+        d = _LayoutDesc()
+        rc = load().qtea_layout_describe(self.handle, ctypes.byref(d))
+        if rc:
+            raise QteaError(rc, "qtea_layout_describe")
+        return {f: getattr(d, f) for f, _ in _LayoutDesc._fields_}
+
+    def set_activation_precision(self, bits: int):
+        """24 (default, exact to 24-bit fixed point) or 16 (fast mode for outlier-free blocks)."""
+        rc = load().qtea_set_activation_precision(self.handle, int(bits))
+        if rc:
+            raise QteaError(rc, "qtea_set_activation_precision")
+        return self
+
+    def free(self):
+        if self._h:
+            load().qtea_free(self._h)
+            self._h = ctypes.c_void_p(None)
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
+def qtea_pack_layout(codes, n_salient: int = 0, group_size: Optional[int] = None, fmt: int = QTEA_FMT_2BIT,
+                     stream=None) -> Layout:
+    """Pack int8 ternary codes [N][K] (CUDA tensor) into a library-owned layout."""
+    import torch
+    if codes.dim() != 2:
+        raise ValueError("codes must be [N][K]")
+    N, K = codes.shape
+    ptr = _ptr(codes, (torch.int8,), "codes")
+    out = ctypes.c_void_p()
+    rc = load().qtea_pack_layout(ptr, N, K, K if group_size is None else group_size, n_salient, fmt,
+                                 _stream(stream), ctypes.byref(out))
+    if rc:
+        raise QteaError(rc, "qtea_pack_layout")
+    return Layout(out.value, N, K, n_salient)
+
+
+def _problem_args(x, layout, row_scale, col_scale, salient_idx, residual_vals, residual_idx, y):
+    import torch
+    f16 = _f16_types()
+    if x.dim() != 2:
+        raise ValueError("x must be [M][K]")
+    M = x.shape[0]
+    N, K, s = layout.N, layout.K, layout.n_salient
+    if y is None:
+        y = torch.empty((M, N), dtype=torch.float32, device=x.device)
+    args = [
+        _ptr(x, f16, "x", (M, K)),
+        layout.handle,
+        _ptr(row_scale.reshape(-1) if row_scale is not None else None, f16, "row_scale", (N,)),
+        _ptr(col_scale, f16, "col_scale", (K,)),
+        _ptr(salient_idx, (torch.int32,), "salient_idx", (s,)) if s else None,
+        _ptr(residual_vals, f16, "residual_vals", (N // 4, s)) if s else None,
+        _ptr(residual_idx, (torch.uint8,), "residual_idx", (N // 4, (s + 3) // 4)) if s else None,
+        _ptr(y, (torch.float32,), "y", (M, N)),
+    ]
+    return args, y, M
+
+
+def qtea_gemv(x, layout: Layout, row_scale, col_scale, salient_idx=None, residual_vals=None, residual_idx=None,
+              y=None, stream=None):
+    """y[M][N] = x[M][K] * W^T (fp32) with the layout's ternary weights and the 1:4 residual."""
+    args, y, M = _problem_args(x, layout, row_scale, col_scale, salient_idx, residual_vals, residual_idx, y)
+    rc = load().qtea_gemv(*args, M, _stream(stream))
+    if rc:
+        raise QteaError(rc, "qtea_gemv")
+    return y
+
+
+def qtea_gemv_grouped(problems, stream=None):
+    """Several independent GEMVs in as few launches as possible.
+
+    `problems` is a sequence of dicts with keys x, layout, row_scale, col_scale and optionally
+    salient_idx, residual_vals, residual_idx, y. Returns the list of y tensors.
+    """
+    ys, arr, M = [], (_Problem * max(len(problems), 1))(), None
+    for i, q in enumerate(problems):
+        args, y, m = _problem_args(q["x"], q["layout"], q["row_scale"], q["col_scale"], q.get("salient_idx"),
+                                   q.get("residual_vals"), q.get("residual_idx"), q.get("y"))
+        if M is None:
+            M = m
+        elif m != M:
+            raise ValueError("all problems of a grouped call need the same batch M")
+        args[1] = args[1].value
+        arr[i] = _Problem(*args)
+        ys.append(y)
+    rc = load().qtea_gemv_grouped(ctypes.cast(arr, ctypes.c_void_p), len(problems), M or 1, _stream(stream))
+    if rc:
+        raise QteaError(rc, "qtea_gemv_grouped")
+    return ys
+
+
+def qtea_device_status(layout: Layout, stream=None) -> int:
+    return load().qtea_device_status(layout.handle, _stream(stream))
+
+
+def packed_bytes(layout: Layout):
+    """Copy of the packed ternary bytes as a CUDA uint8 tensor (for inspection and tests)."""
+    import torch
+    n = layout.describe()["packed_bytes"]
+    out = torch.empty(max(n, 1), dtype=torch.uint8, device="cuda")
+    rc = load().qtea_layout_copy_packed(layout.handle, out.data_ptr(), n, _stream(None))
+    if rc:
+        raise QteaError(rc, "qtea_layout_copy_packed")
+    return out[:n]

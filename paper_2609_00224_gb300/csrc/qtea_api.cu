@@ -1,0 +1,380 @@
+// Host side of the C ABI declared in include/qtea.h: argument validation, layout ownership,
+// launch planning and dispatch. No computation happens on the host.
+#include <cudaTypedefs.h>
+
+#include <cstdlib>
+#include <cstring>
+#include <new>
+
+#include "qtea_internal.h"
+
+using namespace qtea;
+
+namespace {
+
+// Below this many input columns the 16-bit activation mode is not used: with few nonzeros per
+// row its rounding errors average out less.
+constexpr int kMinK16 = 1024;
+
+int round_up(int a, int b) { return (a + b - 1) / b * b; }
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode_tiled() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+void release(qtea_layout* l) {
+  if (!l) return;
+  if (l->packed) cudaFree(l->packed);
+  if (l->workspace) cudaFree(l->workspace);
+  if (l->counters) cudaFree(l->counters);
+  if (l->status) cudaFree(l->status);
+  delete l;
+}
+
+// Resources of the batch-1 kernel for one layout: its TMA descriptor (512-row x 512-column
+// units, two 256-row boxes each) and the split-tile workspace.
+int plan_m1(qtea_layout* l, const cudaDeviceProp& prop) {
+  l->m1_ok = false;
+  l->sm_count = prop.multiProcessorCount;
+  l->smem_optin = prop.sharedMemPerBlockOptin;
+  if (l->N == 0 || l->K == 0) return QTEA_OK;
+  l->n_tiles = (l->N + kTileRows - 1) / kTileRows;
+  l->n_chunks = (l->K_pad + kChunkCols - 1) / kChunkCols;
+  PFN_cuTensorMapEncodeTiled_v12000 encode = get_encode_tiled();
+  if (!encode) return QTEA_OK;
+  cuuint64_t dims[2] = {(cuuint64_t)(l->K_pad / 4), (cuuint64_t)l->N};
+  cuuint64_t strides[1] = {(cuuint64_t)(l->K_pad / 4)};
+  cuuint32_t box[2] = {(cuuint32_t)kChunkRowBytes, (cuuint32_t)kBoxRows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = encode(&l->tmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, l->packed, dims, strides, box, estr,
+                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return QTEA_OK;
+  size_t dyn_max = 0;
+  if (m1_configure(prop.sharedMemPerBlockOptin, &dyn_max) != cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_OK;
+  }
+  l->smem_optin = dyn_max;
+  if (cudaMalloc(&l->workspace, (size_t)l->sm_count * 2 * kTileRows * sizeof(float)) != cudaSuccess)
+    return QTEA_ERR_ALLOC;
+  if (cudaMalloc(&l->counters, (size_t)l->n_tiles * kConsumerWarps * sizeof(unsigned)) != cudaSuccess)
+    return QTEA_ERR_ALLOC;
+  if (cudaMemset(l->counters, 0, (size_t)l->n_tiles * kConsumerWarps * sizeof(unsigned)) != cudaSuccess)
+    return QTEA_ERR_CUDA;
+  l->m1_ok = true;
+  return QTEA_OK;
+}
+
+// Host-side checks of one problem; returns QTEA_OK or the status to report.
+int check_problem(const qtea_gemv_problem& q, int M) {
+  const qtea_layout* l = q.packed_ternary;
+  if (!l) return QTEA_ERR_INVALID_ARG;
+  if (M < 1 || M > QTEA_MAX_M) return QTEA_ERR_INVALID_ARG;
+  if (l->N == 0) return QTEA_OK;
+  if (!q.y || !aligned(q.y, 4)) return QTEA_ERR_INVALID_ARG;
+  if (l->K == 0) return QTEA_OK;
+  if (!q.x || !q.row_scale || !q.col_scale) return QTEA_ERR_INVALID_ARG;
+  if (!aligned(q.x, 2) || !aligned(q.row_scale, 2) || !aligned(q.col_scale, 2)) return QTEA_ERR_INVALID_ARG;
+  if (l->n_salient > 0 && (!q.salient_idx || !q.residual_vals || !q.residual_idx || !aligned(q.salient_idx, 4) ||
+                           !aligned(q.residual_vals, 2)))
+    return QTEA_ERR_INVALID_ARG;
+  return QTEA_OK;
+}
+
+int launch_generic_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
+  const qtea_layout* l = q.packed_ternary;
+  GenericParams p;
+  p.x = q.x;
+  p.packed = l->packed;
+  p.alpha = q.row_scale;
+  p.v = q.col_scale;
+  p.sal = q.salient_idx;
+  p.rvals = q.residual_vals;
+  p.ridx = q.residual_idx;
+  p.y = q.y;
+  p.M = M;
+  p.N = l->N;
+  p.K = l->K;
+  p.K_pad = l->K_pad;
+  p.s = l->n_salient;
+  return launch_generic(p, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+}
+
+// Batch-1 kernel over a group of problems whose layouts all have m1 resources.
+struct M1Group {
+  GroupParams gp;
+  TensorMaps maps;
+  int grid = 0;
+  size_t smem = 0;
+};
+
+void group_reset(M1Group& g) {
+  std::memset(&g.gp, 0, sizeof(g.gp));
+  g.gp.n_problems = 0;
+  g.gp.total_units = 0;
+}
+
+// Add problem q; false if the group is full.
+bool group_add(M1Group& g, const qtea_gemv_problem& q) {
+  if (g.gp.n_problems == kMaxProblems) return false;
+  const qtea_layout* l = q.packed_ternary;
+  ProblemArgs& a = g.gp.prob[g.gp.n_problems];
+  a.x = q.x;
+  a.alpha = q.row_scale;
+  a.v = q.col_scale;
+  a.sal = q.salient_idx;
+  a.rvals = q.residual_vals;
+  a.ridx = q.residual_idx;
+  a.y = q.y;
+  a.ws = l->workspace;
+  a.counters = l->counters;
+  a.N = l->N;
+  a.K = l->K;
+  a.s = l->n_salient;
+  a.n_tiles = l->n_tiles;
+  a.n_chunks = l->n_chunks;
+  a.act_bits = (l->act_bits == 16 && l->K >= kMinK16) ? 16 : 24;
+  a.unit_begin = g.gp.total_units;
+  std::memcpy(&g.maps.m[g.gp.n_problems], &l->tmap, sizeof(CUtensorMap));
+  if (g.gp.n_problems == 0) g.gp.status = l->status;
+  g.gp.total_units += (long long)l->n_tiles * l->n_chunks;
+  g.gp.n_problems += 1;
+  return true;
+}
+
+// Grid, ring depth and shared memory of the group; false if some CTA's staging does not fit.
+bool group_plan(M1Group& g, int sm_count, size_t smem_optin) {
+  if (g.gp.n_problems == 0) return false;
+  if (g.gp.total_units >= (1ll << 30)) return false;
+  g.grid = (int)(g.gp.total_units < sm_count ? g.gp.total_units : sm_count);
+  if (g.grid > kMaxGrid) g.grid = kMaxGrid;
+  for (int b = 0; b <= g.grid; ++b) g.gp.cta_u0[b] = (int)unit_begin_of(b, g.gp.total_units, g.grid);
+  for (int stages = kMaxStages; stages >= kMinStages; --stages) {
+    g.gp.n_stages = stages;
+    size_t need = 0;
+    for (int b = 0; b < g.grid; ++b) {
+      size_t s = cta_smem_plan(g.gp.prob, g.gp.n_problems, g.gp.n_stages, g.gp.cta_u0[b], g.gp.cta_u0[b + 1], nullptr,
+                               nullptr, nullptr);
+      if (s > need) need = s;
+    }
+    if (need <= smem_optin) {
+      g.smem = need;
+      return true;
+    }
+  }
+  return false;
+}
+
+int group_launch(M1Group& g, cudaStream_t st) {
+  return launch_m1(g.maps, g.gp, g.grid, g.smem, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+}
+
+// Batch-1 dispatch: pack as many consecutive problems as fit into each launch.
+int run_m1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st) {
+  int i = 0;
+  while (i < n) {
+    const qtea_layout* l0 = qs[idx[i]].packed_ternary;
+    M1Group g;
+    group_reset(g);
+    int taken = 0;
+    while (i + taken < n) {
+      M1Group trial = g;
+      if (!group_add(trial, qs[idx[i + taken]])) break;
+      if (!group_plan(trial, l0->sm_count, l0->smem_optin)) break;
+      g = trial;
+      ++taken;
+    }
+    if (taken == 0) {
+      // a single problem whose staging does not fit: the generic kernel serves it
+      int rc = launch_generic_problem(qs[idx[i]], 1, st);
+      if (rc) return rc;
+      ++i;
+      continue;
+    }
+    int rc = group_launch(g, st);
+    if (rc) return rc;
+    i += taken;
+  }
+  return QTEA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* qtea_status_string(int status) {
+  switch (status) {
+    case QTEA_OK: return "success";
+    case QTEA_ERR_INVALID_ARG: return "invalid argument";
+    case QTEA_ERR_BAD_CODES: return "ternary code outside {-1, 0, +1}";
+    case QTEA_ERR_UNSUPPORTED: return "unsupported request";
+    case QTEA_ERR_CUDA: return "CUDA runtime error";
+    case QTEA_ERR_ALLOC: return "device allocation failed";
+    case QTEA_ERR_TIMEOUT: return "bounded wait in a kernel timed out";
+    default: return "unknown status";
+  }
+}
+
+int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, int n_salient, int format,
+                     qtea_stream_t stream, qtea_layout** out) {
+  if (!out) return QTEA_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (N < 0 || K < 0 || n_salient < 0 || n_salient > K) return QTEA_ERR_INVALID_ARG;
+  if ((long long)N * K > 0 && !ternary_codes) return QTEA_ERR_INVALID_ARG;
+  if (n_salient > 0 && N % 4 != 0) return QTEA_ERR_INVALID_ARG;
+  if (format != QTEA_FMT_2BIT && format != QTEA_FMT_BASE3) return QTEA_ERR_INVALID_ARG;
+  if (format == QTEA_FMT_BASE3) return QTEA_ERR_UNSUPPORTED;
+  if (group_size != K) return QTEA_ERR_UNSUPPORTED;
+  if ((long long)K + 63 > 0x7fffffffLL) return QTEA_ERR_INVALID_ARG;
+
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) { cudaGetLastError(); return QTEA_ERR_CUDA; }
+  cudaDeviceProp prop;
+  if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) { cudaGetLastError(); return QTEA_ERR_CUDA; }
+
+  qtea_layout* l = new (std::nothrow) qtea_layout;
+  if (!l) return QTEA_ERR_ALLOC;
+  std::memset(l, 0, sizeof(*l));
+  l->N = N;
+  l->K = K;
+  l->K_pad = round_up(K, 64);
+  l->group_size = group_size;
+  l->n_salient = n_salient;
+  l->format = format;
+  l->device = dev;
+  l->act_bits = 24;
+  l->packed_bytes = (size_t)N * (size_t)(l->K_pad / 4);
+  if (cudaMalloc(&l->packed, l->packed_bytes > 0 ? l->packed_bytes : 16) != cudaSuccess ||
+      cudaMalloc(&l->status, 2 * sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    release(l);
+    return QTEA_ERR_ALLOC;
+  }
+  int rc = QTEA_OK;
+  int host_flags[2] = {0, 0};
+  if (cudaMemsetAsync(l->status, 0, 2 * sizeof(int), st) != cudaSuccess ||
+      launch_pack(ternary_codes, N, K, l->K_pad, reinterpret_cast<uint32_t*>(l->packed), l->status + 1, st) !=
+          cudaSuccess ||
+      cudaMemcpyAsync(host_flags, l->status, sizeof(host_flags), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess) {
+    rc = QTEA_ERR_CUDA;
+  } else if (host_flags[1] != 0) {
+    rc = QTEA_ERR_BAD_CODES;
+  } else if (cudaMemsetAsync(l->status, 0, 2 * sizeof(int), st) != cudaSuccess) {
+    rc = QTEA_ERR_CUDA;
+  } else {
+    rc = plan_m1(l, prop);
+  }
+  if (rc == QTEA_OK && cudaStreamSynchronize(st) != cudaSuccess) rc = QTEA_ERR_CUDA;
+  if (rc != QTEA_OK) {
+    cudaGetLastError();
+    release(l);
+    return rc;
+  }
+  *out = l;
+  return QTEA_OK;
+}
+
+int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, qtea_stream_t stream) {
+  if (n_problems < 0 || (n_problems > 0 && !problems)) return QTEA_ERR_INVALID_ARG;
+  if (M < 1 || M > QTEA_MAX_M) return QTEA_ERR_INVALID_ARG;
+  for (int i = 0; i < n_problems; ++i) {
+    int rc = check_problem(problems[i], M);
+    if (rc) return rc;
+    for (int j = 0; j < i; ++j)  // a layout's split-K workspace serves one problem per call
+      if (problems[j].packed_ternary == problems[i].packed_ternary) return QTEA_ERR_INVALID_ARG;
+  }
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int* m1_idx = n_problems > 0 ? static_cast<int*>(std::malloc(sizeof(int) * (size_t)n_problems)) : nullptr;
+  if (n_problems > 0 && !m1_idx) return QTEA_ERR_ALLOC;
+  int n_m1 = 0, rc = QTEA_OK;
+  for (int i = 0; i < n_problems && rc == QTEA_OK; ++i) {
+    const qtea_gemv_problem& q = problems[i];
+    const qtea_layout* l = q.packed_ternary;
+    if (l->N == 0) continue;
+    if (l->K == 0) {
+      if (cudaMemsetAsync(q.y, 0, (size_t)M * l->N * sizeof(float), st) != cudaSuccess) rc = QTEA_ERR_CUDA;
+      continue;
+    }
+    if (M == 1 && l->m1_ok) m1_idx[n_m1++] = i;
+    else rc = launch_generic_problem(q, M, st);
+  }
+  if (rc == QTEA_OK && n_m1 > 0) rc = run_m1(problems, m1_idx, n_m1, st);
+  std::free(m1_idx);
+  if (rc != QTEA_OK) cudaGetLastError();
+  return rc;
+}
+
+int qtea_gemv(const uint16_t* x, const qtea_layout* l, const uint16_t* row_scale, const uint16_t* col_scale,
+              const int32_t* salient_idx, const uint16_t* residual_vals, const uint8_t* residual_idx, float* y, int M,
+              qtea_stream_t stream) {
+  qtea_gemv_problem q;
+  q.x = x;
+  q.packed_ternary = l;
+  q.row_scale = row_scale;
+  q.col_scale = col_scale;
+  q.salient_idx = salient_idx;
+  q.residual_vals = residual_vals;
+  q.residual_idx = residual_idx;
+  q.y = y;
+  return qtea_gemv_grouped(&q, 1, M, stream);
+}
+
+void qtea_free(qtea_layout* layout) { release(layout); }
+
+int qtea_layout_describe(const qtea_layout* l, qtea_layout_desc* out) {
+  if (!l || !out) return QTEA_ERR_INVALID_ARG;
+  out->N = l->N;
+  out->K = l->K;
+  out->K_pad = l->K_pad;
+  out->group_size = l->group_size;
+  out->n_salient = l->n_salient;
+  out->format = l->format;
+  out->packed_bytes = l->packed_bytes;
+  out->packed_data = l->packed;
+  out->batch1_kernel = l->m1_ok ? 1 : 0;
+  return QTEA_OK;
+}
+
+int qtea_set_activation_precision(qtea_layout* l, int bits) {
+  if (!l || (bits != 16 && bits != 24)) return QTEA_ERR_INVALID_ARG;
+  l->act_bits = bits;
+  return QTEA_OK;
+}
+
+int qtea_layout_copy_packed(const qtea_layout* l, void* dst, size_t bytes, qtea_stream_t stream) {
+  if (!l || bytes != l->packed_bytes || (bytes > 0 && !dst)) return QTEA_ERR_INVALID_ARG;
+  if (bytes == 0) return QTEA_OK;
+  if (cudaMemcpyAsync(dst, l->packed, bytes, cudaMemcpyDeviceToDevice, reinterpret_cast<cudaStream_t>(stream)) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_ERR_CUDA;
+  }
+  return QTEA_OK;
+}
+
+int qtea_device_status(const qtea_layout* l, qtea_stream_t stream) {
+  if (!l) return QTEA_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int flag = 0;
+  if (cudaMemcpyAsync(&flag, l->status, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaMemsetAsync(l->status, 0, sizeof(int), st) != cudaSuccess || cudaStreamSynchronize(st) != cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_ERR_CUDA;
+  }
+  return flag == 0 ? QTEA_OK : flag;
+}
+
+}  // extern "C"
