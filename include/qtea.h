@@ -43,7 +43,8 @@ typedef enum qtea_status {
   QTEA_ERR_UNSUPPORTED = 3, /* a valid request this build does not implement */
   QTEA_ERR_CUDA = 4,        /* a CUDA runtime error (no device, launch failure, ...) */
   QTEA_ERR_ALLOC = 5,       /* device memory allocation failed */
-  QTEA_ERR_TIMEOUT = 6      /* a bounded wait inside a kernel gave up (see qtea_device_status) */
+  QTEA_ERR_TIMEOUT = 6,     /* a bounded wait inside a kernel gave up (see qtea_device_status) */
+  QTEA_ERR_SCRATCH_LIMIT = 7 /* larger than the static scratch of qtea_gemv_m1_static allows */
 } qtea_status;
 
 typedef enum qtea_format {
@@ -175,6 +176,48 @@ int qtea_set_activation_precision(qtea_layout* layout, int bits);
  * unspecified). Synchronizes `stream`, reads the flag and clears it.
  */
 int qtea_device_status(const qtea_layout* layout, qtea_stream_t stream);
+
+/*
+ * Allocation-free batch-1 GEMV. The QTEA paper has no counterpart: this is a deployment entry
+ * point of this library, not a step of the method.
+ *
+ * Some callers cannot call cudaMalloc: a serving process whose allocator has already reserved the
+ * GPU's memory for its own pool (a further cudaMalloc fails or escapes its accounting), or code on
+ * a latency-critical path where cudaMalloc and cudaFree may synchronise the device. qtea_gemv needs
+ * a qtea_layout, whose creation allocates. This call instead reads the packed codes from memory the
+ * caller owns and takes its split-tile scratch from a fixed array in the library's static device
+ * memory. It calls no cudaMalloc, cudaFree or other allocating routine.
+ *
+ * Computes, for M = 1, what qtea_gemv computes (Eq. 10 and Eq. 11, one alpha per row, beta = 0),
+ * with the default 24-bit activation precision.
+ *   x, row_scale, col_scale, salient_idx, residual_vals, residual_idx, y
+ *                  as for qtea_gemv, with M = 1
+ *   packed         device, 16-byte aligned, caller-owned: the 2-bit layout qtea_pack_layout
+ *                  writes, N rows of K_pad/4 bytes (K_pad = K rounded up to a multiple of 64),
+ *                  code T+1 four per byte, least significant first, pad columns code 1 (for
+ *                  instance a copy made once with qtea_layout_copy_packed). Codes are not
+ *                  validated: code 3 decodes as T = 2.
+ *   N, K, n_salient  sizes as for qtea_pack_layout (N % 4 == 0 when n_salient > 0)
+ * Limits of the static scratch (663,808 bytes of device memory per device): N <= 131072 (at most
+ * 256 tiles of 512 rows); a larger N returns QTEA_ERR_SCRATCH_LIMIT. At most 160 CTAs are used.
+ * Set-up: the first call on each device, with that device current, looks the scratch up with
+ * cudaGetSymbolAddress and sets the kernel's shared-memory attribute. Make that first call before
+ * any stream capture on the device. Later calls encode a tensor map on the host and launch.
+ * Start state: the split-tile counters in the scratch must be zero when a call starts. Static
+ * device memory is zero when the library's module loads, and every completed call leaves the
+ * counters at zero.
+ * Concurrency: every call on a device shares the one scratch. Calls that may overlap on the
+ * device (different streams without ordering, several host threads) race and give wrong results:
+ * order them, e.g. on one stream.
+ * A bounded wait that times out inside the kernel is recorded in the scratch's status word and is
+ * not reported by this call (qtea_device_status reads layouts only).
+ * Returns QTEA_OK, QTEA_ERR_INVALID_ARG, QTEA_ERR_SCRATCH_LIMIT, QTEA_ERR_UNSUPPORTED (device
+ * ordinal >= 64) or QTEA_ERR_CUDA.
+ */
+int qtea_gemv_m1_static(const uint16_t* x, const uint8_t* packed, int N, int K, int n_salient,
+                        const uint16_t* row_scale, const uint16_t* col_scale, const int32_t* salient_idx,
+                        const uint16_t* residual_vals, const uint8_t* residual_idx, float* y,
+                        qtea_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -4,6 +4,7 @@
 
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <new>
 
 #include "qtea_internal.h"
@@ -209,6 +210,61 @@ int run_m1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st) 
   return QTEA_OK;
 }
 
+// ---------------------------------------------------------------- allocation-free batch-1 entry
+// qtea_gemv_m1_static serves callers that may not allocate device memory. Its split-tile scratch is
+// this fixed array in static device memory (one copy per device), laid out as
+//   [0, kStaticWsBytes)             partial sums   [kStaticGrid][2][kTileRows] float
+//   [kStaticWsBytes, +kStaticCtrBytes)  counters   [kStaticTiles][kConsumerWarps] unsigned, zero between calls
+//   then the status word (int)
+// The counters start at zero because static device memory is zero-initialised when the module
+// is loaded, and every completed call leaves them at zero (the last CTA of a tile resets them).
+constexpr int kStaticGrid = 160;                 // CTAs a call may use (>= the 152 SMs of a GB300)
+constexpr int kStaticTiles = 256;                // 512-row tiles: N <= 131072
+constexpr size_t kStaticWsBytes = (size_t)kStaticGrid * 2 * kTileRows * sizeof(float);    // 655,360
+constexpr size_t kStaticCtrBytes = (size_t)kStaticTiles * kConsumerWarps * sizeof(unsigned);  // 8,192
+constexpr size_t kStaticScratchBytes = kStaticWsBytes + kStaticCtrBytes + 256;              // 663,808
+constexpr int kStaticMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+
+// Per-device set-up, done once with that device current: the scratch address, the SM count and
+// the batch-1 kernel's shared-memory limit.
+struct StaticDevice {
+  bool ready = false;
+  bool m1_ok = false;
+  unsigned char* scratch = nullptr;
+  int sm_count = 0;
+  size_t smem_optin = 0;
+};
+StaticDevice g_static_dev[kStaticMaxDevices];
+std::mutex g_static_mu;
+
+int static_setup(int dev, StaticDevice* out) {
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  StaticDevice& d = g_static_dev[dev];
+  if (!d.ready) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || !p) {
+      cudaGetLastError();
+      return QTEA_ERR_CUDA;
+    }
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess) {
+      cudaGetLastError();
+      return QTEA_ERR_CUDA;
+    }
+    size_t dyn_max = 0;
+    d.m1_ok = get_encode_tiled() != nullptr && m1_configure(prop.sharedMemPerBlockOptin, &dyn_max) == cudaSuccess;
+    if (!d.m1_ok) cudaGetLastError();
+    d.scratch = static_cast<unsigned char*>(p);
+    d.sm_count = prop.multiProcessorCount < kStaticGrid ? prop.multiProcessorCount : kStaticGrid;
+    d.smem_optin = dyn_max;
+    d.ready = true;
+  }
+  *out = d;
+  return QTEA_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -222,6 +278,7 @@ const char* qtea_status_string(int status) {
     case QTEA_ERR_CUDA: return "CUDA runtime error";
     case QTEA_ERR_ALLOC: return "device allocation failed";
     case QTEA_ERR_TIMEOUT: return "bounded wait in a kernel timed out";
+    case QTEA_ERR_SCRATCH_LIMIT: return "problem larger than the static scratch of qtea_gemv_m1_static";
     default: return "unknown status";
   }
 }
@@ -375,6 +432,83 @@ int qtea_device_status(const qtea_layout* l, qtea_stream_t stream) {
     return QTEA_ERR_CUDA;
   }
   return flag == 0 ? QTEA_OK : flag;
+}
+
+int qtea_gemv_m1_static(const uint16_t* x, const uint8_t* packed, int N, int K, int n_salient,
+                        const uint16_t* row_scale, const uint16_t* col_scale, const int32_t* salient_idx,
+                        const uint16_t* residual_vals, const uint8_t* residual_idx, float* y, qtea_stream_t stream) {
+  if (N < 0 || K < 0 || n_salient < 0 || n_salient > K) return QTEA_ERR_INVALID_ARG;
+  if (n_salient > 0 && N % 4 != 0) return QTEA_ERR_INVALID_ARG;
+  if ((long long)K + 63 > 0x7fffffffLL) return QTEA_ERR_INVALID_ARG;
+  if ((N + kTileRows - 1) / kTileRows > kStaticTiles) return QTEA_ERR_SCRATCH_LIMIT;
+  if (N == 0) return QTEA_OK;
+  if (!y || !aligned(y, 4)) return QTEA_ERR_INVALID_ARG;
+  if (K > 0 && (!packed || !aligned(packed, 16))) return QTEA_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (K == 0) {
+    if (cudaMemsetAsync(y, 0, (size_t)N * sizeof(float), st) != cudaSuccess) {
+      cudaGetLastError();
+      return QTEA_ERR_CUDA;
+    }
+    return QTEA_OK;
+  }
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= kStaticMaxDevices) return QTEA_ERR_UNSUPPORTED;
+  StaticDevice d;
+  int rc = static_setup(dev, &d);
+  if (rc) return rc;
+
+  // A layout record on the host stack that borrows the caller's packed codes and points the
+  // split-tile scratch at the static array; the planner and kernels below are the ones qtea_gemv uses.
+  qtea_layout l;
+  std::memset(&l, 0, sizeof(l));
+  l.N = N;
+  l.K = K;
+  l.K_pad = round_up(K, 64);
+  l.group_size = K;
+  l.n_salient = n_salient;
+  l.format = QTEA_FMT_2BIT;
+  l.packed_bytes = (size_t)N * (size_t)(l.K_pad / 4);
+  l.packed = const_cast<uint8_t*>(packed);
+  l.device = dev;
+  l.sm_count = d.sm_count;
+  l.smem_optin = d.smem_optin;
+  l.act_bits = 24;
+  l.n_tiles = (N + kTileRows - 1) / kTileRows;
+  l.n_chunks = (l.K_pad + kChunkCols - 1) / kChunkCols;
+  l.workspace = reinterpret_cast<float*>(d.scratch);
+  l.counters = reinterpret_cast<unsigned*>(d.scratch + kStaticWsBytes);
+  l.status = reinterpret_cast<int*>(d.scratch + kStaticWsBytes + kStaticCtrBytes);
+  l.m1_ok = false;
+  if (d.m1_ok) {
+    cuuint64_t dims[2] = {(cuuint64_t)(l.K_pad / 4), (cuuint64_t)N};
+    cuuint64_t strides[1] = {(cuuint64_t)(l.K_pad / 4)};
+    cuuint32_t box[2] = {(cuuint32_t)kChunkRowBytes, (cuuint32_t)kBoxRows};
+    cuuint32_t estr[2] = {1, 1};
+    l.m1_ok = get_encode_tiled()(&l.tmap, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, l.packed, dims, strides, box, estr,
+                                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
+
+  qtea_gemv_problem q;
+  q.x = x;
+  q.packed_ternary = &l;
+  q.row_scale = row_scale;
+  q.col_scale = col_scale;
+  q.salient_idx = salient_idx;
+  q.residual_vals = residual_vals;
+  q.residual_idx = residual_idx;
+  q.y = y;
+  rc = check_problem(q, 1);
+  if (rc) return rc;
+  const int idx0 = 0;
+  rc = l.m1_ok ? run_m1(&q, &idx0, 1, st) : launch_generic_problem(q, 1, st);
+  if (rc != QTEA_OK) cudaGetLastError();
+  return rc;
 }
 
 }  // extern "C"
