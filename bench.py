@@ -276,8 +276,10 @@ def qtea_arm(args):
     group_args = [[dict(x=g["x"], layout=g["layout"], row_scale=g["alpha"], col_scale=g["v"], salient_idx=g["sal"],
                         residual_vals=g["rv"], residual_idx=g["ri"], y=g["y"]) for g in L] for L in layers]
 
-    def capture(steps, with_events, grouped=True):
-        """One step = the 7 GEMVs of one layer: one grouped launch, or 7 single launches."""
+    def capture(steps, with_events, grouped=True, only=None):
+        """One step = the 7 GEMVs of one layer as one grouped launch, or 7 single launches, or
+        (only = j) GEMV j of the layer alone. Without events, consecutive launches overlap through
+        programmatic dependent launch; event-record nodes between launches serialise them."""
         gr = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gr, stream=stream):
             k = 0
@@ -291,7 +293,9 @@ def qtea_arm(args):
                         ext.record(ev[k][1], stream)
                     k += 1
                     continue
-                for gm in layers[li]:
+                for j, gm in enumerate(layers[li]):
+                    if only is not None and j != only:
+                        continue
                     if with_events:
                         ext.record(ev[k][0], stream)
                     qt.qtea_gemv(gm["x"], gm["layout"], gm["alpha"], gm["v"], gm["sal"], gm["rv"], gm["ri"],
@@ -301,8 +305,20 @@ def qtea_arm(args):
                     k += 1
         return gr
 
+    def timed_replay(gr):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            gr.replay()  # warm replay
+        barrier()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            gr.replay()
+            e1.record(stream)
+        barrier()
+        return e0.elapsed_time(e1)
+
     g_warm = capture(warmup, False)
-    g_timed = capture(args.steps, ext.ok)
+    g_timed = capture(args.steps, False)
     with torch.cuda.stream(stream):
         g_warm.replay()
     barrier()
@@ -319,7 +335,6 @@ def qtea_arm(args):
     barrier()
     clk = clocks.stop()
     total_ms = t_start.elapsed_time(t_end)
-    durs = [a_.elapsed_time(b_) for a_, b_ in ev[:args.steps]] if ext.ok else None
     status = max(qt.qtea_device_status(g["layout"]) for L in layers for g in L)
     if status:
         raise RuntimeError(f"device status {status} after the timed region")
@@ -330,29 +345,32 @@ def qtea_arm(args):
     bytes_all = sum(step_bytes[st % len(layers)] for st in range(args.steps)) * world
     value = bytes_all / (total_ms * 1e-3) / 1e9
 
-    # roofline of the GEMV kernel: the only kernel of the timed region, one grouped launch per step
-    if durs is None:  # no event-record nodes: fall back to the region average
-        durs = [total_ms / args.steps] * args.steps
+    # roofline of the GEMV kernel: the only kernel of the timed region, one grouped launch per
+    # step, launches back to back; its average launch duration is the region time / launches
     kern_bytes = sum(step_bytes[st % len(layers)] for st in range(args.steps))
-    achieved = kern_bytes / (sum(durs) * 1e-3) / 1e9
+    achieved = kern_bytes / (total_ms * 1e-3) / 1e9
     peak, peak_src = load_peaks()
+    # the same launches one at a time (event-record nodes between them), for the isolated duration
+    iso_us = None
+    if ext.ok:
+        g_ev = capture(args.steps, True)
+        timed_replay(g_ev)
+        iso_us = statistics.mean(a_.elapsed_time(b_) for a_, b_ in ev[:args.steps]) * 1e3
+        del g_ev
 
-    # ---- per-GEMV latency: the same steps with one launch per GEMV, each launch timed
+    # ---- per-GEMV latency: each GEMV of the layer alone, launched back to back over the layers
     per_shape = {}
-    if ext.ok and not args.no_per_shape:
-        g_single = capture(args.steps, True, grouped=False)
-        with torch.cuda.stream(stream):
-            g_single.replay()
-        barrier()
-        sd = [a_.elapsed_time(b_) for a_, b_ in ev]
+    if not args.no_per_shape:
         for j, gm in enumerate(layers[0]):
-            d = [sd[st * launches_per_step + j] * 1e3 for st in range(args.steps)]
-            med = statistics.median(d)
-            N, K, bts = gm["N"], gm["K"], gm["bytes"]
-            per_shape[gm["name"]] = {"N": N, "K": K, "s": gm["s"], "us_per_call": round(med, 3),
-                                     "gbs": round(bts / (med * 1e-6) / 1e9, 1),
+            gs = capture(args.steps, False, grouped=False, only=j)
+            ms = timed_replay(gs)
+            del gs
+            us = ms * 1e3 / args.steps
+            N, K = gm["N"], gm["K"]
+            bts = statistics.mean(L[j]["bytes"] for L in layers)
+            per_shape[gm["name"]] = {"N": N, "K": K, "s": gm["s"], "us_per_call": round(us, 3),
+                                     "gbs": round(bts / (us * 1e-6) / 1e9, 1),
                                      "eff_bits_per_weight": round(8 * (bts - 2 * K - 4 * N) / (N * K), 3)}
-        del g_single
 
     # ---- the other activation precision, same steps (reported beside the headline mode)
     alt = {}
@@ -444,7 +462,8 @@ def qtea_arm(args):
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                          "frac": round(achieved / peak, 4), "peak_source": peak_src, "traffic": traffic,
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
-                         "us_per_launch": round(1e3 * sum(durs) / args.steps, 3)},
+                         "us_per_launch": round(1e3 * total_ms / args.steps, 3),
+                         "us_per_launch_isolated": None if iso_us is None else round(iso_us, 3)},
             "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
             "setup_s": round(t_gen, 1),
         }

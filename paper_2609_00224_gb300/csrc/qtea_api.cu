@@ -146,6 +146,8 @@ bool group_add(M1Group& g, const qtea_gemv_problem& q) {
   a.n_tiles = l->n_tiles;
   a.n_chunks = l->n_chunks;
   a.act_bits = (l->act_bits == 16 && l->K >= kMinK16) ? 16 : 24;
+  a.vec_xv = aligned(q.x, 16) && aligned(q.col_scale, 16);
+  a.vec_res = (l->n_salient % kResBlock == 0) && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 2);
   a.unit_begin = g.gp.total_units;
   std::memcpy(&g.maps.m[g.gp.n_problems], &l->tmap, sizeof(CUtensorMap));
   if (g.gp.n_problems == 0) g.gp.status = l->status;
@@ -154,7 +156,7 @@ bool group_add(M1Group& g, const qtea_gemv_problem& q) {
   return true;
 }
 
-// Grid, ring depth and shared memory of the group; false if some CTA's staging does not fit.
+// Grid, ring depth and shared memory of the group; false if the ring does not fit.
 bool group_plan(M1Group& g, int sm_count, size_t smem_optin) {
   if (g.gp.n_problems == 0) return false;
   if (g.gp.total_units >= (1ll << 30)) return false;
@@ -162,15 +164,9 @@ bool group_plan(M1Group& g, int sm_count, size_t smem_optin) {
   if (g.grid > kMaxGrid) g.grid = kMaxGrid;
   for (int b = 0; b <= g.grid; ++b) g.gp.cta_u0[b] = (int)unit_begin_of(b, g.gp.total_units, g.grid);
   for (int stages = kMaxStages; stages >= kMinStages; --stages) {
-    g.gp.n_stages = stages;
-    size_t need = 0;
-    for (int b = 0; b < g.grid; ++b) {
-      size_t s = cta_smem_plan(g.gp.prob, g.gp.n_problems, g.gp.n_stages, g.gp.cta_u0[b], g.gp.cta_u0[b + 1], nullptr,
-                               nullptr, nullptr);
-      if (s > need) need = s;
-    }
-    if (need <= smem_optin) {
-      g.smem = need;
+    if (m1_smem_bytes(stages) <= smem_optin) {
+      g.gp.n_stages = stages;
+      g.smem = m1_smem_bytes(stages);
       return true;
     }
   }
@@ -197,7 +193,7 @@ int run_m1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st) 
       ++taken;
     }
     if (taken == 0) {
-      // a single problem whose staging does not fit: the generic kernel serves it
+      // the ring does not fit this device's shared memory: the generic kernel serves the problem
       int rc = launch_generic_problem(qs[idx[i]], 1, st);
       if (rc) return rc;
       ++i;

@@ -7,23 +7,30 @@
 //    problems form one sequence; one CTA per SM takes an equal contiguous share, so every SM
 //    streams the same number of weight bytes and one launch amortises its fixed costs over
 //    all problems.
-//  * TMA ring: a producer lane fetches each unit as two 256 x 128-byte boxes of packed 2-bit
-//    codes (cp.async.bulk.tensor, 128-byte swizzle) into a shared-memory ring guarded by
-//    mbarriers; eight consumer warps decode from shared memory, each lane owning two rows,
-//    so no cross-lane reduction is needed.
-//  * Decode: v*x (the column rescale of Sec. 3.3, fused into activation staging as the
-//    paper fuses it into its LUT precompute) is held per 512-column chunk as 24-bit fixed
-//    point split into three byte planes. Codes are masked four at a time into byte lanes and
-//    multiplied with dp4a, so sum_j c_j X_j is exact in integers; the ternary value is
-//    c - 1, whose contribution is removed with the chunk's sum of X.
-//  * Residual (Eq. 11): each CTA adds sum_c R x_{S_c} for the salient columns inside the
-//    chunks it decodes (located by binary search of the sorted salient list), so the
-//    residual work is spread like the weight stream; its loads are issued before the unit's
-//    decode to hide their latency. The values are never scaled by alpha or v.
+//  * Roles: eight consumer warps decode from shared memory only, each lane owning two rows of
+//    the tile (no cross-lane reduction). One producer lane keeps S code stages filled by TMA
+//    (two 256 x 128-byte boxes per unit, 128-byte swizzle). Three helper warps take the units
+//    round-robin and write each unit's auxiliary slot, in a ring of six: the chunk's v*x in
+//    fixed point and the unit's share of the residual as one sum per row. A helper starts a unit
+//    as soon as its slot is free, five units ahead of the consumers, so its loads are hidden.
+//  * Decode: v*x (the column rescale of Sec. 3.3, fused into staging as the paper fuses it
+//    into its LUT precompute) is held per 512-column chunk as 24-bit fixed point split into
+//    three byte planes (or 16-bit, two planes, where the caller allows it and the chunk has no
+//    dominant outlier). Codes are masked four at a time into byte lanes and multiplied with
+//    dp4a, so sum_j c_j X_j is exact in integers; the ternary value is c - 1, whose
+//    contribution is removed with the chunk's sum of X.
+//  * Residual (Eq. 11): a tile's salient entries are split over its chunks by index, in blocks
+//    of 8 (chunk ch of nc takes blocks [ch*nb/nc, (ch+1)*nb/nc)), so no search of the salient
+//    list is needed and the work follows the weight stream. The values are never scaled by
+//    alpha or v.
 //  * Split tiles are reduced by the last-arriving CTA (atomic counter, no spin-wait) in a
 //    fixed CTA order, so results are bitwise reproducible.
+//  * Programmatic dependent launch: before griddepcontrol.wait a CTA only initialises its
+//    barriers and starts the TMA of its first units' codes, which the library owns and no other
+//    kernel writes. Everything the caller owns (x, v, alpha, the residual, y) and the split-tile
+//    workspace is touched after the wait. Each CTA lets the next launch start once it is running.
 // Every wait on an mbarrier is bounded: after ~2 s the waiting thread records
-// QTEA_ERR_TIMEOUT in the status word and the CTA abandons its work.
+// QTEA_ERR_TIMEOUT in the status word and its role stops.
 #include <cuda_fp16.h>
 
 #include "qtea_internal.h"
@@ -32,7 +39,6 @@ namespace qtea {
 namespace {
 
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
-constexpr int kResPrefetch = 8;  // residual entries per lane loaded ahead of a unit's decode
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -57,12 +63,16 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
                : "memory");
 }
 
+// One potentially blocking test of the phase with the given parity: the thread may be suspended
+// until the phase completes or about kSuspendNs elapse, so waiting warps do not take issue slots.
+constexpr uint32_t kSuspendNs = 100000;
+
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
-      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(kSuspendNs)
       : "memory");
   return ok != 0;
 }
@@ -71,9 +81,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int* status) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = global_ns();
-  for (uint32_t i = 1;; ++i) {
+  for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0 && global_ns() - t0 > kWaitLimitNs) {
+    if (global_ns() - t0 > kWaitLimitNs) {
       atomicExch(status, (int)QTEA_ERR_TIMEOUT);
       return false;
     }
@@ -94,6 +104,28 @@ __device__ __forceinline__ float h2f(uint16_t b) { return __half2float(__ushort_
 __device__ __forceinline__ int unit_owner(long long u, long long total, int grid) {
   return (int)(((u + 1) * grid - 1) / total);
 }
+
+struct UnitPos {
+  int p, t, ch;  // problem, tile, chunk
+};
+
+__device__ __forceinline__ UnitPos unit_pos(const ProblemArgs* tab, int n_problems, long long u) {
+  int p = 0;
+  while (p + 1 < n_problems && u >= tab[p + 1].unit_begin) ++p;
+  const int v = (int)(u - tab[p].unit_begin);
+  const int nc = tab[p].n_chunks;
+  const int t = v / nc;
+  return {p, t, v - t * nc};
+}
+
+// The two TMA boxes of unit (t, ch) into ring stage `dst`, completing on `bar`.
+__device__ __forceinline__ void issue_unit(const CUtensorMap* map, int t, int ch, uint32_t dst, uint32_t bar) {
+  mbar_arrive_expect_tx(bar, kStageBytes);
+  tma_load_2d(dst, map, ch * kChunkRowBytes, t * kTileRows, bar);
+  tma_load_2d(dst + kBoxBytes, map, ch * kChunkRowBytes, t * kTileRows + kBoxRows, bar);
+}
+
+// ---------------------------------------------------------------- decode (consumers)
 
 // Accumulators of one row for one chunk: [plane][scale set]; scale set 0 holds codes of
 // column groups 0 and 2 (weight 1), set 1 codes of groups 1 and 3 (weight 4).
@@ -191,25 +223,16 @@ __device__ __forceinline__ void decode_unit(const uint4* row0, const uint4* row1
   }
 }
 
-__device__ __forceinline__ void add_residual(float (&rp)[4], uint16_t rv, uint8_t rb, int c, float xv) {
-  const int pos = (rb >> (2 * (c & 3))) & 3;
-  const float val = h2f(rv) * xv;
-  rp[0] += pos == 0 ? val : 0.f;
-  rp[1] += pos == 1 ? val : 0.f;
-  rp[2] += pos == 2 ? val : 0.f;
-  rp[3] += pos == 3 ? val : 0.f;
-}
+// ---------------------------------------------------------------- staging (helpers)
 
-// Activation staging of one 512-column chunk by one warp, 16 columns per lane, in two steps
-// so that the loads of every chunk can be issued before the weight stream starts.
+// x and v of columns 16*lane .. 16*lane+15 of one chunk, as fp16 pairs (zero beyond K).
 struct ChunkLoads {
-  uint32_t x[8], v[8];  // fp16 pairs of columns 16*lane .. 16*lane+15 (zero beyond K)
+  uint32_t x[8], v[8];
 };
 
-__device__ __noinline__ void load_chunk(const ProblemArgs& a, int ch, int lane, ChunkLoads& L) {
+__device__ __forceinline__ void load_chunk(const ProblemArgs& a, int ch, int lane, ChunkLoads& L) {
   const int col0 = ch * kChunkCols + lane * 16;
-  const bool vec_ok = ((reinterpret_cast<uintptr_t>(a.x) | reinterpret_cast<uintptr_t>(a.v)) & 15) == 0;
-  if (vec_ok && col0 + 16 <= a.K) {
+  if (a.vec_xv && col0 + 16 <= a.K) {
     const uint4* xv4 = reinterpret_cast<const uint4*>(a.x + col0);
     const uint4* vv4 = reinterpret_cast<const uint4*>(a.v + col0);
     const uint4 xa = __ldg(xv4), xb = __ldg(xv4 + 1), va = __ldg(vv4), vb = __ldg(vv4 + 1);
@@ -229,10 +252,8 @@ __device__ __noinline__ void load_chunk(const ProblemArgs& a, int ch, int lane, 
   }
 }
 
-// Planes, scale, sum of X, salient range and x at the chunk's first kChunkSalCap salient
-// columns (gathered from the lanes' registers), written to one shared-memory slot.
-__device__ __noinline__ void compute_chunk(const ProblemArgs& a, int ch, const ChunkLoads& L, uint8_t* slot,
-                                              const int* salc, int lane) {
+// The chunk's v*x as fixed point: byte planes of this lane's word, and (lane 0) the metadata.
+__device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLoads& L, uint8_t* ax, int lane) {
   float xt[16];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {  // exact: fp16 x fp16 fits fp32
@@ -264,7 +285,7 @@ __device__ __noinline__ void compute_chunk(const ProblemArgs& a, int ch, const C
     X[i] = __float2int_rn(xt[i] * inv_q);
     sx += X[i];
   }
-  uint4* dst = reinterpret_cast<uint4*>(slot + (size_t)lane * kPlaneBytesPerWord);
+  uint4* dst = reinterpret_cast<uint4*>(ax + (size_t)lane * kPlaneBytesPerWord);
   if (two) {
     uint32_t reg[8];
 #pragma unroll
@@ -297,311 +318,213 @@ __device__ __noinline__ void compute_chunk(const ProblemArgs& a, int ch, const C
   }
 #pragma unroll
   for (int o = 16; o; o >>= 1) sx += __shfl_xor_sync(0xffffffffu, sx, o);
-  // salient entries with column in [512 ch, 512 ch + 512): lanes 0 and 1 search the two bounds
-  int bound = 0;
-  if (lane < 2) {
-    const int lim = (ch + lane) * kChunkCols;
-    int lo = 0, hi = a.s;
-    while (lo < hi) {
-      const int mid = (lo + hi) >> 1;
-      if (salc[mid] < lim) lo = mid + 1;
-      else hi = mid;
-    }
-    bound = lo;
-  }
-  const int c_lo = __shfl_sync(0xffffffffu, bound, 0);
-  const int c_hi = max(__shfl_sync(0xffffffffu, bound, 1), c_lo);
-  const int n_xs = min(c_hi - c_lo, kChunkSalCap);
-  // x at salient column j lives in lane (j mod 512) / 16, element j mod 16
-  float* xs = reinterpret_cast<float*>(slot + kPlaneBytesPerChunk + sizeof(ChunkMeta));
-#pragma unroll
-  for (int r = 0; r < kChunkSalCap / 32; ++r) {
-    const int idx = lane + 32 * r;
-    int col = idx < n_xs ? salc[c_lo + idx] - ch * kChunkCols : 0;
-    col = col < 0 ? 0 : (col > kChunkCols - 1 ? kChunkCols - 1 : col);
-    const int src = col >> 4, word = (col & 15) >> 1;
-    uint32_t got = 0;
-#pragma unroll
-    for (int w = 0; w < 8; ++w) {
-      const uint32_t v = __shfl_sync(0xffffffffu, L.x[w], src);
-      got = (w == word) ? v : got;
-    }
-    if (idx < n_xs) xs[idx] = h2f((uint16_t)((col & 1) ? (got >> 16) : (got & 0xffffu)));
-  }
   if (lane == 0) {
     ChunkMeta mm;
     mm.scale4 = __uint_as_float((uint32_t)(127 + e - qsh - 2) << 23);  // q / 4
-    mm.c_lo = c_lo;
-    mm.c_hi = c_hi;
     mm.planes = two ? 2 : 3;
     mm.sum_x = sx;
-    mm.pad2 = 0;
-    *reinterpret_cast<ChunkMeta*>(slot + kPlaneBytesPerChunk) = mm;
+    mm.pad[0] = mm.pad[1] = 0;
+    *reinterpret_cast<ChunkMeta*>(ax + kAuxMeta) = mm;
   }
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
-    qtea_gemv_m1_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ GroupParams gp) {
-  extern __shared__ uint8_t smem_raw[];
-  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  const int warp = threadIdx.x >> 5;
-  const int lane = threadIdx.x & 31;
-  const int grid = gridDim.x;
-  const int b = blockIdx.x;
-  const int S = gp.n_stages;
-  const int NP = gp.n_problems;
+// Accumulate one salient entry (value r, x at its column xj, position pos in the group of four).
+__device__ __forceinline__ void add_entry(float (&acc)[4], float r, float xj, int pos) {
+  const float val = r * xj;
+  acc[0] += pos == 0 ? val : 0.f;
+  acc[1] += pos == 1 ? val : 0.f;
+  acc[2] += pos == 2 ? val : 0.f;
+  acc[3] += pos == 3 ? val : 0.f;
+}
 
-  // ---- prologue 1: the problem table is copied to shared memory by all threads at once (its
-  //      first reads would otherwise be a chain of constant-cache misses); the copy sits in the
-  //      ring, which no copy has been issued into yet
-  ProblemArgs* prob = reinterpret_cast<ProblemArgs*>(smem);
-  {
-    const uint32_t* src = reinterpret_cast<const uint32_t*>(gp.prob);
-    uint32_t* dst = reinterpret_cast<uint32_t*>(prob);
-    const int words = NP * (int)(sizeof(ProblemArgs) / 4);
-    for (int i = threadIdx.x; i < words; i += blockDim.x) dst[i] = src[i];
+// x at the salient columns of entries e0 .. e0+31 (lane j holds entry e0 + j, zero past e_end).
+__device__ __forceinline__ float gather_salient_x(const ProblemArgs& a, int e0, int e_end, int lane) {
+  const int e = e0 + lane;
+  if (e >= e_end) return 0.f;
+  int col = __ldg(a.sal + e);
+  col = col < 0 ? 0 : (col >= a.K ? a.K - 1 : col);
+  return h2f(__ldg(a.x + col));
+}
+
+// Scalar loads of a residual block, for shapes or pointers the vector loads cannot serve.
+struct ResBlock {
+  uint4 rv;     // 8 fp16 values
+  uint32_t rp;  // 8 positions, 2 bits each
+};
+
+__device__ __noinline__ ResBlock load_block_scalar(const uint16_t* rvals, const uint8_t* ridx, int s, int q, int e0) {
+  const int rs = (s + 3) >> 2;
+  uint32_t h[8];
+  uint32_t pos = 0;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    const int e = e0 + j;
+    h[j] = e < s ? __ldg(rvals + (size_t)q * s + e) : 0u;
+    const uint32_t pb = e < s ? __ldg(ridx + (size_t)q * rs + e / 4) : 0u;
+    pos |= ((pb >> (2 * (e & 3))) & 3u) << (2 * j);
   }
-  if (warp == kProducerWarp && lane < NP)
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.m[lane])) : "memory");
-  const int u0 = gp.cta_u0[b], u1 = gp.cta_u0[b + 1];
+  ResBlock b;
+  b.rv = make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
+  b.rp = pos;
+  return b;
+}
+
+// Values and positions of residual block b (entries 8b .. 8b+7) of group q.
+__device__ __forceinline__ void load_block(const ProblemArgs& a, int q, int b, uint4& rv, uint32_t& rp) {
+  rv = make_uint4(0, 0, 0, 0);
+  rp = 0;
+  if (q >= (a.N >> 2)) return;
+  const int e0 = b * kResBlock;
+  if (a.vec_res) {
+    rv = __ldg(reinterpret_cast<const uint4*>(a.rvals + (size_t)q * a.s + e0));
+    rp = __ldg(reinterpret_cast<const uint16_t*>(a.ridx + (size_t)q * ((a.s + 3) >> 2) + e0 / 4));
+  } else {
+    const ResBlock blk = load_block_scalar(a.rvals, a.ridx, a.s, q, e0);
+    rv = blk.rv;
+    rp = blk.rp;
+  }
+}
+
+// Stage unit (t, ch) of problem *pa into auxiliary slot ax. First the planes and metadata, which
+// need x and v only, then (after the arrival on planes_bar) the residual sums of the tile's 512
+// rows over the unit's salient blocks: the consumers wait for those only after the decode. The
+// residual loads go out after the planes are published, so they never delay them (a unit's first
+// planes are on the critical path of the launch). Lane owns residual groups lane + 32k.
+__device__ __noinline__ void stage_unit(const ProblemArgs* pa, int t, int ch, uint8_t* ax, int lane,
+                                        uint32_t planes_bar) {
+  const ProblemArgs a = *pa;
+  {
+    ChunkLoads L;
+    load_chunk(a, ch, lane, L);
+    write_planes(a, L, ax, lane);
+  }
+  mbar_arrive(planes_bar);
+
+  const int nb = (a.s + kResBlock - 1) / kResBlock;
+  const int b0 = (int)((long long)ch * nb / a.n_chunks), b1 = (int)((long long)(ch + 1) * nb / a.n_chunks);
+  const int e_end = min(b1 * kResBlock, a.s);
+  const int qb = t * (kTileRows / 4) + lane;
+  // the salient indices and the first two residual blocks go out together; x at the salient
+  // columns follows as soon as the indices arrive
+  const bool has_entry = b0 * kResBlock + lane < e_end;  // lane j: entry 8 * b0 + j of the first window
+  int col = has_entry ? __ldg(a.sal + b0 * kResBlock + lane) : 0;
+  uint4 rvA[4], rvB[4];
+  uint32_t rpA[4], rpB[4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    rvA[k] = rvB[k] = make_uint4(0, 0, 0, 0);
+    rpA[k] = rpB[k] = 0;
+    if (b0 < b1) load_block(a, qb + 32 * k, b0, rvA[k], rpA[k]);
+    if (b0 + 1 < b1) load_block(a, qb + 32 * k, b0 + 1, rvB[k], rpB[k]);
+  }
+  col = col < 0 ? 0 : (col >= a.K ? a.K - 1 : col);
+  float xs = has_entry ? h2f(__ldg(a.x + col)) : 0.f;
+
+  float acc[4][4];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) acc[k][0] = acc[k][1] = acc[k][2] = acc[k][3] = 0.f;
+#pragma unroll 1
+  for (int b = b0; b < b1; ++b) {
+    const int w = (b - b0) & 3;  // block within the 32-entry window of xs
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float xj = __shfl_sync(0xffffffffu, xs, w * kResBlock + j);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const uint32_t wd = (j < 2) ? rvA[k].x : (j < 4) ? rvA[k].y : (j < 6) ? rvA[k].z : rvA[k].w;
+        const float r = h2f((uint16_t)((j & 1) ? (wd >> 16) : (wd & 0xffffu)));
+        add_entry(acc[k], r, xj, (int)((rpA[k] >> (2 * j)) & 3u));
+      }
+    }
+    // next block: B moves to A, the one after it is loaded into B; a new window of x every 4
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      rvA[k] = rvB[k];
+      rpA[k] = rpB[k];
+      if (b + 2 < b1) load_block(a, qb + 32 * k, b + 2, rvB[k], rpB[k]);
+    }
+    if (w == 3 && b + 1 < b1) xs = gather_salient_x(a, (b + 1) * kResBlock, e_end, lane);
+  }
+  float4* res = reinterpret_cast<float4*>(ax + kAuxRes);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) res[lane + 32 * k] = make_float4(acc[k][0], acc[k][1], acc[k][2], acc[k][3]);
+}
+
+// ---------------------------------------------------------------- roles
+
+struct Ring {
+  uint8_t* codes;         // [S][kStageBytes]
+  uint8_t* aux;           // [kAuxSlots][kAuxBytes]
+  const ProblemArgs* tab; // [n_problems], copied from the kernel parameters
+  uint64_t* full_c;       // [S] codes landed
+  uint64_t* empty_c;      // [S] consumers released the code stage
+  uint64_t* planes_a;     // [kAuxSlots] planes and metadata of the auxiliary slot written
+  uint64_t* full_a;       // [kAuxSlots] residual sums of the auxiliary slot written
+  uint64_t* empty_a;      // [kAuxSlots] consumers released the auxiliary slot
+  int* last_fill;         // [S] number of fills issued into each code stage
+  int S, n_problems;
+};
+
+// The producer lane: keeps the code stages filled. Fills 0 .. S-1 were issued before the grid
+// dependency wait.
+__device__ __noinline__ void producer_role(const TensorMaps& maps, const Ring r, int u0, int n_units, int* status) {
+  for (int i = r.S; i < n_units; ++i) {
+    const int st = i % r.S, fill = i / r.S;
+    if (!mbar_wait(smem_u32(&r.empty_c[st]), (uint32_t)((fill - 1) & 1), status)) break;
+    const UnitPos up = unit_pos(r.tab, r.n_problems, (long long)u0 + i);
+    issue_unit(&maps.m[up.p], up.t, up.ch, smem_u32(r.codes + (size_t)st * kStageBytes), smem_u32(&r.full_c[st]));
+    r.last_fill[st] = fill + 1;
+  }
+}
+
+// Helper warp h: units h, h + 3, ...; unit i uses auxiliary slot i % 6, so slot h and slot h + 3
+// belong to helper h alone and its waits on them come in order (a parity wait could not tell a
+// phase two ahead from the current one).
+__device__ __noinline__ void helper_role(const Ring r, int u0, int n_units, int h, int lane, int* status) {
+  for (int i = h; i < n_units; i += kHelperWarps) {
+    const int slot = i % kAuxSlots, fill = i / kAuxSlots;
+    if (fill > 0) {
+      const bool ok = mbar_wait(smem_u32(&r.empty_a[slot]), (uint32_t)((fill - 1) & 1), status);
+      if (!__all_sync(0xffffffffu, ok)) break;
+    }
+    const UnitPos up = unit_pos(r.tab, r.n_problems, (long long)u0 + i);
+    stage_unit(&r.tab[up.p], up.t, up.ch, r.aux + (size_t)slot * kAuxBytes, lane, smem_u32(&r.planes_a[slot]));
+    mbar_arrive(smem_u32(&r.full_a[slot]));
+  }
+}
+
+__device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, long long total, int u0, int u1,
+                                           int warp, int lane, int* status) {
   const int n_units = u1 - u0;
-  __syncthreads();
-
-  // ---- prologue 2: thread 0 plans shared memory (chunk slots, salient indices, residual ring,
-  //      barriers); every thread derives the plan's offsets from the shared copy
-  size_t misc_off = 0;
-  int n_slots = 0;
-  cta_smem_plan(prob, NP, S, u0, u1, nullptr, &n_slots, &misc_off);
-  float* rsum = reinterpret_cast<float*>(smem + misc_off);  // per-warp gather of residual sums
-  StageSlot* slots = reinterpret_cast<StageSlot*>(smem + misc_off + kResidFloats * sizeof(float));
-  uint64_t* bars = reinterpret_cast<uint64_t*>(slots + kMaxProblems);
-  uint64_t* full = bars;
-  uint64_t* empty = bars + S;
-  if (threadIdx.x == 0) {
-    cta_smem_plan(prob, NP, S, u0, u1, slots, nullptr, nullptr);
-    for (int i = 0; i < S; ++i) {
-      mbar_init(smem_u32(&full[i]), 1);                // producer arrival + TMA bytes
-      mbar_init(smem_u32(&empty[i]), kConsumerWarps);  // one arrival per consumer warp
-    }
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-  }
-  __syncthreads();
-  // per-problem values the loops need, out of the shared copy into registers
-  int p_ub[kMaxProblems], p_nc[kMaxProblems];
-#pragma unroll
-  for (int p = 0; p < kMaxProblems; ++p) {
-    p_ub[p] = p < NP ? (int)prob[p].unit_begin : 0x7fffffff;
-    p_nc[p] = p < NP ? prob[p].n_chunks : 1;
-  }
-
-  // ---- prologue 3: issue the loads of the salient indices and of the activations of every
-  //      chunk this CTA touches (one warp per chunk, kBatch chunks per warp in flight) before the
-  //      weight stream competes with them for memory bandwidth
-  constexpr int kBatch = 4;
-  constexpr int kSalPerThread = 8;
-  constexpr int kStageWarps = kConsumerWarps + 1;
-  int n_items = 0;
-  for (int j = 0; j < n_slots; ++j) n_items += slots[j].n_ch;
-  // the salient index loads go to registers with compile-time indices (a dynamically indexed
-  // array would live in local memory and every store would wait for its load)
-  int s_tot = 0;
-  for (int j = 0; j < n_slots; ++j) s_tot += slots[j].s;
-  auto sal_load = [&](int e) -> int {
-    int j = 0;
-    while (j + 1 < n_slots && e >= slots[j].s) {
-      e -= slots[j].s;
-      ++j;
-    }
-    return gp.prob[slots[j].p].sal[e];
-  };
-  int sal_val[kSalPerThread];
-#pragma unroll
-  for (int k2 = 0; k2 < kSalPerThread; ++k2) {
-    const int e = threadIdx.x + k2 * blockDim.x;
-    sal_val[k2] = e < s_tot ? sal_load(e) : 0;
-  }
-  auto item_of = [&](int item, int& j, int& k) {
-    j = 0;
-    while (j + 1 < n_slots && item >= slots[j].n_ch) {
-      item -= slots[j].n_ch;
-      ++j;
-    }
-    k = item;
-  };
-  ChunkLoads L[kBatch];
-#pragma unroll 1
-  for (int r = 0; r < kBatch; ++r) {
-    const int item = warp + r * kStageWarps;
-    if (item < n_items) {
-      int j, k;
-      item_of(item, j, k);
-      const ProblemArgs& a = prob[slots[j].p];
-      int ch = slots[j].ch_start + k;
-      if (ch >= a.n_chunks) ch -= a.n_chunks;
-      load_chunk(a, ch, lane, L[r]);
-    }
-  }
-
-  // unit cursor: problem, tile, chunk, slot and slot-local chunk, advanced without division
-  struct Cursor {
-    int p, t, ch, j, li;
-  };
-  Cursor start;
-  {
-    int p = 0;
-    while (p + 1 < NP && u0 >= p_ub[p + 1]) ++p;
-    const int v0 = u0 - p_ub[p];
-    start.p = p;
-    start.t = v0 / p_nc[p];
-    start.ch = v0 - start.t * p_nc[p];
-    start.j = 0;
-    start.li = 0;
-  }
-  auto advance = [&](Cursor& c, int u_next) {
-    const int nc = p_nc[c.p];
-    if (++c.ch == nc) {
-      c.ch = 0;
-      ++c.t;
-    }
-    if (++c.li == nc) c.li = 0;
-    if (c.p + 1 < NP && u_next >= p_ub[c.p + 1]) {
-      ++c.p;
-      c.t = 0;
-      c.ch = 0;
-      c.li = 0;
-      while (c.j + 1 < n_slots && slots[c.j].p != c.p) ++c.j;
-    }
-  };
-  // every field the loops read from the problem table is kept in registers or re-read from
-  // the kernel parameters below, so the ring may be overwritten once everyone is past here
-  __syncthreads();
-
-  // ---- the first ring fills go out now, behind the staging loads
-  auto issue = [&](const Cursor& c, int st) {
-    const uint32_t bar = smem_u32(&full[st]);
-    const uint32_t dst = smem_u32(smem + (size_t)st * kStageBytes);
-    mbar_arrive_expect_tx(bar, kStageBytes);
-    tma_load_2d(dst, &maps.m[c.p], c.ch * kChunkRowBytes, c.t * kTileRows, bar);
-    tma_load_2d(dst + kBoxBytes, &maps.m[c.p], c.ch * kChunkRowBytes, c.t * kTileRows + kBoxRows, bar);
-  };
-  if (warp == kProducerWarp && lane == 0) {
-    Cursor c = start;
-    for (int i = 0; i < n_units && i < S; ++i) {
-      issue(c, i);
-      advance(c, u0 + i + 1);
-    }
-  }
-
-  // ---- prologue 4: salient indices to shared memory, then the planes of every chunk
-  {
-    auto sal_store = [&](int e, int col) {
-      int j = 0;
-      while (j + 1 < n_slots && e >= slots[j].s) {
-        e -= slots[j].s;
-        ++j;
-      }
-      const int K = gp.prob[slots[j].p].K;
-      reinterpret_cast<int*>(smem + slots[j].salc)[e] = col < 0 ? 0 : (col >= K ? K - 1 : col);
-    };
-#pragma unroll
-    for (int k2 = 0; k2 < kSalPerThread; ++k2) {
-      const int e = threadIdx.x + k2 * blockDim.x;
-      if (e < s_tot) sal_store(e, sal_val[k2]);
-    }
-    for (int e = threadIdx.x + kSalPerThread * blockDim.x; e < s_tot; e += blockDim.x) sal_store(e, sal_load(e));
-  }
-  __syncthreads();
-  for (int r0 = 0; r0 * kStageWarps < n_items; r0 += kBatch) {
-#pragma unroll 1
-    for (int r = 0; r < kBatch; ++r) {
-      const int item = warp + (r0 + r) * kStageWarps;
-      if (item < n_items) {
-        int j, k;
-        item_of(item, j, k);
-        const ProblemArgs& a = gp.prob[slots[j].p];
-        int ch = slots[j].ch_start + k;
-        if (ch >= a.n_chunks) ch -= a.n_chunks;
-        if (r0 > 0) load_chunk(a, ch, lane, L[r]);  // chunks beyond the first batch (long ranges)
-        compute_chunk(a, ch, L[r], smem + slots[j].chunks + (size_t)k * kSlotBytes,
-                      reinterpret_cast<const int*>(smem + slots[j].salc), lane);
-      }
-    }
-  }
-  __syncthreads();
-
-  // ---------------------------------------------------------------- producer: the TMA ring
-  if (warp == kProducerWarp) {
-    if (lane != 0) return;
-    Cursor c = start;
-    int st = 0, ph = 0;  // stage and its fill parity
-    int i = 0;
-    bool ok = true;
-    for (; i < n_units; ++i) {
-      if (i >= S) {
-        // wait until the consumers released the previous fill of this stage
-        if (!mbar_wait(smem_u32(&empty[st]), (uint32_t)(ph ^ 1), gp.status)) {
-          ok = false;
-          break;
-        }
-        issue(c, st);
-      }
-      advance(c, u0 + i + 1);
-      if (++st == S) {
-        st = 0;
-        ph ^= 1;
-      }
-    }
-    // drain: no bulk copy may still be writing shared memory when the CTA exits
-    const int n_issued = ok ? n_units : i;
-    for (int s2 = 0; s2 < S && s2 < n_issued; ++s2) {
-      const int fills = (n_issued - s2 + S - 1) / S;  // fills of stage s2
-      if (!mbar_wait(smem_u32(&full[s2]), (uint32_t)((fills - 1) & 1), gp.status)) break;
-    }
-    return;
-  }
-
-  // ---------------------------------------------------------------- consumers: decode
   const int ra = warp * 64 + lane;  // tile rows owned by this lane: ra and ra + 32
   const int sw = lane & 7;          // 128-byte swizzle phase of both rows
-  const int g = lane & 15, half = lane >> 4;  // residual work: group g of the warp's 16, parity half
-  float yacc0 = 0.f, yacc1 = 0.f;
-  float rp[4] = {0.f, 0.f, 0.f, 0.f};
-  Cursor c = start;
-  int st = 0, ph = 0;
-  const long long total = gp.total_units;
+  const int grid = gridDim.x;
+  float yacc0 = 0.f, yacc1 = 0.f, racc0 = 0.f, racc1 = 0.f;
+  uint16_t al0 = 0, al1 = 0;  // raw fp16 bits: converted at the tile's end, so no wait on the load here
+  bool need_alpha = true;
+  UnitPos c = unit_pos(r.tab, r.n_problems, u0);
 
   for (int i = 0; i < n_units; ++i) {
     const int u = u0 + i;
-    const StageSlot& sl = slots[c.j];
-    const uint8_t* slot = smem + sl.chunks + (size_t)c.li * kSlotBytes;
-
-    // this unit's residual entries (salient columns inside the chunk, rows of the lane's
-    // group) are loaded before the decode and used after it
-    const ProblemArgs& a = gp.prob[c.p];
-    const ChunkMeta m = *reinterpret_cast<const ChunkMeta*>(slot + kPlaneBytesPerChunk);
-    const int rs = (a.s + 3) >> 2;
-    const int q = (c.t * kTileRows + warp * 64) / 4 + g;
-    const bool q_ok = q < (a.N >> 2);
-    const uint16_t* rvq = a.rvals + (size_t)q * a.s;
-    const uint8_t* riq = a.ridx + (size_t)q * rs;
-    uint16_t pre_v[kResPrefetch];
-    uint8_t pre_b[kResPrefetch];
-#pragma unroll
-    for (int k = 0; k < kResPrefetch; ++k) {
-      const int cc = m.c_lo + half + 2 * k;
-      const bool okk = q_ok && cc < m.c_hi;
-      pre_v[k] = okk ? __ldg(rvq + cc) : (uint16_t)0;
-      pre_b[k] = okk ? __ldg(riq + (cc >> 2)) : (uint8_t)0;
+    const int st = i % r.S, slot = i % kAuxSlots;
+    const ProblemArgs& a = r.tab[c.p];
+    const int n_chunks = a.n_chunks, N = a.N;
+    const int row0g = c.t * kTileRows + ra, row1g = row0g + 32;
+    if (need_alpha) {  // used at the tile's end; the loads complete during the decode
+      al0 = row0g < N ? __ldg(a.alpha + row0g) : (uint16_t)0;
+      al1 = row1g < N ? __ldg(a.alpha + row1g) : (uint16_t)0;
+      need_alpha = false;
     }
+    bool ok = mbar_wait(smem_u32(&r.full_c[st]), (uint32_t)((i / r.S) & 1), status);
+    ok = ok && mbar_wait(smem_u32(&r.planes_a[slot]), (uint32_t)((i / kAuxSlots) & 1), status);
+    if (!__all_sync(0xffffffffu, ok)) break;
 
-    bool failed = !mbar_wait(smem_u32(&full[st]), (uint32_t)ph, gp.status);
-    // all lanes agree on failure before touching the data or the barriers
-    if (__any_sync(0xffffffffu, failed)) break;
-
-    const uint4* row0 = reinterpret_cast<const uint4*>(smem + (size_t)st * kStageBytes + (size_t)ra * kChunkRowBytes);
+    const uint8_t* ax = r.aux + (size_t)slot * kAuxBytes;
+    const ChunkMeta m = *reinterpret_cast<const ChunkMeta*>(ax + kAuxMeta);
+    const uint4* row0 =
+        reinterpret_cast<const uint4*>(r.codes + (size_t)st * kStageBytes + (size_t)ra * kChunkRowBytes);
     const uint4* row1 = row0 + 32 * (kChunkRowBytes / 16);
-    const uint4* pl = reinterpret_cast<const uint4*>(slot);
+    const uint4* pl = reinterpret_cast<const uint4*>(ax);
     long long d0, d1;
     if (m.planes == 2) {
       RowAcc<2> a0, a1;
@@ -614,96 +537,152 @@ __global__ void __launch_bounds__(kThreads, 1)
       d0 = finish_chunk<3>(a0, m.sum_x);
       d1 = finish_chunk<3>(a1, m.sum_x);
     }
+    ok = mbar_wait(smem_u32(&r.full_a[slot]), (uint32_t)((i / kAuxSlots) & 1), status);
+    if (!__all_sync(0xffffffffu, ok)) break;
+    const float* res = reinterpret_cast<const float*>(ax + kAuxRes);
+    racc0 += res[ra];
+    racc1 += res[ra + 32];
     __syncwarp();
-    if (lane == 0) mbar_arrive(smem_u32(&empty[st]));  // release the stage to the producer
-
+    if (lane == 0) {  // release the code stage and the auxiliary slot
+      mbar_arrive(smem_u32(&r.empty_c[st]));
+      mbar_arrive(smem_u32(&r.empty_a[slot]));
+    }
     yacc0 += (float)d0 * m.scale4;
     yacc1 += (float)d1 * m.scale4;
 
-    // residual (Eq. 11) of the unit's salient columns, unscaled by alpha and v
-    {
-      const float* xs = reinterpret_cast<const float*>(slot + kPlaneBytesPerChunk + sizeof(ChunkMeta));
-      const int* salc = reinterpret_cast<const int*>(smem + sl.salc);
-#pragma unroll
-      for (int k = 0; k < kResPrefetch; ++k) {
-        const int cc = m.c_lo + half + 2 * k;
-        if (q_ok && cc < m.c_hi) {
-          const float xv = (cc - m.c_lo < kChunkSalCap) ? xs[cc - m.c_lo] : h2f(__ldg(a.x + salc[cc]));
-          add_residual(rp, pre_v[k], pre_b[k], cc, xv);
-        }
-      }
-      if (q_ok) {
-        for (int cc = m.c_lo + 2 * kResPrefetch + half; cc < m.c_hi; cc += 2) {
-          const float xv = (cc - m.c_lo < kChunkSalCap) ? xs[cc - m.c_lo] : h2f(__ldg(a.x + salc[cc]));
-          add_residual(rp, __ldg(rvq + cc), __ldg(riq + (cc >> 2)), cc, xv);
-        }
-      }
-    }
-
     // ---- tile epilogue once this CTA's part of tile t is done
-    if (c.ch == p_nc[c.p] - 1 || u == u1 - 1) {
+    if (c.ch == n_chunks - 1 || u == u1 - 1) {
       const int t = c.t;
-      const long long A = (long long)p_ub[c.p] + (long long)t * p_nc[c.p], B = A + p_nc[c.p];
-      // per-row residual sums: lane (g, half) holds positions 0..3 of group g; gather by row
-      float* rw = rsum + (size_t)warp * (16 * 2 * 4);
-#pragma unroll
-      for (int k = 0; k < 4; ++k) rw[(g * 2 + half) * 4 + k] = rp[k];
-      __syncwarp();
-      // row ra of the warp is local row `lane` -> group lane/4, position lane%4; ra+32 -> group 8 + lane/4
-      const float res0 = rw[((lane >> 2) * 2 + 0) * 4 + (lane & 3)] + rw[((lane >> 2) * 2 + 1) * 4 + (lane & 3)];
-      const float res1 =
-          rw[((8 + (lane >> 2)) * 2 + 0) * 4 + (lane & 3)] + rw[((8 + (lane >> 2)) * 2 + 1) * 4 + (lane & 3)];
-      __syncwarp();
-      rp[0] = rp[1] = rp[2] = rp[3] = 0.f;
-      const int row0g = t * kTileRows + ra, row1g = row0g + 32;
-      const float al0 = row0g < a.N ? h2f(a.alpha[row0g]) : 0.f;
-      const float al1 = row1g < a.N ? h2f(a.alpha[row1g]) : 0.f;
-      const float val0 = al0 * yacc0 + res0;
-      const float val1 = al1 * yacc1 + res1;
+      const long long A = a.unit_begin + (long long)t * n_chunks, B = A + n_chunks;
+      const float val0 = h2f(al0) * yacc0 + racc0;
+      const float val1 = h2f(al1) * yacc1 + racc1;
+      float* y = a.y;
       if (A >= u0 && B <= u1) {
-        if (row0g < a.N) a.y[row0g] = val0;
-        if (row1g < a.N) a.y[row1g] = val1;
+        if (row0g < N) y[row0g] = val0;
+        if (row1g < N) y[row1g] = val1;
       } else {
         // partial tile: publish this warp's 64 rows, then the last of the tile's contributors
         // (per warp: counter t * kConsumerWarps + warp) sums all partials in CTA order. Slot 0
         // of a CTA holds the tile its range starts in, slot 1 the tile its range ends in.
+        float* ws = a.ws;
         const int my_slot = (u0 >= A) ? 0 : 1;
-        float* wsp = a.ws + ((size_t)b * 2 + my_slot) * kTileRows;
+        float* wsp = ws + ((size_t)blockIdx.x * 2 + my_slot) * kTileRows;
         wsp[ra] = val0;
         wsp[ra + 32] = val1;
-        __threadfence();
         __syncwarp();
         const int bf = unit_owner(A, total, grid), bl = unit_owner(B - 1, total, grid);
         int last = 0;
         if (lane == 0) {
+          // acq_rel at gpu scope: the warp's partials (ordered before by __syncwarp) are published
+          // with the increment, and the last arriver sees every other contributor's partials
           unsigned* ctr = a.counters + (size_t)t * kConsumerWarps + warp;
-          const unsigned prev = atomicAdd(ctr, 1u);
+          unsigned prev;
+          asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], 1;" : "=r"(prev) : "l"(ctr) : "memory");
           last = (prev == (unsigned)(bl - bf));  // every CTA in [bf, bl] holds units of this tile
-          if (last) {
-            __threadfence();
-            *ctr = 0u;  // self-reset for the next call
-          }
+          if (last) *ctr = 0u;                   // self-reset for the next call
         }
         last = __shfl_sync(0xffffffffu, last, 0);
+        __syncwarp();
         if (last) {
           float s0 = 0.f, s1 = 0.f;
           for (int cb = bf; cb <= bl; ++cb) {
-            const int cslot = (gp.cta_u0[cb] >= A) ? 0 : 1;
-            const float* src = a.ws + ((size_t)cb * 2 + cslot) * kTileRows;
+            const int cslot = (cta_u0[cb] >= A) ? 0 : 1;
+            const float* src = ws + ((size_t)cb * 2 + cslot) * kTileRows;
             s0 += __ldcg(src + ra);
             s1 += __ldcg(src + ra + 32);
           }
-          if (row0g < a.N) a.y[row0g] = s0;
-          if (row1g < a.N) a.y[row1g] = s1;
+          if (row0g < N) y[row0g] = s0;
+          if (row1g < N) y[row1g] = s1;
         }
       }
-      yacc0 = 0.f;
-      yacc1 = 0.f;
+      yacc0 = yacc1 = racc0 = racc1 = 0.f;
+      need_alpha = true;
     }
-    advance(c, u + 1);
-    if (++st == S) {
-      st = 0;
-      ph ^= 1;
+    if (++c.ch == n_chunks) {
+      c.ch = 0;
+      if (++c.t == a.n_tiles) {
+        c.t = 0;
+        ++c.p;
+      }
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    qtea_gemv_m1_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ GroupParams gp) {
+  extern __shared__ uint8_t smem_raw[];
+  // 1024-byte aligned base, formed by indexing (not through an integer) so that the compiler keeps
+  // the shared address space and the hot loops use shared-memory loads
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int S = gp.n_stages;
+  const int NP = gp.n_problems;
+  const int u0 = gp.cta_u0[blockIdx.x], u1 = gp.cta_u0[blockIdx.x + 1];
+  const int n_units = u1 - u0;
+
+  Ring r;
+  r.S = S;
+  r.n_problems = NP;
+  r.codes = smem;
+  r.aux = smem + (size_t)S * kStageBytes;
+  ProblemArgs* tab = reinterpret_cast<ProblemArgs*>(r.aux + (size_t)kAuxSlots * kAuxBytes);
+  r.tab = tab;
+  r.full_c = reinterpret_cast<uint64_t*>(tab + kMaxProblems);
+  r.empty_c = r.full_c + S;
+  r.planes_a = r.empty_c + S;
+  r.full_a = r.planes_a + kAuxSlots;
+  r.empty_a = r.full_a + kAuxSlots;
+  r.last_fill = reinterpret_cast<int*>(r.empty_a + kAuxSlots);
+
+  // the problem table goes to shared memory in one step (every thread one word): reading it
+  // from the parameter space field by field would be a chain of constant-cache misses
+  {
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(gp.prob);
+    uint32_t* dst = reinterpret_cast<uint32_t*>(tab);
+    const int words = NP * (int)(sizeof(ProblemArgs) / 4);
+    for (int i = threadIdx.x; i < words; i += kThreads) dst[i] = src[i];
+  }
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < S; ++i) {
+      mbar_init(smem_u32(&r.full_c[i]), 1);                // the producer's arrival with the TMA bytes
+      mbar_init(smem_u32(&r.empty_c[i]), kConsumerWarps);  // one arrival per consumer warp
+      r.last_fill[i] = 0;
+    }
+    for (int i = 0; i < kAuxSlots; ++i) {
+      mbar_init(smem_u32(&r.planes_a[i]), 32);             // every lane of the helper
+      mbar_init(smem_u32(&r.full_a[i]), 32);
+      mbar_init(smem_u32(&r.empty_a[i]), kConsumerWarps);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == kProducerWarp && lane < NP)
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.m[lane])) : "memory");
+  __syncthreads();
+
+  // the first fill of every code stage: library-owned codes only, so it may start before the wait
+  if (warp == kProducerWarp && lane == 0) {
+    for (int i = 0; i < S && i < n_units; ++i) {
+      const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
+      issue_unit(&maps.m[up.p], up.t, up.ch, smem_u32(r.codes + (size_t)i * kStageBytes), smem_u32(&r.full_c[i]));
+      r.last_fill[i] = 1;
+    }
+  }
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+
+  if (warp < kConsumerWarps) consumer_role(r, gp.cta_u0, gp.total_units, u0, u1, warp, lane, gp.status);
+  else if (warp < kProducerWarp) helper_role(r, u0, n_units, warp - kConsumerWarps, lane, gp.status);
+  else if (lane == 0) producer_role(maps, r, u0, n_units, gp.status);
+
+  // no bulk copy may still be writing shared memory when the CTA exits (after a timeout the
+  // consumers may not have waited for every fill)
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int s2 = 0; s2 < S; ++s2) {
+      const int f = r.last_fill[s2];
+      if (f > 0 && !mbar_wait(smem_u32(&r.full_c[s2]), (uint32_t)((f - 1) & 1), gp.status)) break;
     }
   }
 }
@@ -721,9 +700,20 @@ cudaError_t m1_configure(size_t smem_optin, size_t* dyn_max) {
   return cudaFuncSetAttribute(qtea_gemv_m1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
 }
 
+// Programmatic stream serialisation lets this launch start while the previous kernel on the
+// stream drains; the kernel waits for it (griddepcontrol.wait) before touching caller memory.
 cudaError_t launch_m1(const TensorMaps& maps, const GroupParams& p, int grid, size_t smem, cudaStream_t st) {
-  qtea_gemv_m1_kernel<<<grid, kThreads, smem, st>>>(maps, p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel, maps, p);
 }
 
 }  // namespace qtea

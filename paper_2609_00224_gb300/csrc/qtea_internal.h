@@ -11,16 +11,19 @@
 namespace qtea {
 
 // ---------------------------------------------------------------- batch-1 grouped stream-K kernel
-// One CTA per SM: 8 consumer warps (each lane owns 2 rows of a 512-row tile) and 1 producer
-// warp whose lane 0 drives the TMA ring. A unit of work is one (tile, chunk) pair of one
-// problem: 512 rows x 512 columns = 512 x 128 bytes of 2-bit codes, fetched as two 2D TMA
-// boxes of 256 rows with the 128-byte swizzle. One launch serves up to kMaxProblems
+// One CTA per SM: 8 consumer warps decode (each lane owns 2 rows of a 512-row tile), 3 helper
+// warps stage activations and residual sums, 1 producer warp drives the TMA. A unit of work is
+// one (tile, chunk) pair of one problem: 512 rows x 512 columns = 512 x 128 bytes of 2-bit codes,
+// fetched by TMA as two 2D boxes of 256 rows with the 128-byte swizzle into a code stage. Its
+// auxiliary slot (in a deeper ring of its own) holds the chunk's fixed-point v*x planes and the
+// unit's share of the residual as one sum per row. One launch serves up to kMaxProblems
 // independent GEMVs; their units form one sequence that is split evenly over the CTAs.
 constexpr int kMaxProblems = 8;
 constexpr int kMaxGrid = 1024;                                 // CTAs a launch may use
 constexpr int kConsumerWarps = 8;
-constexpr int kProducerWarp = kConsumerWarps;
-constexpr int kThreads = (kConsumerWarps + 1) * 32;
+constexpr int kHelperWarps = 3;                                // activation / residual staging
+constexpr int kProducerWarp = kConsumerWarps + kHelperWarps;  // TMA issue
+constexpr int kThreads = (kProducerWarp + 1) * 32;             // 384
 constexpr int kTileRows = 512;
 constexpr int kBoxRows = 256;
 constexpr int kChunkCols = 512;
@@ -32,21 +35,20 @@ constexpr int kPlaneBytesPerWord = 48;                         // 4 groups x 3 b
 constexpr int kPlaneBytesPerChunk = kWordsPerChunk * kPlaneBytesPerWord;  // 1536
 constexpr int kMaxStages = 3;
 constexpr int kMinStages = 2;
-constexpr int kResidFloats = kConsumerWarps * 16 * 2 * 4;      // per-warp gather of residual sums
-
-constexpr int kChunkSalCap = 64;                             // salient x values kept per staged chunk
+constexpr int kAuxSlots = 2 * kHelperWarps;                    // each helper owns two slots
+constexpr int kResBlock = 8;                                   // salient entries per residual block
 
 struct ChunkMeta {
   float scale4;      // q / 4, q the fixed-point quantum of v*x in this chunk (a power of two)
-  int c_lo, c_hi;    // salient entries whose column lies in the chunk
   int planes;        // byte planes of the chunk's fixed-point v*x: 3 (24-bit) or 2 (16-bit)
   long long sum_x;   // sum of the chunk's fixed-point v*x values
-  long long pad2;
+  long long pad[2];
 };
 
-// One staged chunk: activation planes, metadata, and x at (up to kChunkSalCap of) the
-// chunk's salient columns, in the order of the salient list.
-constexpr int kSlotBytes = kPlaneBytesPerChunk + (int)sizeof(ChunkMeta) + kChunkSalCap * 4;  // 1824
+// Auxiliary slot: planes [32 words][48 bytes], metadata, residual sums [512 rows].
+constexpr int kAuxMeta = kPlaneBytesPerChunk;
+constexpr int kAuxRes = kAuxMeta + (int)sizeof(ChunkMeta);
+constexpr int kAuxBytes = kAuxRes + kTileRows * (int)sizeof(float);  // 3616
 
 struct ProblemArgs {
   const uint16_t* x;        // [K] (M = 1)
@@ -60,6 +62,8 @@ struct ProblemArgs {
   unsigned* counters;       // [n_tiles][kConsumerWarps], zero between calls
   int N, K, s, n_tiles, n_chunks;
   int act_bits;             // 24: v*x in 24-bit fixed point; 16: 16-bit where a chunk allows it
+  int vec_xv;               // x and v are 16-byte aligned (vector loads)
+  int vec_res;              // s % 8 == 0 and rvals 16-byte / ridx 2-byte aligned (vector loads)
   long long unit_begin;     // first global unit of this problem
 };
 
@@ -80,53 +84,12 @@ __host__ __device__ inline long long unit_begin_of(int b, long long total, int g
   return (long long)b * total / grid;
 }
 
-// Per-problem staging of one CTA: the cyclic range of chunks its units touch.
-struct StageSlot {
-  int p;         // problem index
-  int ch_start;  // first chunk (cyclic range)
-  int n_ch;      // number of chunks staged
-  int s;         // salient count of the problem
-  int chunks;    // byte offset of n_ch chunk slots of kSlotBytes
-  int salc;      // byte offset of the clamped salient column indices (s ints)
-  int first_unit;  // first unit of this problem in the CTA's range
-  int pad;
-};
-
-// Shared-memory plan of the CTA whose units are [u0, u1). Identical on host (for the launch
-// size) and device.
-__host__ __device__ inline size_t cta_smem_plan(const ProblemArgs* prob, int n_problems, int n_stages, int u0, int u1,
-                                                StageSlot* slots, int* n_slots, size_t* misc_off) {
-  size_t off = (size_t)n_stages * kStageBytes;  // ring first, at the 1024-aligned base
-  int ns = 0;
-  for (int p = 0; p < n_problems; ++p) {
-    const ProblemArgs& a = prob[p];
-    const int pb = (int)a.unit_begin, pe = (int)a.unit_begin + a.n_tiles * a.n_chunks;
-    const int lo = u0 > pb ? u0 : pb, hi = u1 < pe ? u1 : pe;
-    if (lo >= hi) continue;
-    StageSlot sl;
-    sl.p = p;
-    sl.ch_start = (lo - pb) % a.n_chunks;
-    const int n = hi - lo;
-    sl.n_ch = n >= a.n_chunks ? a.n_chunks : n;
-    sl.s = a.s;
-    sl.first_unit = lo;
-    sl.pad = 0;
-    off = (off + 15) & ~(size_t)15;
-    sl.chunks = (int)off;
-    off += (size_t)sl.n_ch * kSlotBytes;
-    sl.salc = (int)off;
-    off += (size_t)(a.s > 0 ? a.s : 1) * sizeof(int);
-    if (slots) slots[ns] = sl;
-    ++ns;
-  }
-  off = (off + 15) & ~(size_t)15;
-  if (misc_off) *misc_off = off;
-  // misc: residual gather floats, staging table, barriers (ring full/empty)
-  off += (size_t)kResidFloats * sizeof(float);
-  off += (size_t)kMaxProblems * sizeof(StageSlot);
-  off += (size_t)2 * n_stages * sizeof(unsigned long long);
-  if (n_slots) *n_slots = ns;
-  return off + 1024;  // slack to align the dynamic smem base to 1024 bytes
+// Dynamic shared memory of the batch-1 kernel with S code stages: codes, auxiliary slots, the
+// problem table, the barriers (code stages: full, empty; auxiliary slots: planes written, residual
+// written, empty), the fills issued per code stage (for the drain), and 1024 bytes of slack.
+__host__ __device__ constexpr size_t m1_smem_bytes(int S) {
+  return (size_t)S * kStageBytes + (size_t)kAuxSlots * kAuxBytes + (size_t)kMaxProblems * sizeof(ProblemArgs) +
+         (size_t)(2 * S + 3 * kAuxSlots) * sizeof(unsigned long long) + (size_t)kMaxStages * sizeof(int) + 1024;
 }
 
 // ---------------------------------------------------------------- generic kernel (any M)
