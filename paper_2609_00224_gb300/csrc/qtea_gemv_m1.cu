@@ -328,15 +328,6 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
   }
 }
 
-// Accumulate one salient entry (value r, x at its column xj, position pos in the group of four).
-__device__ __forceinline__ void add_entry(float (&acc)[4], float r, float xj, int pos) {
-  const float val = r * xj;
-  acc[0] += pos == 0 ? val : 0.f;
-  acc[1] += pos == 1 ? val : 0.f;
-  acc[2] += pos == 2 ? val : 0.f;
-  acc[3] += pos == 3 ? val : 0.f;
-}
-
 // x at the salient columns of entries e0 .. e0+31 (lane j holds entry e0 + j, zero past e_end).
 __device__ __forceinline__ float gather_salient_x(const ProblemArgs& a, int e0, int e_end, int lane) {
   const int e = e0 + lane;
@@ -391,7 +382,7 @@ __device__ __forceinline__ void load_block(const ProblemArgs& a, int q, int b, u
 // residual loads go out after the planes are published, so they never delay them (a unit's first
 // planes are on the critical path of the launch). Lane owns residual groups lane + 32k.
 __device__ __noinline__ void stage_unit(const ProblemArgs* pa, int t, int ch, uint8_t* ax, int lane,
-                                        uint32_t planes_bar) {
+                                        uint32_t planes_bar, float4* onehot) {
   const ProblemArgs a = *pa;
   {
     ChunkLoads L;
@@ -426,16 +417,27 @@ __device__ __noinline__ void stage_unit(const ProblemArgs* pa, int t, int ch, ui
 #pragma unroll 1
   for (int b = b0; b < b1; ++b) {
     const int w = (b - b0) & 3;  // block within the 32-entry window of xs
+    {
+      // lane 4j + p writes T[j][p] = x_j * e_p for the block's entries j
+      const float xj = __shfl_sync(0xffffffffu, xs, w * kResBlock + (lane >> 2));
+      const int pp = lane & 3;
+      onehot[lane] = make_float4(pp == 0 ? xj : 0.f, pp == 1 ? xj : 0.f, pp == 2 ? xj : 0.f, pp == 3 ? xj : 0.f);
+      __syncwarp();
+    }
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const float xj = __shfl_sync(0xffffffffu, xs, w * kResBlock + j);
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
         const uint32_t wd = (j < 2) ? rvA[k].x : (j < 4) ? rvA[k].y : (j < 6) ? rvA[k].z : rvA[k].w;
-        const float r = h2f((uint16_t)((j & 1) ? (wd >> 16) : (wd & 0xffffu)));
-        add_entry(acc[k], r, xj, (int)((rpA[k] >> (2 * j)) & 3u));
+        const float rr = h2f((uint16_t)((j & 1) ? (wd >> 16) : (wd & 0xffffu)));
+        const float4 oh = onehot[4 * j + (int)((rpA[k] >> (2 * j)) & 3u)];
+        acc[k][0] = fmaf(rr, oh.x, acc[k][0]);
+        acc[k][1] = fmaf(rr, oh.y, acc[k][1]);
+        acc[k][2] = fmaf(rr, oh.z, acc[k][2]);
+        acc[k][3] = fmaf(rr, oh.w, acc[k][3]);
       }
     }
+    __syncwarp();  // every lane has read the table before the next block rewrites it
     // next block: B moves to A, the one after it is loaded into B; a new window of x every 4
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
@@ -455,6 +457,7 @@ __device__ __noinline__ void stage_unit(const ProblemArgs* pa, int t, int ch, ui
 struct Ring {
   uint8_t* codes;         // [S][kStageBytes]
   uint8_t* aux;           // [kAuxSlots][kAuxBytes]
+  float4* onehot;         // [kHelperWarps][kResBlock * 4]
   const ProblemArgs* tab; // [n_problems], copied from the kernel parameters
   uint64_t* full_c;       // [S] codes landed
   uint64_t* empty_c;      // [S] consumers released the code stage
@@ -488,7 +491,8 @@ __device__ __noinline__ void helper_role(const Ring r, int u0, int n_units, int 
       if (!__all_sync(0xffffffffu, ok)) break;
     }
     const UnitPos up = unit_pos(r.tab, r.n_problems, (long long)u0 + i);
-    stage_unit(&r.tab[up.p], up.t, up.ch, r.aux + (size_t)slot * kAuxBytes, lane, smem_u32(&r.planes_a[slot]));
+    stage_unit(&r.tab[up.p], up.t, up.ch, r.aux + (size_t)slot * kAuxBytes, lane, smem_u32(&r.planes_a[slot]),
+               r.onehot + h * (kOneHotBytes / 16));
     mbar_arrive(smem_u32(&r.full_a[slot]));
   }
 }
@@ -626,7 +630,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   r.n_problems = NP;
   r.codes = smem;
   r.aux = smem + (size_t)S * kStageBytes;
-  ProblemArgs* tab = reinterpret_cast<ProblemArgs*>(r.aux + (size_t)kAuxSlots * kAuxBytes);
+  r.onehot = reinterpret_cast<float4*>(r.aux + (size_t)kAuxSlots * kAuxBytes);
+  ProblemArgs* tab = reinterpret_cast<ProblemArgs*>(r.aux + (size_t)kAuxSlots * kAuxBytes +
+                                                    (size_t)kHelperWarps * kOneHotBytes);
   r.tab = tab;
   r.full_c = reinterpret_cast<uint64_t*>(tab + kMaxProblems);
   r.empty_c = r.full_c + S;

@@ -49,6 +49,9 @@ struct ChunkMeta {
 constexpr int kAuxMeta = kPlaneBytesPerChunk;
 constexpr int kAuxRes = kAuxMeta + (int)sizeof(ChunkMeta);
 constexpr int kAuxBytes = kAuxRes + kTileRows * (int)sizeof(float);  // 3616
+// Per helper: x at one residual block's 8 entries spread over the 4 positions of a group,
+// T[entry][position] = x * one-hot(position), so that an entry adds with 4 FMAs and no selects.
+constexpr int kOneHotBytes = kResBlock * 4 * 16;               // 512
 
 struct ProblemArgs {
   const uint16_t* x;        // [K] (M = 1)
@@ -85,10 +88,11 @@ __host__ __device__ inline long long unit_begin_of(int b, long long total, int g
 }
 
 // Dynamic shared memory of the batch-1 kernel with S code stages: codes, auxiliary slots, the
-// problem table, the barriers (code stages: full, empty; auxiliary slots: planes written, residual
+// helpers' one-hot tables, the problem table, the barriers (code stages: full, empty; auxiliary slots: planes written, residual
 // written, empty), the fills issued per code stage (for the drain), and 1024 bytes of slack.
 __host__ __device__ constexpr size_t m1_smem_bytes(int S) {
-  return (size_t)S * kStageBytes + (size_t)kAuxSlots * kAuxBytes + (size_t)kMaxProblems * sizeof(ProblemArgs) +
+  return (size_t)S * kStageBytes + (size_t)kAuxSlots * kAuxBytes + (size_t)kHelperWarps * kOneHotBytes +
+         (size_t)kMaxProblems * sizeof(ProblemArgs) +
          (size_t)(2 * S + 3 * kAuxSlots) * sizeof(unsigned long long) + (size_t)kMaxStages * sizeof(int) + 1024;
 }
 

@@ -114,6 +114,21 @@ def test_parity_small(qt, N, K, s, M):
     assert_within(y, y_ref, b, f"N={N} K={K} s={s} M={M}")
 
 
+DENSE_SALIENT = [  # more than 16 salient entries per unit (residual summed by the staging warps),
+    # s not a multiple of 8 (scalar residual loads), every column salient
+    (512, 1024, 400), (300, 2048, 100), (1024, 1024, 1024), (2048, 4096, 600), (4, 64, 64), (516, 700, 36),
+]
+
+
+@pytest.mark.parametrize("N,K,s", DENSE_SALIENT)
+def test_parity_dense_salient(qt, N, K, s):
+    p = synth.make_problem("t", N, K, 1, s, seed=N + 3 * K + 5 * s)
+    d = Dev(qt, p)
+    y = d.run(qt)
+    y_ref, b = oracle_ref(p)
+    assert_within(y, y_ref, b, f"N={N} K={K} s={s}")
+
+
 def test_config0_tiny(qt):
     p = synth.config_problem(0, 0)
     d = Dev(qt, p)
