@@ -63,16 +63,14 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t byt
                : "memory");
 }
 
-// One potentially blocking test of the phase with the given parity: the thread may be suspended
-// until the phase completes or about kSuspendNs elapse, so waiting warps do not take issue slots.
-constexpr uint32_t kSuspendNs = 100000;
-
+// One potentially blocking test of the phase with the given parity (the thread may be suspended
+// for a system-dependent time until the phase completes).
 __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
-      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
+      "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
       : "=r"(ok)
-      : "r"(bar), "r"(parity), "r"(kSuspendNs)
+      : "r"(bar), "r"(parity)
       : "memory");
   return ok != 0;
 }
@@ -196,7 +194,7 @@ __device__ __forceinline__ void decode_unit(const uint4* row0, const uint4* row1
   for (int k = 0; k < P; ++k) { a0.a[k][0] = a0.a[k][1] = 0; a1.a[k][0] = a1.a[k][1] = 0; }
   uint4 P0 = pl[0], P1 = pl[1], P2 = kW == 3 ? pl[2] : make_uint4(0, 0, 0, 0);
   uint4 c0 = row0[0 ^ sw], c1 = row1[0 ^ sw];
-#pragma unroll 1
+#pragma unroll 2  // two chunks per iteration: the code and plane registers alternate without copies
   for (int jj = 0; jj < 8; ++jj) {
     const uint4 n0 = row0[((jj + 1) & 7) ^ sw];
     const uint4 n1 = row1[((jj + 1) & 7) ^ sw];
