@@ -5,8 +5,9 @@ Workload: the seven linear layers of one Llama3-8B decoder layer (q/k/v/o/gate/u
 = 4096x4096, 1024x4096, 1024x4096, 4096x4096, 14336x4096, 14336x4096, 4096x14336) at batch M = 1,
 with synthetic weights drawn like the paper's models would be stored (ternary codes
 P(-1,0,+1) = (0.3,0.4,0.3), alpha ~ U(0.01,0.05), v ~ U(0.8,1.2), 3% salient columns, residual
-~ N(0,0.02), x ~ N(0,1)). `--layers` independent layers are resident in HBM and the steps
-rotate through them, so every step reads weights that are not in L2.
+~ N(0,0.02), x ~ N(0,1)). `--layers` independent layers are resident in HBM (default 32: the
+whole decoder stack, 1.87 GB of codes) and the steps rotate through them, so every step reads
+weights that are not in L2; `layers` consecutive steps are one token's linear layers.
 
 A step = the seven GEMVs of one layer. value = algorithmic bytes moved per step (packed ternary
 codes, alpha, v, salient indices, residual values and positions, x, y) x steps / device time.
@@ -187,6 +188,22 @@ def oracle_sample_seconds(problems, rows_stride, budget_s):
 
 # ---------------------------------------------------------------------------- arms
 
+def max_over_ranks(ms, world, device):
+    """The slowest rank's time in ms (every rank receives it); ms itself on a single rank."""
+    if world <= 1:
+        return ms
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(bytes_per_rank, world, ms):
+    """Whole-job GB/s: the bytes all ranks processed over the slowest rank's time (weak scaling)."""
+    return bytes_per_rank * world / (ms * 1e-3) / 1e9
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -338,12 +355,10 @@ def qtea_arm(args):
     status = max(qt.qtea_device_status(g["layout"]) for L in layers for g in L)
     if status:
         raise RuntimeError(f"device status {status} after the timed region")
-    if world > 1:
-        t = torch.tensor([total_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
-    bytes_all = sum(step_bytes[st % len(layers)] for st in range(args.steps)) * world
-    value = bytes_all / (total_ms * 1e-3) / 1e9
+    total_ms = max_over_ranks(total_ms, world, "cuda")
+    bytes_rank = sum(step_bytes[st % len(layers)] for st in range(args.steps))
+    bytes_all = bytes_rank * world
+    value = job_throughput(bytes_rank, world, total_ms)
 
     # roofline of the GEMV kernel: the only kernel of the timed region, one grouped launch per
     # step, launches back to back; its average launch duration is the region time / launches
@@ -430,12 +445,48 @@ def qtea_arm(args):
             e1.record(stream)
         barrier()
         e2e_ms = e0.elapsed_time(e1)
-        if world > 1:
-            t = torch.tensor([e2e_ms], device="cuda")
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            e2e_ms = float(t.item())
-        e2e = {"value": round(bytes_all / (e2e_ms * 1e-3) / 1e9, 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
+        e2e_ms = max_over_ranks(e2e_ms, world, "cuda")
+        e2e = {"value": round(job_throughput(bytes_rank, world, e2e_ms), 1), "unit": "GB/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": round(e2e_ms / args.steps, 5)}
+
+    # ---- dense fp16 GEMV through cuBLAS (torch.mm) on the same seven shapes: the
+    #      unquantized baseline, weights in enough copies that every step reads them from HBM
+    dense = None
+    if not args.no_dense:
+        copies = max(2, -(-4 * l2 // sum(2 * g["N"] * g["K"] for g in layers[0])))
+        dw = [[torch.randn((g["N"], g["K"]), dtype=torch.float16, device="cuda") for g in layers[0]]
+              for _ in range(copies)]
+        dx = [torch.randn((1, g["K"]), dtype=torch.float16, device="cuda") for g in layers[0]]
+        dy = [torch.empty((1, g["N"]), dtype=torch.float16, device="cuda") for g in layers[0]]
+
+        with torch.cuda.stream(stream):  # cuBLAS creates its handle and workspace outside the capture
+            for j in range(len(dx)):
+                torch.mm(dx[j], dw[0][j].t(), out=dy[j])
+        barrier()
+
+        def dense_graph(only=None):
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=stream):
+                for st in range(args.steps):
+                    for j in range(len(dx)):
+                        if only is None or j == only:
+                            torch.mm(dx[j], dw[st % copies][j].t(), out=dy[j])
+            return gr
+
+        gd = dense_graph()
+        dms = timed_replay(gd)
+        del gd
+        dbytes = sum(2 * g["N"] * g["K"] + 2 * g["K"] + 2 * g["N"] for g in layers[0])
+        dense = {"us_per_step": round(dms * 1e3 / args.steps, 3), "value": round(dbytes * args.steps / (dms * 1e-3) / 1e9, 1),
+                 "unit": "GB/s", "weight_copies": copies, "us_per_call": {}}
+        if not args.no_per_shape:
+            for j, g in enumerate(layers[0]):
+                gs = dense_graph(only=j)
+                dense["us_per_call"][g["name"]] = round(timed_replay(gs) * 1e3 / args.steps, 3)
+                del gs
+        dense["qtea_speedup_per_step"] = round(dense["us_per_step"] / (1e3 * total_ms / args.steps), 2)
+        del dw, dx, dy
+        torch.cuda.empty_cache()
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -456,6 +507,7 @@ def qtea_arm(args):
             "data": "synthetic",
             "config": {"workload": WORKLOAD, "M": 1, "shapes": [[g["name"], g["N"], g["K"], g["s"]] for g in layers[0]],
                        "layers_resident": args.layers, "resident_weight_bytes": resident, "l2_bytes": l2,
+                       "linear_tokens_per_s": round(args.steps / args.layers / (total_ms * 1e-3), 1),
                        "l2": "inputs larger than L2: steps rotate over the resident layers",
                        "parallelism": "replicas" if world > 1 else "single"},
             "us_per_call": per_shape,
@@ -464,7 +516,7 @@ def qtea_arm(args):
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
                          "us_per_launch": round(1e3 * total_ms / args.steps, 3),
                          "us_per_launch_isolated": None if iso_us is None else round(iso_us, 3)},
-            "cpu_baseline": cpu, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
+            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
             "setup_s": round(t_gen, 1),
         }
         print(json.dumps(line), flush=True)
@@ -479,7 +531,9 @@ def main():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["qtea", "reference"], default="qtea")
-    ap.add_argument("--layers", type=int, default=16)
+    ap.add_argument("--no-dense", action="store_true", help="skip the dense fp16 cuBLAS baseline")
+    ap.add_argument("--layers", type=int, default=32,
+                    help="independent resident layers the steps rotate over (32 = the whole Llama3-8B stack)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")

@@ -290,6 +290,20 @@ def test_grouped_llama3_8b_layer(qt):
         assert torch.equal(y, y2)
 
 
+@pytest.mark.parametrize("layer", [0, 17, 31])
+def test_grouped_llama3_8b_stack_layers(qt, layer):
+    """Layers of the 32-layer stack (independent seeds per layer), as the benchmark launches them."""
+    ps = [synth.config_problem(4, m, layer=layer) for m in range(7)]
+    ds = [Dev(qt, p) for p in ps]
+    ys = qt.qtea_gemv_grouped([problem_dict(d) for d in ds])
+    torch.cuda.synchronize()
+    assert qt.qtea_device_status(ds[0].layout) == 0
+    for m, (p, y) in enumerate(zip(ps, ys)):
+        rows = sample_rows(p.N, n=12, seed=layer * 7 + m)
+        y_ref, b = oracle_ref(p, rows=rows)
+        assert_within(y.cpu().numpy().astype(np.float64)[:, rows], y_ref, b, f"{p.name} layer {layer}")
+
+
 def test_grouped_rejects_shared_layout_and_mixed_batch(qt):
     p = synth.make_problem("g", 64, 128, 1, 8, seed=1)
     d = Dev(qt, p)
