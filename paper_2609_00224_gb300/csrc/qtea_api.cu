@@ -67,6 +67,17 @@ int plan_m1(qtea_layout* l, const cudaDeviceProp& prop) {
     return QTEA_OK;
   }
   l->smem_optin = dyn_max;
+  {
+    // low batch: the same codes in boxes of 128 rows for the tensor-core kernel
+    cuuint32_t box_mb[2] = {(cuuint32_t)kChunkRowBytes, 128};
+    size_t mb_dyn = 0;
+    l->mb_ok = encode(&l->tmap_mb, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, l->packed, dims, strides, box_mb, estr,
+                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS &&
+               mb_configure(prop.sharedMemPerBlockOptin, &mb_dyn) == cudaSuccess;
+    if (!l->mb_ok) cudaGetLastError();
+    l->mb_smem_optin = mb_dyn;
+  }
   if (cudaMalloc(&l->workspace, (size_t)l->sm_count * 2 * kTileRows * sizeof(float)) != cudaSuccess)
     return QTEA_ERR_ALLOC;
   if (cudaMalloc(&l->counters, (size_t)l->n_tiles * kConsumerWarps * sizeof(unsigned)) != cudaSuccess)
@@ -110,6 +121,60 @@ int launch_generic_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
   p.K_pad = l->K_pad;
   p.s = l->n_salient;
   return launch_generic(p, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+}
+
+// Low-batch (2 <= M <= 16) problem on the tensor-core kernel; returns QTEA_ERR_UNSUPPORTED when the
+// shapes or pointers do not allow it (the caller then uses the generic kernel).
+int launch_mb_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
+  const qtea_layout* l = q.packed_ternary;
+  if (!l->mb_ok || M < 2 || M > 16 || l->K % 8 != 0 || l->n_salient > kMaxSalientMb) return QTEA_ERR_UNSUPPORTED;
+  if (!aligned(q.x, 16) || !aligned(q.col_scale, 16)) return QTEA_ERR_UNSUPPORTED;
+  PFN_cuTensorMapEncodeTiled_v12000 encode = get_encode_tiled();
+  if (!encode) return QTEA_ERR_UNSUPPORTED;
+  MbMaps maps;
+  std::memcpy(&maps.codes, &l->tmap_mb, sizeof(CUtensorMap));
+  {
+    cuuint64_t dims[2] = {(cuuint64_t)l->K, (cuuint64_t)M};
+    cuuint64_t strides[1] = {(cuuint64_t)l->K * 2};
+    cuuint32_t box[2] = {64, 16};
+    cuuint32_t estr[2] = {1, 1};
+    if (encode(&maps.x, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint16_t*>(q.x), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return QTEA_ERR_UNSUPPORTED;
+  }
+  {
+    cuuint64_t dims[2] = {(cuuint64_t)l->K, 1};
+    cuuint64_t strides[1] = {(cuuint64_t)l->K * 2};
+    cuuint32_t box[2] = {256, 1};
+    cuuint32_t estr[2] = {1, 1};
+    if (encode(&maps.v, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint16_t*>(q.col_scale), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return QTEA_ERR_UNSUPPORTED;
+  }
+  MbParams p;
+  p.x = q.x;
+  p.alpha = q.row_scale;
+  p.sal = q.salient_idx;
+  p.rvals = q.residual_vals;
+  p.ridx = q.residual_idx;
+  p.y = q.y;
+  p.status = l->status;
+  p.N = l->N;
+  p.K = l->K;
+  p.M = M;
+  p.s = l->n_salient;
+  p.s_pad = round_up(l->n_salient, 16) + 8;
+  p.n_tiles = (l->N + 127) / 128;
+  p.n_chunks = l->n_chunks;
+  p.vec_res = (l->n_salient % 8 == 0) && aligned(q.residual_vals, 16);
+  int S = kMaxStagesMb;
+  while (S >= kMinStagesMb && mb_smem_bytes(S, p.s_pad) > l->mb_smem_optin) --S;
+  if (S < kMinStagesMb) return QTEA_ERR_UNSUPPORTED;
+  p.n_stages = S;
+  const int grid = p.n_tiles < l->sm_count ? p.n_tiles : l->sm_count;
+  return launch_mb(maps, p, grid, mb_smem_bytes(S, p.s_pad), st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
 }
 
 // Batch-1 kernel over a group of problems whose layouts all have m1 resources.
@@ -361,8 +426,12 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
       if (cudaMemsetAsync(q.y, 0, (size_t)M * l->N * sizeof(float), st) != cudaSuccess) rc = QTEA_ERR_CUDA;
       continue;
     }
-    if (M == 1 && l->m1_ok) m1_idx[n_m1++] = i;
-    else rc = launch_generic_problem(q, M, st);
+    if (M == 1 && l->m1_ok) {
+      m1_idx[n_m1++] = i;
+    } else {
+      rc = launch_mb_problem(q, M, st);
+      if (rc == QTEA_ERR_UNSUPPORTED) rc = launch_generic_problem(q, M, st);
+    }
   }
   if (rc == QTEA_OK && n_m1 > 0) rc = run_m1(problems, m1_idx, n_m1, st);
   std::free(m1_idx);

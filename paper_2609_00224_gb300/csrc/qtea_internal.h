@@ -96,6 +96,33 @@ __host__ __device__ constexpr size_t m1_smem_bytes(int S) {
          (size_t)(2 * S + 3 * kAuxSlots) * sizeof(unsigned long long) + (size_t)kMaxStages * sizeof(int) + 1024;
 }
 
+// ---------------------------------------------------------------- low-batch tensor-core kernel (2 <= M <= 16)
+constexpr int kMaxStagesMb = 6;
+constexpr int kMinStagesMb = 2;
+constexpr int kMaxSalientMb = 1024;  // x at the salient columns is staged in shared memory
+
+struct MbMaps {
+  CUtensorMap codes;  // packed codes [N][K_pad/4] bytes, box 128 bytes x 128 rows, 128-byte swizzle
+  CUtensorMap x;      // activations [M][K] fp16, box 64 x 16 rows, 128-byte swizzle
+  CUtensorMap v;      // column rescale [1][K] fp16, box 256 x 1
+};
+
+struct MbParams {
+  const uint16_t* x;        // [M][K]
+  const uint16_t* alpha;    // [N]
+  const int32_t* sal;       // [s]
+  const uint16_t* rvals;    // [N/4][s]
+  const uint8_t* ridx;      // [N/4][ceil(s/4)]
+  float* y;                 // [M][N]
+  int* status;
+  int N, K, M, s, s_pad, n_tiles, n_chunks, n_stages;
+  int vec_res;              // s % 8 == 0 and rvals 16-byte aligned: 8-byte residual loads
+};
+
+size_t mb_smem_bytes(int S, int s_pad);
+cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max);
+cudaError_t launch_mb(const MbMaps& maps, const MbParams& p, int grid, size_t smem, cudaStream_t st);
+
 // ---------------------------------------------------------------- generic kernel (any M)
 struct GenericParams {
   const uint16_t* x;        // [M][K]
@@ -132,4 +159,8 @@ struct qtea_layout {
   unsigned* counters;    // [n_tiles][kConsumerWarps]
   int* status;
   CUtensorMap tmap;
+  // low-batch kernel resources
+  bool mb_ok;
+  size_t mb_smem_optin;
+  CUtensorMap tmap_mb;   // codes, box 128 bytes x 128 rows
 };
