@@ -169,12 +169,24 @@ int launch_mb_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
   p.n_tiles = (l->N + 127) / 128;
   p.n_chunks = l->n_chunks;
   p.vec_res = (l->n_salient % 8 == 0) && aligned(q.residual_vals, 16);
+  // clusters of C CTAs split a tile's chunks when there are fewer tiles than SMs
+  int C = l->sm_count / p.n_tiles;
+  if (C > 8) C = 8;
+  if (C > p.n_chunks) C = p.n_chunks;
+  if (C < 1) C = 1;
   int S = kMaxStagesMb;
-  while (S >= kMinStagesMb && mb_smem_bytes(S, p.s_pad) > l->mb_smem_optin) --S;
+  for (;;) {
+    while (S >= kMinStagesMb && mb_smem_bytes(S, p.s_pad, C, M) > l->mb_smem_optin) --S;
+    if (S >= kMinStagesMb || C == 1) break;
+    --C;
+    S = kMaxStagesMb;
+  }
   if (S < kMinStagesMb) return QTEA_ERR_UNSUPPORTED;
   p.n_stages = S;
-  const int grid = p.n_tiles < l->sm_count ? p.n_tiles : l->sm_count;
-  return launch_mb(maps, p, grid, mb_smem_bytes(S, p.s_pad), st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+  p.cluster = C;
+  int n_cl = l->sm_count / C;
+  if (n_cl > p.n_tiles) n_cl = p.n_tiles;
+  return launch_mb(maps, p, n_cl * C, mb_smem_bytes(S, p.s_pad, C, M), st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
 }
 
 // Batch-1 kernel over a group of problems whose layouts all have m1 resources.

@@ -14,10 +14,12 @@
 //    salient column, A holds the fp16 residual value of the row's group where the stored
 //    position is the row and 0 elsewhere, and B holds x at the salient column. It is accumulated
 //    apart, since alpha does not scale it.
-// Work: a unit is a 128-row tile of the full width K (no split of K over CTAs, hence no partial
-// sums in global memory and a fixed summation order). Eight consumer warps each own 16 rows of
-// the tile; a producer lane streams the tile's 512-column chunks through a ring of shared-memory
-// stages by TMA: 128 rows x 128 bytes of codes (128-byte swizzle), the 16 x 512 block of x
+// Work: a unit is a 128-row tile. A cluster of C CTAs (C chosen so that tiles x C fills the GPU)
+// shares a tile: CTA rank r takes chunks [r n/C, (r+1) n/C) and residual steps r, r + C, ...; the
+// ranks' partial rows go through distributed shared memory into rank 0, which adds them in rank
+// order (no partial sums in global memory, a fixed summation order). Eight consumer warps each
+// own 16 rows of the tile; a producer lane streams the CTA's 512-column chunks through a ring of
+// shared-memory stages by TMA: 128 rows x 128 bytes of codes (128-byte swizzle), the 16 x 512 block of x
 // (128-byte swizzle, rows beyond M read as zero) and 512 values of v. x at the salient columns is
 // gathered once per CTA. The k order inside each 16-column step is permuted so that a thread's
 // four k slots are four consecutive columns, i.e. one byte of codes.
@@ -119,6 +121,75 @@ __device__ __forceinline__ void decode_byte(uint32_t word, uint32_t q, uint32_t 
   a23 = h2_as_u32(__hmul2(t23, u32_as_h2(v23)));
 }
 
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t cluster_id() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t n_clusters() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+
+__device__ __forceinline__ void st_cluster_v4(uint32_t addr, float a, float b, float c, float d) {
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t remote_bar) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote_bar) : "memory");
+}
+
+// Wait for a phase completed by arrivals from other CTAs of the cluster (acquire at cluster scope).
+__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, int* status) {
+  const unsigned long long t0 = global_ns();
+  for (;;) {
+    uint32_t ok;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    if (ok) return true;
+    if (global_ns() - t0 > kWaitLimitNs) {
+      atomicExch(status, (int)QTEA_ERR_TIMEOUT);
+      return false;
+    }
+  }
+}
+
+// Shared memory of the kernel: S stages, x at the salient columns [16][s_pad] fp16, the rank-0
+// CTA's slots for the other ranks' partial rows [C-1][256 threads][4 MT] floats, and barriers.
+struct MbSmem {
+  uint8_t* stages;
+  __half* xs;
+  float* slots;
+  uint64_t* full;          // [S] stage landed
+  uint64_t* empty;         // [S] consumers released the stage
+  uint64_t* red_full;      // rank 0: every other rank wrote its partial rows of the tile
+  uint64_t* red_empty;     // other ranks: rank 0 has read this rank's partial rows
+  int* last_fill;          // [kMaxStagesMb]
+};
+
 template <int MT>  // n8 tiles of the batch: 1 for M <= 8, 2 for M <= 16
 __global__ void __launch_bounds__(kMbThreads, 1)
     qtea_gemv_mb_kernel(const __grid_constant__ MbMaps maps, const __grid_constant__ MbParams p) {
@@ -127,22 +198,33 @@ __global__ void __launch_bounds__(kMbThreads, 1)
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int S = p.n_stages;
-  uint8_t* stages = smem;                                            // [S][kMbStageBytes]
-  __half* xs = reinterpret_cast<__half*>(smem + (size_t)S * kMbStageBytes);  // [16][s_pad]
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + (size_t)S * kMbStageBytes + (size_t)16 * p.s_pad * 2);
-  uint64_t* empty = full + S;
-  int* last_fill = reinterpret_cast<int*>(empty + S);
+  const int C = p.cluster;                 // CTAs of a cluster share a tile, each a range of chunks
+  const int rank = (int)cluster_rank();
+  MbSmem sm;
+  sm.stages = smem;
+  sm.xs = reinterpret_cast<__half*>(smem + (size_t)S * kMbStageBytes);
+  sm.slots = reinterpret_cast<float*>(smem + (size_t)S * kMbStageBytes + (size_t)16 * p.s_pad * 2);
+  sm.full = reinterpret_cast<uint64_t*>(sm.slots + (size_t)(C - 1) * kMbConsumerWarps * 32 * 4 * MT);
+  sm.empty = sm.full + S;
+  sm.red_full = sm.empty + S;
+  sm.red_empty = sm.red_full + 1;
+  sm.last_fill = reinterpret_cast<int*>(sm.red_empty + 1);
 
-  // units of this CTA: tiles blockIdx.x, blockIdx.x + gridDim.x, ...
-  const int n_my_tiles = p.n_tiles > (int)blockIdx.x ? (p.n_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
-  const int n_fills = n_my_tiles * p.n_chunks;
+  // tiles of this cluster: cluster_id, + n_clusters, ...; chunks of this CTA: [c0, c1)
+  const int cid = (int)cluster_id(), ncl = (int)n_clusters();
+  const int n_my_tiles = p.n_tiles > cid ? (p.n_tiles - 1 - cid) / ncl + 1 : 0;
+  const int c0 = rank * p.n_chunks / C, c1 = (rank + 1) * p.n_chunks / C;
+  const int my_chunks = c1 - c0;
+  const int n_fills = n_my_tiles * my_chunks;
 
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
-      mbar_init(smem_u32(&full[i]), 1);
-      mbar_init(smem_u32(&empty[i]), kMbConsumerWarps);
-      last_fill[i] = 0;
+      mbar_init(smem_u32(&sm.full[i]), 1);
+      mbar_init(smem_u32(&sm.empty[i]), kMbConsumerWarps);
+      sm.last_fill[i] = 0;
     }
+    mbar_init(smem_u32(sm.red_full), (uint32_t)(C > 1 ? (C - 1) * kMbConsumerWarps * 32 : 1));  // unused if C == 1
+    mbar_init(smem_u32(sm.red_empty), (uint32_t)(kMbConsumerWarps * 32));
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -150,7 +232,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
     const CUtensorMap* m = lane == 0 ? &maps.codes : (lane == 1 ? &maps.x : &maps.v);
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
   }
-  __syncthreads();
+  cluster_sync();  // barriers initialised in every CTA of the cluster before any remote arrival
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
@@ -159,10 +241,10 @@ __global__ void __launch_bounds__(kMbThreads, 1)
     if (lane == 0) {
       for (int f = 0; f < n_fills; ++f) {
         const int st = f % S, ph = f / S;
-        if (ph > 0 && !mbar_wait(smem_u32(&empty[st]), (uint32_t)((ph - 1) & 1), p.status)) break;
-        const int t = (int)blockIdx.x + (f / p.n_chunks) * (int)gridDim.x, ch = f % p.n_chunks;
-        uint8_t* sb = stages + (size_t)st * kMbStageBytes;
-        const uint32_t bar = smem_u32(&full[st]);
+        if (ph > 0 && !mbar_wait(smem_u32(&sm.empty[st]), (uint32_t)((ph - 1) & 1), p.status)) break;
+        const int t = cid + (f / my_chunks) * ncl, ch = c0 + f % my_chunks;
+        uint8_t* sb = sm.stages + (size_t)st * kMbStageBytes;
+        const uint32_t bar = smem_u32(&sm.full[st]);
         mbar_arrive_expect_tx(bar, kMbCodeBytes + kMbXBytes + kMbVBytes);
         tma_load_2d(smem_u32(sb), &maps.codes, ch * kChunkRowBytes, t * kMbTileRows, bar);
 #pragma unroll
@@ -170,7 +252,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
           tma_load_2d(smem_u32(sb + kMbCodeBytes + j * 2048), &maps.x, ch * kChunkCols + j * kMbXBoxCols, 0, bar);
         tma_load_2d(smem_u32(sb + kMbCodeBytes + kMbXBytes), &maps.v, ch * kChunkCols, 0, bar);
         tma_load_2d(smem_u32(sb + kMbCodeBytes + kMbXBytes + 512), &maps.v, ch * kChunkCols + 256, 0, bar);
-        last_fill[st] = ph + 1;
+        sm.last_fill[st] = ph + 1;
       }
     }
   } else {
@@ -184,15 +266,17 @@ __global__ void __launch_bounds__(kMbThreads, 1)
         col = col < 0 ? 0 : (col >= p.K ? p.K - 1 : col);
         v = __ushort_as_half(__ldg(p.x + (size_t)m * p.K + col));
       }
-      xs[i] = v;
+      sm.xs[i] = v;
     }
     asm volatile("bar.sync 1, %0;" ::"n"(kMbConsumerWarps * 32) : "memory");
 
     const int g = lane >> 2, q = lane & 3;
     const int r0 = warp * 16 + g;  // tile rows of the thread: r0 and r0 + 8
+    const int tid = threadIdx.x;   // consumer index 0 .. 255
     int f = 0;
-    for (int ti = 0; ti < n_my_tiles; ++ti) {
-      const int t = (int)blockIdx.x + ti * (int)gridDim.x;
+    bool ok = true;
+    for (int ti = 0; ti < n_my_tiles && ok; ++ti) {
+      const int t = cid + ti * ncl;
       const int row0 = t * kMbTileRows + r0, row1 = row0 + 8;
       const uint16_t al0 = row0 < p.N ? __ldg(p.alpha + row0) : (uint16_t)0;
       const uint16_t al1 = row1 < p.N ? __ldg(p.alpha + row1) : (uint16_t)0;
@@ -202,12 +286,14 @@ __global__ void __launch_bounds__(kMbThreads, 1)
 #pragma unroll
         for (int e = 0; e < 4; ++e) acc[j][e] = res[j][e] = 0.f;
 
-      bool ok = true;
-      for (int ch = 0; ch < p.n_chunks; ++ch, ++f) {
+      for (int ch = c0; ch < c1; ++ch, ++f) {
         const int st = f % S;
-        ok = mbar_wait(smem_u32(&full[st]), (uint32_t)((f / S) & 1), p.status);
-        if (!__all_sync(0xffffffffu, ok)) break;
-        const uint8_t* sb = stages + (size_t)st * kMbStageBytes;
+        ok = mbar_wait(smem_u32(&sm.full[st]), (uint32_t)((f / S) & 1), p.status);
+        if (!__all_sync(0xffffffffu, ok)) {
+          ok = false;
+          break;
+        }
+        const uint8_t* sb = sm.stages + (size_t)st * kMbStageBytes;
         const uint8_t* c0p = sb + (size_t)r0 * kChunkRowBytes;
         const uint8_t* c1p = c0p + 8 * kChunkRowBytes;
         const uint8_t* xb = sb + kMbCodeBytes;
@@ -225,7 +311,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
             uint32_t a0, a1, a2, a3;
             decode_byte(wa[e], (uint32_t)q, vv.x, vv.y, a0, a2);
             decode_byte(wb[e], (uint32_t)q, vv.x, vv.y, a1, a3);
-            // x box k4 / 2 holds columns 64 (kb / 4) .. +63; the step's 4q .. 4q+3 within it
+            // x box kb / 4 holds columns 64 (kb / 4) .. +63; the step's 4q .. 4q+3 within it
             const int chunk = (kb & 3) * 2 + (q >> 1);
 #pragma unroll
             for (int j = 0; j < MT; ++j) {
@@ -237,16 +323,16 @@ __global__ void __launch_bounds__(kMbThreads, 1)
           }
         }
         __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
+        if (lane == 0) mbar_arrive(smem_u32(&sm.empty[st]));
       }
-      if (!__all_sync(0xffffffffu, ok)) break;
+      if (!ok) break;
 
-      // ---- residual (Eq. 11): virtual columns, 16 salient entries per step
+      // ---- residual (Eq. 11): virtual columns, 16 salient entries per step, steps split over ranks
       if (p.s > 0) {
         const int gq0 = row0 >> 2, gq1 = row1 >> 2, pos = row0 & 3;  // row1 & 3 == pos
         const bool v0 = gq0 < (p.N >> 2), v1 = gq1 < (p.N >> 2);
         const int rs = (p.s + 3) >> 2;
-        for (int eb = 0; eb * 16 < p.s; ++eb) {
+        for (int eb = rank; eb * 16 < p.s; eb += C) {
           const int e0 = eb * 16 + 4 * q;  // the thread's entries e0 .. e0 + 3
           uint2 r0v = make_uint2(0, 0), r1v = make_uint2(0, 0);
           uint32_t p0 = 0, p1 = 0;
@@ -289,44 +375,82 @@ __global__ void __launch_bounds__(kMbThreads, 1)
 #pragma unroll
           for (int j = 0; j < MT; ++j) {
             const int n = 8 * j + g;
-            const uint2 bb = *reinterpret_cast<const uint2*>(xs + (size_t)n * p.s_pad + e0);
+            const uint2 bb = *reinterpret_cast<const uint2*>(sm.xs + (size_t)n * p.s_pad + e0);
             mma_16816(res[j], a0, a1, a2, a3, bb.x, bb.y);
           }
         }
       }
 
-      // ---- epilogue: y[n][row] = alpha[row] * acc + res for the thread's rows and batch columns
+      // ---- this CTA's part of the tile: alpha * acc + res (alpha scales only the ternary part)
       const float fa0 = __half2float(__ushort_as_half(al0)), fa1 = __half2float(__ushort_as_half(al1));
+      float part[MT][4];
+#pragma unroll
+      for (int j = 0; j < MT; ++j) {
+        part[j][0] = fa0 * acc[j][0] + res[j][0];
+        part[j][1] = fa0 * acc[j][1] + res[j][1];
+        part[j][2] = fa1 * acc[j][2] + res[j][2];
+        part[j][3] = fa1 * acc[j][3] + res[j][3];
+      }
+      if (rank != 0) {
+        // into rank 0's slot for this rank, once rank 0 has read the previous tile's
+        if (ti > 0 && !mbar_wait_cluster(smem_u32(sm.red_empty), (uint32_t)((ti - 1) & 1), p.status)) break;
+        const uint32_t dst = map_rank(smem_u32(sm.slots + ((size_t)(rank - 1) * kMbConsumerWarps * 32 + tid) * 4 * MT), 0);
+#pragma unroll
+        for (int j = 0; j < MT; ++j) st_cluster_v4(dst + 16 * j, part[j][0], part[j][1], part[j][2], part[j][3]);
+        mbar_arrive_cluster(map_rank(smem_u32(sm.red_full), 0));
+        continue;
+      }
+      if (C > 1) {
+        // rank 0: add the other ranks' parts in rank order, then give their slots back
+        if (!mbar_wait_cluster(smem_u32(sm.red_full), (uint32_t)(ti & 1), p.status)) break;
+        for (int rr = 1; rr < C; ++rr) {
+          const float* src = sm.slots + ((size_t)(rr - 1) * kMbConsumerWarps * 32 + tid) * 4 * MT;
+#pragma unroll
+          for (int j = 0; j < MT; ++j) {
+            const float4 v4 = *reinterpret_cast<const float4*>(src + 4 * j);
+            part[j][0] += v4.x;
+            part[j][1] += v4.y;
+            part[j][2] += v4.z;
+            part[j][3] += v4.w;
+          }
+        }
+        for (int rr = 1; rr < C; ++rr) mbar_arrive_cluster(map_rank(smem_u32(sm.red_empty), (uint32_t)rr));
+      }
+      // ---- y[n][row] for the thread's rows and batch columns
 #pragma unroll
       for (int j = 0; j < MT; ++j) {
         const int n0 = 8 * j + 2 * q;
         if (row0 < p.N) {
-          if (n0 < p.M) p.y[(size_t)n0 * p.N + row0] = fa0 * acc[j][0] + res[j][0];
-          if (n0 + 1 < p.M) p.y[(size_t)(n0 + 1) * p.N + row0] = fa0 * acc[j][1] + res[j][1];
+          if (n0 < p.M) p.y[(size_t)n0 * p.N + row0] = part[j][0];
+          if (n0 + 1 < p.M) p.y[(size_t)(n0 + 1) * p.N + row0] = part[j][1];
         }
         if (row1 < p.N) {
-          if (n0 < p.M) p.y[(size_t)n0 * p.N + row1] = fa1 * acc[j][2] + res[j][2];
-          if (n0 + 1 < p.M) p.y[(size_t)(n0 + 1) * p.N + row1] = fa1 * acc[j][3] + res[j][3];
+          if (n0 < p.M) p.y[(size_t)n0 * p.N + row1] = part[j][2];
+          if (n0 + 1 < p.M) p.y[(size_t)(n0 + 1) * p.N + row1] = part[j][3];
         }
       }
     }
   }
 
-  // no bulk copy may still be writing shared memory when the CTA exits
+  // no bulk copy may still be writing shared memory when the CTA exits, and no CTA of the
+  // cluster may exit while another may still write its shared memory
   __syncthreads();
   if (threadIdx.x == 0) {
     for (int s2 = 0; s2 < S; ++s2) {
-      const int lf = last_fill[s2];
-      if (lf > 0 && !mbar_wait(smem_u32(&full[s2]), (uint32_t)((lf - 1) & 1), p.status)) break;
+      const int lf = sm.last_fill[s2];
+      if (lf > 0 && !mbar_wait(smem_u32(&sm.full[s2]), (uint32_t)((lf - 1) & 1), p.status)) break;
     }
   }
+  cluster_sync();
 }
 
 }  // namespace
 
-size_t mb_smem_bytes(int S, int s_pad) {
-  return (size_t)S * kMbStageBytes + (size_t)16 * s_pad * 2 + (size_t)2 * S * sizeof(unsigned long long) +
-         (size_t)kMaxStagesMb * sizeof(int) + 1024;
+size_t mb_smem_bytes(int S, int s_pad, int cluster, int M) {
+  const int mt = M <= 8 ? 1 : 2;
+  return (size_t)S * kMbStageBytes + (size_t)16 * s_pad * 2 +
+         (size_t)(cluster - 1) * kMbConsumerWarps * 32 * 4 * mt * sizeof(float) +
+         (size_t)(2 * S + 2) * sizeof(unsigned long long) + (size_t)kMaxStagesMb * sizeof(int) + 1024;
 }
 
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max) {
@@ -349,11 +473,15 @@ cudaError_t launch_mb(const MbMaps& maps, const MbParams& p, int grid, size_t sm
   cfg.blockDim = dim3(kMbThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = (unsigned)p.cluster;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   if (p.M <= 8) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1>, maps, p);
   return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2>, maps, p);
 }

@@ -117,9 +117,10 @@ struct MbParams {
   int* status;
   int N, K, M, s, s_pad, n_tiles, n_chunks, n_stages;
   int vec_res;              // s % 8 == 0 and rvals 16-byte aligned: 8-byte residual loads
+  int cluster;              // CTAs per cluster sharing a tile (1 .. 8)
 };
 
-size_t mb_smem_bytes(int S, int s_pad);
+size_t mb_smem_bytes(int S, int s_pad, int cluster, int M);
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max);
 cudaError_t launch_mb(const MbMaps& maps, const MbParams& p, int grid, size_t smem, cudaStream_t st);
 
