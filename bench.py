@@ -488,6 +488,72 @@ def qtea_arm(args):
         del dw, dx, dy
         torch.cuda.empty_cache()
 
+    # ---- Qwen3-14B layer shapes at batch M = 1 .. 16 (reported beside the batch-1 workload): the seven
+    #      GEMVs of a layer per step, rotating over resident layers; the dense fp16 GEMM on the same shapes
+    msweep = None
+    if not args.no_m_sweep:
+        msweep = {"workload": "qwen3_14b_layer_gemvs", "layers_resident": 4, "us_per_layer": {}}
+        qlayers = []
+        for li in range(4):
+            L = []
+            for mi, (name, N, K) in enumerate(synth.config_shapes(2)):
+                pq = synth.config_problem(2, mi, M=16, layer=li)
+                f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
+                T = torch.from_numpy(pq.T).cuda()
+                lay = qt.qtea_pack_layout(T, n_salient=pq.s)
+                del T
+                L.append(dict(layout=lay, x=f16(pq.x), alpha=f16(pq.alpha.reshape(-1)), v=f16(pq.v),
+                              sal=torch.from_numpy(pq.salient_idx).cuda(), rv=f16(pq.residual_vals),
+                              ri=torch.from_numpy(pq.residual_idx).cuda(), N=N, K=K))
+            qlayers.append(L)
+        qcopies = 2
+        qw = [[torch.randn((g["N"], g["K"]), dtype=torch.float16, device="cuda") for g in qlayers[0]]
+              for _ in range(qcopies)]
+        nsteps = 32
+        for M in (1, 2, 4, 8, 16):
+            ys = [[torch.empty((M, g["N"]), dtype=torch.float32, device="cuda") for g in L] for L in qlayers]
+            yd = [torch.empty((M, g["N"]), dtype=torch.float16, device="cuda") for g in qlayers[0]]
+            xs = [[g["x"][:M].contiguous() for g in L] for L in qlayers]
+
+            def qstep(st):
+                L = qlayers[st % len(qlayers)]
+                if M == 1:
+                    qt.qtea_gemv_grouped([dict(x=xs[st % len(qlayers)][j], layout=g["layout"], row_scale=g["alpha"],
+                                               col_scale=g["v"], salient_idx=g["sal"], residual_vals=g["rv"],
+                                               residual_idx=g["ri"], y=ys[st % len(qlayers)][j])
+                                          for j, g in enumerate(L)], stream=stream)
+                else:
+                    for j, g in enumerate(L):
+                        qt.qtea_gemv(xs[st % len(qlayers)][j], g["layout"], g["alpha"], g["v"], g["sal"], g["rv"],
+                                     g["ri"], y=ys[st % len(qlayers)][j], stream=stream)
+
+            def dstep(st):
+                for j in range(len(yd)):
+                    torch.mm(xs[0][j], qw[st % qcopies][j].t(), out=yd[j])
+
+            with torch.cuda.stream(stream):
+                qstep(0)
+                dstep(0)
+            barrier()
+            gq = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gq, stream=stream):
+                for st in range(nsteps):
+                    qstep(st)
+            tq = timed_replay(gq) * 1e3 / nsteps
+            gdd = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gdd, stream=stream):
+                for st in range(nsteps):
+                    dstep(st)
+            tdn = timed_replay(gdd) * 1e3 / nsteps
+            del gq, gdd
+            msweep["us_per_layer"][str(M)] = {"qtea": round(tq, 2), "dense_fp16": round(tdn, 2),
+                                              "speedup": round(tdn / tq, 2)}
+        status = max(qt.qtea_device_status(g["layout"]) for L in qlayers for g in L)
+        if status:
+            raise RuntimeError(f"device status {status} after the batch sweep")
+        del qlayers, qw
+        torch.cuda.empty_cache()
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         probs = [g["host"] for g in layers[0]]
@@ -516,7 +582,7 @@ def qtea_arm(args):
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
                          "us_per_launch": round(1e3 * total_ms / args.steps, 3),
                          "us_per_launch_isolated": None if iso_us is None else round(iso_us, 3)},
-            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
+            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
             "setup_s": round(t_gen, 1),
         }
         print(json.dumps(line), flush=True)
@@ -532,6 +598,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["qtea", "reference"], default="qtea")
     ap.add_argument("--no-dense", action="store_true", help="skip the dense fp16 cuBLAS baseline")
+    ap.add_argument("--no-m-sweep", action="store_true", help="skip the Qwen3-14B batch sweep (M = 1 .. 16)")
     ap.add_argument("--layers", type=int, default=32,
                     help="independent resident layers the steps rotate over (32 = the whole Llama3-8B stack)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
