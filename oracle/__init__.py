@@ -38,8 +38,12 @@ def load(path: str | None = None):
     i32 = ctypes.c_int
     lib.qo_half_to_double.restype = ctypes.c_double
     lib.qo_half_to_double.argtypes = [ctypes.c_uint16]
+    lib.qo_e4m3_to_double.restype = ctypes.c_double
+    lib.qo_e4m3_to_double.argtypes = [ctypes.c_uint8]
     lib.qo_gemv.restype = i32
     lib.qo_gemv.argtypes = [i32, i32, i32, i32, P, P, P, P, P, i32, P, P, P, P, i32, P, P]
+    lib.qo_gemv_ex.restype = i32
+    lib.qo_gemv_ex.argtypes = [i32, i32, i32, i32, P, P, P, P, P, i32, P, P, i32, P, P, i32, P, P]
     for name in ("qo_pack_2bit", "qo_unpack_2bit", "qo_pack_base3", "qo_unpack_base3"):
         getattr(lib, name).restype = i32
         getattr(lib, name).argtypes = [P, i32, i32, P]
@@ -72,12 +76,17 @@ def half_to_double(h: int, lib=None) -> float:
     return (lib or load()).qo_half_to_double(int(h) & 0xFFFF)
 
 
+def e4m3_to_double(b: int, lib=None) -> float:
+    return (lib or load()).qo_e4m3_to_double(int(b) & 0xFF)
+
+
 def gemv(x, T, alpha, v, salient_idx=None, residual_vals=None, residual_idx=None, beta=None,
-         group_size=None, rows=None, want_bound=True, lib=None):
+         group_size=None, rows=None, want_bound=True, residual_fp8=False, lib=None):
     """y = x * W^T per Eq. 10/11 in fp64. fp16 inputs are given as uint16 bit patterns.
 
-    x [M][K] uint16, T [N][K] int8, alpha [N][G] uint16, v [K] uint16,
-    salient_idx [s] int32, residual_vals [N/4][s] uint16, residual_idx [N/4][ceil(s/4)] uint8.
+    x [M][K] uint16, T [N][K] int8, alpha [N][G] uint16, v [K] uint16, beta [N][G] uint16 or None,
+    salient_idx [s] int32, residual_vals [N/4][s] uint16 (uint8 FP8 E4M3 bytes with
+    residual_fp8), residual_idx [N/4][ceil(s/4)] uint8.
     Returns (y, bound), each float64 [M][n_out].
     """
     lib = lib or load()
@@ -99,10 +108,11 @@ def gemv(x, T, alpha, v, salient_idx=None, residual_vals=None, residual_idx=None
     beta = _c(beta, np.uint16)
     v = _c(v, np.uint16)
     si = _c(salient_idx, np.int32) if s else None
-    rv = _c(residual_vals, np.uint16) if s else None
+    rv = _c(residual_vals, np.uint8 if residual_fp8 else np.uint16) if s else None
     ri = _c(residual_idx, np.uint8) if s else None
-    rc = lib.qo_gemv(M, N, K, group_size, _ptr(T), _ptr(x), _ptr(alpha), _ptr(beta), _ptr(v), s,
-                     _ptr(si), _ptr(rv), _ptr(ri), _ptr(rows_a), n_out, _ptr(y), _ptr(b))
+    rc = lib.qo_gemv_ex(M, N, K, group_size, _ptr(T), _ptr(x), _ptr(alpha), _ptr(beta), _ptr(v), s,
+                        _ptr(si), _ptr(rv), int(bool(residual_fp8)), _ptr(ri), _ptr(rows_a), n_out, _ptr(y),
+                        _ptr(b))
     if rc != 0:
         raise OracleError(f"qo_gemv returned {rc}")
     return y, b

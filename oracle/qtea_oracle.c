@@ -33,7 +33,11 @@
  *                         least significant digit). Byte 25 covers 3 real columns and 2 pad
  *                         digits; pad digits and columns >= K hold digit 1 (T = 0).
  *   salient_idx           int32 [s], strictly ascending, each < K
- *   residual_vals         fp16 [N/4][s]: value of group q (rows 4q..4q+3) in salient column c
+ *   residual_vals         fp16 [N/4][s]: value of group q (rows 4q..4q+3) in salient column c;
+ *                         or, where the paper's storage is used (Sec. 4.1: FP8 residual), one
+ *                         byte per value in the FP8 E4M3 format: sign bit 7, exponent bits 6-3
+ *                         with bias 7, mantissa bits 2-0; exponent 0 is subnormal (m * 2^-9);
+ *                         0x7F and 0xFF are NaN; there is no infinity
  *   residual_idx          uint8 [N/4][ceil(s/4)]: 2-bit position of that value inside its
  *                         group, entry (q, c) at bits 2*(c%4) of byte q*ceil(s/4) + c/4
  *
@@ -65,6 +69,29 @@ double qo_half_to_double(uint16_t h) {
   return sign ? -mag : mag;
 }
 
+/* FP8 E4M3 -> double, exact (every E4M3 value is a double). */
+double qo_e4m3_to_double(uint8_t b) {
+  int sign = (b >> 7) & 1;
+  int expo = (b >> 3) & 0xf;
+  int frac = b & 7;
+  double mag;
+  if (expo == 0xf && frac == 7) {
+    mag = NAN;
+  } else if (expo == 0) {
+    mag = ldexp((double)frac, -9); /* subnormal: frac/8 * 2^-6 */
+  } else {
+    mag = ldexp((double)(8 + frac), expo - 10); /* (1 + frac/8) * 2^(expo-7) */
+  }
+  return sign ? -mag : mag;
+}
+
+/* Value of residual entry (q, c): fp16 or, with fp8 set, FP8 E4M3. */
+static double residual_value(const void* residual_vals, int fp8, int s, int q, int c) {
+  size_t i = (size_t)q * s + c;
+  return fp8 ? qo_e4m3_to_double(((const uint8_t*)residual_vals)[i])
+             : qo_half_to_double(((const uint16_t*)residual_vals)[i]);
+}
+
 static int residual_stride(int s) { return (s + 3) / 4; }
 
 static int residual_position(const uint8_t* ridx, int s, int q, int c) {
@@ -83,11 +110,12 @@ static int residual_position(const uint8_t* ridx, int s, int q, int c) {
  *             + sum_{c < s} [ residual position of (o/4, c) == o % 4 ] R[o/4][c] x[m][S_c]
  * bound[m][o] = sum_j | x[m][j] * W^[o][j] |, W^ the dense dequantized row including the
  *               residual entries, the scale of the comparison tolerance.
+ * residual_fp8 selects FP8 E4M3 residual values (one byte each) instead of fp16.
  */
-int qo_gemv(int M, int N, int K, int group_size, const int8_t* T, const uint16_t* x,
-            const uint16_t* alpha, const uint16_t* beta, const uint16_t* v, int s,
-            const int32_t* salient_idx, const uint16_t* residual_vals, const uint8_t* residual_idx,
-            const int32_t* rows, int n_rows, double* y, double* bound) {
+int qo_gemv_ex(int M, int N, int K, int group_size, const int8_t* T, const uint16_t* x,
+               const uint16_t* alpha, const uint16_t* beta, const uint16_t* v, int s,
+               const int32_t* salient_idx, const void* residual_vals, int residual_fp8,
+               const uint8_t* residual_idx, const int32_t* rows, int n_rows, double* y, double* bound) {
   if (M < 0 || N < 0 || K < 0 || s < 0 || group_size <= 0) return QO_BAD_ARG;
   if (s > 0 && (N % 4 != 0 || !salient_idx || !residual_vals || !residual_idx)) return QO_BAD_ARG;
   for (int c = 0; c < s; ++c) {
@@ -116,7 +144,7 @@ int qo_gemv(int M, int N, int K, int group_size, const int8_t* T, const uint16_t
     }
     for (int c = 0; c < s; ++c) {
       if (residual_position(residual_idx, s, o / 4, c) == o % 4)
-        w_row[salient_idx[c]] += qo_half_to_double(residual_vals[(size_t)(o / 4) * s + c]);
+        w_row[salient_idx[c]] += residual_value(residual_vals, residual_fp8, s, o / 4, c);
     }
     for (int m = 0; m < M; ++m) {
       const uint16_t* xm = x + (size_t)m * K;
@@ -138,7 +166,7 @@ int qo_gemv(int M, int N, int K, int group_size, const int8_t* T, const uint16_t
       /* Eq. 11, the sparse residual over the salient columns */
       for (int c = 0; c < s; ++c) {
         if (residual_position(residual_idx, s, o / 4, c) == o % 4)
-          acc += qo_half_to_double(residual_vals[(size_t)(o / 4) * s + c]) *
+          acc += residual_value(residual_vals, residual_fp8, s, o / 4, c) *
                  qo_half_to_double(xm[salient_idx[c]]);
       }
       y[(size_t)m * n_out + i] = acc;
@@ -151,6 +179,15 @@ int qo_gemv(int M, int N, int K, int group_size, const int8_t* T, const uint16_t
   }
   free(w_row);
   return status;
+}
+
+/* The same with fp16 residual values. */
+int qo_gemv(int M, int N, int K, int group_size, const int8_t* T, const uint16_t* x,
+            const uint16_t* alpha, const uint16_t* beta, const uint16_t* v, int s,
+            const int32_t* salient_idx, const uint16_t* residual_vals, const uint8_t* residual_idx,
+            const int32_t* rows, int n_rows, double* y, double* bound) {
+  return qo_gemv_ex(M, N, K, group_size, T, x, alpha, beta, v, s, salient_idx, residual_vals, 0, residual_idx,
+                    rows, n_rows, y, bound);
 }
 
 /* ---------------------------- packed layouts ---------------------------- */

@@ -25,7 +25,7 @@ _LIB_PATH = os.path.join(_HERE, "libqtea_synth.so")
 _lib = None
 
 # stream ids, one per tensor kind
-S_CODES, S_ALPHA, S_V, S_X, S_SALIENT, S_RVALS, S_RIDX = 1, 2, 3, 4, 5, 6, 7
+S_CODES, S_ALPHA, S_V, S_X, S_SALIENT, S_RVALS, S_RIDX, S_BETA = 1, 2, 3, 4, 5, 6, 7, 8
 
 
 def build(force: bool = False) -> str:
@@ -49,6 +49,10 @@ def _load():
     for n in ("synth_uniform_f16", "synth_normal_f16", "synth_laplace_f16"):
         getattr(lib, n).restype = None
         getattr(lib, n).argtypes = [u64, u64, sz, d, d, P]
+    lib.synth_e4m3_from_double.restype = ctypes.c_uint8
+    lib.synth_e4m3_from_double.argtypes = [d]
+    lib.synth_normal_e4m3.restype = None
+    lib.synth_normal_e4m3.argtypes = [u64, u64, sz, d, d, P]
     lib.synth_salient.restype = i32
     lib.synth_salient.argtypes = [u64, u64, i32, i32, P]
     lib.synth_residual_idx.restype = None
@@ -68,6 +72,16 @@ def f16_from_double(v: float) -> int:
 def codes(seed, stream, shape, p_neg, p_zero) -> np.ndarray:
     out = np.empty(shape, np.int8)
     _load().synth_codes(seed, stream, out.size, p_neg, p_zero, _p(out))
+    return out
+
+
+def e4m3_from_double(v: float) -> int:
+    return int(_load().synth_e4m3_from_double(float(v)))
+
+
+def normal_e4m3(seed, stream, shape, mean, std) -> np.ndarray:
+    out = np.empty(shape, np.uint8)
+    _load().synth_normal_e4m3(seed, stream, out.size, mean, std, _p(out))
     return out
 
 
@@ -126,21 +140,39 @@ class Problem:
     alpha: np.ndarray        # fp16 bits [N][1]
     v: np.ndarray            # fp16 bits [K]
     salient_idx: np.ndarray  # int32 [s]
-    residual_vals: np.ndarray  # fp16 bits [N/4][s]
+    residual_vals: np.ndarray  # fp16 bits [N/4][s] (uint8 FP8 E4M3 bytes when residual_fp8)
     residual_idx: np.ndarray   # uint8 [N/4][ceil(s/4)]
+    group_size: int = 0        # columns per alpha (and beta) group; 0 = K (one per row)
+    beta: Optional[np.ndarray] = None  # fp16 bits [N][G], or None (= 0)
+    residual_fp8: bool = False
+
+    @property
+    def G(self) -> int:
+        g = self.group_size or self.K
+        return (self.K + g - 1) // g if self.K else 1
 
 
 def make_problem(name: str, N: int, K: int, M: int, s: int, seed: int, p_neg: float = 0.3,
                  p_zero: float = 0.4, residual: str = "normal", residual_scale: float = 0.02,
-                 alpha_range=(0.01, 0.05), v_range=(0.8, 1.2)) -> Problem:
+                 alpha_range=(0.01, 0.05), v_range=(0.8, 1.2), group_size: int = 0, beta_std: float = 0.0,
+                 residual_fp8: bool = False) -> Problem:
+    """Seeded operands. group_size > 0 gives one alpha per (row, group of group_size columns),
+    beta_std > 0 a per-(row, group) beta drawn N(0, beta_std), and residual_fp8 residual values
+    rounded to FP8 E4M3 instead of fp16: the paper's own storage (Sec. 3.3, Eq. 4; Sec. 4.1)."""
     if s > 0 and N % 4:
         raise ValueError("N must be a multiple of 4 when there is a residual")
+    g = group_size or K
+    G = (K + g - 1) // g if K else 1
     T = codes(seed, S_CODES, (N, K), p_neg, p_zero)
-    alpha = uniform_f16(seed, S_ALPHA, (N, 1), *alpha_range)
+    alpha = uniform_f16(seed, S_ALPHA, (N, G), *alpha_range)
     v = uniform_f16(seed, S_V, (K,), *v_range)
     x = normal_f16(seed, S_X, (M, K), 0.0, 1.0)
     sal = salient(seed, S_SALIENT, K, s)
-    if residual == "normal":
+    if residual_fp8:
+        if residual != "normal":
+            raise ValueError("FP8 residual values are drawn from a normal distribution")
+        rv = normal_e4m3(seed, S_RVALS, (N // 4, s), 0.0, residual_scale)
+    elif residual == "normal":
         rv = normal_f16(seed, S_RVALS, (N // 4, s), 0.0, residual_scale)
     elif residual == "laplace":
         rv = laplace_f16(seed, S_RVALS, (N // 4, s), 0.0, residual_scale)
@@ -149,7 +181,8 @@ def make_problem(name: str, N: int, K: int, M: int, s: int, seed: int, p_neg: fl
     else:
         raise ValueError(residual)
     ri = residual_idx(seed, S_RIDX, N // 4, s)
-    return Problem(name, N, K, M, s, seed, T, x, alpha, v, sal, rv, ri)
+    beta = normal_f16(seed, S_BETA, (N, G), 0.0, beta_std) if beta_std > 0 else None
+    return Problem(name, N, K, M, s, seed, T, x, alpha, v, sal, rv, ri, group_size, beta, residual_fp8)
 
 
 # Layer shapes (out x in) of the three model families the workloads are modelled on.
@@ -189,6 +222,23 @@ def config_problem(config: int, matrix: int, M: Optional[int] = None, layer: int
     p_neg, p_zero = cfg["p"]
     return make_problem(f"{cfg['name']}/{name}", N, K, M, s, config_seed(config, layer, matrix), p_neg, p_zero,
                         cfg["residual"], cfg["residual_scale"])
+
+
+# The paper's own storage of a layer (Sec. 3.3 and Sec. 4.1): alpha and beta per row and group of
+# 128 columns, FP8 E4M3 residual values, base-3 codes. beta is drawn N(0, 0.002), a tenth of the
+# typical |alpha * v| (the paper gives no distribution).
+PAPER_FORMAT = dict(group_size=128, beta_std=0.002, residual_fp8=True)
+
+
+def paper_problem(config: int, matrix: int, M: Optional[int] = None, layer: int = 0) -> Problem:
+    """config_problem's operands in the paper's storage (same seed, hence the same codes, x and v)."""
+    cfg = CONFIGS[config]
+    name, N, K = cfg["shapes"][matrix]
+    s = cfg.get("fixed_s") or salient_count(K)
+    M = cfg["M"][0] if M is None else M
+    p_neg, p_zero = cfg["p"]
+    return make_problem(f"{cfg['name']}/{name}/paper_format", N, K, M, s, config_seed(config, layer, matrix), p_neg,
+                        p_zero, "normal", cfg["residual_scale"], **PAPER_FORMAT)
 
 
 def config_shapes(config: int) -> List[Tuple[str, int, int]]:

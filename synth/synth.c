@@ -61,6 +61,32 @@ uint16_t synth_f16_from_double(double v) {
   return sign | (uint16_t)((ue + 15) << 10) | (uint16_t)((int)q - 1024);
 }
 
+/* double -> FP8 E4M3 bits (sign, 4 exponent bits with bias 7, 3 mantissa bits; no infinity),
+ * round to nearest, ties to even; magnitudes beyond the largest finite value 448 saturate. */
+uint8_t synth_e4m3_from_double(double v) {
+  uint8_t sign = signbit(v) ? 0x80 : 0;
+  double a = fabs(v);
+  if (isnan(v)) return 0x7f;
+  if (a == 0.0) return sign;
+  if (a >= 448.0) return sign | 0x7e;
+  int e;
+  frexp(a, &e);
+  int ue = e - 1;
+  if (ue < -6) {
+    /* subnormal range: units of 2^-9 */
+    double q = nearbyint(a * 0x1.0p9);
+    if (q >= 8.0) return sign | 0x08; /* rounded up to the smallest normal */
+    return sign | (uint8_t)q;
+  }
+  double q = nearbyint(ldexp(a, 3 - ue)); /* significand in [8, 16] */
+  if (q >= 16.0) {
+    q = 8.0;
+    ue += 1;
+  }
+  if (ue > 8 || (ue == 8 && q > 14.0)) return sign | 0x7e; /* 448 is the largest finite value */
+  return sign | (uint8_t)((ue + 7) << 3) | (uint8_t)((int)q - 8);
+}
+
 /* ------------------------------------------------------------------ threads */
 
 typedef struct {
@@ -71,7 +97,7 @@ typedef struct {
   void* out;
 } job_t;
 
-enum { K_CODES = 0, K_UNIFORM = 1, K_NORMAL = 2, K_LAPLACE = 3 };
+enum { K_CODES = 0, K_UNIFORM = 1, K_NORMAL = 2, K_LAPLACE = 3, K_NORMAL_E4M3 = 4 };
 
 static void run_job(job_t* j) {
   for (size_t i = j->lo; i < j->hi; ++i) {
@@ -91,6 +117,13 @@ static void run_job(job_t* j) {
         double u2 = u01(j->base, 2 * i + 1);
         double z = sqrt(-2.0 * log(u1)) * cos(6.283185307179586 * u2);
         ((uint16_t*)j->out)[i] = synth_f16_from_double(j->a + j->b * z);
+        break;
+      }
+      case K_NORMAL_E4M3: {
+        double u1 = 1.0 - u01(j->base, 2 * i); /* (0, 1] */
+        double u2 = u01(j->base, 2 * i + 1);
+        double z = sqrt(-2.0 * log(u1)) * cos(6.283185307179586 * u2);
+        ((uint8_t*)j->out)[i] = synth_e4m3_from_double(j->a + j->b * z);
         break;
       }
       case K_LAPLACE: {
@@ -143,6 +176,10 @@ void synth_uniform_f16(uint64_t seed, uint64_t stream, size_t n, double lo, doub
 
 void synth_normal_f16(uint64_t seed, uint64_t stream, size_t n, double mean, double std, uint16_t* out) {
   run_parallel(K_NORMAL, stream_base(seed, stream), n, mean, std, out);
+}
+
+void synth_normal_e4m3(uint64_t seed, uint64_t stream, size_t n, double mean, double std, uint8_t* out) {
+  run_parallel(K_NORMAL_E4M3, stream_base(seed, stream), n, mean, std, out);
 }
 
 void synth_laplace_f16(uint64_t seed, uint64_t stream, size_t n, double loc, double scale, uint16_t* out) {

@@ -98,6 +98,100 @@ def test_group_scales_and_bias_match_dense(K, g):
     assert np.allclose(y, f(p.x) @ W.T, rtol=1e-12, atol=1e-13)
 
 
+# ---------------------------------------------------------------- FP8 E4M3 residual values
+
+def _golden_e4m3():
+    path = os.path.join(os.path.dirname(__file__), "golden", "e4m3_values.txt")
+    rows = []
+    for line in open(path):
+        line = line.strip()
+        if line and not line.startswith("#"):
+            b, v = line.split()
+            rows.append((int(b, 16), float(v)))
+    return rows
+
+
+def test_e4m3_decode_matches_the_format_table():
+    """Values the FP8 E4M3 definition fixes (tests/golden/e4m3_values.txt, OFP8 Table 1)."""
+    for b, v in _golden_e4m3():
+        got = oracle.e4m3_to_double(b)
+        if np.isnan(v):
+            assert np.isnan(got), hex(b)
+        else:
+            assert got == v and np.signbit(got) == np.signbit(v), (hex(b), got, v)
+
+
+def test_e4m3_values_are_exact_binary16_and_ordered():
+    """Every finite E4M3 value is a binary16 value (numpy round trip is exact); the positive
+    codes 0x00..0x7e are strictly increasing and the negative codes mirror them."""
+    vals = np.array([oracle.e4m3_to_double(b) for b in range(256)])
+    finite = ~np.isnan(vals)
+    assert finite.sum() == 254
+    assert np.array_equal(vals[finite].astype(F16).astype(np.float64), vals[finite])
+    pos = vals[:0x7f]
+    assert np.all(np.diff(pos) > 0)
+    assert np.array_equal(vals[0x80:0xff], -pos)
+
+
+def test_fp8_residual_equals_the_same_values_in_fp16():
+    """The FP8 path adds the decoded value and nothing else: converting each E4M3 value to its
+    (exactly equal) binary16 pattern gives the same y and bound."""
+    N, K, M, s = 16, 256, 2, 24
+    p = synth.make_problem("t", N, K, M, s, seed=77, residual_fp8=True)
+    y8, b8 = run(p, residual_fp8=True)
+    as16 = h([oracle.e4m3_to_double(b) for b in p.residual_vals.ravel()]).reshape(p.residual_vals.shape)
+    y16, b16 = oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, as16, p.residual_idx)
+    assert np.array_equal(y8, y16) and np.array_equal(b8, b16)
+
+
+def test_paper_storage_matches_dense():
+    """The paper's own storage end to end: alpha and beta per (row, 128-column group), FP8 E4M3
+    residual values; brute-force dense W^ (E4M3 decoded by the pinned routine) times x."""
+    p = synth.paper_problem(0, 0)
+    p.T, p.x = p.T[:64, :300], p.x[:, :300]  # a ragged last group
+    N, K = p.T.shape
+    G = -(-K // 128)
+    p.alpha, p.beta = p.alpha[:N, :G], p.beta[:N, :G]
+    p.v = p.v[:K]
+    keep = p.salient_idx < K
+    p.salient_idx, p.s = p.salient_idx[keep], int(keep.sum())
+    cols = np.flatnonzero(keep)
+    p.residual_vals = np.ascontiguousarray(p.residual_vals[:N // 4][:, cols])
+    pos = synth.residual_positions(p.residual_idx[:N // 4], 32)[:, cols]
+    packed = np.zeros((N // 4, -(-p.s // 4)), np.uint8)
+    for c in range(p.s):
+        packed[:, c // 4] |= (pos[:, c] << (2 * (c % 4))).astype(np.uint8)
+    p.residual_idx = packed
+    y, _ = run(p, beta=p.beta, group_size=128, residual_fp8=True)
+    alpha, beta = f(p.alpha), f(p.beta)
+    g = np.arange(K) // 128
+    W = alpha[:, g] * f(p.v)[None, :] * p.T + beta[:, g]
+    for q in range(N // 4):
+        for c in range(p.s):
+            W[4 * q + pos[q, c], p.salient_idx[c]] += oracle.e4m3_to_double(p.residual_vals[q, c])
+    assert np.allclose(y, f(p.x) @ W.T, rtol=1e-12, atol=1e-13)
+
+
+def test_generator_e4m3_rounding_is_nearest_even():
+    """The input generator's FP8 rounding against brute force over every finite E4M3 value
+    (nearest, ties to the even code), with saturation at 448."""
+    codes = [b for b in range(0x7f)]
+    vals = np.array([oracle.e4m3_to_double(b) for b in codes])
+    rng = np.random.default_rng(3)
+    xs = np.concatenate([rng.normal(0, 0.02, 2000), rng.normal(0, 30, 2000), (vals[:-1] + vals[1:]) / 2,
+                         vals, [500.0, 1e-12, 2.0 ** -10, 3 * 2.0 ** -11]])
+    for x in xs:
+        a = abs(x)
+        if a >= 448:
+            want = 0x7e
+        else:
+            d = np.abs(vals - a)
+            cand = np.flatnonzero(d == d.min())
+            want = int(cand[0]) if len(cand) == 1 else int([c for c in cand if c % 2 == 0][0])
+        want |= 0x80 if np.signbit(x) else 0
+        assert synth.e4m3_from_double(x) == want, (x, hex(want))
+
+
 # ---------------------------------------------------------------- closed forms
 
 def test_unit_vector_extracts_a_column():

@@ -77,6 +77,21 @@ def pin_failures(lib):
     T = np.zeros((1, 128), np.int8)
     T[0, :5] = [1, -1, 0, 0, 0]
     check("pack3", int(oracle.pack(T, "base3", lib=lib)[0]) == 119)
+    # FP8 E4M3 residual values: the format's defining values, and a dense brute force with them
+    table = {0x01: 2.0 ** -9, 0x07: 7 * 2.0 ** -9, 0x08: 2.0 ** -6, 0x38: 1.0, 0x7e: 448.0, 0xb8: -1.0}
+    check("e4m3", all(lib.qo_e4m3_to_double(b) == v for b, v in table.items()) and
+          np.isnan(lib.qo_e4m3_to_double(0x7f)))
+    p = synth.make_problem("m", 8, 64, 2, 8, seed=91, residual_fp8=True)
+    y, _ = oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx, residual_fp8=True,
+                       lib=lib)
+    W = f(p.alpha) * f(p.v)[None] * p.T
+    pos = synth.residual_positions(p.residual_idx, p.s)
+    dec = {b: lib.qo_e4m3_to_double(int(b)) for b in range(256)} if "e4m3" not in fails else None
+    if dec is not None:
+        for q in range(2):
+            for c in range(p.s):
+                W[4 * q + pos[q, c], p.salient_idx[c]] += dec[int(p.residual_vals[q, c])]
+        check("fp8_residual", np.allclose(y, f(p.x) @ W.T, rtol=1e-12, atol=1e-13))
     # LUT symmetry and single-digit entries
     xs = np.array([0.3, -1.25, 2.0, 0.125, -0.5])
     lut = oracle.lut5(xs, lib=lib)
@@ -85,7 +100,10 @@ def pin_failures(lib):
 
 
 MUTANTS = {
-    "drop_residual_term": [("acc += qo_half_to_double(residual_vals", "acc += 0.0 * qo_half_to_double(residual_vals")],
+    "drop_residual_term": [("acc += residual_value(", "acc += 0.0 * residual_value(")],
+    "e4m3_exponent_bias": [("expo - 10); /* (1 + frac/8)", "expo - 9); /* (1 + frac/8)")],
+    "e4m3_subnormal_scale": [("ldexp((double)frac, -9);", "ldexp((double)frac, -10);")],
+    "e4m3_nan_range": [("if (expo == 0xf && frac == 7) {", "if (expo == 0xf && frac >= 6) {")],
     "wrong_residual_row": [("== o % 4)\n          acc +=", "== (o + 1) % 4)\n          acc +=")],
     "ternary_sign_flip": [("tvx += (double)T[", "tvx -= (double)T[")],
     "rescale_index_shift": [("qo_half_to_double(v[j]) * xj", "qo_half_to_double(v[(j + 1) % K]) * xj")],
