@@ -11,7 +11,10 @@
  * the bias beta being zero) plus the column-semi-sparse residual of Sec. 3.2 / Sec. 3.5: in
  * each salient column S_c, every group of four consecutive output rows holds exactly one
  * residual value and its 2-bit position inside the group (1:4 sparsity along the rows).
- * One scale per output row is supported (group size = K); per-group alpha/beta is not.
+ * The paper's own storage is available too (Sec. 3.3 Eq. 4 and Sec. 3.5): alpha, and optionally
+ * the bias beta, per row and group of 128 columns; base-3 codes; FP8 E4M3 residual values:
+ *   y[m][o] = sum_g ( alpha[o][g] sum_{j in g} T v x + beta[o][g] sum_{j in g} x[m][j] ) + residual
+ * (see qtea_pack_layout and qtea_set_layout_options).
  *
  * Conventions for every entry point:
  *   - fp16 tensors are IEEE 754 binary16 bit patterns passed as uint16_t.
@@ -48,9 +51,16 @@ typedef enum qtea_status {
 } qtea_status;
 
 typedef enum qtea_format {
-  QTEA_FMT_2BIT = 0, /* 4 codes per byte; the only format qtea_gemv consumes */
-  QTEA_FMT_BASE3 = 1 /* 5 codes per byte, 26 bytes per 128 columns (Sec. 3.5); not implemented */
+  QTEA_FMT_2BIT = 0, /* 4 codes per byte, this library's layout */
+  QTEA_FMT_BASE3 = 1 /* 5 codes per byte, 26 bytes per 128 columns: the paper's layout (Sec. 3.5) */
 } qtea_format;
+
+/* Layout options (qtea_set_layout_options), the paper's own storage of the scales and residual. */
+typedef enum qtea_option {
+  QTEA_OPT_BIAS = 1,        /* row_scale holds (alpha, beta) pairs: fp16 [N][G][2] (Eq. 4's beta) */
+  QTEA_OPT_RESIDUAL_FP8 = 2 /* residual_vals holds FP8 E4M3 bytes [N/4][s] (Sec. 4.1), passed
+                               through the same pointer argument */
+} qtea_option;
 
 /* Largest batch (rows of x) one qtea_gemv call accepts. */
 #define QTEA_MAX_M 16
@@ -61,15 +71,24 @@ typedef enum qtea_format {
  *
  *   ternary_codes  device int8 [N][K], values -1, 0, +1 (read only; may be freed afterwards)
  *   N, K           output rows and input columns, N >= 0, K >= 0
- *   group_size     must equal K (one alpha per row); anything else -> QTEA_ERR_UNSUPPORTED
+ *   group_size     K (one alpha per row) or 128 (alpha per row and group of 128 columns,
+ *                  G = ceil(K/128) groups, the last one possibly shorter); anything else ->
+ *                  QTEA_ERR_UNSUPPORTED
  *   n_salient      number of salient columns s the layout will be used with, s >= 0;
  *                  if s > 0, N must be a multiple of 4 (groups of four rows)
- *   format         QTEA_FMT_2BIT (QTEA_FMT_BASE3 -> QTEA_ERR_UNSUPPORTED)
+ *   format         QTEA_FMT_2BIT or QTEA_FMT_BASE3
  *   out            receives the new layout on success, NULL on failure
  *
  * Packed layout (2-bit): K_pad = K rounded up to a multiple of 64. Row r occupies bytes
  * [r*K_pad/4, (r+1)*K_pad/4); column k sits in byte r*K_pad/4 + k/4 at bits 2*(k%4) and
  * 2*(k%4)+1 (least significant first) as the code T+1; columns k >= K hold code 1.
+ * Base-3 layout: K_pad = K rounded up to a multiple of 128; each row is K_pad/128 groups of 26
+ * bytes; byte q of group h holds columns 128h + 5q + d, d = 0..4, as sum_d (T+1) 3^d (lowest
+ * column in the least significant digit); byte 25 holds three columns and two pad digits; pad
+ * digits and columns >= K are digit 1.
+ * Layouts other than 2-bit with group_size = K and no options (the paper's storage) run on a
+ * general kernel for every M; the TMA batch-1 and tensor-core low-batch kernels serve the
+ * 2-bit, one-scale-per-row layout.
  *
  * The call validates every code on the device and synchronizes `stream` once to read the
  * result; invalid codes give QTEA_ERR_BAD_CODES and no layout. It allocates the packed
@@ -84,10 +103,12 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
  *
  *   x              device fp16 [M][K], activations
  *   packed_ternary layout from qtea_pack_layout
- *   row_scale      device fp16 [N], alpha_o (one scale per output row)
+ *   row_scale      device fp16 [N][G], alpha (G = 1 unless the layout's group_size is 128);
+ *                  with QTEA_OPT_BIAS, [N][G][2]: alpha then beta of each group
  *   col_scale      device fp16 [K], v_j, the column-wise rescale factors (Sec. 3.3, Eq. 4)
  *   salient_idx    device int32 [s], strictly ascending column indices, each in [0, K)
  *   residual_vals  device fp16 [N/4][s]: R of group q (rows 4q..4q+3) in salient column c
+ *                  (FP8 E4M3 bytes [N/4][s] with QTEA_OPT_RESIDUAL_FP8)
  *   residual_idx   device uint8 [N/4][ceil(s/4)]: 2-bit position of that value in its
  *                  group; entry (q, c) at bits 2*(c%4) of byte q*ceil(s/4) + c/4
  *   y              device fp32 [M][N], overwritten
@@ -150,6 +171,7 @@ typedef struct qtea_layout_desc {
   const void* packed_data;  /* device pointer to the packed ternary weights */
   int batch1_kernel;        /* 1 if M = 1 calls run the TMA stream-K batch-1 kernel, 0 if they
                                fall back to the general kernel (e.g. no tensor-map support) */
+  int options;              /* QTEA_OPT_* flags */
 } qtea_layout_desc;
 
 int qtea_layout_describe(const qtea_layout* layout, qtea_layout_desc* out);
@@ -169,6 +191,15 @@ int qtea_layout_copy_packed(const qtea_layout* layout, void* dst, size_t bytes, 
  * Returns QTEA_ERR_INVALID_ARG for other values. Batch sizes M > 1 are not affected.
  */
 int qtea_set_activation_precision(qtea_layout* layout, int bits);
+
+/*
+ * Storage options of the scales and residual values qtea_gemv reads with this layout: any
+ * combination of QTEA_OPT_BIAS and QTEA_OPT_RESIDUAL_FP8 (0 restores fp16 alpha only and fp16
+ * residual values). Other bits -> QTEA_ERR_INVALID_ARG. With any option set, calls run on the
+ * general kernel (see qtea_pack_layout). Set it before the calls that use it; it takes effect
+ * for calls made afterwards.
+ */
+int qtea_set_layout_options(qtea_layout* layout, int options);
 
 /*
  * Status written by the kernels of this layout: QTEA_OK, or QTEA_ERR_TIMEOUT if a bounded

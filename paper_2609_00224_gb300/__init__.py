@@ -24,6 +24,8 @@ QTEA_ERR_TIMEOUT = 6
 QTEA_ERR_SCRATCH_LIMIT = 7
 QTEA_FMT_2BIT = 0
 QTEA_FMT_BASE3 = 1
+QTEA_OPT_BIAS = 1
+QTEA_OPT_RESIDUAL_FP8 = 2
 QTEA_MAX_M = 16
 
 _lib = None
@@ -44,7 +46,7 @@ class _Problem(ctypes.Structure):
 class _LayoutDesc(ctypes.Structure):
     _fields_ = [("N", ctypes.c_int), ("K", ctypes.c_int), ("K_pad", ctypes.c_int), ("group_size", ctypes.c_int),
                 ("n_salient", ctypes.c_int), ("format", ctypes.c_int), ("packed_bytes", ctypes.c_size_t),
-                ("packed_data", ctypes.c_void_p), ("batch1_kernel", ctypes.c_int)]
+                ("packed_data", ctypes.c_void_p), ("batch1_kernel", ctypes.c_int), ("options", ctypes.c_int)]
 
 
 def library_path() -> str:
@@ -77,6 +79,8 @@ def load(build_if_missing: bool = True):
     lib.qtea_gemv_grouped.argtypes = [P, i32, i32, P]
     lib.qtea_set_activation_precision.restype = i32
     lib.qtea_set_activation_precision.argtypes = [P, i32]
+    lib.qtea_set_layout_options.restype = i32
+    lib.qtea_set_layout_options.argtypes = [P, i32]
     lib.qtea_layout_copy_packed.restype = i32
     lib.qtea_layout_copy_packed.argtypes = [P, P, ctypes.c_size_t, P]
     lib.qtea_gemv_m1_static.restype = i32
@@ -119,9 +123,16 @@ def _f16_types():
 class Layout:
     """Owner of a qtea_layout handle (packed ternary weights + split-K workspace)."""
 
-    def __init__(self, handle: int, N: int, K: int, n_salient: int):
+    def __init__(self, handle: int, N: int, K: int, n_salient: int, group_size: Optional[int] = None):
         self._h = ctypes.c_void_p(handle)
         self.N, self.K, self.n_salient = N, K, n_salient
+        self.group_size = K if group_size is None else group_size
+        self.options = 0
+
+    @property
+    def G(self) -> int:
+        g = self.group_size or 1
+        return (self.K + g - 1) // g if self.K else 1
 
     @property
     def handle(self):
@@ -141,6 +152,14 @@ class Layout:
         rc = load().qtea_set_activation_precision(self.handle, int(bits))
         if rc:
             raise QteaError(rc, "qtea_set_activation_precision")
+        return self
+
+    def set_options(self, options: int):
+        """QTEA_OPT_BIAS and/or QTEA_OPT_RESIDUAL_FP8: the paper's storage of beta and residual values."""
+        rc = load().qtea_set_layout_options(self.handle, int(options))
+        if rc:
+            raise QteaError(rc, "qtea_set_layout_options")
+        self.options = int(options)
         return self
 
     def free(self):
@@ -168,7 +187,7 @@ def qtea_pack_layout(codes, n_salient: int = 0, group_size: Optional[int] = None
                                  _stream(stream), ctypes.byref(out))
     if rc:
         raise QteaError(rc, "qtea_pack_layout")
-    return Layout(out.value, N, K, n_salient)
+    return Layout(out.value, N, K, n_salient, K if group_size is None else group_size)
 
 
 def _problem_args(x, layout, row_scale, col_scale, salient_idx, residual_vals, residual_idx, y):
@@ -183,10 +202,12 @@ def _problem_args(x, layout, row_scale, col_scale, salient_idx, residual_vals, r
     args = [
         _ptr(x, f16, "x", (M, K)),
         layout.handle,
-        _ptr(row_scale.reshape(-1) if row_scale is not None else None, f16, "row_scale", (N,)),
+        _ptr(row_scale.reshape(-1) if row_scale is not None else None, f16, "row_scale",
+             (N * layout.G * (2 if layout.options & QTEA_OPT_BIAS else 1),)),
         _ptr(col_scale, f16, "col_scale", (K,)),
         _ptr(salient_idx, (torch.int32,), "salient_idx", (s,)) if s else None,
-        _ptr(residual_vals, f16, "residual_vals", (N // 4, s)) if s else None,
+        _ptr(residual_vals, (torch.uint8,) if layout.options & QTEA_OPT_RESIDUAL_FP8 else f16, "residual_vals",
+             (N // 4, s)) if s else None,
         _ptr(residual_idx, (torch.uint8,), "residual_idx", (N // 4, (s + 3) // 4)) if s else None,
         _ptr(y, (torch.float32,), "y", (M, N)),
     ]

@@ -98,10 +98,38 @@ int check_problem(const qtea_gemv_problem& q, int M) {
   if (l->K == 0) return QTEA_OK;
   if (!q.x || !q.row_scale || !q.col_scale) return QTEA_ERR_INVALID_ARG;
   if (!aligned(q.x, 2) || !aligned(q.row_scale, 2) || !aligned(q.col_scale, 2)) return QTEA_ERR_INVALID_ARG;
+  const size_t rv_align = (l->options & QTEA_OPT_RESIDUAL_FP8) ? 1 : 2;
   if (l->n_salient > 0 && (!q.salient_idx || !q.residual_vals || !q.residual_idx || !aligned(q.salient_idx, 4) ||
-                           !aligned(q.residual_vals, 2)))
+                           !aligned(q.residual_vals, rv_align)))
     return QTEA_ERR_INVALID_ARG;
   return QTEA_OK;
+}
+
+// The paper's own storage: base-3 codes, groups of 128 columns, beta or FP8 residual values.
+bool is_paper(const qtea_layout* l) { return l->format != QTEA_FMT_2BIT || l->group_size != l->K || l->options != 0; }
+
+int launch_paper_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
+  const qtea_layout* l = q.packed_ternary;
+  PaperParams p;
+  p.x = q.x;
+  p.packed = l->packed;
+  p.scales = q.row_scale;
+  p.v = q.col_scale;
+  p.sal = q.salient_idx;
+  p.rvals = q.residual_vals;
+  p.ridx = q.residual_idx;
+  p.y = q.y;
+  p.M = M;
+  p.N = l->N;
+  p.K = l->K;
+  p.s = l->n_salient;
+  p.group_size = l->group_size > 0 ? l->group_size : 1;
+  p.G = (l->K + p.group_size - 1) / p.group_size;
+  p.row_bytes = l->row_bytes;
+  p.format = l->format;
+  p.bias = (l->options & QTEA_OPT_BIAS) ? 1 : 0;
+  p.residual_fp8 = (l->options & QTEA_OPT_RESIDUAL_FP8) ? 1 : 0;
+  return launch_paper(p, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
 }
 
 int launch_generic_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
@@ -364,8 +392,7 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
   if ((long long)N * K > 0 && !ternary_codes) return QTEA_ERR_INVALID_ARG;
   if (n_salient > 0 && N % 4 != 0) return QTEA_ERR_INVALID_ARG;
   if (format != QTEA_FMT_2BIT && format != QTEA_FMT_BASE3) return QTEA_ERR_INVALID_ARG;
-  if (format == QTEA_FMT_BASE3) return QTEA_ERR_UNSUPPORTED;
-  if (group_size != K) return QTEA_ERR_UNSUPPORTED;
+  if (group_size != K && group_size != 128) return QTEA_ERR_UNSUPPORTED;
   if ((long long)K + 63 > 0x7fffffffLL) return QTEA_ERR_INVALID_ARG;
 
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -379,13 +406,15 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
   std::memset(l, 0, sizeof(*l));
   l->N = N;
   l->K = K;
-  l->K_pad = round_up(K, 64);
+  l->K_pad = format == QTEA_FMT_BASE3 ? round_up(K, 128) : round_up(K, 64);
   l->group_size = group_size;
   l->n_salient = n_salient;
   l->format = format;
+  l->options = 0;
+  l->row_bytes = format == QTEA_FMT_BASE3 ? l->K_pad / 128 * 26 : l->K_pad / 4;
   l->device = dev;
   l->act_bits = 24;
-  l->packed_bytes = (size_t)N * (size_t)(l->K_pad / 4);
+  l->packed_bytes = (size_t)N * (size_t)l->row_bytes;
   if (cudaMalloc(&l->packed, l->packed_bytes > 0 ? l->packed_bytes : 16) != cudaSuccess ||
       cudaMalloc(&l->status, 2 * sizeof(int)) != cudaSuccess) {
     cudaGetLastError();
@@ -395,7 +424,9 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
   int rc = QTEA_OK;
   int host_flags[2] = {0, 0};
   if (cudaMemsetAsync(l->status, 0, 2 * sizeof(int), st) != cudaSuccess ||
-      launch_pack(ternary_codes, N, K, l->K_pad, reinterpret_cast<uint32_t*>(l->packed), l->status + 1, st) !=
+      (format == QTEA_FMT_BASE3
+           ? launch_pack_base3(ternary_codes, N, K, l->packed, l->status + 1, st)
+           : launch_pack(ternary_codes, N, K, l->K_pad, reinterpret_cast<uint32_t*>(l->packed), l->status + 1, st)) !=
           cudaSuccess ||
       cudaMemcpyAsync(host_flags, l->status, sizeof(host_flags), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
       cudaStreamSynchronize(st) != cudaSuccess) {
@@ -404,8 +435,8 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
     rc = QTEA_ERR_BAD_CODES;
   } else if (cudaMemsetAsync(l->status, 0, 2 * sizeof(int), st) != cudaSuccess) {
     rc = QTEA_ERR_CUDA;
-  } else {
-    rc = plan_m1(l, prop);
+  } else if (format == QTEA_FMT_2BIT && group_size == K) {
+    rc = plan_m1(l, prop);  // the batch-1 and low-batch kernels' resources
   }
   if (rc == QTEA_OK && cudaStreamSynchronize(st) != cudaSuccess) rc = QTEA_ERR_CUDA;
   if (rc != QTEA_OK) {
@@ -438,7 +469,9 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
       if (cudaMemsetAsync(q.y, 0, (size_t)M * l->N * sizeof(float), st) != cudaSuccess) rc = QTEA_ERR_CUDA;
       continue;
     }
-    if (M == 1 && l->m1_ok) {
+    if (is_paper(l)) {
+      rc = launch_paper_problem(q, M, st);
+    } else if (M == 1 && l->m1_ok) {
       m1_idx[n_m1++] = i;
     } else {
       rc = launch_mb_problem(q, M, st);
@@ -478,7 +511,14 @@ int qtea_layout_describe(const qtea_layout* l, qtea_layout_desc* out) {
   out->format = l->format;
   out->packed_bytes = l->packed_bytes;
   out->packed_data = l->packed;
-  out->batch1_kernel = l->m1_ok ? 1 : 0;
+  out->batch1_kernel = (l->m1_ok && !is_paper(l)) ? 1 : 0;
+  out->options = l->options;
+  return QTEA_OK;
+}
+
+int qtea_set_layout_options(qtea_layout* l, int options) {
+  if (!l || (options & ~(QTEA_OPT_BIAS | QTEA_OPT_RESIDUAL_FP8)) != 0) return QTEA_ERR_INVALID_ARG;
+  l->options = options;
   return QTEA_OK;
 }
 

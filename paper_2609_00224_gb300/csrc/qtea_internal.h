@@ -137,6 +137,22 @@ struct GenericParams {
   int M, N, K, K_pad, s;
 };
 
+// Layouts in the paper's own storage (base-3 codes, scale groups of 128 columns, beta, FP8
+// residual values): one warp per output row, any batch.
+struct PaperParams {
+  const uint16_t* x;        // [M][K]
+  const uint8_t* packed;    // [N][row_bytes]: 2-bit (K_pad/4 bytes per row) or base-3 (26 per 128 columns)
+  const uint16_t* scales;   // [N][G] alpha, or [N][G][2] (alpha, beta) with bias
+  const uint16_t* v;        // [K]
+  const int32_t* sal;       // [s]
+  const void* rvals;        // [N/4][s] fp16, or FP8 E4M3 bytes with residual_fp8
+  const uint8_t* ridx;      // [N/4][ceil(s/4)]
+  float* y;                 // [M][N]
+  int M, N, K, s, G, group_size, row_bytes, format, bias, residual_fp8;
+};
+
+cudaError_t launch_paper(const PaperParams& p, cudaStream_t st);
+cudaError_t launch_pack_base3(const int8_t* codes, int N, int K, uint8_t* packed, int* bad_flag, cudaStream_t st);
 cudaError_t launch_m1(const TensorMaps& maps, const GroupParams& p, int grid, size_t smem, cudaStream_t st);
 cudaError_t m1_configure(size_t smem_optin, size_t* dyn_max);
 cudaError_t launch_generic(const GenericParams& p, cudaStream_t st);
@@ -147,6 +163,8 @@ cudaError_t launch_pack(const int8_t* codes, int N, int K, int K_pad, uint32_t* 
 
 struct qtea_layout {
   int N, K, K_pad, group_size, n_salient, format;
+  int options;           // QTEA_OPT_* flags (qtea_set_layout_options)
+  int row_bytes;         // packed bytes per row
   size_t packed_bytes;
   uint8_t* packed;
   int device;

@@ -42,10 +42,11 @@ def test_host_side_argument_checks_need_no_gpu():
     assert lib.qtea_pack_layout(None, -1, 8, 8, 0, 0, None, ctypes.byref(out)) == qt.QTEA_ERR_INVALID_ARG
     assert lib.qtea_pack_layout(None, 6, 8, 8, 4, 0, None, ctypes.byref(out)) == qt.QTEA_ERR_INVALID_ARG  # N % 4
     assert lib.qtea_pack_layout(None, 4, 8, 8, 9, 0, None, ctypes.byref(out)) == qt.QTEA_ERR_INVALID_ARG  # s > K
-    assert lib.qtea_pack_layout(ctypes.c_void_p(16), 4, 8, 8, 0, qt.QTEA_FMT_BASE3, None,
-                                ctypes.byref(out)) == qt.QTEA_ERR_UNSUPPORTED
-    assert lib.qtea_pack_layout(ctypes.c_void_p(16), 4, 256, 128, 0, 0, None,
-                                ctypes.byref(out)) == qt.QTEA_ERR_UNSUPPORTED  # group-wise alpha
+    assert lib.qtea_pack_layout(ctypes.c_void_p(16), 4, 8, 8, 0, 7, None,
+                                ctypes.byref(out)) == qt.QTEA_ERR_INVALID_ARG  # no such format
+    assert lib.qtea_pack_layout(ctypes.c_void_p(16), 4, 256, 64, 0, 0, None,
+                                ctypes.byref(out)) == qt.QTEA_ERR_UNSUPPORTED  # groups other than K or 128
+    assert lib.qtea_set_layout_options(None, qt.QTEA_OPT_BIAS) == qt.QTEA_ERR_INVALID_ARG
     assert lib.qtea_gemv(None, None, None, None, None, None, None, None, 1, None) == qt.QTEA_ERR_INVALID_ARG
     lib.qtea_free(None)
 

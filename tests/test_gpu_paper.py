@@ -1,0 +1,129 @@
+"""GPU parity for layouts in the paper's own storage (Sec. 3.3 Eq. 4, Sec. 3.5, Sec. 4.1):
+base-3 codes, alpha and beta per row and group of 128 columns, FP8 E4M3 residual values.
+
+Same pass rule as test_gpu_parity: |y - y_ref| <= 1e-4 * sum_j |x_j * W^[o][j]| + 1e-6 per output
+element, W^ including beta and the residual; base-3 packing bit-identical to the oracle's packer.
+"""
+import itertools
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+REL, ABS = 1e-4, 1e-6
+
+
+@pytest.fixture(scope="module")
+def qt():
+    import paper_2609_00224_gb300 as m
+    m.load()
+    return m
+
+
+def dev(a, dtype=None):
+    t = torch.from_numpy(np.ascontiguousarray(a))
+    if dtype is not None:
+        t = t.view(dtype)
+    return t.cuda()
+
+
+def scales(p, bias):
+    """row_scale as the ABI wants it: [N][G] alpha, or [N][G][2] (alpha, beta) pairs."""
+    if not bias:
+        return p.alpha.reshape(-1)
+    return np.stack([p.alpha.reshape(p.N, -1), p.beta.reshape(p.N, -1)], axis=-1).reshape(-1)
+
+
+def run_paper(qt, p, fmt, bias, M=None):
+    layout = qt.qtea_pack_layout(dev(p.T), n_salient=p.s, group_size=p.group_size or p.K, fmt=fmt)
+    opts = (qt.QTEA_OPT_BIAS if bias else 0) | (qt.QTEA_OPT_RESIDUAL_FP8 if p.residual_fp8 else 0)
+    layout.set_options(opts)
+    default = fmt == qt.QTEA_FMT_2BIT and not p.group_size and opts == 0  # the library's own storage
+    assert layout.describe()["batch1_kernel"] == int(default) and layout.describe()["options"] == opts
+    x = p.x if M is None else p.x[:M]
+    rv = dev(p.residual_vals) if p.residual_fp8 else dev(p.residual_vals.view(np.int16), torch.float16)
+    y = qt.qtea_gemv(dev(x.view(np.int16), torch.float16), layout, dev(scales(p, bias).view(np.int16), torch.float16),
+                     dev(p.v.view(np.int16), torch.float16), dev(p.salient_idx) if p.s else None,
+                     rv if p.s else None, dev(p.residual_idx) if p.s else None)
+    torch.cuda.synchronize()
+    assert qt.qtea_device_status(layout) == 0
+    return y.cpu().numpy().astype(np.float64), layout
+
+
+def reference(p, bias, rows=None, M=None):
+    x = p.x if M is None else p.x[:M]
+    return oracle.gemv(x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx,
+                       beta=p.beta if bias else None, group_size=p.group_size or p.K, rows=rows,
+                       residual_fp8=p.residual_fp8)
+
+
+def assert_within(y, y_ref, bound, what=""):
+    err = np.abs(y - y_ref)
+    lim = REL * bound + ABS
+    bad = np.argwhere(err > lim)
+    assert bad.size == 0, (f"{what}: {len(bad)} elements out of tolerance; worst normalised error "
+                           f"{(err / lim).max():.3g} at {bad[0].tolist()}")
+    return float((err / lim).max())
+
+
+@pytest.mark.parametrize("N,K", [(4, 128), (8, 1), (12, 300), (64, 1024), (33, 5)])
+def test_base3_pack_is_bit_identical_to_oracle(qt, N, K):
+    T = synth.codes(N * 1000 + K, 1, (N, K), 0.3, 0.4)
+    layout = qt.qtea_pack_layout(dev(T), fmt=qt.QTEA_FMT_BASE3)
+    d = layout.describe()
+    assert d["K_pad"] == -(-K // 128) * 128 and d["packed_bytes"] == N * (-(-K // 128)) * 26
+    got = qt.packed_bytes(layout)
+    torch.cuda.synchronize()
+    assert np.array_equal(got.cpu().numpy(), oracle.pack(T, "base3").reshape(-1))
+
+
+def test_base3_pack_rejects_invalid_codes(qt):
+    T = np.zeros((4, 256), np.int8)
+    T[2, 200] = 2
+    with pytest.raises(qt.QteaError) as e:
+        qt.qtea_pack_layout(dev(T), fmt=qt.QTEA_FMT_BASE3)
+    assert e.value.status == qt.QTEA_ERR_BAD_CODES
+
+
+@pytest.mark.parametrize("fmt,group,bias,fp8", list(itertools.product([0, 1], [0, 128], [0, 1], [0, 1])))
+def test_paper_storage_parity_small(qt, fmt, group, bias, fp8):
+    """Every combination of code format, scale groups, beta and FP8 residual, K ragged against both
+    the 128-column groups and the 64-column 2-bit padding, batch sizes 1, 3 and 16."""
+    N, K, s = 64, 300, 16
+    p = synth.make_problem("t", N, K, 16, s, seed=1 + fmt + 2 * bool(group) + 4 * bias + 8 * fp8,
+                           group_size=group, beta_std=0.002 if bias else 0.0, residual_fp8=bool(fp8))
+    for M in (1, 3, 16):
+        y, _ = run_paper(qt, p, fmt, bias, M=M)
+        y_ref, b = reference(p, bias, M=M)
+        assert_within(y, y_ref, b, f"fmt {fmt} group {group} bias {bias} fp8 {fp8} M {M}")
+
+
+def test_options_switch_a_default_layout_to_the_paper_path(qt):
+    """A 2-bit, one-alpha-per-row layout with QTEA_OPT_BIAS reads (alpha, beta) pairs; clearing the
+    options returns it to the batch-1 kernel."""
+    N, K = 256, 1024
+    p = synth.make_problem("t", N, K, 1, 32, seed=5, beta_std=0.002)
+    y, layout = run_paper(qt, p, qt.QTEA_FMT_2BIT, True)
+    y_ref, b = reference(p, True)
+    assert_within(y, y_ref, b, "2-bit with beta")
+    layout.set_options(0)
+    assert layout.describe()["batch1_kernel"] == 1
+    with pytest.raises(qt.QteaError):
+        layout.set_options(4)
+
+
+@pytest.mark.parametrize("matrix", range(7))
+@pytest.mark.parametrize("M", [1, 4])
+def test_paper_storage_llama3_8b_layer(qt, matrix, M):
+    """The Llama3-8B layer GEMVs in the paper's storage (base-3, 128-column groups with beta, FP8
+    residual), on 48 sampled output rows."""
+    p = synth.paper_problem(1, matrix, M=M)
+    y, _ = run_paper(qt, p, qt.QTEA_FMT_BASE3, True)
+    rows = np.sort(np.random.default_rng(matrix).choice(p.N, size=48, replace=False)).astype(np.int32)
+    y_ref, b = reference(p, True, rows=rows)
+    assert_within(y[:, rows], y_ref, b, p.name)
