@@ -40,6 +40,14 @@ def algorithmic_bytes(N, K, s, M=1):
             + 2 * M * K + 4 * M * N)
 
 
+def paper_algorithmic_bytes(N, K, s, M=1, group=128):
+    """Bytes one call must move in the paper's storage: base-3 codes (26 bytes per 128 columns),
+    alpha and beta per (row, group), v, salient list, FP8 residual values, positions, x, y."""
+    G = -(-K // group)
+    return (N * (-(-K // 128)) * 26 + 2 * 2 * N * G + 2 * K + 4 * s + (N // 4) * s + (N // 4) * ((s + 3) // 4)
+            + 2 * M * K + 4 * M * N)
+
+
 def profiled_traffic():
     """DRAM bytes per launch from the committed ncu summary, if the kernel source still
     matches the one that was profiled (else None)."""
@@ -554,6 +562,54 @@ def qtea_arm(args):
         del qlayers, qw
         torch.cuda.empty_cache()
 
+    # ---- the Llama3-8B layer in the paper's own storage (base-3 codes, alpha and beta per 128-column
+    #      group, FP8 residual values): the seven GEMVs per step on the general kernel, rotating over
+    #      resident layers
+    paper = None
+    if not args.no_paper:
+        n_res = 4
+        players = []
+        for li in range(n_res):
+            L = []
+            for mi in range(7):
+                pp = synth.paper_problem(1, mi, layer=li)
+                f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
+                T = torch.from_numpy(pp.T).cuda()
+                lay = qt.qtea_pack_layout(T, n_salient=pp.s, group_size=128, fmt=qt.QTEA_FMT_BASE3)
+                lay.set_options(qt.QTEA_OPT_BIAS | qt.QTEA_OPT_RESIDUAL_FP8)
+                del T
+                sc = np.stack([pp.alpha.reshape(pp.N, -1), pp.beta.reshape(pp.N, -1)], axis=-1).reshape(-1)
+                L.append(dict(x=f16(pp.x), layout=lay, row_scale=f16(sc), col_scale=f16(pp.v),
+                              salient_idx=torch.from_numpy(pp.salient_idx).cuda(),
+                              residual_vals=torch.from_numpy(pp.residual_vals).cuda(),
+                              residual_idx=torch.from_numpy(pp.residual_idx).cuda(),
+                              y=torch.empty((1, pp.N), dtype=torch.float32, device="cuda")))
+            players.append(L)
+        pbytes = sum(paper_algorithmic_bytes(N, K, synth.salient_count(K)) for _, N, K in synth.config_shapes(1))
+        nsteps = 16
+        with torch.cuda.stream(stream):
+            for g in players[0]:
+                qt.qtea_gemv(g["x"], g["layout"], g["row_scale"], g["col_scale"], g["salient_idx"],
+                             g["residual_vals"], g["residual_idx"], y=g["y"], stream=stream)
+        gp = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gp, stream=stream):
+            for st in range(nsteps):
+                for g in players[st % n_res]:
+                    qt.qtea_gemv(g["x"], g["layout"], g["row_scale"], g["col_scale"], g["salient_idx"],
+                                 g["residual_vals"], g["residual_idx"], y=g["y"], stream=stream)
+        tp = timed_replay(gp) * 1e3 / nsteps
+        del gp
+        status = max(qt.qtea_device_status(g["layout"]) for L in players for g in L)
+        if status:
+            raise RuntimeError(f"device status {status} in the paper-storage steps")
+        w = sum(N * K for _, N, K in synth.config_shapes(1))
+        paper = {"workload": "llama3_8b_layer_paper_storage", "us_per_step": round(tp, 2),
+                 "GBps": round(pbytes / (tp * 1e-6) / 1e9, 1), "bytes_per_step": pbytes,
+                 "bits_per_weight": round(8 * (pbytes - sum(2 * K + 4 * N for _, N, K in synth.config_shapes(1))) / w, 3),
+                 "kernel": "qtea_gemv_paper_kernel (general, one warp per row)", "layers_resident": n_res}
+        del players
+        torch.cuda.empty_cache()
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         probs = [g["host"] for g in layers[0]]
@@ -582,7 +638,7 @@ def qtea_arm(args):
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
                          "us_per_launch": round(1e3 * total_ms / args.steps, 3),
                          "us_per_launch_isolated": None if iso_us is None else round(iso_us, 3)},
-            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
+            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
             "setup_s": round(t_gen, 1),
         }
         print(json.dumps(line), flush=True)
@@ -599,6 +655,7 @@ def main():
     ap.add_argument("--impl", choices=["qtea", "reference"], default="qtea")
     ap.add_argument("--no-dense", action="store_true", help="skip the dense fp16 cuBLAS baseline")
     ap.add_argument("--no-m-sweep", action="store_true", help="skip the Qwen3-14B batch sweep (M = 1 .. 16)")
+    ap.add_argument("--no-paper", action="store_true", help="skip the layer in the paper's own storage")
     ap.add_argument("--layers", type=int, default=32,
                     help="independent resident layers the steps rotate over (32 = the whole Llama3-8B stack)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)

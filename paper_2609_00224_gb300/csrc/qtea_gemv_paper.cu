@@ -8,11 +8,12 @@
 // paper's base-3 layout (five codes per byte, 26 bytes per 128 columns), and residual values in
 // fp16 or in the paper's FP8 E4M3.
 //
-// One warp per output row. Lane l takes the row's 128-column blocks l, l + 32, ...; a block lies in
-// one scale group (groups are 128 columns or the whole row), so the lane adds
-// alpha * sum T v x + beta * sum x once per block and batch row. Base-3 bytes are expanded to five
-// 2-bit codes through a 243-entry table in shared memory. v*x is exact in fp32; sums are fp32.
-// The same warp adds the residual of the row's group of four.
+// One warp per output row, walking the row's 128-column blocks; a block lies in one scale group
+// (groups are 128 columns or the whole row). Lane l takes code byte l of the block and adds
+// alpha * sum T v x + beta * sum x over its columns for every batch row; the lanes' sums are added
+// once at the end. Base-3 bytes are expanded to five 2-bit codes through a 243-entry table in shared
+// memory. v*x is exact in fp32; sums are fp32. The same warp adds the residual of the row's group
+// of four.
 #include <cuda_fp16.h>
 
 #include "qtea_internal.h"
@@ -39,35 +40,6 @@ __device__ __forceinline__ float e4m3_to_float(uint32_t b) {
   return (b & 0x80u) ? -mag : mag;
 }
 
-// Codes (T + 1, 2 bits each, lowest column first) of the 128-column block `blk` of row `row`:
-// 8 words. Columns at or beyond K hold code 1.
-__device__ __forceinline__ void block_codes(const PaperParams& p, int row, int blk, const uint16_t* lut,
-                                            uint32_t (&w)[8]) {
-  if (p.format == QTEA_FMT_2BIT) {
-    // rows are K_pad/4 bytes, K_pad a multiple of 64: the last block may have only 64 columns
-    const uint4* src = reinterpret_cast<const uint4*>(p.packed + (size_t)row * p.row_bytes + (size_t)blk * 32);
-    const uint4 a = __ldg(src);
-    const uint4 b = blk * 32 + 16 < p.row_bytes ? __ldg(src + 1) : make_uint4(0x55555555u, 0x55555555u, 0x55555555u,
-                                                                              0x55555555u);
-    w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
-    w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
-  } else {
-    // 26 bytes: byte q holds columns 5q .. 5q+4 as base-3 digits; byte 25 covers columns 125-127
-    const uint8_t* src = p.packed + (size_t)row * p.row_bytes + (size_t)blk * 26;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) w[i] = 0;
-#pragma unroll
-    for (int q = 0; q < 26; ++q) {
-      const uint32_t c5 = lut[min((uint32_t)__ldg(src + q), 242u)];  // five 2-bit codes (bytes are < 243)
-#pragma unroll
-      for (int d = 0; d < 5; ++d) {
-        const int col = 5 * q + d;
-        if (col < 128) w[col >> 4] |= ((c5 >> (2 * d)) & 3u) << (2 * (col & 15));
-      }
-    }
-  }
-}
-
 template <int MB>
 __global__ void __launch_bounds__(kPaperWarps * 32) qtea_gemv_paper_kernel(const PaperParams p) {
   __shared__ uint16_t lut[243];  // base-3 byte -> five 2-bit codes
@@ -89,26 +61,37 @@ __global__ void __launch_bounds__(kPaperWarps * 32) qtea_gemv_paper_kernel(const
 #pragma unroll
   for (int m = 0; m < MB; ++m) acc[m] = res[m] = 0.f;
 
+  // The row's 128-column blocks in order; within a block lane l takes code byte l (base-3: columns
+  // 5l .. 5l+4 for l < 26; 2-bit: columns 4l .. 4l+3), so the warp's loads of codes, x and v are
+  // contiguous. alpha and beta of the block's group are the same for every lane.
   const int n_blocks = (p.K + 127) / 128;
-  for (int blk = lane; blk < n_blocks; blk += 32) {
-    uint32_t w[8];
-    block_codes(p, o, blk, lut, w);
+  const uint8_t* row = p.packed + (size_t)o * p.row_bytes;
+  const bool b3 = p.format == QTEA_FMT_BASE3;
+  const int per = b3 ? 5 : 4, bytes = b3 ? 26 : 32;
+  const int lane_cols = per * lane;
+  const bool lane_in = lane < bytes;
+#pragma unroll 4
+  for (int blk = 0; blk < n_blocks; ++blk) {
     const int g = (blk * 128) / p.group_size;
     const uint16_t* sc = p.scales + ((size_t)o * p.G + g) * (p.bias ? 2 : 1);
     const float al = h2f(__ldg(sc)), be = p.bias ? h2f(__ldg(sc + 1)) : 0.f;
+    const int c0 = blk * 128 + lane_cols;
+    const bool on = lane_in && c0 < p.K && blk * bytes + lane < p.row_bytes;
+    const uint32_t byte = on ? (uint32_t)__ldg(row + (size_t)blk * bytes + lane) : 0x55u;
+    const uint32_t codes = b3 ? (uint32_t)lut[min(byte, 242u)] : byte;  // 2-bit codes, lowest column first
     float tvx[MB], sx[MB];
 #pragma unroll
     for (int m = 0; m < MB; ++m) tvx[m] = sx[m] = 0.f;
-    const int c0 = blk * 128;
-    for (int i = 0; i < 128; ++i) {
-      const int col = c0 + i;
-      if (col >= p.K) break;
-      const int t = (int)((w[i >> 4] >> (2 * (i & 15))) & 3u) - 1;
-      const float vj = h2f(__ldg(p.v + col));
+#pragma unroll
+    for (int d = 0; d < 5; ++d) {
+      const int col = c0 + d;
+      const bool cin = on && d < per && col < p.K && lane_cols + d < 128;
+      const int t = (int)((codes >> (2 * d)) & 3u) - 1;
+      const float vj = cin ? h2f(__ldg(p.v + col)) : 0.f;
 #pragma unroll
       for (int m = 0; m < MB; ++m) {
         if (m < M) {
-          const float xj = h2f(__ldg(p.x + (size_t)m * p.K + col));
+          const float xj = cin ? h2f(__ldg(p.x + (size_t)m * p.K + col)) : 0.f;
           sx[m] += xj;
           const float xv = vj * xj;  // exact in fp32
           tvx[m] += t > 0 ? xv : (t < 0 ? -xv : 0.f);
