@@ -525,15 +525,10 @@ def qtea_arm(args):
 
             def qstep(st):
                 L = qlayers[st % len(qlayers)]
-                if M == 1:
-                    qt.qtea_gemv_grouped([dict(x=xs[st % len(qlayers)][j], layout=g["layout"], row_scale=g["alpha"],
-                                               col_scale=g["v"], salient_idx=g["sal"], residual_vals=g["rv"],
-                                               residual_idx=g["ri"], y=ys[st % len(qlayers)][j])
-                                          for j, g in enumerate(L)], stream=stream)
-                else:
-                    for j, g in enumerate(L):
-                        qt.qtea_gemv(xs[st % len(qlayers)][j], g["layout"], g["alpha"], g["v"], g["sal"], g["rv"],
-                                     g["ri"], y=ys[st % len(qlayers)][j], stream=stream)
+                qt.qtea_gemv_grouped([dict(x=xs[st % len(qlayers)][j], layout=g["layout"], row_scale=g["alpha"],
+                                           col_scale=g["v"], salient_idx=g["sal"], residual_vals=g["rv"],
+                                           residual_idx=g["ri"], y=ys[st % len(qlayers)][j])
+                                      for j, g in enumerate(L)], stream=stream)
 
             def dstep(st):
                 for j in range(len(yd)):

@@ -39,6 +39,9 @@ void release(qtea_layout* l) {
   if (l->workspace) cudaFree(l->workspace);
   if (l->counters) cudaFree(l->counters);
   if (l->status) cudaFree(l->status);
+  if (l->mb_ws) cudaFree(l->mb_ws);
+  if (l->mb_part) cudaFree(l->mb_part);
+  if (l->mb_counters) cudaFree(l->mb_counters);
   delete l;
 }
 
@@ -68,15 +71,25 @@ int plan_m1(qtea_layout* l, const cudaDeviceProp& prop) {
   }
   l->smem_optin = dyn_max;
   {
-    // low batch: the same codes in boxes of 128 rows for the tensor-core kernel
-    cuuint32_t box_mb[2] = {(cuuint32_t)kChunkRowBytes, 128};
+    // low batch: the same descriptor (256-row boxes); v and x in fragment order per 512-column chunk,
+    // then x at the salient columns; partial rows and counters of split 256-row tiles
     size_t mb_dyn = 0;
-    l->mb_ok = encode(&l->tmap_mb, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, l->packed, dims, strides, box_mb, estr,
-                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS &&
-               mb_configure(prop.sharedMemPerBlockOptin, &mb_dyn) == cudaSuccess;
+    const int mb_tiles = (l->N + kMbTileRows - 1) / kMbTileRows;
+    const size_t ws = (size_t)l->n_chunks * kMbChunkWsBytes +
+                      (l->n_salient > 0 ? (size_t)mb_tiles * kMbResFloatsPerTile * sizeof(float) : 0);
+    const size_t ctr = (size_t)mb_tiles * kMbConsumerWarps * sizeof(unsigned);
+    l->mb_ok = mb_configure(prop.sharedMemPerBlockOptin, &mb_dyn) == cudaSuccess &&
+               mb_prep_configure(prop.sharedMemPerBlockOptin) == cudaSuccess;
+    l->prep_smem_optin = prop.sharedMemPerBlockOptin;
     if (!l->mb_ok) cudaGetLastError();
     l->mb_smem_optin = mb_dyn;
+    if (l->mb_ok) {
+      if (cudaMalloc(&l->mb_ws, ws) != cudaSuccess ||
+          cudaMalloc(&l->mb_part, (size_t)l->sm_count * kMbPartFloatsPerCta * sizeof(float)) != cudaSuccess ||
+          cudaMalloc(&l->mb_counters, ctr) != cudaSuccess)
+        return QTEA_ERR_ALLOC;
+      if (cudaMemset(l->mb_counters, 0, ctr) != cudaSuccess) return QTEA_ERR_CUDA;
+    }
   }
   if (cudaMalloc(&l->workspace, (size_t)l->sm_count * 2 * kTileRows * sizeof(float)) != cudaSuccess)
     return QTEA_ERR_ALLOC;
@@ -151,70 +164,128 @@ int launch_generic_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
   return launch_generic(p, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
 }
 
-// Low-batch (2 <= M <= 16) problem on the tensor-core kernel; returns QTEA_ERR_UNSUPPORTED when the
-// shapes or pointers do not allow it (the caller then uses the generic kernel).
-int launch_mb_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
+// Low-batch (2 <= M <= 16) problems on the tensor-core kernel, up to kMaxProblems per launch: one
+// prep launch writes v and x of every problem in fragment order into the layouts' workspaces, one
+// main launch streams the codes of all of them.
+struct MbGroup {
+  MbGroupParams gp;
+  MbPrepGroup pg;
+  TensorMaps maps;
+  int grid = 0;
+  size_t smem = 0;
+  size_t prep_smem_optin = 0;
+};
+
+void mb_group_reset(MbGroup& g, int M, size_t prep_smem_optin) {
+  std::memset(&g.gp, 0, sizeof(g.gp));
+  std::memset(&g.pg, 0, sizeof(g.pg));
+  std::memset(&g.maps, 0, sizeof(g.maps));
+  g.gp.M = M;
+  g.pg.M = M;
+  g.pg.mt = M <= 8 ? 1 : 2;
+  g.grid = 0;
+  g.smem = 0;
+  g.prep_smem_optin = prep_smem_optin;
+}
+
+bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
+  if (g.gp.n_problems == kMaxProblems) return false;
   const qtea_layout* l = q.packed_ternary;
-  if (!l->mb_ok || M < 2 || M > 16 || l->K % 8 != 0 || l->n_salient > kMaxSalientMb) return QTEA_ERR_UNSUPPORTED;
-  if (!aligned(q.x, 16) || !aligned(q.col_scale, 16)) return QTEA_ERR_UNSUPPORTED;
-  PFN_cuTensorMapEncodeTiled_v12000 encode = get_encode_tiled();
-  if (!encode) return QTEA_ERR_UNSUPPORTED;
-  MbMaps maps;
-  std::memcpy(&maps.codes, &l->tmap_mb, sizeof(CUtensorMap));
-  {
-    cuuint64_t dims[2] = {(cuuint64_t)l->K, (cuuint64_t)M};
-    cuuint64_t strides[1] = {(cuuint64_t)l->K * 2};
-    cuuint32_t box[2] = {64, 16};
-    cuuint32_t estr[2] = {1, 1};
-    if (encode(&maps.x, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint16_t*>(q.x), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return QTEA_ERR_UNSUPPORTED;
+  const int k = g.gp.n_problems;
+  const int n_tiles = (l->N + kMbTileRows - 1) / kMbTileRows;
+  float* yres = l->n_salient > 0 ? reinterpret_cast<float*>(l->mb_ws + (size_t)l->n_chunks * kMbChunkWsBytes) : nullptr;
+  MbPrepProblem& pp = g.pg.prob[k];
+  pp.x = q.x;
+  pp.v = q.col_scale;
+  pp.sal = q.salient_idx;
+  pp.rvals = q.residual_vals;
+  pp.ridx = q.residual_idx;
+  pp.ws = l->mb_ws;
+  pp.yres = yres;
+  pp.N = l->N;
+  pp.K = l->K;
+  pp.s = l->n_salient;
+  pp.n_chunks = l->n_chunks;
+  pp.n_tiles = n_tiles;
+  pp.native = l->n_salient > 0 && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 16) &&
+              mb_prep_smem_bytes(l->n_salient, true) <= g.prep_smem_optin;
+  const size_t need = mb_prep_smem_bytes(l->n_salient, pp.native != 0);
+  if (need > g.pg.smem) g.pg.smem = need;
+  pp.block_begin = g.pg.n_blocks;
+  MbProblemArgs& a = g.gp.prob[k];
+  a.alpha = q.row_scale;
+  a.ws = l->mb_ws;
+  a.yres = yres;
+  a.y = q.y;
+  a.part = l->mb_part;
+  a.counters = l->mb_counters;
+  a.N = l->N;
+  a.n_tiles = n_tiles;
+  a.n_chunks = l->n_chunks;
+  a.unit_begin = g.gp.total_units;
+  std::memcpy(&g.maps.m[k], &l->tmap, sizeof(CUtensorMap));
+  if (k == 0) g.gp.status = l->status;
+  g.gp.total_units += (long long)a.n_tiles * a.n_chunks;
+  g.pg.n_blocks += l->n_chunks + (l->n_salient > 0 ? n_tiles : 0);
+  g.gp.n_problems += 1;
+  g.pg.n_problems += 1;
+  return true;
+}
+
+// Grid, ring depth and shared memory of the group; false if the ring does not fit or the group
+// needs more CTAs than every layout's partial-row slots serve.
+bool mb_group_plan(MbGroup& g, int sm_count, size_t smem_optin) {
+  if (g.gp.n_problems == 0) return false;
+  if (g.gp.total_units >= (1ll << 30)) return false;
+  g.grid = (int)(g.gp.total_units < sm_count ? g.gp.total_units : sm_count);
+  if (g.grid > kMaxGrid) g.grid = kMaxGrid;
+  for (int b = 0; b <= g.grid; ++b) g.gp.cta_u0[b] = (int)unit_begin_of(b, g.gp.total_units, g.grid);
+  for (int S = kMaxStagesMb; S >= kMinStagesMb; --S) {
+    if (mb_smem_bytes(S, g.gp.M) <= smem_optin) {
+      g.gp.n_stages = S;
+      g.smem = mb_smem_bytes(S, g.gp.M);
+      return true;
+    }
   }
-  {
-    cuuint64_t dims[2] = {(cuuint64_t)l->K, 1};
-    cuuint64_t strides[1] = {(cuuint64_t)l->K * 2};
-    cuuint32_t box[2] = {256, 1};
-    cuuint32_t estr[2] = {1, 1};
-    if (encode(&maps.v, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint16_t*>(q.col_scale), dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return QTEA_ERR_UNSUPPORTED;
+  return false;
+}
+
+int mb_group_launch(MbGroup& g, cudaStream_t st) {
+  if (launch_mb_prep(g.pg, st) != cudaSuccess) return QTEA_ERR_CUDA;
+  return launch_mb(g.maps, g.gp, g.grid, g.smem, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+}
+
+bool mb_capable(const qtea_layout* l, int M) { return l->mb_ok && l->m1_ok && M >= 2 && M <= 16; }
+
+// Low-batch dispatch: as many consecutive problems per launch as fit; a problem the kernel cannot
+// serve goes to the generic kernel.
+int run_mb(const qtea_gemv_problem* qs, const int* idx, int n, int M, cudaStream_t st) {
+  int i = 0;
+  while (i < n) {
+    const qtea_layout* l0 = qs[idx[i]].packed_ternary;
+    MbGroup g;
+    mb_group_reset(g, M, l0->prep_smem_optin);
+    int taken = 0;
+    while (i + taken < n) {
+      const qtea_layout* li = qs[idx[i + taken]].packed_ternary;
+      if (li->sm_count != l0->sm_count) break;  // partial-row slots are sized by the SM count
+      MbGroup trial = g;
+      if (!mb_group_add(trial, qs[idx[i + taken]])) break;
+      if (!mb_group_plan(trial, l0->sm_count, l0->mb_smem_optin)) break;
+      g = trial;
+      ++taken;
+    }
+    if (taken == 0) {
+      int rc = launch_generic_problem(qs[idx[i]], M, st);
+      if (rc) return rc;
+      ++i;
+      continue;
+    }
+    int rc = mb_group_launch(g, st);
+    if (rc) return rc;
+    i += taken;
   }
-  MbParams p;
-  p.x = q.x;
-  p.alpha = q.row_scale;
-  p.sal = q.salient_idx;
-  p.rvals = q.residual_vals;
-  p.ridx = q.residual_idx;
-  p.y = q.y;
-  p.status = l->status;
-  p.N = l->N;
-  p.K = l->K;
-  p.M = M;
-  p.s = l->n_salient;
-  p.s_pad = round_up(l->n_salient, 16) + 8;
-  p.n_tiles = (l->N + 127) / 128;
-  p.n_chunks = l->n_chunks;
-  p.vec_res = (l->n_salient % 8 == 0) && aligned(q.residual_vals, 16);
-  // clusters of C CTAs split a tile's chunks when there are fewer tiles than SMs
-  int C = l->sm_count / p.n_tiles;
-  if (C > 8) C = 8;
-  if (C > p.n_chunks) C = p.n_chunks;
-  if (C < 1) C = 1;
-  int S = kMaxStagesMb;
-  for (;;) {
-    while (S >= kMinStagesMb && mb_smem_bytes(S, p.s_pad, C, M) > l->mb_smem_optin) --S;
-    if (S >= kMinStagesMb || C == 1) break;
-    --C;
-    S = kMaxStagesMb;
-  }
-  if (S < kMinStagesMb) return QTEA_ERR_UNSUPPORTED;
-  p.n_stages = S;
-  p.cluster = C;
-  int n_cl = l->sm_count / C;
-  if (n_cl > p.n_tiles) n_cl = p.n_tiles;
-  return launch_mb(maps, p, n_cl * C, mb_smem_bytes(S, p.s_pad, C, M), st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+  return QTEA_OK;
 }
 
 // Batch-1 kernel over a group of problems whose layouts all have m1 resources.
@@ -458,9 +529,10 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
       if (problems[j].packed_ternary == problems[i].packed_ternary) return QTEA_ERR_INVALID_ARG;
   }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  int* m1_idx = n_problems > 0 ? static_cast<int*>(std::malloc(sizeof(int) * (size_t)n_problems)) : nullptr;
+  int* m1_idx = n_problems > 0 ? static_cast<int*>(std::malloc(sizeof(int) * 2 * (size_t)n_problems)) : nullptr;
   if (n_problems > 0 && !m1_idx) return QTEA_ERR_ALLOC;
-  int n_m1 = 0, rc = QTEA_OK;
+  int* mb_idx = m1_idx + n_problems;
+  int n_m1 = 0, n_mb = 0, rc = QTEA_OK;
   for (int i = 0; i < n_problems && rc == QTEA_OK; ++i) {
     const qtea_gemv_problem& q = problems[i];
     const qtea_layout* l = q.packed_ternary;
@@ -473,12 +545,14 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
       rc = launch_paper_problem(q, M, st);
     } else if (M == 1 && l->m1_ok) {
       m1_idx[n_m1++] = i;
+    } else if (mb_capable(l, M)) {
+      mb_idx[n_mb++] = i;
     } else {
-      rc = launch_mb_problem(q, M, st);
-      if (rc == QTEA_ERR_UNSUPPORTED) rc = launch_generic_problem(q, M, st);
+      rc = launch_generic_problem(q, M, st);
     }
   }
   if (rc == QTEA_OK && n_m1 > 0) rc = run_m1(problems, m1_idx, n_m1, st);
+  if (rc == QTEA_OK && n_mb > 0) rc = run_mb(problems, mb_idx, n_mb, M, st);
   std::free(m1_idx);
   if (rc != QTEA_OK) cudaGetLastError();
   return rc;

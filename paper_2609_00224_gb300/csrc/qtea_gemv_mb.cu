@@ -4,26 +4,32 @@
 // Computes Eq. 10 (one alpha per row, beta = 0) plus Eq. 11 of the QTEA paper (Sec. 3.5) for a
 // batch of M activation rows. With M rows the product is a skinny dense contraction, so it runs
 // on mma.sync m16n8k16 (fp16 operands, fp32 accumulation), exactly:
-//  * A = T * v: the ternary code times the column rescale of Sec. 3.3. T is -1, 0 or +1 and v an
-//    fp16 value, so every element of A is an fp16 value, formed in registers from the 2-bit codes
-//    (byte permute, a multiply that spreads the byte, the 0x6400 magic exponent, two fp16 fix-ups
-//    and a multiply by v).
-//  * B = x, the fp16 activations, unchanged; each product A * B is exact in fp32 and the sums
-//    accumulate in fp32.
+//  * A = 2T * v. A 32-bit code word holds the codes c = T + 1 of 16 consecutive columns; shifting
+//    it left by 14 - 2i puts the codes of columns i and i + 8 at bits 14-15 and 30-31, and one
+//    LOP3 (~w & 0xC000C000) turns each into the fp16 value -2, -0 or +2 (sign bit and the top
+//    exponent bit). One multiply by the pair (v_i, v_{i+8}) gives 2T * v exactly (a power-of-two
+//    multiple of an fp16 value). The accumulator is halved once at the end.
+//  * B = x, the fp16 activations, unchanged; each product is exact in fp32 and the sums
+//    accumulate in fp32. The contraction index runs over the columns in the order that pairing
+//    gives (columns i and i + 8 of a word side by side), so a prep kernel writes, once per call and
+//    512-column chunk, v and x in exactly the register order the fragments need ("fragment
+//    order"): one 8-byte shared load per thread and step.
 //  * The residual of Eq. 11 is an exact contraction too: over "virtual columns", one per
 //    salient column, A holds the fp16 residual value of the row's group where the stored
-//    position is the row and 0 elsewhere, and B holds x at the salient column. It is accumulated
-//    apart, since alpha does not scale it.
-// Work: a unit is a 128-row tile. A cluster of C CTAs (C chosen so that tiles x C fills the GPU)
-// shares a tile: CTA rank r takes chunks [r n/C, (r+1) n/C) and residual steps r, r + C, ...; the
-// ranks' partial rows go through distributed shared memory into rank 0, which adds them in rank
-// order (no partial sums in global memory, a fixed summation order). Eight consumer warps each
-// own 16 rows of the tile; a producer lane streams the CTA's 512-column chunks through a ring of
-// shared-memory stages by TMA: 128 rows x 128 bytes of codes (128-byte swizzle), the 16 x 512 block of x
-// (128-byte swizzle, rows beyond M read as zero) and 512 values of v. x at the salient columns is
-// gathered once per CTA. The k order inside each 16-column step is permuted so that a thread's
-// four k slots are four consecutive columns, i.e. one byte of codes.
-// Every wait on an mbarrier is bounded (~2 s, then QTEA_ERR_TIMEOUT in the status word).
+//    position is the row and 0 elsewhere, and B holds x at the salient column. The prep kernel
+//    computes it per 256-row tile (its loads are scattered and would stall the decode) and the
+//    main kernel adds it, unscaled by alpha, at the tile's end.
+// Work: a unit is 256 rows x 512 columns of one problem; the units of every problem of a group
+// form one sequence that is split evenly over persistent CTAs (one launch for all the GEMVs of a
+// group). Each of eight consumer warps owns two 16-row blocks of a unit, so every B fragment it
+// loads feeds two MMAs; two accumulator sets alternate between steps so that consecutive MMAs do
+// not wait on each other. A tile whose units span several
+// CTAs is finished by the last of them (per warp, counted with an acq_rel atomic): it adds the
+// partial rows in CTA order, so results do not depend on timing. A producer lane streams the
+// CTA's units through a ring of shared-memory stages: 256 rows x 128 bytes of codes by TMA
+// (128-byte swizzle) and the chunk's v and x in fragment order by bulk copy.
+// |v| must stay below 32768 (2v is formed in fp16). Every wait on an mbarrier is bounded (~2 s,
+// then QTEA_ERR_TIMEOUT in the status word).
 #include <cuda_fp16.h>
 
 #include "qtea_internal.h"
@@ -32,14 +38,8 @@ namespace qtea {
 namespace {
 
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
-constexpr int kMbConsumerWarps = 8;
 constexpr int kMbThreads = (kMbConsumerWarps + 1) * 32;
-constexpr int kMbTileRows = 128;
-constexpr int kMbCodeBytes = kMbTileRows * kChunkRowBytes;  // 16384
-constexpr int kMbXBoxCols = 64;                              // 128-byte rows of fp16
-constexpr int kMbXBytes = 16 * kChunkCols * 2;               // 16384: 8 boxes of 16 x 64
-constexpr int kMbVBytes = kChunkCols * 2;                    // 1024
-constexpr int kMbStageBytes = 34816;                         // codes, x, v, rounded to 1024
+constexpr int kMbCodeBytes = kMbTileRows * kChunkRowBytes;  // 32768
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -94,6 +94,13 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       : "memory");
 }
 
+// 1-D bulk copy of `bytes` (a multiple of 16, both addresses 16-byte aligned) into shared memory.
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
 __device__ __forceinline__ void mma_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
                                           uint32_t b0, uint32_t b1) {
   asm volatile(
@@ -105,352 +112,536 @@ __device__ __forceinline__ void mma_16816(float (&c)[4], uint32_t a0, uint32_t a
 __device__ __forceinline__ uint32_t h2_as_u32(__half2 h) { return *reinterpret_cast<uint32_t*>(&h); }
 __device__ __forceinline__ __half2 u32_as_h2(uint32_t u) { return *reinterpret_cast<__half2*>(&u); }
 
-// The four codes of byte q of a code word as two fp16 pairs of T * v (columns 4q, 4q+1 and
-// 4q+2, 4q+3 of the 16-column step): a code c = T + 1 is placed in the mantissa of 1024
-// (0x6400), 1025 is subtracted (c in bits 0-1) or the value is scaled by 1/16 and 65 subtracted
-// (c in bits 4-5), and the result, exactly -1, 0 or 1, multiplies v.
-__device__ __forceinline__ void decode_byte(uint32_t word, uint32_t q, uint32_t v01, uint32_t v23, uint32_t& a01,
-                                            uint32_t& a23) {
-  const uint32_t b = __byte_perm(word, 0u, 0x4440u | q);  // byte q alone
-  const uint32_t s = b * 0x4001u;                           // b in bits 0-7 and 14-21
-  const uint32_t w01 = (s & 0x00030003u) | 0x64006400u;     // 1024 + c0 | 1024 + c1
-  const uint32_t w23 = (s & 0x00300030u) | 0x64006400u;     // 1024 + 16 c2 | 1024 + 16 c3
-  const __half2 t01 = __hsub2(u32_as_h2(w01), __float2half2_rn(1025.f));
-  const __half2 t23 = __hfma2(u32_as_h2(w23), __float2half2_rn(0.0625f), __float2half2_rn(-65.f));
-  a01 = h2_as_u32(__hmul2(t01, u32_as_h2(v01)));
-  a23 = h2_as_u32(__hmul2(t23, u32_as_h2(v23)));
+// Codes of columns I and I + 8 of word w as fp16 -2, -0 or +2 (2T), times the pair of v.
+template <int I>
+__device__ __forceinline__ uint32_t a_reg(uint32_t w, uint32_t vpair) {
+  const uint32_t t2 = ~(w << (14 - 2 * I)) & 0xC000C000u;
+  return h2_as_u32(__hmul2(u32_as_h2(t2), u32_as_h2(vpair)));
 }
 
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
+__device__ __forceinline__ float h2f(uint16_t b) { return __half2float(__ushort_as_half(b)); }
+
+// CTA whose range contains unit u (the inverse of the balanced split cta_u0[b] = b * total / grid).
+__device__ __forceinline__ int unit_owner(long long u, long long total, int grid) {
+  return (int)(((u + 1) * grid - 1) / total);
 }
 
-__device__ __forceinline__ uint32_t cluster_id() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
-  return r;
+struct UnitPos {
+  int p, t, ch;  // problem, tile, chunk
+};
+
+__device__ __forceinline__ UnitPos unit_pos(const MbProblemArgs* tab, int n_problems, long long u) {
+  int p = 0;
+  while (p + 1 < n_problems && u >= tab[p + 1].unit_begin) ++p;
+  const int v = (int)(u - tab[p].unit_begin);
+  const int nc = tab[p].n_chunks;
+  const int t = v / nc;
+  return {p, t, v - t * nc};
 }
 
-__device__ __forceinline__ uint32_t n_clusters() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
-  return r;
+// ---------------------------------------------------------------- prep kernel
+
+// Residual (Eq. 11) of one 16-entry step for a consumer thread's rows: the values whose stored
+// position is the row (fp16 lanes all-ones or zero) as A, x at the salient columns as B. Entries
+// e0 .. e0 + 3 (e0 = 16 step + 4q) of the row groups of rows r, r + 8 of block b (r = tr + 16b + g)
+// come from the staged tile: rv [64 groups][rvs] fp16, ri [64][ris] position bytes (entry e of a
+// group in bits 2(e % 4) of byte e / 4), xr [16 batch rows][xrs] fp16 (zero past the valid
+// entries); only entries below ne count.
+__device__ __forceinline__ void res_step(const uint16_t* rv, int rvs, const uint8_t* ri, int ris, const uint16_t* xr,
+                                         int xrs, int ne, int step, int tr, int g, int q, int mt, bool quad_loads,
+                                         float (&res)[kMbBlocks][2][4]) {
+  const int e0 = step * 16 + 4 * q;
+  const uint32_t pos = (uint32_t)(g & 3);  // row & 3 for every row of the thread
+  uint2 xb[2];
+#pragma unroll
+  for (int j = 0; j < 2; ++j) xb[j] = *reinterpret_cast<const uint2*>(xr + (8 * j + g) * xrs + e0);
+#pragma unroll
+  for (int b = 0; b < kMbBlocks; ++b) {
+    uint32_t a[4];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int gl = (tr + 16 * b + 8 * h + g) >> 2;
+      // match bits: field k of d is zero where entry e0 + k is stored at this row's position;
+      // nz holds bit 2k set where it is not
+      const uint32_t d = (uint32_t)ri[gl * ris + (e0 >> 2)] ^ (pos * 0x55u);
+      const uint32_t nz = (d | (d >> 1)) & 0x55u;
+      uint32_t lo, hi;
+      if (quad_loads) {  // the four values in one 8-byte load (rvs % 4 == 0, e0 + 3 < ne or zero)
+        uint2 v = make_uint2(0, 0);
+        if (e0 < ne) v = *reinterpret_cast<const uint2*>(rv + gl * rvs + e0);
+        lo = v.x;
+        hi = v.y;
+      } else {
+        uint32_t v4[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) v4[k] = e0 + k < ne ? (uint32_t)rv[gl * rvs + e0 + k] : 0u;
+        lo = v4[0] | (v4[1] << 16);
+        hi = v4[2] | (v4[3] << 16);
+      }
+      // keep a 16-bit lane where its match bit is clear: (bit - 1) is all ones exactly then
+      const uint32_t k0 = ((nz & 1u) - 1u) & 0x0000ffffu, k1 = (((nz >> 2) & 1u) - 1u) & 0xffff0000u;
+      const uint32_t k2 = (((nz >> 4) & 1u) - 1u) & 0x0000ffffu, k3 = (((nz >> 6) & 1u) - 1u) & 0xffff0000u;
+      a[h] = lo & (k0 | k1);
+      a[2 + h] = hi & (k2 | k3);
+    }
+    mma_16816(res[b][0], a[0], a[1], a[2], a[3], xb[0].x, xb[0].y);
+    if (mt == 2) mma_16816(res[b][1], a[0], a[1], a[2], a[3], xb[1].x, xb[1].y);
+  }
 }
 
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+// Blocks of a problem: its chunks, then (with salient columns) its 256-row tiles.
+// Chunk ch's 512 columns: entry (step s, quad lane q) of the v block holds the pairs
+// (v[16W + i], v[16W + i + 8]) for i = 2(s & 3) and i + 1, W = 8q + (s >> 2); entry (step s,
+// lane 4g + q) of x block j holds the same two pairs of x[8j + g]. Columns >= K and batch rows >= M
+// are zero.
+// Tile t: the residual of its 256 rows for every batch row, computed with the main kernel's thread
+// mapping (thread tid holds rows tr + 16b + g and + 8, batch rows 8j + 2q and + 1) and stored in
+// that order, so that each main-kernel thread reads its part with vector loads. The tile's values
+// and position bytes are one contiguous range each, starting on a 16-byte boundary (64 groups x s
+// x 2 bytes and 64 groups x ceil(s/4) bytes before it); with `native` they are copied as they are
+// by 16-byte loads, otherwise (too large for shared memory, or not 16-byte aligned) in passes of
+// kMbResEntries entries by 2-byte loads.
+__global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant__ MbPrepGroup gr) {
+  static_assert(kMbConsumerWarps * 32 == 256, "the prep kernel's residual blocks mirror the consumers");
+  extern __shared__ __align__(16) uint8_t sm[];
+  // the main kernel may launch now and prefetch its codes; it reads this kernel's output only after
+  // its own grid dependency wait, which waits for this grid to complete
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  int pi = 0;
+  while (pi + 1 < gr.n_problems && (int)blockIdx.x >= gr.prob[pi + 1].block_begin) ++pi;
+  // the problem's fields in registers, read once (field-by-field reads from the parameter space
+  // with a dynamic index would each be a constant-cache miss)
+  const MbPrepProblem p = gr.prob[pi];
+  const int M = gr.M;
+  const int local = (int)blockIdx.x - p.block_begin;
+  const int tid = threadIdx.x;
+  if (local >= p.n_chunks) {
+    // ---- residual of tile t
+    const int t = local - p.n_chunks;
+    const int g0 = t * (kMbTileRows / 4), ng = min(kMbTileRows / 4, p.N / 4 - g0);
+    const int rs = (p.s + 3) >> 2;
+    const int warp = tid >> 5, lane = tid & 31, g = lane >> 2, q = lane & 3;
+    const int tr = warp * 16 * kMbBlocks;
+    float res[kMbBlocks][2][4];
+#pragma unroll
+    for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+#pragma unroll
+        for (int k = 0; k < 4; ++k) res[b][j][k] = 0.f;
+    const int E = p.native ? p.s : kMbResEntries;       // entries per pass
+    const int xrs = (E + 15) & ~15;                       // staged x row stride
+    const int ris = p.native ? rs : kMbResEntries / 4;  // staged position-byte row stride
+    uint16_t* rv = reinterpret_cast<uint16_t*>(sm);
+    uint8_t* ri = sm + (((size_t)64 * E * 2 + 15) & ~(size_t)15);
+    uint16_t* xr = reinterpret_cast<uint16_t*>(ri + (((size_t)64 * ris + 15) & ~(size_t)15));
+    for (int e_base = 0; e_base < p.s; e_base += E) {
+      const int ne = min(E, p.s - e_base);
+      if (p.native) {
+        // whole 16-byte vectors by vector loads (all in flight at once), the tails by 2-byte and
+        // 1-byte loads: no load past the caller's arrays
+        const uint4* src = reinterpret_cast<const uint4*>(p.rvals + (size_t)g0 * p.s);
+        uint4* dst = reinterpret_cast<uint4*>(rv);
+        const int nv = (ng * p.s) >> 3;
+#pragma unroll 16
+        for (int i = tid; i < nv; i += 256) dst[i] = __ldg(src + i);
+        for (int i = 8 * nv + tid; i < ng * p.s; i += 256) rv[i] = __ldg(p.rvals + (size_t)g0 * p.s + i);
+        const uint4* srci = reinterpret_cast<const uint4*>(p.ridx + (size_t)g0 * rs);
+        uint4* dsti = reinterpret_cast<uint4*>(ri);
+        const int nvi = (ng * rs) >> 4;
+#pragma unroll 4
+        for (int i = tid; i < nvi; i += 256) dsti[i] = __ldg(srci + i);
+        for (int i = 16 * nvi + tid; i < ng * rs; i += 256) ri[i] = __ldg(p.ridx + (size_t)g0 * rs + i);
+      } else {
+#pragma unroll 8
+        for (int i = tid; i < 64 * kMbResEntries; i += 256) {
+          const int gg = i / kMbResEntries, e = i % kMbResEntries;
+          rv[i] = (gg < ng && e < ne) ? __ldg(p.rvals + (size_t)(g0 + gg) * p.s + e_base + e) : (uint16_t)0;
+        }
+#pragma unroll 8
+        for (int i = tid; i < 64 * (kMbResEntries / 4); i += 256) {
+          const int gg = i / (kMbResEntries / 4), e4 = i % (kMbResEntries / 4);
+          ri[i] = (gg < ng && 4 * e4 < ne) ? __ldg(p.ridx + (size_t)(g0 + gg) * rs + (e_base >> 2) + e4) : (uint8_t)0;
+        }
+      }
+      // x at the pass's salient columns (zero past ne): up to four entries per thread, their
+      // column indices first, then all their x loads at once
+      for (int e_lo = 0; e_lo < xrs; e_lo += 1024) {
+        int col[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int e = e_lo + tid + 256 * k;
+          col[k] = e < ne ? __ldg(p.sal + e_base + e) : 0;
+          col[k] = col[k] < 0 ? 0 : (col[k] >= p.K ? p.K - 1 : col[k]);
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int e = e_lo + tid + 256 * k;
+          if (e >= xrs) break;
+          uint16_t xv[16];
+#pragma unroll
+          for (int m = 0; m < 16; ++m) xv[m] = (m < M && e < ne) ? __ldg(p.x + (size_t)m * p.K + col[k]) : (uint16_t)0;
+#pragma unroll
+          for (int m = 0; m < 16; ++m) xr[m * xrs + e] = xv[m];
+        }
+      }
+      __syncthreads();
+      // groups past ng are never read: their rows lie past N, which the main kernel does not write
+      const int rvs = p.native ? p.s : kMbResEntries;
+      // 8-byte value loads where a row's entries start on 8-byte boundaries and the last quad is
+      // whole (staged rows in passes are padded with zeros)
+      const bool quad = (rvs & 3) == 0 && (p.native ? (ne & 3) == 0 : true);
+      if (quad) {
+        for (int step = 0; step * 16 < ne; ++step) res_step(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, true, res);
+      } else {
+        for (int step = 0; step * 16 < ne; ++step) res_step(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, false, res);
+      }
+      __syncthreads();
+    }
+    float4* dst = reinterpret_cast<float4*>(p.yres + ((size_t)t * 256 + tid) * 4 * kMbBlocks * gr.mt);
+#pragma unroll
+    for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+      for (int j = 0; j < 2; ++j)
+        if (j < gr.mt) dst[b * gr.mt + j] = make_float4(res[b][j][0], res[b][j][1], res[b][j][2], res[b][j][3]);
+    return;
+  }
+  // ---- v and x of chunk ch in fragment order
+  uint16_t(*xsm)[kChunkCols] = reinterpret_cast<uint16_t(*)[kChunkCols]>(sm);
+  uint16_t* vsm = reinterpret_cast<uint16_t*>(sm + 16 * kChunkCols * 2);
+  const int ch = local, col0 = ch * kChunkCols;
+#pragma unroll 2
+  for (int i = tid; i < kChunkCols; i += 256) {
+    const int col = col0 + i;
+    const bool in = col < p.K;
+    vsm[i] = in ? __ldg(p.v + col) : (uint16_t)0;
+    uint16_t xv[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) xv[m] = (in && m < M) ? __ldg(p.x + (size_t)m * p.K + col) : (uint16_t)0;
+#pragma unroll
+    for (int m = 0; m < 16; ++m) xsm[m][i] = xv[m];
+  }
+  __syncthreads();
+  uint8_t* out = p.ws + (size_t)ch * kMbChunkWsBytes;
+  auto pair = [](const uint16_t* row, int c) { return (uint32_t)row[c] | ((uint32_t)row[c + 8] << 16); };
+  if (tid < 128) {
+    const int s = tid >> 2, q = tid & 3;
+    const int base = 16 * (8 * q + (s >> 2)), i0 = 2 * (s & 3);
+    reinterpret_cast<uint2*>(out)[tid] = make_uint2(pair(vsm, base + i0), pair(vsm, base + i0 + 1));
+  }
+  for (int e = tid; e < gr.mt * 1024; e += 256) {
+    const int j = e >> 10, s = (e >> 5) & 31, lane = e & 31, g = lane >> 2, q = lane & 3;
+    const int base = 16 * (8 * q + (s >> 2)), i0 = 2 * (s & 3);
+    const uint16_t* row = xsm[8 * j + g];
+    reinterpret_cast<uint2*>(out + kMbVBytes)[e] = make_uint2(pair(row, base + i0), pair(row, base + i0 + 1));
+  }
 }
 
-// Address of the same shared-memory location in CTA `rank` of the cluster.
-__device__ __forceinline__ uint32_t map_rank(uint32_t addr, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
-  return r;
-}
+// ---------------------------------------------------------------- decode of one unit
 
-__device__ __forceinline__ void st_cluster_v4(uint32_t addr, float a, float b, float c, float d) {
-  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
-               : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t remote_bar) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote_bar) : "memory");
-}
-
-// Wait for a phase completed by arrivals from other CTAs of the cluster (acquire at cluster scope).
-__device__ __forceinline__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, int* status) {
-  const unsigned long long t0 = global_ns();
-  for (;;) {
-    uint32_t ok;
-    asm volatile(
-        "{ .reg .pred p; mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2; selp.u32 %0, 1, 0, p; }"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    if (ok) return true;
-    if (global_ns() - t0 > kWaitLimitNs) {
-      atomicExch(status, (int)QTEA_ERR_TIMEOUT);
-      return false;
+// The unit's 32 steps of 16 columns for the warp's 16-row blocks (rows tr + 16b + g and + 8 of the
+// stage); even steps accumulate into acc[0], odd steps into acc[1].
+template <int MT>
+__device__ __forceinline__ void decode_unit(const uint8_t* sb, int tr, int g, int q, int lane,
+                                            float (&acc)[2][kMbBlocks][MT][4]) {
+  const uint8_t* vblk = sb + kMbCodeBytes;
+  const uint8_t* xblk = vblk + kMbVBytes;
+  // the thread's 32 code bytes (8 words) of each of its four rows (128-byte swizzle)
+  uint32_t wr[kMbBlocks][2][8];
+#pragma unroll
+  for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const uint8_t* rp = sb + (size_t)(tr + 16 * b + 8 * h + g) * kChunkRowBytes;
+      const uint4 u0 = *reinterpret_cast<const uint4*>(rp + (((2 * q) ^ g) << 4));
+      const uint4 u1 = *reinterpret_cast<const uint4*>(rp + (((2 * q + 1) ^ g) << 4));
+      wr[b][h][0] = u0.x; wr[b][h][1] = u0.y; wr[b][h][2] = u0.z; wr[b][h][3] = u0.w;
+      wr[b][h][4] = u1.x; wr[b][h][5] = u1.y; wr[b][h][6] = u1.z; wr[b][h][7] = u1.w;
+    }
+#pragma unroll
+  for (int w = 0; w < 8; ++w) {
+#pragma unroll
+    for (int tq = 0; tq < 4; ++tq) {
+      const int s = 4 * w + tq;
+      const uint2 vp = *reinterpret_cast<const uint2*>(vblk + (s * 4 + q) * 8);
+      // k slots 2q, 2q+1: columns i, i + 8 with i = 2tq; slots 2q+8, 2q+9: i = 2tq + 1
+      uint32_t a[kMbBlocks][4];
+#pragma unroll
+      for (int b = 0; b < kMbBlocks; ++b) {
+        if (tq == 0) {
+          a[b][0] = a_reg<0>(wr[b][0][w], vp.x); a[b][1] = a_reg<0>(wr[b][1][w], vp.x);
+          a[b][2] = a_reg<1>(wr[b][0][w], vp.y); a[b][3] = a_reg<1>(wr[b][1][w], vp.y);
+        } else if (tq == 1) {
+          a[b][0] = a_reg<2>(wr[b][0][w], vp.x); a[b][1] = a_reg<2>(wr[b][1][w], vp.x);
+          a[b][2] = a_reg<3>(wr[b][0][w], vp.y); a[b][3] = a_reg<3>(wr[b][1][w], vp.y);
+        } else if (tq == 2) {
+          a[b][0] = a_reg<4>(wr[b][0][w], vp.x); a[b][1] = a_reg<4>(wr[b][1][w], vp.x);
+          a[b][2] = a_reg<5>(wr[b][0][w], vp.y); a[b][3] = a_reg<5>(wr[b][1][w], vp.y);
+        } else {
+          a[b][0] = a_reg<6>(wr[b][0][w], vp.x); a[b][1] = a_reg<6>(wr[b][1][w], vp.x);
+          a[b][2] = a_reg<7>(wr[b][0][w], vp.y); a[b][3] = a_reg<7>(wr[b][1][w], vp.y);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < MT; ++j) {
+        const uint2 bx = *reinterpret_cast<const uint2*>(xblk + j * kMbXTileBytes + (s * 32 + lane) * 8);
+#pragma unroll
+        for (int b = 0; b < kMbBlocks; ++b) mma_16816(acc[s & 1][b][j], a[b][0], a[b][1], a[b][2], a[b][3], bx.x, bx.y);
+      }
     }
   }
 }
 
-// Shared memory of the kernel: S stages, x at the salient columns [16][s_pad] fp16, the rank-0
-// CTA's slots for the other ranks' partial rows [C-1][256 threads][4 MT] floats, and barriers.
-struct MbSmem {
-  uint8_t* stages;
-  __half* xs;
-  float* slots;
-  uint64_t* full;          // [S] stage landed
-  uint64_t* empty;         // [S] consumers released the stage
-  uint64_t* red_full;      // rank 0: every other rank wrote its partial rows of the tile
-  uint64_t* red_empty;     // other ranks: rank 0 has read this rank's partial rows
-  int* last_fill;          // [kMaxStagesMb]
-};
+// ---------------------------------------------------------------- main kernel
 
 template <int MT>  // n8 tiles of the batch: 1 for M <= 8, 2 for M <= 16
 __global__ void __launch_bounds__(kMbThreads, 1)
-    qtea_gemv_mb_kernel(const __grid_constant__ MbMaps maps, const __grid_constant__ MbParams p) {
+    qtea_gemv_mb_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ MbGroupParams gp) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  constexpr int kStage = mb_stage_bytes(MT);
+  constexpr uint32_t kFill = kMbCodeBytes + kMbVBytes + MT * kMbXTileBytes;
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int S = p.n_stages;
-  const int C = p.cluster;                 // CTAs of a cluster share a tile, each a range of chunks
-  const int rank = (int)cluster_rank();
-  MbSmem sm;
-  sm.stages = smem;
-  sm.xs = reinterpret_cast<__half*>(smem + (size_t)S * kMbStageBytes);
-  sm.slots = reinterpret_cast<float*>(smem + (size_t)S * kMbStageBytes + (size_t)16 * p.s_pad * 2);
-  sm.full = reinterpret_cast<uint64_t*>(sm.slots + (size_t)(C - 1) * kMbConsumerWarps * 32 * 4 * MT);
-  sm.empty = sm.full + S;
-  sm.red_full = sm.empty + S;
-  sm.red_empty = sm.red_full + 1;
-  sm.last_fill = reinterpret_cast<int*>(sm.red_empty + 1);
+  const int S = gp.n_stages;
+  const int NP = gp.n_problems;
+  const int u0 = gp.cta_u0[blockIdx.x], u1 = gp.cta_u0[blockIdx.x + 1];
+  const int n_units = u1 - u0;
+  uint8_t* stages = smem;
+  MbProblemArgs* tab = reinterpret_cast<MbProblemArgs*>(smem + (size_t)S * kStage);
+  uint64_t* full = reinterpret_cast<uint64_t*>(tab + kMaxProblems);  // [S] stage landed
+  uint64_t* empty = full + S;                                         // [S] consumers released it
+  int* last_fill = reinterpret_cast<int*>(empty + S);                 // [S] fills issued per stage
 
-  // tiles of this cluster: cluster_id, + n_clusters, ...; chunks of this CTA: [c0, c1)
-  const int cid = (int)cluster_id(), ncl = (int)n_clusters();
-  const int n_my_tiles = p.n_tiles > cid ? (p.n_tiles - 1 - cid) / ncl + 1 : 0;
-  const int c0 = rank * p.n_chunks / C, c1 = (rank + 1) * p.n_chunks / C;
-  const int my_chunks = c1 - c0;
-  const int n_fills = n_my_tiles * my_chunks;
-
+  // the problem table goes to shared memory in one step (every thread one word)
+  {
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(gp.prob);
+    uint32_t* dst = reinterpret_cast<uint32_t*>(tab);
+    const int words = NP * (int)(sizeof(MbProblemArgs) / 4);
+    for (int i = threadIdx.x; i < words; i += kMbThreads) dst[i] = src[i];
+  }
   if (threadIdx.x == 0) {
     for (int i = 0; i < S; ++i) {
-      mbar_init(smem_u32(&sm.full[i]), 1);
-      mbar_init(smem_u32(&sm.empty[i]), kMbConsumerWarps);
-      sm.last_fill[i] = 0;
+      mbar_init(smem_u32(&full[i]), 1);
+      mbar_init(smem_u32(&empty[i]), kMbConsumerWarps);
+      last_fill[i] = 0;
     }
-    mbar_init(smem_u32(sm.red_full), (uint32_t)(C > 1 ? (C - 1) * kMbConsumerWarps * 32 : 1));  // unused if C == 1
-    mbar_init(smem_u32(sm.red_empty), (uint32_t)(kMbConsumerWarps * 32));
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
-  if (warp == kMbConsumerWarps && lane < 3) {
-    const CUtensorMap* m = lane == 0 ? &maps.codes : (lane == 1 ? &maps.x : &maps.v);
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(m)) : "memory");
+  if (warp == kMbConsumerWarps && lane < NP)
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.m[lane])) : "memory");
+  __syncthreads();
+  // the codes of the first stages are the library's and no kernel writes them: they may load before
+  // the grid dependency wait; v and x in fragment order come from the prep kernel, after it
+  if (warp == kMbConsumerWarps && lane == 0) {
+    for (int i = 0; i < S && i < n_units; ++i) {
+      const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
+      const uint32_t bar = smem_u32(&full[i]);
+      mbar_arrive_expect_tx(bar, kFill);
+      tma_load_2d(smem_u32(stages + (size_t)i * kStage), &maps.m[up.p], up.ch * kChunkRowBytes, up.t * kMbTileRows,
+                  bar);
+      last_fill[i] = 1;
+    }
   }
-  cluster_sync();  // barriers initialised in every CTA of the cluster before any remote arrival
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
   if (warp == kMbConsumerWarps) {
     // ---------------------------------------------------------------- producer lane
     if (lane == 0) {
-      for (int f = 0; f < n_fills; ++f) {
-        const int st = f % S, ph = f / S;
-        if (ph > 0 && !mbar_wait(smem_u32(&sm.empty[st]), (uint32_t)((ph - 1) & 1), p.status)) break;
-        const int t = cid + (f / my_chunks) * ncl, ch = c0 + f % my_chunks;
-        uint8_t* sb = sm.stages + (size_t)st * kMbStageBytes;
-        const uint32_t bar = smem_u32(&sm.full[st]);
-        mbar_arrive_expect_tx(bar, kMbCodeBytes + kMbXBytes + kMbVBytes);
-        tma_load_2d(smem_u32(sb), &maps.codes, ch * kChunkRowBytes, t * kMbTileRows, bar);
-#pragma unroll
-        for (int j = 0; j < kChunkCols / kMbXBoxCols; ++j)
-          tma_load_2d(smem_u32(sb + kMbCodeBytes + j * 2048), &maps.x, ch * kChunkCols + j * kMbXBoxCols, 0, bar);
-        tma_load_2d(smem_u32(sb + kMbCodeBytes + kMbXBytes), &maps.v, ch * kChunkCols, 0, bar);
-        tma_load_2d(smem_u32(sb + kMbCodeBytes + kMbXBytes + 512), &maps.v, ch * kChunkCols + 256, 0, bar);
-        sm.last_fill[st] = ph + 1;
+      for (int i = 0; i < n_units; ++i) {
+        const int st = i % S, ph = i / S;
+        const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
+        uint8_t* sb = stages + (size_t)st * kStage;
+        const uint32_t bar = smem_u32(&full[st]);
+        if (ph > 0) {
+          if (!mbar_wait(smem_u32(&empty[st]), (uint32_t)((ph - 1) & 1), gp.status)) break;
+          mbar_arrive_expect_tx(bar, kFill);
+          tma_load_2d(smem_u32(sb), &maps.m[up.p], up.ch * kChunkRowBytes, up.t * kMbTileRows, bar);
+          last_fill[st] = ph + 1;
+        }
+        bulk_load(smem_u32(sb + kMbCodeBytes), tab[up.p].ws + (size_t)up.ch * kMbChunkWsBytes,
+                  (uint32_t)(kMbVBytes + MT * kMbXTileBytes), bar);
       }
     }
   } else {
     // ---------------------------------------------------------------- consumers
-    // x at the salient columns, rows beyond M and columns beyond s zero
-    for (int i = threadIdx.x; i < 16 * p.s_pad; i += kMbConsumerWarps * 32) {
-      const int m = i / p.s_pad, c = i - m * p.s_pad;
-      __half v = __float2half(0.f);
-      if (m < p.M && c < p.s) {
-        int col = __ldg(p.sal + c);
-        col = col < 0 ? 0 : (col >= p.K ? p.K - 1 : col);
-        v = __ushort_as_half(__ldg(p.x + (size_t)m * p.K + col));
-      }
-      sm.xs[i] = v;
-    }
-    asm volatile("bar.sync 1, %0;" ::"n"(kMbConsumerWarps * 32) : "memory");
-
     const int g = lane >> 2, q = lane & 3;
-    const int r0 = warp * 16 + g;  // tile rows of the thread: r0 and r0 + 8
-    const int tid = threadIdx.x;   // consumer index 0 .. 255
-    int f = 0;
-    bool ok = true;
-    for (int ti = 0; ti < n_my_tiles && ok; ++ti) {
-      const int t = cid + ti * ncl;
-      const int row0 = t * kMbTileRows + r0, row1 = row0 + 8;
-      const uint16_t al0 = row0 < p.N ? __ldg(p.alpha + row0) : (uint16_t)0;
-      const uint16_t al1 = row1 < p.N ? __ldg(p.alpha + row1) : (uint16_t)0;
-      float acc[MT][4], res[MT][4];
+    const int tr = warp * 16 * kMbBlocks;  // first row of the warp's 16-row blocks
+    const int tid = threadIdx.x;           // consumer index
+    const int grid = gridDim.x;
+    const int M = gp.M;
+    float acc[2][kMbBlocks][MT][4], res[kMbBlocks][MT][4];
 #pragma unroll
-      for (int j = 0; j < MT; ++j)
+    for (int e = 0; e < 2; ++e)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) acc[j][e] = res[j][e] = 0.f;
+      for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+        for (int j = 0; j < MT; ++j)
+#pragma unroll
+          for (int k = 0; k < 4; ++k) acc[e][b][j][k] = res[b][j][k] = 0.f;
+    uint16_t al[kMbBlocks][2] = {};
+    bool need_alpha = true;
+    UnitPos c = unit_pos(tab, NP, u0);
+    for (int i = 0; i < n_units; ++i) {
+      const int u = u0 + i, st = i % S;
+      const MbProblemArgs& a = tab[c.p];
+      const int tile_row = c.t * kMbTileRows + tr;
+      if (need_alpha) {  // used at the tile's end; the loads complete during the decode
+#pragma unroll
+        for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int row = tile_row + 16 * b + 8 * h + g;
+            al[b][h] = row < a.N ? __ldg(a.alpha + row) : (uint16_t)0;
+          }
+        need_alpha = false;
+      }
+      if (c.ch == 0 && a.yres) {
+        // the tile's residual (Eq. 11), added once: by the CTA that decodes its first chunk
+        const float4* src = reinterpret_cast<const float4*>(a.yres + ((size_t)c.t * 256 + tid) * 4 * kMbBlocks * MT);
+#pragma unroll
+        for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+          for (int j = 0; j < MT; ++j) {
+            const float4 r4 = __ldcg(src + b * MT + j);
+            res[b][j][0] = r4.x;
+            res[b][j][1] = r4.y;
+            res[b][j][2] = r4.z;
+            res[b][j][3] = r4.w;
+          }
+      }
+      const bool ok = mbar_wait(smem_u32(&full[st]), (uint32_t)((i / S) & 1), gp.status);
+      if (!__all_sync(0xffffffffu, ok)) break;
+      decode_unit<MT>(stages + (size_t)st * kStage, tr, g, q, lane, acc);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
 
-      for (int ch = c0; ch < c1; ++ch, ++f) {
-        const int st = f % S;
-        ok = mbar_wait(smem_u32(&sm.full[st]), (uint32_t)((f / S) & 1), p.status);
-        if (!__all_sync(0xffffffffu, ok)) {
-          ok = false;
-          break;
-        }
-        const uint8_t* sb = sm.stages + (size_t)st * kMbStageBytes;
-        const uint8_t* c0p = sb + (size_t)r0 * kChunkRowBytes;
-        const uint8_t* c1p = c0p + 8 * kChunkRowBytes;
-        const uint8_t* xb = sb + kMbCodeBytes;
-        const uint32_t* vb = reinterpret_cast<const uint32_t*>(sb + kMbCodeBytes + kMbXBytes);
-#pragma unroll 2
-        for (int k4 = 0; k4 < 8; ++k4) {  // 16-byte chunk of codes = 4 steps of 16 columns
-          const uint4 w0 = *reinterpret_cast<const uint4*>(c0p + ((k4 ^ (r0 & 7)) << 4));
-          const uint4 w1 = *reinterpret_cast<const uint4*>(c1p + ((k4 ^ (r0 & 7)) << 4));
-          const uint32_t wa[4] = {w0.x, w0.y, w0.z, w0.w};
-          const uint32_t wb[4] = {w1.x, w1.y, w1.z, w1.w};
+      // ---- tile epilogue once this CTA's part of tile c.t is done
+      if (c.ch == a.n_chunks - 1 || u == u1 - 1) {
+        const int t = c.t;
+        // this CTA's part: alpha * acc / 2 + res (alpha scales only the ternary part)
+        float part[kMbBlocks][MT][4];
 #pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            const int kb = 4 * k4 + e;
-            const uint2 vv = *reinterpret_cast<const uint2*>(vb + 8 * kb + 2 * q);  // v at 16kb + 4q .. +3
-            uint32_t a0, a1, a2, a3;
-            decode_byte(wa[e], (uint32_t)q, vv.x, vv.y, a0, a2);
-            decode_byte(wb[e], (uint32_t)q, vv.x, vv.y, a1, a3);
-            // x box kb / 4 holds columns 64 (kb / 4) .. +63; the step's 4q .. 4q+3 within it
-            const int chunk = (kb & 3) * 2 + (q >> 1);
+        for (int b = 0; b < kMbBlocks; ++b) {
+          const float fa0 = 0.5f * h2f(al[b][0]), fa1 = 0.5f * h2f(al[b][1]);
+#pragma unroll
+          for (int j = 0; j < MT; ++j) {
+            part[b][j][0] = fa0 * (acc[0][b][j][0] + acc[1][b][j][0]) + res[b][j][0];
+            part[b][j][1] = fa0 * (acc[0][b][j][1] + acc[1][b][j][1]) + res[b][j][1];
+            part[b][j][2] = fa1 * (acc[0][b][j][2] + acc[1][b][j][2]) + res[b][j][2];
+            part[b][j][3] = fa1 * (acc[0][b][j][3] + acc[1][b][j][3]) + res[b][j][3];
+          }
+        }
+        const long long A = a.unit_begin + (long long)t * a.n_chunks, B = A + a.n_chunks;
+        bool write = true;
+        if (!(A >= u0 && B <= u1)) {
+          // partial tile: publish this warp's rows, then the last of the tile's contributors (per
+          // warp: counter t * 8 + warp) adds all partials in CTA order. Slot 0 of a CTA holds the
+          // tile its range starts in, slot 1 the tile its range ends in.
+          const int my_slot = (u0 >= A) ? 0 : 1;
+          float4* mine = reinterpret_cast<float4*>(
+              a.part + (((size_t)blockIdx.x * 2 + my_slot) * kMbConsumerWarps * 32 + tid) * 4 * kMbBlocks * MT);
+#pragma unroll
+          for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+            for (int j = 0; j < MT; ++j)
+              mine[b * MT + j] = make_float4(part[b][j][0], part[b][j][1], part[b][j][2], part[b][j][3]);
+          __syncwarp();
+          const int bf = unit_owner(A, gp.total_units, grid), bl = unit_owner(B - 1, gp.total_units, grid);
+          int last = 0;
+          if (lane == 0) {
+            // acq_rel at gpu scope: the warp's partials (ordered before by __syncwarp) are published
+            // with the increment, and the last arriver sees every other contributor's partials
+            unsigned* ctr = a.counters + (size_t)t * kMbConsumerWarps + warp;
+            unsigned prev;
+            asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], 1;" : "=r"(prev) : "l"(ctr) : "memory");
+            last = (prev == (unsigned)(bl - bf));  // every CTA in [bf, bl] holds units of this tile
+            if (last) *ctr = 0u;                   // self-reset for the next call
+          }
+          last = __shfl_sync(0xffffffffu, last, 0);
+          __syncwarp();
+          write = last != 0;
+          if (write) {
+#pragma unroll
+            for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+              for (int j = 0; j < MT; ++j)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) part[b][j][k] = 0.f;
+            for (int cb = bf; cb <= bl; ++cb) {
+              const int cslot = (gp.cta_u0[cb] >= A) ? 0 : 1;
+              const float4* src = reinterpret_cast<const float4*>(
+                  a.part + (((size_t)cb * 2 + cslot) * kMbConsumerWarps * 32 + tid) * 4 * kMbBlocks * MT);
+#pragma unroll
+              for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+                for (int j = 0; j < MT; ++j) {
+                  const float4 v4 = __ldcg(src + b * MT + j);
+                  part[b][j][0] += v4.x;
+                  part[b][j][1] += v4.y;
+                  part[b][j][2] += v4.z;
+                  part[b][j][3] += v4.w;
+                }
+            }
+          }
+        }
+        if (write) {
+#pragma unroll
+          for (int b = 0; b < kMbBlocks; ++b)
 #pragma unroll
             for (int j = 0; j < MT; ++j) {
-              const int n = 8 * j + g;
-              const uint2 bb = *reinterpret_cast<const uint2*>(xb + (kb >> 2) * 2048 + n * 128 +
-                                                               ((chunk ^ (n & 7)) << 4) + 8 * (q & 1));
-              mma_16816(acc[j], a0, a1, a2, a3, bb.x, bb.y);
-            }
-          }
-        }
-        __syncwarp();
-        if (lane == 0) mbar_arrive(smem_u32(&sm.empty[st]));
-      }
-      if (!ok) break;
-
-      // ---- residual (Eq. 11): virtual columns, 16 salient entries per step, steps split over ranks
-      if (p.s > 0) {
-        const int gq0 = row0 >> 2, gq1 = row1 >> 2, pos = row0 & 3;  // row1 & 3 == pos
-        const bool v0 = gq0 < (p.N >> 2), v1 = gq1 < (p.N >> 2);
-        const int rs = (p.s + 3) >> 2;
-        for (int eb = rank; eb * 16 < p.s; eb += C) {
-          const int e0 = eb * 16 + 4 * q;  // the thread's entries e0 .. e0 + 3
-          uint2 r0v = make_uint2(0, 0), r1v = make_uint2(0, 0);
-          uint32_t p0 = 0, p1 = 0;
-          if (p.vec_res) {
-            if (v0 && e0 < p.s) {
-              r0v = __ldg(reinterpret_cast<const uint2*>(p.rvals + (size_t)gq0 * p.s + e0));
-              p0 = __ldg(p.ridx + (size_t)gq0 * rs + (e0 >> 2));
-            }
-            if (v1 && e0 < p.s) {
-              r1v = __ldg(reinterpret_cast<const uint2*>(p.rvals + (size_t)gq1 * p.s + e0));
-              p1 = __ldg(p.ridx + (size_t)gq1 * rs + (e0 >> 2));
-            }
-          } else {
-            uint32_t h0[4] = {0, 0, 0, 0}, h1[4] = {0, 0, 0, 0};
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const int e = e0 + j;
-              if (e < p.s) {
-                if (v0) {
-                  h0[j] = __ldg(p.rvals + (size_t)gq0 * p.s + e);
-                  p0 |= ((uint32_t)(__ldg(p.ridx + (size_t)gq0 * rs + (e >> 2)) >> (2 * (e & 3))) & 3u) << (2 * j);
-                }
-                if (v1) {
-                  h1[j] = __ldg(p.rvals + (size_t)gq1 * p.s + e);
-                  p1 |= ((uint32_t)(__ldg(p.ridx + (size_t)gq1 * rs + (e >> 2)) >> (2 * (e & 3))) & 3u) << (2 * j);
-                }
+              const int n0 = 8 * j + 2 * q;
+              const int row0 = c.t * kMbTileRows + tr + 16 * b + g, row1 = row0 + 8;
+              if (row0 < a.N) {
+                if (n0 < M) a.y[(size_t)n0 * a.N + row0] = part[b][j][0];
+                if (n0 + 1 < M) a.y[(size_t)(n0 + 1) * a.N + row0] = part[b][j][1];
+              }
+              if (row1 < a.N) {
+                if (n0 < M) a.y[(size_t)n0 * a.N + row1] = part[b][j][2];
+                if (n0 + 1 < M) a.y[(size_t)(n0 + 1) * a.N + row1] = part[b][j][3];
               }
             }
-            r0v = make_uint2(h0[0] | (h0[1] << 16), h0[2] | (h0[3] << 16));
-            r1v = make_uint2(h1[0] | (h1[1] << 16), h1[2] | (h1[3] << 16));
-          }
-          // keep the values whose stored position is this row (fp16 lanes all-ones or zero)
-          auto keep = [&](uint32_t pb, int j0) -> uint32_t {
-            const uint32_t lo = (((pb >> (2 * j0)) & 3u) == (uint32_t)pos) ? 0x0000ffffu : 0u;
-            const uint32_t hi = (((pb >> (2 * j0 + 2)) & 3u) == (uint32_t)pos) ? 0xffff0000u : 0u;
-            return lo | hi;
-          };
-          const uint32_t a0 = r0v.x & keep(p0, 0), a2 = r0v.y & keep(p0, 2);
-          const uint32_t a1 = r1v.x & keep(p1, 0), a3 = r1v.y & keep(p1, 2);
-#pragma unroll
-          for (int j = 0; j < MT; ++j) {
-            const int n = 8 * j + g;
-            const uint2 bb = *reinterpret_cast<const uint2*>(sm.xs + (size_t)n * p.s_pad + e0);
-            mma_16816(res[j], a0, a1, a2, a3, bb.x, bb.y);
-          }
         }
-      }
-
-      // ---- this CTA's part of the tile: alpha * acc + res (alpha scales only the ternary part)
-      const float fa0 = __half2float(__ushort_as_half(al0)), fa1 = __half2float(__ushort_as_half(al1));
-      float part[MT][4];
 #pragma unroll
-      for (int j = 0; j < MT; ++j) {
-        part[j][0] = fa0 * acc[j][0] + res[j][0];
-        part[j][1] = fa0 * acc[j][1] + res[j][1];
-        part[j][2] = fa1 * acc[j][2] + res[j][2];
-        part[j][3] = fa1 * acc[j][3] + res[j][3];
-      }
-      if (rank != 0) {
-        // into rank 0's slot for this rank, once rank 0 has read the previous tile's
-        if (ti > 0 && !mbar_wait_cluster(smem_u32(sm.red_empty), (uint32_t)((ti - 1) & 1), p.status)) break;
-        const uint32_t dst = map_rank(smem_u32(sm.slots + ((size_t)(rank - 1) * kMbConsumerWarps * 32 + tid) * 4 * MT), 0);
+        for (int e = 0; e < 2; ++e)
 #pragma unroll
-        for (int j = 0; j < MT; ++j) st_cluster_v4(dst + 16 * j, part[j][0], part[j][1], part[j][2], part[j][3]);
-        mbar_arrive_cluster(map_rank(smem_u32(sm.red_full), 0));
-        continue;
-      }
-      if (C > 1) {
-        // rank 0: add the other ranks' parts in rank order, then give their slots back
-        if (!mbar_wait_cluster(smem_u32(sm.red_full), (uint32_t)(ti & 1), p.status)) break;
-        for (int rr = 1; rr < C; ++rr) {
-          const float* src = sm.slots + ((size_t)(rr - 1) * kMbConsumerWarps * 32 + tid) * 4 * MT;
+          for (int b = 0; b < kMbBlocks; ++b)
 #pragma unroll
-          for (int j = 0; j < MT; ++j) {
-            const float4 v4 = *reinterpret_cast<const float4*>(src + 4 * j);
-            part[j][0] += v4.x;
-            part[j][1] += v4.y;
-            part[j][2] += v4.z;
-            part[j][3] += v4.w;
-          }
-        }
-        for (int rr = 1; rr < C; ++rr) mbar_arrive_cluster(map_rank(smem_u32(sm.red_empty), (uint32_t)rr));
-      }
-      // ---- y[n][row] for the thread's rows and batch columns
+            for (int j = 0; j < MT; ++j)
 #pragma unroll
-      for (int j = 0; j < MT; ++j) {
-        const int n0 = 8 * j + 2 * q;
-        if (row0 < p.N) {
-          if (n0 < p.M) p.y[(size_t)n0 * p.N + row0] = part[j][0];
-          if (n0 + 1 < p.M) p.y[(size_t)(n0 + 1) * p.N + row0] = part[j][1];
-        }
-        if (row1 < p.N) {
-          if (n0 < p.M) p.y[(size_t)n0 * p.N + row1] = part[j][2];
-          if (n0 + 1 < p.M) p.y[(size_t)(n0 + 1) * p.N + row1] = part[j][3];
+              for (int k = 0; k < 4; ++k) acc[e][b][j][k] = res[b][j][k] = 0.f;
+        need_alpha = true;
+      }
+      if (++c.ch == a.n_chunks) {
+        c.ch = 0;
+        if (++c.t == a.n_tiles) {
+          c.t = 0;
+          ++c.p;
         }
       }
     }
   }
 
-  // no bulk copy may still be writing shared memory when the CTA exits, and no CTA of the
-  // cluster may exit while another may still write its shared memory
+  // no bulk copy may still be writing shared memory when the CTA exits (after a timeout the
+  // consumers may not have waited for every fill)
   __syncthreads();
   if (threadIdx.x == 0) {
     for (int s2 = 0; s2 < S; ++s2) {
-      const int lf = sm.last_fill[s2];
-      if (lf > 0 && !mbar_wait(smem_u32(&sm.full[s2]), (uint32_t)((lf - 1) & 1), p.status)) break;
+      const int lf = last_fill[s2];
+      if (lf > 0 && !mbar_wait(smem_u32(&full[s2]), (uint32_t)((lf - 1) & 1), gp.status)) break;
     }
   }
-  cluster_sync();
 }
 
 }  // namespace
 
-size_t mb_smem_bytes(int S, int s_pad, int cluster, int M) {
+size_t mb_smem_bytes(int S, int M) {
   const int mt = M <= 8 ? 1 : 2;
-  return (size_t)S * kMbStageBytes + (size_t)16 * s_pad * 2 +
-         (size_t)(cluster - 1) * kMbConsumerWarps * 32 * 4 * mt * sizeof(float) +
-         (size_t)(2 * S + 2) * sizeof(unsigned long long) + (size_t)kMaxStagesMb * sizeof(int) + 1024;
+  return (size_t)S * mb_stage_bytes(mt) + (size_t)kMaxProblems * sizeof(MbProblemArgs) +
+         (size_t)(2 * S) * sizeof(unsigned long long) + (size_t)kMaxStagesMb * sizeof(int) + 1024;
 }
 
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max) {
@@ -467,21 +658,48 @@ cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max) {
   return cudaFuncSetAttribute(qtea_gemv_mb_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
 }
 
-cudaError_t launch_mb(const MbMaps& maps, const MbParams& p, int grid, size_t smem, cudaStream_t st) {
+// Both launches use programmatic stream serialisation: the prep kernel starts while the previous
+// kernel on the stream drains, and the main kernel while the prep kernel runs; each waits
+// (griddepcontrol.wait) before it touches memory that an earlier kernel writes.
+size_t mb_prep_smem_bytes(int s, bool native) {
+  const size_t E = native ? (size_t)s : (size_t)kMbResEntries;
+  const size_t ris = native ? (size_t)((s + 3) / 4) : (size_t)kMbResEntries / 4;
+  const size_t res = ((64 * E * 2 + 15) & ~(size_t)15) + ((64 * ris + 15) & ~(size_t)15) + 16 * ((E + 15) & ~(size_t)15) * 2;
+  const size_t chunk = (size_t)16 * kChunkCols * 2 + (size_t)kChunkCols * 2;
+  return s > 0 && res > chunk ? res : chunk;
+}
+
+cudaError_t mb_prep_configure(size_t smem_optin) {
+  cudaError_t e = cudaFuncSetAttribute(qtea_mb_prep_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_optin);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(qtea_mb_prep_kernel, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+}
+
+cudaError_t launch_mb_prep(const MbPrepGroup& g, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)g.n_blocks);
+  cfg.blockDim = dim3(256);
+  cfg.dynamicSmemBytes = g.smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, qtea_mb_prep_kernel, g);
+}
+
+cudaError_t launch_mb(const TensorMaps& maps, const MbGroupParams& p, int grid, size_t smem, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(kMbThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[2];
+  cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
-  attr[1].id = cudaLaunchAttributeClusterDimension;
-  attr[1].val.clusterDim.x = (unsigned)p.cluster;
-  attr[1].val.clusterDim.y = 1;
-  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = 1;
   if (p.M <= 8) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1>, maps, p);
   return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2>, maps, p);
 }

@@ -99,30 +99,75 @@ __host__ __device__ constexpr size_t m1_smem_bytes(int S) {
 // ---------------------------------------------------------------- low-batch tensor-core kernel (2 <= M <= 16)
 constexpr int kMaxStagesMb = 6;
 constexpr int kMinStagesMb = 2;
-constexpr int kMaxSalientMb = 1024;  // x at the salient columns is staged in shared memory
+constexpr int kMbTileRows = 256;                               // rows of a unit (one TMA box)
+constexpr int kMbVBytes = 1024;                                // v of a chunk in fragment order
+constexpr int kMbXTileBytes = 8192;                            // x of a chunk, 8 batch rows, fragment order
+constexpr int kMbChunkWsBytes = kMbVBytes + 2 * kMbXTileBytes; // 17408 per 512-column chunk
 
-struct MbMaps {
-  CUtensorMap codes;  // packed codes [N][K_pad/4] bytes, box 128 bytes x 128 rows, 128-byte swizzle
-  CUtensorMap x;      // activations [M][K] fp16, box 64 x 16 rows, 128-byte swizzle
-  CUtensorMap v;      // column rescale [1][K] fp16, box 256 x 1
-};
+// One shared-memory stage of the low-batch kernel: codes [256 rows][128 bytes], the chunk's v block
+// and MT x blocks, rounded to 1024 bytes (the 128-byte swizzle of the next stage's codes).
+__host__ __device__ constexpr int mb_stage_bytes(int mt) {
+  return (kMbTileRows * kChunkRowBytes + kMbVBytes + mt * kMbXTileBytes + 1023) / 1024 * 1024;
+}
 
-struct MbParams {
+// Prep kernel: v and x of every 512-column chunk in fragment order, and the residual (Eq. 11) of
+// every 256-row tile in the consumers' accumulator order, for every problem of a group in one launch.
+constexpr int kMbResEntries = 256;  // salient entries staged per pass of a residual block
+
+struct MbPrepProblem {
   const uint16_t* x;        // [M][K]
-  const uint16_t* alpha;    // [N]
+  const uint16_t* v;        // [K]
   const int32_t* sal;       // [s]
   const uint16_t* rvals;    // [N/4][s]
   const uint8_t* ridx;      // [N/4][ceil(s/4)]
-  float* y;                 // [M][N]
-  int* status;
-  int N, K, M, s, s_pad, n_tiles, n_chunks, n_stages;
-  int vec_res;              // s % 8 == 0 and rvals 16-byte aligned: 8-byte residual loads
-  int cluster;              // CTAs per cluster sharing a tile (1 .. 8)
+  uint8_t* ws;              // [n_chunks][kMbChunkWsBytes]
+  float* yres;              // [n_tiles][256 threads][4 kMbBlocks MT] residual in accumulator order
+  int N, K, s, n_chunks, n_tiles;
+  int native;               // residual staged as stored (16-byte vector loads), else in passes
+  int block_begin;          // first block of this problem in the launch
 };
 
-size_t mb_smem_bytes(int S, int s_pad, int cluster, int M);
+struct MbPrepGroup {
+  MbPrepProblem prob[kMaxProblems];
+  int n_problems, M, mt, n_blocks;
+  size_t smem;              // dynamic shared memory of a block
+};
+
+constexpr int kMbBlocks = 2;                                   // 16-row blocks per consumer warp
+constexpr int kMbConsumerWarps = kMbTileRows / 16 / kMbBlocks;  // 8
+
+// One problem of a grouped low-batch launch; units (tile of 256 rows, chunk of 512 columns) of all
+// problems form one sequence split evenly over the CTAs, as in the batch-1 kernel.
+struct MbProblemArgs {
+  const uint16_t* alpha;    // [N]
+  const uint8_t* ws;        // the prep kernel's chunks
+  const float* yres;        // the prep kernel's residual, or null without salient columns
+  float* y;                 // [M][N]
+  float* part;              // [grid][2][256 threads][4 kMbBlocks MT] partial rows of split tiles
+  unsigned* counters;       // [n_tiles][kMbConsumerWarps], zero between calls
+  int N, n_tiles, n_chunks;
+  long long unit_begin;
+};
+
+struct MbGroupParams {
+  MbProblemArgs prob[kMaxProblems];
+  int n_problems, n_stages, M;
+  int* status;              // device status word (the first layout's)
+  long long total_units;
+  int cta_u0[kMaxGrid + 1];
+};
+
+// Partial-row slots of the low-batch kernel per layout: [sm_count][2][256 threads][16] floats.
+constexpr size_t kMbPartFloatsPerCta = 2 * 256 * 16;
+// Residual of one 256-row tile in accumulator order: [256 threads][16] floats.
+constexpr size_t kMbResFloatsPerTile = 256 * 16;
+
+size_t mb_smem_bytes(int S, int M);
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max);
-cudaError_t launch_mb(const MbMaps& maps, const MbParams& p, int grid, size_t smem, cudaStream_t st);
+size_t mb_prep_smem_bytes(int s, bool native);
+cudaError_t mb_prep_configure(size_t smem_optin);
+cudaError_t launch_mb_prep(const MbPrepGroup& g, cudaStream_t st);
+cudaError_t launch_mb(const TensorMaps& maps, const MbGroupParams& p, int grid, size_t smem, cudaStream_t st);
 
 // ---------------------------------------------------------------- generic kernel (any M)
 struct GenericParams {
@@ -181,5 +226,9 @@ struct qtea_layout {
   // low-batch kernel resources
   bool mb_ok;
   size_t mb_smem_optin;
-  CUtensorMap tmap_mb;   // codes, box 128 bytes x 128 rows
+  size_t prep_smem_optin;  // dynamic shared memory the prep kernel may use
+  uint8_t* mb_ws;        // [n_chunks][kMbChunkWsBytes] v and x in fragment order, then the residual
+                         // of every 256-row tile [n_tiles][kMbResFloatsPerTile]
+  float* mb_part;        // [sm_count][kMbPartFloatsPerCta] partial rows of split tiles
+  unsigned* mb_counters; // [n_tiles of 256 rows][kMbConsumerWarps]
 };

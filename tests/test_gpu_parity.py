@@ -121,12 +121,35 @@ DENSE_SALIENT = [  # more than 16 salient entries per unit (residual summed by t
 
 
 @pytest.mark.parametrize("N,K,s", DENSE_SALIENT)
-def test_parity_dense_salient(qt, N, K, s):
-    p = synth.make_problem("t", N, K, 1, s, seed=N + 3 * K + 5 * s)
+@pytest.mark.parametrize("M", [1, 3, 12])
+def test_parity_dense_salient(qt, N, K, s, M):
+    p = synth.make_problem("t", N, K, M, s, seed=N + 3 * K + 5 * s + M)
     d = Dev(qt, p)
     y = d.run(qt)
     y_ref, b = oracle_ref(p)
-    assert_within(y, y_ref, b, f"N={N} K={K} s={s}")
+    assert_within(y, y_ref, b, f"N={N} K={K} s={s} M={M}")
+
+
+@pytest.mark.parametrize("M", [2, 9])
+def test_low_batch_unaligned_operands(qt, M):
+    """x and v starting 2 bytes past a 16-byte boundary, K odd, residual values 2 bytes past an
+    8-byte boundary (scalar residual loads)."""
+    N, K, s = 516, 777, 12
+    p = synth.make_problem("t", N, K, M, s, seed=40 + M)
+    d = Dev(qt, p)
+
+    def shifted(t):
+        buf = torch.zeros(t.numel() + 1, dtype=t.dtype, device=t.device)
+        buf[1:] = t.reshape(-1)
+        return buf[1:].view(t.shape)
+
+    x, v, rv = shifted(d.x), shifted(d.v), shifted(d.rv)
+    assert x.data_ptr() % 16 == 2 and rv.data_ptr() % 8 == 2
+    y = qt.qtea_gemv(x, d.layout, d.alpha, v, d.sal, rv, d.ri)
+    torch.cuda.synchronize()
+    assert qt.qtea_device_status(d.layout) == 0
+    y_ref, b = oracle_ref(p)
+    assert_within(y.cpu().numpy().astype(np.float64), y_ref, b, f"unaligned M={M}")
 
 
 def test_config0_tiny(qt):
