@@ -75,8 +75,12 @@ int plan_m1(qtea_layout* l, const cudaDeviceProp& prop) {
     // then x at the salient columns; partial rows and counters of split 256-row tiles
     size_t mb_dyn = 0;
     const int mb_tiles = (l->N + kMbTileRows - 1) / kMbTileRows;
+    // chunks, then (with salient columns) the prep kernel's residual per tile and x at the salient
+    // columns for the helper warps
     const size_t ws = (size_t)l->n_chunks * kMbChunkWsBytes +
-                      (l->n_salient > 0 ? (size_t)mb_tiles * kMbResFloatsPerTile * sizeof(float) : 0);
+                      (l->n_salient > 0 ? (size_t)mb_tiles * kMbResFloatsPerTile * sizeof(float) +
+                                              (size_t)16 * round_up(l->n_salient, 16) * 2
+                                        : 0);
     const size_t ctr = (size_t)mb_tiles * kMbConsumerWarps * sizeof(unsigned);
     l->mb_ok = mb_configure(prop.sharedMemPerBlockOptin, &mb_dyn) == cudaSuccess &&
                mb_prep_configure(prop.sharedMemPerBlockOptin) == cudaSuccess;
@@ -174,9 +178,10 @@ struct MbGroup {
   int grid = 0;
   size_t smem = 0;
   size_t prep_smem_optin = 0;
+  size_t smem_optin = 0;  // the main kernel's dynamic shared memory limit
 };
 
-void mb_group_reset(MbGroup& g, int M, size_t prep_smem_optin) {
+void mb_group_reset(MbGroup& g, int M, size_t prep_smem_optin, size_t smem_optin) {
   std::memset(&g.gp, 0, sizeof(g.gp));
   std::memset(&g.pg, 0, sizeof(g.pg));
   std::memset(&g.maps, 0, sizeof(g.maps));
@@ -186,6 +191,7 @@ void mb_group_reset(MbGroup& g, int M, size_t prep_smem_optin) {
   g.grid = 0;
   g.smem = 0;
   g.prep_smem_optin = prep_smem_optin;
+  g.smem_optin = smem_optin;
 }
 
 bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
@@ -193,7 +199,20 @@ bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
   const qtea_layout* l = q.packed_ternary;
   const int k = g.gp.n_problems;
   const int n_tiles = (l->N + kMbTileRows - 1) / kMbTileRows;
-  float* yres = l->n_salient > 0 ? reinterpret_cast<float*>(l->mb_ws + (size_t)l->n_chunks * kMbChunkWsBytes) : nullptr;
+  const int s = l->n_salient, s16 = round_up(s, 16);
+  const int mt = g.gp.M <= 8 ? 1 : 2;
+  uint8_t* res_base = l->mb_ws + (size_t)l->n_chunks * kMbChunkWsBytes;
+  float* yres = s > 0 ? reinterpret_cast<float*>(res_base) : nullptr;
+  uint16_t* xs = s > 0 ? reinterpret_cast<uint16_t*>(res_base + (size_t)n_tiles * kMbResFloatsPerTile * sizeof(float))
+                       : nullptr;
+  // residual by the main kernel's helpers when the caller's arrays allow bulk copies and a pass over a
+  // half or quarter of a tile's row groups fits beside two code stages; else by the prep kernel
+  int mode = s > 0 ? kMbResPrep : kMbResNone, passes = 0;
+  if (s > 0 && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 16)) {
+    for (int p = 1; p <= 4 && !passes; p *= 2)
+      if (mb_smem_layout(kMinStagesMb, mt, (int)mb_res_stage_bytes(s, p)).total <= g.smem_optin) passes = p;
+    if (passes) mode = kMbResHelpers;
+  }
   MbPrepProblem& pp = g.pg.prob[k];
   pp.x = q.x;
   pp.v = q.col_scale;
@@ -202,38 +221,51 @@ bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
   pp.ridx = q.residual_idx;
   pp.ws = l->mb_ws;
   pp.yres = yres;
+  pp.xs = xs;
   pp.N = l->N;
   pp.K = l->K;
-  pp.s = l->n_salient;
+  pp.s = s;
+  pp.s16 = s16;
   pp.n_chunks = l->n_chunks;
   pp.n_tiles = n_tiles;
-  pp.native = l->n_salient > 0 && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 16) &&
-              mb_prep_smem_bytes(l->n_salient, true) <= g.prep_smem_optin;
-  const size_t need = mb_prep_smem_bytes(l->n_salient, pp.native != 0);
-  if (need > g.pg.smem) g.pg.smem = need;
+  pp.res_mode = mode;
+  pp.native = mode == kMbResPrep && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 16) &&
+              mb_prep_smem_bytes(s, true) <= g.prep_smem_optin;
   pp.block_begin = g.pg.n_blocks;
+  const size_t need = mb_prep_smem_bytes(mode == kMbResPrep ? s : 0, pp.native != 0);
+  if (need > g.pg.smem) g.pg.smem = need;
   MbProblemArgs& a = g.gp.prob[k];
   a.alpha = q.row_scale;
   a.ws = l->mb_ws;
   a.yres = yres;
+  a.rvals = q.residual_vals;
+  a.ridx = q.residual_idx;
+  a.xs = xs;
   a.y = q.y;
   a.part = l->mb_part;
   a.counters = l->mb_counters;
   a.N = l->N;
   a.n_tiles = n_tiles;
   a.n_chunks = l->n_chunks;
+  a.s = s;
+  a.s16 = s16;
+  a.res_mode = mode;
+  a.res_passes = passes;
   a.unit_begin = g.gp.total_units;
+  if (mode == kMbResHelpers) {
+    const int rsb = (int)mb_res_stage_bytes(s, passes);
+    if (rsb > g.gp.res_stage_bytes) g.gp.res_stage_bytes = rsb;
+  }
   std::memcpy(&g.maps.m[k], &l->tmap, sizeof(CUtensorMap));
   if (k == 0) g.gp.status = l->status;
   g.gp.total_units += (long long)a.n_tiles * a.n_chunks;
-  g.pg.n_blocks += l->n_chunks + (l->n_salient > 0 ? n_tiles : 0);
+  g.pg.n_blocks += l->n_chunks + (mode == kMbResPrep ? n_tiles : mode == kMbResHelpers ? (s16 + 255) / 256 : 0);
   g.gp.n_problems += 1;
   g.pg.n_problems += 1;
   return true;
 }
 
-// Grid, ring depth and shared memory of the group; false if the ring does not fit or the group
-// needs more CTAs than every layout's partial-row slots serve.
+// Grid, ring depth and shared memory of the group; false if the ring does not fit.
 bool mb_group_plan(MbGroup& g, int sm_count, size_t smem_optin) {
   if (g.gp.n_problems == 0) return false;
   if (g.gp.total_units >= (1ll << 30)) return false;
@@ -241,9 +273,10 @@ bool mb_group_plan(MbGroup& g, int sm_count, size_t smem_optin) {
   if (g.grid > kMaxGrid) g.grid = kMaxGrid;
   for (int b = 0; b <= g.grid; ++b) g.gp.cta_u0[b] = (int)unit_begin_of(b, g.gp.total_units, g.grid);
   for (int S = kMaxStagesMb; S >= kMinStagesMb; --S) {
-    if (mb_smem_bytes(S, g.gp.M) <= smem_optin) {
+    const size_t bytes = mb_smem_bytes(S, g.gp.M, g.gp.res_stage_bytes);
+    if (bytes <= smem_optin) {
       g.gp.n_stages = S;
-      g.smem = mb_smem_bytes(S, g.gp.M);
+      g.smem = bytes;
       return true;
     }
   }
@@ -264,7 +297,7 @@ int run_mb(const qtea_gemv_problem* qs, const int* idx, int n, int M, cudaStream
   while (i < n) {
     const qtea_layout* l0 = qs[idx[i]].packed_ternary;
     MbGroup g;
-    mb_group_reset(g, M, l0->prep_smem_optin);
+    mb_group_reset(g, M, l0->prep_smem_optin, l0->mb_smem_optin);
     int taken = 0;
     while (i + taken < n) {
       const qtea_layout* li = qs[idx[i + taken]].packed_ternary;

@@ -38,7 +38,7 @@ namespace qtea {
 namespace {
 
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
-constexpr int kMbThreads = (kMbConsumerWarps + 1) * 32;
+constexpr int kMbThreads = (kMbConsumerWarps + 1 + kMbHelperWarps) * 32;  // consumers, producer, helpers
 constexpr int kMbCodeBytes = kMbTileRows * kChunkRowBytes;  // 32768
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
@@ -147,16 +147,17 @@ __device__ __forceinline__ UnitPos unit_pos(const MbProblemArgs* tab, int n_prob
 // come from the staged tile: rv [64 groups][rvs] fp16, ri [64][ris] position bytes (entry e of a
 // group in bits 2(e % 4) of byte e / 4), xr [16 batch rows][xrs] fp16 (zero past the valid
 // entries); only entries below ne count.
+template <int NB>
 __device__ __forceinline__ void res_step(const uint16_t* rv, int rvs, const uint8_t* ri, int ris, const uint16_t* xr,
                                          int xrs, int ne, int step, int tr, int g, int q, int mt, bool quad_loads,
-                                         float (&res)[kMbBlocks][2][4]) {
+                                         float (&res)[NB][2][4]) {
   const int e0 = step * 16 + 4 * q;
   const uint32_t pos = (uint32_t)(g & 3);  // row & 3 for every row of the thread
   uint2 xb[2];
 #pragma unroll
   for (int j = 0; j < 2; ++j) xb[j] = *reinterpret_cast<const uint2*>(xr + (8 * j + g) * xrs + e0);
 #pragma unroll
-  for (int b = 0; b < kMbBlocks; ++b) {
+  for (int b = 0; b < NB; ++b) {
     uint32_t a[4];
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
@@ -189,7 +190,9 @@ __device__ __forceinline__ void res_step(const uint16_t* rv, int rvs, const uint
   }
 }
 
-// Blocks of a problem: its chunks, then (with salient columns) its 256-row tiles.
+// Blocks of a problem: its chunks; then, for a residual left to the prep kernel, its 256-row tiles;
+// or, for a residual of the main kernel's helpers, blocks that gather x at the salient columns
+// (xs[m][c], zero beyond s or M), 256 columns each.
 // Chunk ch's 512 columns: entry (step s, quad lane q) of the v block holds the pairs
 // (v[16W + i], v[16W + i + 8]) for i = 2(s & 3) and i + 1, W = 8q + (s >> 2); entry (step s,
 // lane 4g + q) of x block j holds the same two pairs of x[8j + g]. Columns >= K and batch rows >= M
@@ -216,6 +219,20 @@ __global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant
   const int M = gr.M;
   const int local = (int)blockIdx.x - p.block_begin;
   const int tid = threadIdx.x;
+  if (local >= p.n_chunks && p.res_mode == kMbResHelpers) {
+    // ---- x at 256 salient columns, all 16 batch rows
+    const int c = (local - p.n_chunks) * 256 + tid;
+    if (c < p.s16) {
+      int col = c < p.s ? __ldg(p.sal + c) : 0;
+      col = col < 0 ? 0 : (col >= p.K ? p.K - 1 : col);
+      uint16_t xv[16];
+#pragma unroll
+      for (int m = 0; m < 16; ++m) xv[m] = (c < p.s && m < M) ? __ldg(p.x + (size_t)m * p.K + col) : (uint16_t)0;
+#pragma unroll
+      for (int m = 0; m < 16; ++m) p.xs[(size_t)m * p.s16 + c] = xv[m];
+    }
+    return;
+  }
   if (local >= p.n_chunks) {
     // ---- residual of tile t
     const int t = local - p.n_chunks;
@@ -293,9 +310,11 @@ __global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant
       // whole (staged rows in passes are padded with zeros)
       const bool quad = (rvs & 3) == 0 && (p.native ? (ne & 3) == 0 : true);
       if (quad) {
-        for (int step = 0; step * 16 < ne; ++step) res_step(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, true, res);
+        for (int step = 0; step * 16 < ne; ++step)
+          res_step<kMbBlocks>(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, true, res);
       } else {
-        for (int step = 0; step * 16 < ne; ++step) res_step(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, false, res);
+        for (int step = 0; step * 16 < ne; ++step)
+          res_step<kMbBlocks>(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, false, res);
       }
       __syncthreads();
     }
@@ -393,6 +412,102 @@ __device__ __forceinline__ void decode_unit(const uint8_t* sb, int tr, int g, in
   }
 }
 
+// ---------------------------------------------------------------- helper warps (residual)
+
+__device__ __forceinline__ void helpers_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kMbHelperWarps * 32) : "memory"); }
+
+// The residual (Eq. 11) of every tile whose first chunk this CTA decodes, in the order the consumers
+// reach those tiles, into a ring of two result slots laid out in the consumers' accumulator order
+// ([256 consumer threads][4 kMbBlocks MT] floats). Per tile, in 1, 2 or 4 passes over its row
+// groups: the pass's values and position bytes (one contiguous range each, starting on a 16-byte
+// boundary) and, once per tile, x at the salient columns come by bulk copy (the last < 16 bytes by
+// plain loads); then helper warp hw takes 16-row blocks hw, hw + 4, ... of the pass with the same
+// virtual-column MMA as the prep kernel. A wait that times out is recorded in the status word and
+// the helpers carry on, so that every helper reaches every named barrier.
+template <int MT>
+__device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u0, int n_units, float* rslot,
+                                         uint8_t* rstage, uint64_t* res_full, uint64_t* res_empty, uint64_t* staged,
+                                         int hw, int lane, int* status) {
+  const int g = lane >> 2, q = lane & 3;
+  const int htid = hw * 32 + lane;
+  UnitPos c = unit_pos(tab, NP, u0);
+  int k = 0, sphase = 0;
+  bool failed = false;
+  for (int i = 0; i < n_units; ++i) {
+    const MbProblemArgs& a = tab[c.p];
+    if (c.ch == 0 && a.res_mode == kMbResHelpers) {
+      const int slot = k & 1;
+      const int s = a.s, rs = (s + 3) >> 2, s16 = a.s16;
+      const int passes = a.res_passes, gpp = (kMbTileRows / 4) / passes;
+      const int g0 = c.t * (kMbTileRows / 4), ng_tile = min(kMbTileRows / 4, a.N / 4 - g0);
+      uint16_t* rv = reinterpret_cast<uint16_t*>(rstage);
+      uint8_t* ri = rstage + (((size_t)gpp * s * 2 + 15) & ~(size_t)15);
+      uint16_t* xr = reinterpret_cast<uint16_t*>(ri + (((size_t)gpp * rs + 15) & ~(size_t)15));
+      float* out = rslot + (size_t)slot * 256 * 8 * MT;
+      if (k >= 2 && !mbar_wait(smem_u32(&res_empty[slot]), (uint32_t)(((k >> 1) - 1) & 1), status)) failed = true;
+      const bool quad = (s & 3) == 0;
+      for (int pass = 0; pass < passes; ++pass) {
+        const int G0 = pass * gpp;
+        const int ng = max(0, min(gpp, ng_tile - G0));
+        helpers_sync();  // every helper is done with the staging buffer
+        const size_t vb = (size_t)ng * s * 2, ib = (size_t)ng * rs;
+        const size_t vsrc = (size_t)(g0 + G0) * s, isrc = (size_t)(g0 + G0) * rs;
+        if (htid == 0) {
+          const uint32_t vbb = (uint32_t)(vb & ~(size_t)15), ibb = (uint32_t)(ib & ~(size_t)15);
+          const uint32_t xbb = pass == 0 ? (uint32_t)(32 * s16) : 0u;
+          const uint32_t bar = smem_u32(staged);
+          // the helpers' reads of the previous pass (generic proxy) before the copies (async proxy)
+          asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          mbar_arrive_expect_tx(bar, vbb + ibb + xbb);
+          if (vbb) bulk_load(smem_u32(rv), a.rvals + vsrc, vbb, bar);
+          if (ibb) bulk_load(smem_u32(ri), a.ridx + isrc, ibb, bar);
+          if (xbb) bulk_load(smem_u32(xr), a.xs, xbb, bar);
+        }
+        {
+          const int vt = (int)((vb & 15) >> 1), it = (int)(ib & 15);
+          const size_t v0 = (vb & ~(size_t)15) >> 1, i0 = ib & ~(size_t)15;
+          if (htid < vt) rv[v0 + htid] = __ldg(a.rvals + vsrc + v0 + htid);
+          if (htid >= 32 && htid - 32 < it) ri[i0 + htid - 32] = __ldg(a.ridx + isrc + i0 + htid - 32);
+        }
+        if (!mbar_wait(smem_u32(staged), (uint32_t)(sphase & 1), status)) failed = true;
+        ++sphase;
+        helpers_sync();  // the tails are visible to every helper
+        if (ng == 0) continue;  // rows past N: never written
+        for (int jb = 0; jb < gpp / 16; ++jb) {
+          const int rb = G0 / 4 + hw + 4 * jb;  // 16-row block of the tile
+          float res[1][2][4];
+#pragma unroll
+          for (int j = 0; j < 2; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) res[0][j][e] = 0.f;
+          const int tr = 16 * (rb - G0 / 4);  // first row of the block within the pass
+          if (quad) {
+            for (int step = 0; step * 16 < s; ++step) res_step<1>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, true, res);
+          } else {
+            for (int step = 0; step * 16 < s; ++step) res_step<1>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, false, res);
+          }
+          // consumer thread 32 (rb / 2) + lane holds these rows as its block rb % 2
+          float4* dst = reinterpret_cast<float4*>(out + (size_t)(32 * (rb >> 1) + lane) * 8 * MT);
+#pragma unroll
+          for (int j = 0; j < MT; ++j) dst[(rb & 1) * MT + j] = make_float4(res[0][j][0], res[0][j][1], res[0][j][2], res[0][j][3]);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&res_full[slot]));
+      ++k;
+    }
+    if (++c.ch == a.n_chunks) {
+      c.ch = 0;
+      if (++c.t == a.n_tiles) {
+        c.t = 0;
+        ++c.p;
+      }
+    }
+  }
+  // no bulk copy may still be writing shared memory when the CTA exits
+  if (failed && htid == 0 && sphase > 0) mbar_wait(smem_u32(staged), (uint32_t)((sphase - 1) & 1), status);
+}
+
 // ---------------------------------------------------------------- main kernel
 
 template <int MT>  // n8 tiles of the batch: 1 for M <= 8, 2 for M <= 16
@@ -408,11 +523,17 @@ __global__ void __launch_bounds__(kMbThreads, 1)
   const int NP = gp.n_problems;
   const int u0 = gp.cta_u0[blockIdx.x], u1 = gp.cta_u0[blockIdx.x + 1];
   const int n_units = u1 - u0;
+  const MbSmem lay = mb_smem_layout(S, MT, gp.res_stage_bytes);
   uint8_t* stages = smem;
-  MbProblemArgs* tab = reinterpret_cast<MbProblemArgs*>(smem + (size_t)S * kStage);
-  uint64_t* full = reinterpret_cast<uint64_t*>(tab + kMaxProblems);  // [S] stage landed
-  uint64_t* empty = full + S;                                         // [S] consumers released it
-  int* last_fill = reinterpret_cast<int*>(empty + S);                 // [S] fills issued per stage
+  MbProblemArgs* tab = reinterpret_cast<MbProblemArgs*>(smem + lay.tab);
+  float* rslot = reinterpret_cast<float*>(smem + lay.rslot);      // [2][256][8 MT] helpers' results
+  uint8_t* rstage = smem + lay.rstage;                             // helpers' staging
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + lay.bars);   // [S] stage landed
+  uint64_t* empty = full + S;                                      // [S] consumers released it
+  uint64_t* res_full = empty + S;                                  // [2] helpers wrote the slot
+  uint64_t* res_empty = res_full + 2;                              // [2] consumers read the slot
+  uint64_t* staged = res_empty + 2;                                // helpers' bulk copies landed
+  int* last_fill = reinterpret_cast<int*>(smem + lay.last_fill);   // [S] fills issued per stage
 
   // the problem table goes to shared memory in one step (every thread one word)
   {
@@ -427,6 +548,11 @@ __global__ void __launch_bounds__(kMbThreads, 1)
       mbar_init(smem_u32(&empty[i]), kMbConsumerWarps);
       last_fill[i] = 0;
     }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&res_full[i]), kMbHelperWarps);
+      mbar_init(smem_u32(&res_empty[i]), kMbConsumerWarps);
+    }
+    mbar_init(smem_u32(staged), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   }
@@ -448,7 +574,10 @@ __global__ void __launch_bounds__(kMbThreads, 1)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
-  if (warp == kMbConsumerWarps) {
+  if (warp > kMbConsumerWarps) {
+    helper_role<MT>(tab, NP, u0, n_units, rslot, rstage, res_full, res_empty, staged, warp - kMbConsumerWarps - 1,
+                    lane, gp.status);
+  } else if (warp == kMbConsumerWarps) {
     // ---------------------------------------------------------------- producer lane
     if (lane == 0) {
       for (int i = 0; i < n_units; ++i) {
@@ -484,6 +613,8 @@ __global__ void __launch_bounds__(kMbThreads, 1)
           for (int k = 0; k < 4; ++k) acc[e][b][j][k] = res[b][j][k] = 0.f;
     uint16_t al[kMbBlocks][2] = {};
     bool need_alpha = true;
+    bool own_res = false;  // the helpers compute this tile's residual
+    int kc = 0;            // helper result slots taken so far
     UnitPos c = unit_pos(tab, NP, u0);
     for (int i = 0; i < n_units; ++i) {
       const int u = u0 + i, st = i % S;
@@ -499,19 +630,22 @@ __global__ void __launch_bounds__(kMbThreads, 1)
           }
         need_alpha = false;
       }
-      if (c.ch == 0 && a.yres) {
-        // the tile's residual (Eq. 11), added once: by the CTA that decodes its first chunk
-        const float4* src = reinterpret_cast<const float4*>(a.yres + ((size_t)c.t * 256 + tid) * 4 * kMbBlocks * MT);
+      if (c.ch == 0) {
+        // the tile's residual (Eq. 11) is added once, by the CTA that decodes its first chunk
+        own_res = a.res_mode == kMbResHelpers;
+        if (a.res_mode == kMbResPrep) {
+          const float4* src = reinterpret_cast<const float4*>(a.yres + ((size_t)c.t * 256 + tid) * 4 * kMbBlocks * MT);
 #pragma unroll
-        for (int b = 0; b < kMbBlocks; ++b)
+          for (int b = 0; b < kMbBlocks; ++b)
 #pragma unroll
-          for (int j = 0; j < MT; ++j) {
-            const float4 r4 = __ldcg(src + b * MT + j);
-            res[b][j][0] = r4.x;
-            res[b][j][1] = r4.y;
-            res[b][j][2] = r4.z;
-            res[b][j][3] = r4.w;
-          }
+            for (int j = 0; j < MT; ++j) {
+              const float4 r4 = __ldcg(src + b * MT + j);
+              res[b][j][0] = r4.x;
+              res[b][j][1] = r4.y;
+              res[b][j][2] = r4.z;
+              res[b][j][3] = r4.w;
+            }
+        }
       }
       const bool ok = mbar_wait(smem_u32(&full[st]), (uint32_t)((i / S) & 1), gp.status);
       if (!__all_sync(0xffffffffu, ok)) break;
@@ -522,6 +656,26 @@ __global__ void __launch_bounds__(kMbThreads, 1)
       // ---- tile epilogue once this CTA's part of tile c.t is done
       if (c.ch == a.n_chunks - 1 || u == u1 - 1) {
         const int t = c.t;
+        if (own_res) {
+          const int slot = kc & 1;
+          const bool rok = mbar_wait(smem_u32(&res_full[slot]), (uint32_t)((kc >> 1) & 1), gp.status);
+          if (!__all_sync(0xffffffffu, rok)) break;
+          const float4* src = reinterpret_cast<const float4*>(rslot + ((size_t)slot * 256 + tid) * 8 * MT);
+#pragma unroll
+          for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+            for (int j = 0; j < MT; ++j) {
+              const float4 r4 = src[b * MT + j];
+              res[b][j][0] += r4.x;
+              res[b][j][1] += r4.y;
+              res[b][j][2] += r4.z;
+              res[b][j][3] += r4.w;
+            }
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&res_empty[slot]));
+          ++kc;
+          own_res = false;
+        }
         // this CTA's part: alpha * acc / 2 + res (alpha scales only the ternary part)
         float part[kMbBlocks][MT][4];
 #pragma unroll
@@ -638,10 +792,8 @@ __global__ void __launch_bounds__(kMbThreads, 1)
 
 }  // namespace
 
-size_t mb_smem_bytes(int S, int M) {
-  const int mt = M <= 8 ? 1 : 2;
-  return (size_t)S * mb_stage_bytes(mt) + (size_t)kMaxProblems * sizeof(MbProblemArgs) +
-         (size_t)(2 * S) * sizeof(unsigned long long) + (size_t)kMaxStagesMb * sizeof(int) + 1024;
+size_t mb_smem_bytes(int S, int M, int res_stage_bytes) {
+  return mb_smem_layout(S, M <= 8 ? 1 : 2, res_stage_bytes).total;
 }
 
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max) {

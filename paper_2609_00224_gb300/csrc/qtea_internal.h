@@ -114,6 +114,10 @@ __host__ __device__ constexpr int mb_stage_bytes(int mt) {
 // every 256-row tile in the consumers' accumulator order, for every problem of a group in one launch.
 constexpr int kMbResEntries = 256;  // salient entries staged per pass of a residual block
 
+// How a problem's residual (Eq. 11) is computed: not at all (s = 0), by the main kernel's helper
+// warps from bulk copies, or per tile by the prep kernel.
+enum MbResMode { kMbResNone = 0, kMbResHelpers = 1, kMbResPrep = 2 };
+
 struct MbPrepProblem {
   const uint16_t* x;        // [M][K]
   const uint16_t* v;        // [K]
@@ -121,9 +125,11 @@ struct MbPrepProblem {
   const uint16_t* rvals;    // [N/4][s]
   const uint8_t* ridx;      // [N/4][ceil(s/4)]
   uint8_t* ws;              // [n_chunks][kMbChunkWsBytes]
-  float* yres;              // [n_tiles][256 threads][4 kMbBlocks MT] residual in accumulator order
-  int N, K, s, n_chunks, n_tiles;
-  int native;               // residual staged as stored (16-byte vector loads), else in passes
+  float* yres;              // kMbResPrep: [n_tiles][256 threads][4 kMbBlocks MT] residual in accumulator order
+  uint16_t* xs;             // kMbResHelpers: x at the salient columns [16][s16]
+  int N, K, s, s16, n_chunks, n_tiles;
+  int res_mode;
+  int native;               // kMbResPrep: residual staged as stored (16-byte vector loads), else in passes
   int block_begin;          // first block of this problem in the launch
 };
 
@@ -135,23 +141,29 @@ struct MbPrepGroup {
 
 constexpr int kMbBlocks = 2;                                   // 16-row blocks per consumer warp
 constexpr int kMbConsumerWarps = kMbTileRows / 16 / kMbBlocks;  // 8
+constexpr int kMbHelperWarps = 4;                              // residual of the tiles a CTA starts
 
 // One problem of a grouped low-batch launch; units (tile of 256 rows, chunk of 512 columns) of all
 // problems form one sequence split evenly over the CTAs, as in the batch-1 kernel.
 struct MbProblemArgs {
   const uint16_t* alpha;    // [N]
   const uint8_t* ws;        // the prep kernel's chunks
-  const float* yres;        // the prep kernel's residual, or null without salient columns
+  const float* yres;        // kMbResPrep: the prep kernel's residual per tile
+  const uint16_t* rvals;    // kMbResHelpers: [N/4][s], 16-byte aligned
+  const uint8_t* ridx;      // kMbResHelpers: [N/4][ceil(s/4)], 16-byte aligned
+  const uint16_t* xs;       // kMbResHelpers: the prep kernel's x at the salient columns [16][s16]
   float* y;                 // [M][N]
   float* part;              // [grid][2][256 threads][4 kMbBlocks MT] partial rows of split tiles
   unsigned* counters;       // [n_tiles][kMbConsumerWarps], zero between calls
-  int N, n_tiles, n_chunks;
+  int N, n_tiles, n_chunks, s, s16, res_mode;
+  int res_passes;           // kMbResHelpers: a tile's row groups are staged in 1, 2 or 4 passes
   long long unit_begin;
 };
 
 struct MbGroupParams {
   MbProblemArgs prob[kMaxProblems];
   int n_problems, n_stages, M;
+  int res_stage_bytes;      // the helpers' staging buffer
   int* status;              // device status word (the first layout's)
   long long total_units;
   int cta_u0[kMaxGrid + 1];
@@ -162,7 +174,29 @@ constexpr size_t kMbPartFloatsPerCta = 2 * 256 * 16;
 // Residual of one 256-row tile in accumulator order: [256 threads][16] floats.
 constexpr size_t kMbResFloatsPerTile = 256 * 16;
 
-size_t mb_smem_bytes(int S, int M);
+// Helpers' staging of one pass over a tile's residual: the values and position bytes of 64 / passes
+// row groups as stored, and x at the salient columns [16][s16].
+__host__ __device__ inline size_t mb_res_stage_bytes(int s, int passes) {
+  const size_t g = (size_t)(kMbTileRows / 4 / passes), rs = (size_t)((s + 3) / 4), s16 = (size_t)((s + 15) / 16 * 16);
+  return ((g * s * 2 + 15) & ~(size_t)15) + ((g * rs + 15) & ~(size_t)15) + 16 * s16 * 2;
+}
+
+// Shared memory of the low-batch kernel (offsets from the 1024-byte aligned base).
+struct MbSmem {
+  size_t tab, rslot, rstage, bars, last_fill, total;
+};
+__host__ __device__ inline MbSmem mb_smem_layout(int S, int mt, int res_stage_bytes) {
+  MbSmem o;
+  o.tab = (size_t)S * mb_stage_bytes(mt);
+  o.rslot = (o.tab + kMaxProblems * sizeof(MbProblemArgs) + 127) & ~(size_t)127;
+  o.rstage = (o.rslot + (size_t)2 * 256 * 8 * mt * sizeof(float) + 127) & ~(size_t)127;
+  o.bars = (o.rstage + (size_t)res_stage_bytes + 127) & ~(size_t)127;
+  o.last_fill = o.bars + (size_t)(2 * S + 5) * 8;  // full, empty [S]; res_full, res_empty [2]; staged
+  o.total = o.last_fill + (size_t)kMaxStagesMb * sizeof(int) + 1024;
+  return o;
+}
+
+size_t mb_smem_bytes(int S, int M, int res_stage_bytes);
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max);
 size_t mb_prep_smem_bytes(int s, bool native);
 cudaError_t mb_prep_configure(size_t smem_optin);
