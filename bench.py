@@ -549,8 +549,10 @@ def qtea_arm(args):
                     dstep(st)
             tdn = timed_replay(gdd) * 1e3 / nsteps
             del gq, gdd
+            lb = sum(algorithmic_bytes(g["N"], g["K"], g["sal"].numel(), M) for g in qlayers[0])
             msweep["us_per_layer"][str(M)] = {"qtea": round(tq, 2), "dense_fp16": round(tdn, 2),
-                                              "speedup": round(tdn / tq, 2)}
+                                              "speedup": round(tdn / tq, 2), "GBps": round(lb / tq / 1e3, 1),
+                                              "frac_of_measured_hbm": round(lb / tq / 1e3 / peak, 3)}
         status = max(qt.qtea_device_status(g["layout"]) for L in qlayers for g in L)
         if status:
             raise RuntimeError(f"device status {status} after the batch sweep")
