@@ -644,6 +644,35 @@ def qtea_arm(args):
     return 0
 
 
+def profile_case(args):
+    """A small fixed workload for ncu captures: the Qwen3-14B layer's seven GEMVs at batch M as one
+    grouped call, `--calls` times, then a status check. Prints one line; times nothing."""
+    import numpy as np
+    import torch
+    import paper_2609_00224_gb300 as qt
+    import synth
+    qt.load()
+
+    def f16(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
+
+    M = args.m
+    probs = []
+    for mi in range(7):
+        p = synth.config_problem(2, mi, M=M)
+        lay = qt.qtea_pack_layout(torch.from_numpy(p.T).cuda(), n_salient=p.s)
+        probs.append(dict(x=f16(p.x), layout=lay, row_scale=f16(p.alpha.reshape(-1)), col_scale=f16(p.v),
+                          salient_idx=torch.from_numpy(p.salient_idx).cuda(), residual_vals=f16(p.residual_vals),
+                          residual_idx=torch.from_numpy(p.residual_idx).cuda(),
+                          y=torch.empty((M, p.N), dtype=torch.float32, device="cuda")))
+    for _ in range(args.calls):
+        qt.qtea_gemv_grouped(probs)
+    torch.cuda.synchronize()
+    status = qt.qtea_device_status(probs[0]["layout"])
+    print(json.dumps({"profile_case": args.profile_case, "M": M, "calls": args.calls, "status": status}))
+    return 1 if status else 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -661,7 +690,13 @@ def main():
     ap.add_argument("--no-per-shape", action="store_true")
     ap.add_argument("--act-bits", type=int, choices=[16, 24], default=24,
                     help="activation precision of the timed region (24 = exact default, 16 = fast mode)")
+    ap.add_argument("--profile-case", choices=["qwen3_14b_layer"], default=None,
+                    help="run a small fixed workload for profilers instead of the benchmark")
+    ap.add_argument("--m", type=int, default=2, help="batch of --profile-case")
+    ap.add_argument("--calls", type=int, default=3, help="grouped calls of --profile-case")
     args = ap.parse_args()
+    if args.profile_case:
+        return profile_case(args)
     if args.impl == "reference":
         return reference_arm(args)
     return qtea_arm(args)
