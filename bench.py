@@ -560,52 +560,62 @@ def qtea_arm(args):
         torch.cuda.empty_cache()
 
     # ---- the Llama3-8B layer in the paper's own storage (base-3 codes, alpha and beta per 128-column
-    #      group, FP8 residual values): the seven GEMVs per step on the general kernel, rotating over
-    #      resident layers
-    paper = None
-    if not args.no_paper:
+    #      group, FP8 residual values), and with the paper's scale groups on 2-bit codes and fp16
+    #      residual values: the seven GEMVs per step as one grouped call, rotating over resident layers
+    def paper_leg(fmt, fp8):
         n_res = 4
         players = []
         for li in range(n_res):
             L = []
             for mi in range(7):
-                pp = synth.paper_problem(1, mi, layer=li)
+                pp = synth.paper_problem(1, mi, layer=li, residual_fp8=fp8)
                 f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
                 T = torch.from_numpy(pp.T).cuda()
-                lay = qt.qtea_pack_layout(T, n_salient=pp.s, group_size=128, fmt=qt.QTEA_FMT_BASE3)
-                lay.set_options(qt.QTEA_OPT_BIAS | qt.QTEA_OPT_RESIDUAL_FP8)
+                lay = qt.qtea_pack_layout(T, n_salient=pp.s, group_size=128, fmt=fmt)
+                lay.set_options(qt.QTEA_OPT_BIAS | (qt.QTEA_OPT_RESIDUAL_FP8 if fp8 else 0))
                 del T
                 sc = np.stack([pp.alpha.reshape(pp.N, -1), pp.beta.reshape(pp.N, -1)], axis=-1).reshape(-1)
+                rv = torch.from_numpy(pp.residual_vals).cuda() if fp8 else f16(pp.residual_vals)
                 L.append(dict(x=f16(pp.x), layout=lay, row_scale=f16(sc), col_scale=f16(pp.v),
-                              salient_idx=torch.from_numpy(pp.salient_idx).cuda(),
-                              residual_vals=torch.from_numpy(pp.residual_vals).cuda(),
+                              salient_idx=torch.from_numpy(pp.salient_idx).cuda(), residual_vals=rv,
                               residual_idx=torch.from_numpy(pp.residual_idx).cuda(),
                               y=torch.empty((1, pp.N), dtype=torch.float32, device="cuda")))
             players.append(L)
-        pbytes = sum(paper_algorithmic_bytes(N, K, synth.salient_count(K)) for _, N, K in synth.config_shapes(1))
+        shapes = synth.config_shapes(1)
+        if fmt == qt.QTEA_FMT_BASE3 and fp8:
+            pbytes = sum(paper_algorithmic_bytes(N, K, synth.salient_count(K)) for _, N, K in shapes)
+        else:
+            # 2-bit codes and fp16 residual values with (alpha, beta) per 128-column group
+            pbytes = sum(algorithmic_bytes(N, K, synth.salient_count(K)) + 4 * N * (-(-K // 128)) - 2 * N
+                         for _, N, K in shapes)
         nsteps = 16
         with torch.cuda.stream(stream):
-            for g in players[0]:
-                qt.qtea_gemv(g["x"], g["layout"], g["row_scale"], g["col_scale"], g["salient_idx"],
-                             g["residual_vals"], g["residual_idx"], y=g["y"], stream=stream)
+            qt.qtea_gemv_grouped(players[0], stream=stream)
         gp = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gp, stream=stream):
             for st in range(nsteps):
-                for g in players[st % n_res]:
-                    qt.qtea_gemv(g["x"], g["layout"], g["row_scale"], g["col_scale"], g["salient_idx"],
-                                 g["residual_vals"], g["residual_idx"], y=g["y"], stream=stream)
+                qt.qtea_gemv_grouped(players[st % n_res], stream=stream)
         tp = timed_replay(gp) * 1e3 / nsteps
         del gp
         status = max(qt.qtea_device_status(g["layout"]) for L in players for g in L)
         if status:
             raise RuntimeError(f"device status {status} in the paper-storage steps")
-        w = sum(N * K for _, N, K in synth.config_shapes(1))
-        paper = {"workload": "llama3_8b_layer_paper_storage", "us_per_step": round(tp, 2),
-                 "GBps": round(pbytes / (tp * 1e-6) / 1e9, 1), "bytes_per_step": pbytes,
-                 "bits_per_weight": round(8 * (pbytes - sum(2 * K + 4 * N for _, N, K in synth.config_shapes(1))) / w, 3),
-                 "kernel": "qtea_gemv_paper_kernel (general, one warp per row)", "layers_resident": n_res}
+        w = sum(N * K for _, N, K in shapes)
+        res = {"us_per_step": round(tp, 2), "GBps": round(pbytes / (tp * 1e-6) / 1e9, 1),
+               "frac_of_measured_hbm": round(pbytes / (tp * 1e-6) / 1e9 / peak, 3), "bytes_per_step": pbytes,
+               "bits_per_weight": round(8 * (pbytes - sum(2 * K + 4 * N for _, N, K in shapes)) / w, 3),
+               "layers_resident": n_res}
         del players
         torch.cuda.empty_cache()
+        return res
+
+    paper = None
+    if not args.no_paper:
+        paper = {"workload": "llama3_8b_layer_paper_storage", "M": 1,
+                 "base3_fp8": dict(paper_leg(qt.QTEA_FMT_BASE3, True),
+                                   kernel="qtea_gemv_paper_kernel (general, one warp per row)"),
+                 "2bit_fp16_residual": dict(paper_leg(qt.QTEA_FMT_2BIT, False),
+                                            kernel="qtea_gemv_mb_kernel (tensor cores, scale groups)")}
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:

@@ -179,12 +179,16 @@ struct MbGroup {
   size_t smem = 0;
   size_t prep_smem_optin = 0;
   size_t smem_optin = 0;  // the main kernel's dynamic shared memory limit
+  TensorMaps ab_maps;     // scale groups: alpha (and beta) per row and 128-column group
+  bool grp = false;       // the group's problems have scale groups (one kernel variant per launch)
 };
 
 void mb_group_reset(MbGroup& g, int M, size_t prep_smem_optin, size_t smem_optin) {
   std::memset(&g.gp, 0, sizeof(g.gp));
   std::memset(&g.pg, 0, sizeof(g.pg));
   std::memset(&g.maps, 0, sizeof(g.maps));
+  std::memset(&g.ab_maps, 0, sizeof(g.ab_maps));
+  g.grp = false;
   g.gp.M = M;
   g.pg.M = M;
   g.pg.mt = M <= 8 ? 1 : 2;
@@ -194,10 +198,31 @@ void mb_group_reset(MbGroup& g, int M, size_t prep_smem_optin, size_t smem_optin
   g.smem_optin = smem_optin;
 }
 
+// Scale groups of the low-batch kernel: row_scale as [N][G] alpha or [N][2G] (alpha, beta) fp16
+// for TMA boxes of 8 values x 256 rows; false if its address or row stride does not allow them.
+bool encode_ab_map(const qtea_layout* l, const uint16_t* row_scale, CUtensorMap* out) {
+  PFN_cuTensorMapEncodeTiled_v12000 encode = get_encode_tiled();
+  if (!encode || !aligned(row_scale, 16)) return false;
+  const int G = (l->K + 127) / 128;
+  const int cols = G * ((l->options & QTEA_OPT_BIAS) ? 2 : 1);
+  if ((cols * 2) % 16 != 0) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)l->N};
+  cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  cuuint32_t box[2] = {8, (cuuint32_t)kMbTileRows};
+  cuuint32_t estr[2] = {1, 1};
+  return encode(out, CU_TENSOR_MAP_DATA_TYPE_UINT16, 2, const_cast<uint16_t*>(row_scale), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
   if (g.gp.n_problems == kMaxProblems) return false;
   const qtea_layout* l = q.packed_ternary;
   const int k = g.gp.n_problems;
+  const bool grp = l->group_size != l->K;
+  if (k > 0 && grp != g.grp) return false;
+  if (grp && !encode_ab_map(l, q.row_scale, &g.ab_maps.m[k])) return false;
+  g.grp = grp;
   const int n_tiles = (l->N + kMbTileRows - 1) / kMbTileRows;
   const int s = l->n_salient, s16 = round_up(s, 16);
   const int mt = g.gp.M <= 8 ? 1 : 2;
@@ -210,7 +235,7 @@ bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
   int mode = s > 0 ? kMbResPrep : kMbResNone, passes = 0;
   if (s > 0 && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 16)) {
     for (int p = 1; p <= 4 && !passes; p *= 2)
-      if (mb_smem_layout(kMinStagesMb, mt, (int)mb_res_stage_bytes(s, p)).total <= g.smem_optin) passes = p;
+      if (mb_smem_layout(kMinStagesMb, mt, grp, (int)mb_res_stage_bytes(s, p)).total <= g.smem_optin) passes = p;
     if (passes) mode = kMbResHelpers;
   }
   MbPrepProblem& pp = g.pg.prob[k];
@@ -251,6 +276,7 @@ bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
   a.s16 = s16;
   a.res_mode = mode;
   a.res_passes = passes;
+  a.bias = (l->options & QTEA_OPT_BIAS) ? 1 : 0;
   a.unit_begin = g.gp.total_units;
   if (mode == kMbResHelpers) {
     const int rsb = (int)mb_res_stage_bytes(s, passes);
@@ -273,7 +299,7 @@ bool mb_group_plan(MbGroup& g, int sm_count, size_t smem_optin) {
   if (g.grid > kMaxGrid) g.grid = kMaxGrid;
   for (int b = 0; b <= g.grid; ++b) g.gp.cta_u0[b] = (int)unit_begin_of(b, g.gp.total_units, g.grid);
   for (int S = kMaxStagesMb; S >= kMinStagesMb; --S) {
-    const size_t bytes = mb_smem_bytes(S, g.gp.M, g.gp.res_stage_bytes);
+    const size_t bytes = mb_smem_bytes(S, g.gp.M, g.grp, g.gp.res_stage_bytes);
     if (bytes <= smem_optin) {
       g.gp.n_stages = S;
       g.smem = bytes;
@@ -285,13 +311,21 @@ bool mb_group_plan(MbGroup& g, int sm_count, size_t smem_optin) {
 
 int mb_group_launch(MbGroup& g, cudaStream_t st) {
   if (launch_mb_prep(g.pg, st) != cudaSuccess) return QTEA_ERR_CUDA;
-  return launch_mb(g.maps, g.gp, g.grid, g.smem, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+  return launch_mb(g.maps, g.ab_maps, g.gp, g.grp, g.grid, g.smem, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
 }
 
-bool mb_capable(const qtea_layout* l, int M) { return l->mb_ok && l->m1_ok && M >= 2 && M <= 16; }
+// The low-batch kernel serves the library's own layouts at 2 <= M <= 16 and, at any M, layouts in
+// the paper's storage with 2-bit codes, fp16 residual values, and one alpha per row or alpha (and
+// beta) per 128-column group.
+bool mb_capable(const qtea_layout* l, int M) {
+  if (!l->mb_ok || !l->m1_ok || M < 1 || M > 16) return false;
+  if (!is_paper(l)) return M >= 2;
+  if (l->format != QTEA_FMT_2BIT || (l->options & QTEA_OPT_RESIDUAL_FP8)) return false;
+  return l->group_size == 128 || !(l->options & QTEA_OPT_BIAS);
+}
 
-// Low-batch dispatch: as many consecutive problems per launch as fit; a problem the kernel cannot
-// serve goes to the generic kernel.
+// Low-batch dispatch: as many consecutive problems per launch as fit (one kernel variant per
+// launch); a problem the kernel cannot take goes to the paper-storage or the generic kernel.
 int run_mb(const qtea_gemv_problem* qs, const int* idx, int n, int M, cudaStream_t st) {
   int i = 0;
   while (i < n) {
@@ -309,7 +343,7 @@ int run_mb(const qtea_gemv_problem* qs, const int* idx, int n, int M, cudaStream
       ++taken;
     }
     if (taken == 0) {
-      int rc = launch_generic_problem(qs[idx[i]], M, st);
+      int rc = is_paper(l0) ? launch_paper_problem(qs[idx[i]], M, st) : launch_generic_problem(qs[idx[i]], M, st);
       if (rc) return rc;
       ++i;
       continue;
@@ -539,7 +573,7 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
     rc = QTEA_ERR_BAD_CODES;
   } else if (cudaMemsetAsync(l->status, 0, 2 * sizeof(int), st) != cudaSuccess) {
     rc = QTEA_ERR_CUDA;
-  } else if (format == QTEA_FMT_2BIT && group_size == K) {
+  } else if (format == QTEA_FMT_2BIT) {
     rc = plan_m1(l, prop);  // the batch-1 and low-batch kernels' resources
   }
   if (rc == QTEA_OK && cudaStreamSynchronize(st) != cudaSuccess) rc = QTEA_ERR_CUDA;
@@ -574,12 +608,12 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
       if (cudaMemsetAsync(q.y, 0, (size_t)M * l->N * sizeof(float), st) != cudaSuccess) rc = QTEA_ERR_CUDA;
       continue;
     }
-    if (is_paper(l)) {
-      rc = launch_paper_problem(q, M, st);
-    } else if (M == 1 && l->m1_ok) {
+    if (M == 1 && l->m1_ok && !is_paper(l)) {
       m1_idx[n_m1++] = i;
     } else if (mb_capable(l, M)) {
       mb_idx[n_mb++] = i;
+    } else if (is_paper(l)) {
+      rc = launch_paper_problem(q, M, st);
     } else {
       rc = launch_generic_problem(q, M, st);
     }

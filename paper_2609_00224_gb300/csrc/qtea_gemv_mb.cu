@@ -194,9 +194,9 @@ __device__ __forceinline__ void res_step(const uint16_t* rv, int rvs, const uint
 // or, for a residual of the main kernel's helpers, blocks that gather x at the salient columns
 // (xs[m][c], zero beyond s or M), 256 columns each.
 // Chunk ch's 512 columns: entry (step s, quad lane q) of the v block holds the pairs
-// (v[16W + i], v[16W + i + 8]) for i = 2(s & 3) and i + 1, W = 8q + (s >> 2); entry (step s,
+// (v[16W + i], v[16W + i + 8]) for i = 2(s & 3) and i + 1, W = 4(s >> 2) + q; entry (step s,
 // lane 4g + q) of x block j holds the same two pairs of x[8j + g]. Columns >= K and batch rows >= M
-// are zero.
+// are zero. Steps 8k .. 8k + 7 cover columns 128k .. 128k + 127 (words 8k .. 8k + 7) only.
 // Tile t: the residual of its 256 rows for every batch row, computed with the main kernel's thread
 // mapping (thread tid holds rows tr + 16b + g and + 8, batch rows 8j + 2q and + 1) and stored in
 // that order, so that each main-kernel thread reads its part with vector loads. The tile's values
@@ -346,37 +346,78 @@ __global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant
   auto pair = [](const uint16_t* row, int c) { return (uint32_t)row[c] | ((uint32_t)row[c + 8] << 16); };
   if (tid < 128) {
     const int s = tid >> 2, q = tid & 3;
-    const int base = 16 * (8 * q + (s >> 2)), i0 = 2 * (s & 3);
+    const int base = 16 * (4 * (s >> 2) + q), i0 = 2 * (s & 3);
     reinterpret_cast<uint2*>(out)[tid] = make_uint2(pair(vsm, base + i0), pair(vsm, base + i0 + 1));
   }
   for (int e = tid; e < gr.mt * 1024; e += 256) {
     const int j = e >> 10, s = (e >> 5) & 31, lane = e & 31, g = lane >> 2, q = lane & 3;
-    const int base = 16 * (8 * q + (s >> 2)), i0 = 2 * (s & 3);
+    const int base = 16 * (4 * (s >> 2) + q), i0 = 2 * (s & 3);
     const uint16_t* row = xsm[8 * j + g];
-    reinterpret_cast<uint2*>(out + kMbVBytes)[e] = make_uint2(pair(row, base + i0), pair(row, base + i0 + 1));
+    reinterpret_cast<uint2*>(out + kMbChunkHead)[e] = make_uint2(pair(row, base + i0), pair(row, base + i0 + 1));
+  }
+  {
+    // sum of x over each 128-column group k of the chunk for batch row m (the beta term of Eq. 10):
+    // four lanes per (k, m) add 32 columns each, then a fixed butterfly
+    const int k = tid >> 6, m = (tid >> 2) & 15, part = tid & 3;
+    float sxv = 0.f;
+#pragma unroll 8
+    for (int c = 0; c < 32; ++c) sxv += __half2float(__ushort_as_half(xsm[m][128 * k + 32 * part + c]));
+    sxv += __shfl_xor_sync(0xffffffffu, sxv, 1);
+    sxv += __shfl_xor_sync(0xffffffffu, sxv, 2);
+    if (part == 0) reinterpret_cast<float*>(out + kMbVBytes)[16 * k + m] = sxv;
   }
 }
 
 // ---------------------------------------------------------------- decode of one unit
 
-// The unit's 32 steps of 16 columns for the warp's 16-row blocks (rows tr + 16b + g and + 8 of the
-// stage); even steps accumulate into acc[0], odd steps into acc[1].
+// Group k of the unit done: run += alpha_k * (acc[0] + acc[1]) / 2 + beta_k * sum_k(x), acc = 0.
+// alpha and beta of row r come from the unit's scale block (8 fp16 per row: (alpha, beta) of groups
+// 0 .. 3 with beta, else alpha of groups 0 .. 7 of the chunk pair), the group sums from the chunk.
 template <int MT>
-__device__ __forceinline__ void decode_unit(const uint8_t* sb, int tr, int g, int q, int lane,
-                                            float (&acc)[2][kMbBlocks][MT][4]) {
+__device__ __forceinline__ void group_fold(const uint8_t* sb, int tr, int g, int q, int k, int ch_odd, bool bias,
+                                           float (&acc)[2][kMbBlocks][MT][4], float (&run)[kMbBlocks][MT][4]) {
+  const uint16_t* ab = reinterpret_cast<const uint16_t*>(sb + kMbCodeBytes + kMbChunkHead + MT * kMbXTileBytes);
+  const float* sx = reinterpret_cast<const float*>(sb + kMbCodeBytes + kMbVBytes) + 16 * k;
+  float2 sxm[MT];
+#pragma unroll
+  for (int j = 0; j < MT; ++j) sxm[j] = *reinterpret_cast<const float2*>(sx + 8 * j + 2 * q);
+#pragma unroll
+  for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const uint16_t* r = ab + (tr + 16 * b + 8 * h + g) * 8;
+      const float al = 0.5f * __half2float(__ushort_as_half(bias ? r[2 * k] : r[4 * ch_odd + k]));
+      const float be = bias ? __half2float(__ushort_as_half(r[2 * k + 1])) : 0.f;
+#pragma unroll
+      for (int j = 0; j < MT; ++j) {
+        run[b][j][2 * h] += al * (acc[0][b][j][2 * h] + acc[1][b][j][2 * h]) + be * sxm[j].x;
+        run[b][j][2 * h + 1] += al * (acc[0][b][j][2 * h + 1] + acc[1][b][j][2 * h + 1]) + be * sxm[j].y;
+        acc[0][b][j][2 * h] = acc[1][b][j][2 * h] = 0.f;
+        acc[0][b][j][2 * h + 1] = acc[1][b][j][2 * h + 1] = 0.f;
+      }
+    }
+}
+
+// The unit's 32 steps of 16 columns for the warp's 16-row blocks (rows tr + 16b + g and + 8 of the
+// stage); even steps accumulate into acc[0], odd steps into acc[1]. With scale groups (GRP) the
+// steps of each 128-column group k (8k .. 8k + 7) are folded into run after the group's last step:
+// run += alpha_k * acc / 2 + beta_k * sum_k(x), acc = 0 (Eq. 10 per group).
+template <int MT, bool GRP>
+__device__ __forceinline__ void decode_unit(const uint8_t* sb, int tr, int g, int q, int lane, int ch_odd, bool bias,
+                                            float (&acc)[2][kMbBlocks][MT][4], float (&run)[kMbBlocks][MT][4]) {
   const uint8_t* vblk = sb + kMbCodeBytes;
-  const uint8_t* xblk = vblk + kMbVBytes;
-  // the thread's 32 code bytes (8 words) of each of its four rows (128-byte swizzle)
+  const uint8_t* xblk = vblk + kMbChunkHead;
+  // the thread's code words 4w + q (w = 0 .. 7) of each of its rows: word 4w + q sits in 16-byte
+  // segment w of the row, stored at segment w ^ (row & 7) (128-byte swizzle); the 32 lanes of a load
+  // hit 32 different banks
   uint32_t wr[kMbBlocks][2][8];
 #pragma unroll
   for (int b = 0; b < kMbBlocks; ++b)
 #pragma unroll
     for (int h = 0; h < 2; ++h) {
-      const uint8_t* rp = sb + (size_t)(tr + 16 * b + 8 * h + g) * kChunkRowBytes;
-      const uint4 u0 = *reinterpret_cast<const uint4*>(rp + (((2 * q) ^ g) << 4));
-      const uint4 u1 = *reinterpret_cast<const uint4*>(rp + (((2 * q + 1) ^ g) << 4));
-      wr[b][h][0] = u0.x; wr[b][h][1] = u0.y; wr[b][h][2] = u0.z; wr[b][h][3] = u0.w;
-      wr[b][h][4] = u1.x; wr[b][h][5] = u1.y; wr[b][h][6] = u1.z; wr[b][h][7] = u1.w;
+      const uint8_t* rp = sb + (size_t)(tr + 16 * b + 8 * h + g) * kChunkRowBytes + 4 * q;
+#pragma unroll
+      for (int w = 0; w < 8; ++w) wr[b][h][w] = *reinterpret_cast<const uint32_t*>(rp + ((w ^ g) << 4));
     }
 #pragma unroll
   for (int w = 0; w < 8; ++w) {
@@ -408,6 +449,7 @@ __device__ __forceinline__ void decode_unit(const uint8_t* sb, int tr, int g, in
 #pragma unroll
         for (int b = 0; b < kMbBlocks; ++b) mma_16816(acc[s & 1][b][j], a[b][0], a[b][1], a[b][2], a[b][3], bx.x, bx.y);
       }
+      if (GRP && (w & 1) && tq == 3) group_fold<MT>(sb, tr, g, q, w >> 1, ch_odd, bias, acc, run);
     }
   }
 }
@@ -510,20 +552,23 @@ __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u
 
 // ---------------------------------------------------------------- main kernel
 
-template <int MT>  // n8 tiles of the batch: 1 for M <= 8, 2 for M <= 16
+// MT: n8 tiles of the batch (1 for M <= 8, 2 for M <= 16). GRP: alpha (and beta) per row and
+// 128-column group, loaded per unit by TMA, instead of one alpha per row.
+template <int MT, bool GRP>
 __global__ void __launch_bounds__(kMbThreads, 1)
-    qtea_gemv_mb_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ MbGroupParams gp) {
+    qtea_gemv_mb_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ TensorMaps ab_maps,
+                        const __grid_constant__ MbGroupParams gp) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  constexpr int kStage = mb_stage_bytes(MT);
-  constexpr uint32_t kFill = kMbCodeBytes + kMbVBytes + MT * kMbXTileBytes;
+  constexpr int kStage = mb_stage_bytes(MT, GRP);
+  constexpr uint32_t kFill = kMbCodeBytes + kMbChunkHead + MT * kMbXTileBytes + (GRP ? kMbAbBytes : 0);
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   const int S = gp.n_stages;
   const int NP = gp.n_problems;
   const int u0 = gp.cta_u0[blockIdx.x], u1 = gp.cta_u0[blockIdx.x + 1];
   const int n_units = u1 - u0;
-  const MbSmem lay = mb_smem_layout(S, MT, gp.res_stage_bytes);
+  const MbSmem lay = mb_smem_layout(S, MT, GRP, gp.res_stage_bytes);
   uint8_t* stages = smem;
   MbProblemArgs* tab = reinterpret_cast<MbProblemArgs*>(smem + lay.tab);
   float* rslot = reinterpret_cast<float*>(smem + lay.rslot);      // [2][256][8 MT] helpers' results
@@ -558,6 +603,8 @@ __global__ void __launch_bounds__(kMbThreads, 1)
   }
   if (warp == kMbConsumerWarps && lane < NP)
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.m[lane])) : "memory");
+  if (GRP && warp == kMbConsumerWarps && lane >= 16 && lane - 16 < NP)
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&ab_maps.m[lane - 16])) : "memory");
   __syncthreads();
   // the codes of the first stages are the library's and no kernel writes them: they may load before
   // the grid dependency wait; v and x in fragment order come from the prep kernel, after it
@@ -592,7 +639,13 @@ __global__ void __launch_bounds__(kMbThreads, 1)
           last_fill[st] = ph + 1;
         }
         bulk_load(smem_u32(sb + kMbCodeBytes), tab[up.p].ws + (size_t)up.ch * kMbChunkWsBytes,
-                  (uint32_t)(kMbVBytes + MT * kMbXTileBytes), bar);
+                  (uint32_t)(kMbChunkHead + MT * kMbXTileBytes), bar);
+        if (GRP) {
+          // the unit's alpha (and beta): 8 fp16 per row from column 8 ch (pairs) or 8 (ch / 2)
+          const int xa = tab[up.p].bias ? 8 * up.ch : 8 * (up.ch >> 1);
+          tma_load_2d(smem_u32(sb + kMbCodeBytes + kMbChunkHead + MT * kMbXTileBytes), &ab_maps.m[up.p], xa,
+                      up.t * kMbTileRows, bar);
+        }
       }
     }
   } else {
@@ -602,7 +655,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
     const int tid = threadIdx.x;           // consumer index
     const int grid = gridDim.x;
     const int M = gp.M;
-    float acc[2][kMbBlocks][MT][4], res[kMbBlocks][MT][4];
+    float acc[2][kMbBlocks][MT][4], res[kMbBlocks][MT][4], run[kMbBlocks][MT][4];
 #pragma unroll
     for (int e = 0; e < 2; ++e)
 #pragma unroll
@@ -610,7 +663,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
 #pragma unroll
         for (int j = 0; j < MT; ++j)
 #pragma unroll
-          for (int k = 0; k < 4; ++k) acc[e][b][j][k] = res[b][j][k] = 0.f;
+          for (int k = 0; k < 4; ++k) acc[e][b][j][k] = res[b][j][k] = run[b][j][k] = 0.f;
     uint16_t al[kMbBlocks][2] = {};
     bool need_alpha = true;
     bool own_res = false;  // the helpers compute this tile's residual
@@ -620,7 +673,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
       const int u = u0 + i, st = i % S;
       const MbProblemArgs& a = tab[c.p];
       const int tile_row = c.t * kMbTileRows + tr;
-      if (need_alpha) {  // used at the tile's end; the loads complete during the decode
+      if (!GRP && need_alpha) {  // used at the tile's end; the loads complete during the decode
 #pragma unroll
         for (int b = 0; b < kMbBlocks; ++b)
 #pragma unroll
@@ -649,7 +702,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
       }
       const bool ok = mbar_wait(smem_u32(&full[st]), (uint32_t)((i / S) & 1), gp.status);
       if (!__all_sync(0xffffffffu, ok)) break;
-      decode_unit<MT>(stages + (size_t)st * kStage, tr, g, q, lane, acc);
+      decode_unit<MT, GRP>(stages + (size_t)st * kStage, tr, g, q, lane, c.ch & 1, a.bias != 0, acc, run);
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
 
@@ -676,17 +729,26 @@ __global__ void __launch_bounds__(kMbThreads, 1)
           ++kc;
           own_res = false;
         }
-        // this CTA's part: alpha * acc / 2 + res (alpha scales only the ternary part)
+        // this CTA's part: alpha * acc / 2 + res (alpha scales only the ternary part), or with scale
+        // groups the folded sum
         float part[kMbBlocks][MT][4];
 #pragma unroll
         for (int b = 0; b < kMbBlocks; ++b) {
-          const float fa0 = 0.5f * h2f(al[b][0]), fa1 = 0.5f * h2f(al[b][1]);
+          const float fa0 = GRP ? 0.f : 0.5f * h2f(al[b][0]), fa1 = GRP ? 0.f : 0.5f * h2f(al[b][1]);
 #pragma unroll
           for (int j = 0; j < MT; ++j) {
-            part[b][j][0] = fa0 * (acc[0][b][j][0] + acc[1][b][j][0]) + res[b][j][0];
-            part[b][j][1] = fa0 * (acc[0][b][j][1] + acc[1][b][j][1]) + res[b][j][1];
-            part[b][j][2] = fa1 * (acc[0][b][j][2] + acc[1][b][j][2]) + res[b][j][2];
-            part[b][j][3] = fa1 * (acc[0][b][j][3] + acc[1][b][j][3]) + res[b][j][3];
+            if (GRP) {
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                part[b][j][e] = run[b][j][e] + res[b][j][e];
+                run[b][j][e] = 0.f;
+              }
+            } else {
+              part[b][j][0] = fa0 * (acc[0][b][j][0] + acc[1][b][j][0]) + res[b][j][0];
+              part[b][j][1] = fa0 * (acc[0][b][j][1] + acc[1][b][j][1]) + res[b][j][1];
+              part[b][j][2] = fa1 * (acc[0][b][j][2] + acc[1][b][j][2]) + res[b][j][2];
+              part[b][j][3] = fa1 * (acc[0][b][j][3] + acc[1][b][j][3]) + res[b][j][3];
+            }
           }
         }
         const long long A = a.unit_begin + (long long)t * a.n_chunks, B = A + a.n_chunks;
@@ -792,27 +854,33 @@ __global__ void __launch_bounds__(kMbThreads, 1)
 
 }  // namespace
 
-size_t mb_smem_bytes(int S, int M, int res_stage_bytes) {
-  return mb_smem_layout(S, M <= 8 ? 1 : 2, res_stage_bytes).total;
+size_t mb_smem_bytes(int S, int M, bool grp, int res_stage_bytes) {
+  return mb_smem_layout(S, M <= 8 ? 1 : 2, grp, res_stage_bytes).total;
 }
 
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max) {
-  cudaFuncAttributes a1, a2;
-  cudaError_t e = cudaFuncGetAttributes(&a1, qtea_gemv_mb_kernel<1>);
-  if (e != cudaSuccess) return e;
-  e = cudaFuncGetAttributes(&a2, qtea_gemv_mb_kernel<2>);
-  if (e != cudaSuccess) return e;
-  const size_t st = a1.sharedSizeBytes > a2.sharedSizeBytes ? a1.sharedSizeBytes : a2.sharedSizeBytes;
+  cudaFuncAttributes a[4];
+  cudaError_t e;
+  if ((e = cudaFuncGetAttributes(&a[0], qtea_gemv_mb_kernel<1, false>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&a[1], qtea_gemv_mb_kernel<2, false>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&a[2], qtea_gemv_mb_kernel<1, true>)) != cudaSuccess) return e;
+  if ((e = cudaFuncGetAttributes(&a[3], qtea_gemv_mb_kernel<2, true>)) != cudaSuccess) return e;
+  size_t st = 0;
+  for (int i = 0; i < 4; ++i) st = a[i].sharedSizeBytes > st ? a[i].sharedSizeBytes : st;
   const size_t dyn = smem_optin > st ? smem_optin - st : 0;
   *dyn_max = dyn;
-  e = cudaFuncSetAttribute(qtea_gemv_mb_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(qtea_gemv_mb_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  if ((e = cudaFuncSetAttribute(qtea_gemv_mb_kernel<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn)) !=
+      cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(qtea_gemv_mb_kernel<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn)) !=
+      cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(qtea_gemv_mb_kernel<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn)) !=
+      cudaSuccess)
+    return e;
+  return cudaFuncSetAttribute(qtea_gemv_mb_kernel<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
 }
 
-// Both launches use programmatic stream serialisation: the prep kernel starts while the previous
-// kernel on the stream drains, and the main kernel while the prep kernel runs; each waits
-// (griddepcontrol.wait) before it touches memory that an earlier kernel writes.
 size_t mb_prep_smem_bytes(int s, bool native) {
   const size_t E = native ? (size_t)s : (size_t)kMbResEntries;
   const size_t ris = native ? (size_t)((s + 3) / 4) : (size_t)kMbResEntries / 4;
@@ -841,7 +909,8 @@ cudaError_t launch_mb_prep(const MbPrepGroup& g, cudaStream_t st) {
   return cudaLaunchKernelEx(&cfg, qtea_mb_prep_kernel, g);
 }
 
-cudaError_t launch_mb(const TensorMaps& maps, const MbGroupParams& p, int grid, size_t smem, cudaStream_t st) {
+cudaError_t launch_mb(const TensorMaps& maps, const TensorMaps& ab_maps, const MbGroupParams& p, bool grp, int grid,
+                      size_t smem, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(kMbThreads);
@@ -852,8 +921,12 @@ cudaError_t launch_mb(const TensorMaps& maps, const MbGroupParams& p, int grid, 
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  if (p.M <= 8) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1>, maps, p);
-  return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2>, maps, p);
+  if (grp) {
+    if (p.M <= 8) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, true>, maps, ab_maps, p);
+    return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2, true>, maps, ab_maps, p);
+  }
+  if (p.M <= 8) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, false>, maps, ab_maps, p);
+  return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2, false>, maps, ab_maps, p);
 }
 
 }  // namespace qtea

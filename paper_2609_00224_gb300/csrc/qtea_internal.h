@@ -101,13 +101,18 @@ constexpr int kMaxStagesMb = 6;
 constexpr int kMinStagesMb = 2;
 constexpr int kMbTileRows = 256;                               // rows of a unit (one TMA box)
 constexpr int kMbVBytes = 1024;                                // v of a chunk in fragment order
+constexpr int kMbSxBytes = 256;                                // sum of x per 128-column group and batch row [4][16] fp32
+constexpr int kMbChunkHead = kMbVBytes + kMbSxBytes;           // the x blocks start here
 constexpr int kMbXTileBytes = 8192;                            // x of a chunk, 8 batch rows, fragment order
-constexpr int kMbChunkWsBytes = kMbVBytes + 2 * kMbXTileBytes; // 17408 per 512-column chunk
+constexpr int kMbChunkWsBytes = kMbChunkHead + 2 * kMbXTileBytes;  // 17664 per 512-column chunk
+constexpr int kMbAbBytes = 256 * 16;                           // alpha (and beta) of a unit's rows, 8 fp16 per row
 
-// One shared-memory stage of the low-batch kernel: codes [256 rows][128 bytes], the chunk's v block
-// and MT x blocks, rounded to 1024 bytes (the 128-byte swizzle of the next stage's codes).
-__host__ __device__ constexpr int mb_stage_bytes(int mt) {
-  return (kMbTileRows * kChunkRowBytes + kMbVBytes + mt * kMbXTileBytes + 1023) / 1024 * 1024;
+// One shared-memory stage of the low-batch kernel: codes [256 rows][128 bytes], the chunk's v block,
+// group sums of x and MT x blocks, with scale groups the unit's alpha (and beta), rounded to 1024
+// bytes (the 128-byte swizzle of the next stage's codes).
+__host__ __device__ constexpr int mb_stage_bytes(int mt, bool grp) {
+  return (kMbTileRows * kChunkRowBytes + kMbChunkHead + mt * kMbXTileBytes + (grp ? kMbAbBytes : 0) + 1023) / 1024 *
+         1024;
 }
 
 // Prep kernel: v and x of every 512-column chunk in fragment order, and the residual (Eq. 11) of
@@ -157,6 +162,7 @@ struct MbProblemArgs {
   unsigned* counters;       // [n_tiles][kMbConsumerWarps], zero between calls
   int N, n_tiles, n_chunks, s, s16, res_mode;
   int res_passes;           // kMbResHelpers: a tile's row groups are staged in 1, 2 or 4 passes
+  int bias;                 // scale groups: row_scale holds (alpha, beta) pairs
   long long unit_begin;
 };
 
@@ -185,9 +191,9 @@ __host__ __device__ inline size_t mb_res_stage_bytes(int s, int passes) {
 struct MbSmem {
   size_t tab, rslot, rstage, bars, last_fill, total;
 };
-__host__ __device__ inline MbSmem mb_smem_layout(int S, int mt, int res_stage_bytes) {
+__host__ __device__ inline MbSmem mb_smem_layout(int S, int mt, bool grp, int res_stage_bytes) {
   MbSmem o;
-  o.tab = (size_t)S * mb_stage_bytes(mt);
+  o.tab = (size_t)S * mb_stage_bytes(mt, grp);
   o.rslot = (o.tab + kMaxProblems * sizeof(MbProblemArgs) + 127) & ~(size_t)127;
   o.rstage = (o.rslot + (size_t)2 * 256 * 8 * mt * sizeof(float) + 127) & ~(size_t)127;
   o.bars = (o.rstage + (size_t)res_stage_bytes + 127) & ~(size_t)127;
@@ -196,12 +202,15 @@ __host__ __device__ inline MbSmem mb_smem_layout(int S, int mt, int res_stage_by
   return o;
 }
 
-size_t mb_smem_bytes(int S, int M, int res_stage_bytes);
+size_t mb_smem_bytes(int S, int M, bool grp, int res_stage_bytes);
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max);
 size_t mb_prep_smem_bytes(int s, bool native);
 cudaError_t mb_prep_configure(size_t smem_optin);
 cudaError_t launch_mb_prep(const MbPrepGroup& g, cudaStream_t st);
-cudaError_t launch_mb(const TensorMaps& maps, const MbGroupParams& p, int grid, size_t smem, cudaStream_t st);
+// Scale groups (grp): alpha, or (alpha, beta) pairs, per row and 128-column group, loaded per unit
+// by TMA through `ab_maps` (row_scale as [N][G] or [N][2G] fp16, box 8 x 256).
+cudaError_t launch_mb(const TensorMaps& maps, const TensorMaps& ab_maps, const MbGroupParams& p, bool grp, int grid,
+                      size_t smem, cudaStream_t st);
 
 // ---------------------------------------------------------------- generic kernel (any M)
 struct GenericParams {

@@ -230,15 +230,18 @@ def config_problem(config: int, matrix: int, M: Optional[int] = None, layer: int
 PAPER_FORMAT = dict(group_size=128, beta_std=0.002, residual_fp8=True)
 
 
-def paper_problem(config: int, matrix: int, M: Optional[int] = None, layer: int = 0) -> Problem:
-    """config_problem's operands in the paper's storage (same seed, hence the same codes, x and v)."""
+def paper_problem(config: int, matrix: int, M: Optional[int] = None, layer: int = 0,
+                  residual_fp8: bool = True) -> Problem:
+    """config_problem's operands in the paper's storage (same seed, hence the same codes, x and v);
+    residual_fp8=False keeps fp16 residual values with the paper's scale groups."""
     cfg = CONFIGS[config]
     name, N, K = cfg["shapes"][matrix]
     s = cfg.get("fixed_s") or salient_count(K)
     M = cfg["M"][0] if M is None else M
     p_neg, p_zero = cfg["p"]
+    fmt = dict(PAPER_FORMAT, residual_fp8=residual_fp8)
     return make_problem(f"{cfg['name']}/{name}/paper_format", N, K, M, s, config_seed(config, layer, matrix), p_neg,
-                        p_zero, "normal", cfg["residual_scale"], **PAPER_FORMAT)
+                        p_zero, "normal", cfg["residual_scale"], **fmt)
 
 
 def config_shapes(config: int) -> List[Tuple[str, int, int]]:

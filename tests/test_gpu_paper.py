@@ -127,3 +127,42 @@ def test_paper_storage_llama3_8b_layer(qt, matrix, M):
     rows = np.sort(np.random.default_rng(matrix).choice(p.N, size=48, replace=False)).astype(np.int32)
     y_ref, b = reference(p, True, rows=rows)
     assert_within(y[:, rows], y_ref, b, p.name)
+
+
+@pytest.mark.parametrize("bias", [0, 1])
+@pytest.mark.parametrize("N,K,s", [(512, 2048, 24), (516, 3072, 40), (1024, 1024, 0), (260, 1536, 7)])
+def test_group_scales_through_the_tensor_core_kernel(qt, N, K, s, bias):
+    """2-bit codes with alpha (and beta) per 128-column group, row_scale rows a multiple of 16 bytes
+    (the shapes the tensor-core kernel takes): batch 1, 5 and 16, several tiles, ragged N, s not a
+    multiple of 4."""
+    p = synth.make_problem("t", N, K, 16, s, seed=N + K + s + 7 * bias, group_size=128,
+                           beta_std=0.002 if bias else 0.0)
+    for M in (1, 5, 16):
+        y, _ = run_paper(qt, p, qt.QTEA_FMT_2BIT, bias, M=M)
+        y_ref, b = reference(p, bias, M=M)
+        assert_within(y, y_ref, b, f"N {N} K {K} s {s} bias {bias} M {M}")
+
+
+def test_group_scales_llama3_8b_layer_2bit(qt):
+    """The Llama3-8B layer with 2-bit codes, alpha and beta per 128-column group and fp16 residual, at
+    batch 4, grouped in one call, on sampled rows."""
+    ps = [synth.make_problem("g", N, K, 4, s, seed=3000 + m, group_size=128, beta_std=0.002)
+          for m, (N, K, s) in enumerate([(4096, 4096, 120), (1024, 4096, 120), (14336, 4096, 120),
+                                         (4096, 14336, 432)])]
+    probs, lays = [], []
+    for p in ps:
+        lay = qt.qtea_pack_layout(dev(p.T), n_salient=p.s, group_size=128, fmt=qt.QTEA_FMT_2BIT)
+        lay.set_options(qt.QTEA_OPT_BIAS)
+        lays.append(lay)
+        probs.append(dict(x=dev(p.x.view(np.int16), torch.float16), layout=lay,
+                          row_scale=dev(scales(p, True).view(np.int16), torch.float16),
+                          col_scale=dev(p.v.view(np.int16), torch.float16), salient_idx=dev(p.salient_idx),
+                          residual_vals=dev(p.residual_vals.view(np.int16), torch.float16),
+                          residual_idx=dev(p.residual_idx)))
+    ys = qt.qtea_gemv_grouped(probs)
+    torch.cuda.synchronize()
+    assert qt.qtea_device_status(lays[0]) == 0
+    for m, (p, y) in enumerate(zip(ps, ys)):
+        rows = np.sort(np.random.default_rng(m).choice(p.N, size=32, replace=False)).astype(np.int32)
+        y_ref, b = reference(p, True, rows=rows)
+        assert_within(y.cpu().numpy().astype(np.float64)[:, rows], y_ref, b, f"{p.N}x{p.K}")
