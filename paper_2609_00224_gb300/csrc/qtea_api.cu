@@ -232,12 +232,14 @@ bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
                        : nullptr;
   // residual by the main kernel's helpers when the caller's arrays allow bulk copies and a pass over a
   // half or quarter of a tile's row groups fits beside two code stages; else by the prep kernel
+  const bool fp8 = (l->options & QTEA_OPT_RESIDUAL_FP8) != 0;
   int mode = s > 0 ? kMbResPrep : kMbResNone, passes = 0;
   if (s > 0 && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 16)) {
     for (int p = 1; p <= 4 && !passes; p *= 2)
-      if (mb_smem_layout(kMinStagesMb, mt, grp, (int)mb_res_stage_bytes(s, p)).total <= g.smem_optin) passes = p;
+      if (mb_smem_layout(kMinStagesMb, mt, grp, (int)mb_res_stage_bytes(s, p, fp8)).total <= g.smem_optin) passes = p;
     if (passes) mode = kMbResHelpers;
   }
+  if (fp8 && mode == kMbResPrep) return false;  // FP8 values only through the helpers
   MbPrepProblem& pp = g.pg.prob[k];
   pp.x = q.x;
   pp.v = q.col_scale;
@@ -277,9 +279,10 @@ bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
   a.res_mode = mode;
   a.res_passes = passes;
   a.bias = (l->options & QTEA_OPT_BIAS) ? 1 : 0;
+  a.fp8 = fp8 ? 1 : 0;
   a.unit_begin = g.gp.total_units;
   if (mode == kMbResHelpers) {
-    const int rsb = (int)mb_res_stage_bytes(s, passes);
+    const int rsb = (int)mb_res_stage_bytes(s, passes, fp8);
     if (rsb > g.gp.res_stage_bytes) g.gp.res_stage_bytes = rsb;
   }
   std::memcpy(&g.maps.m[k], &l->tmap, sizeof(CUtensorMap));
@@ -315,12 +318,12 @@ int mb_group_launch(MbGroup& g, cudaStream_t st) {
 }
 
 // The low-batch kernel serves the library's own layouts at 2 <= M <= 16 and, at any M, layouts in
-// the paper's storage with 2-bit codes, fp16 residual values, and one alpha per row or alpha (and
-// beta) per 128-column group.
+// the paper's storage with 2-bit codes, fp16 or FP8 residual values, and one alpha per row or alpha
+// (and beta) per 128-column group.
 bool mb_capable(const qtea_layout* l, int M) {
   if (!l->mb_ok || !l->m1_ok || M < 1 || M > 16) return false;
   if (!is_paper(l)) return M >= 2;
-  if (l->format != QTEA_FMT_2BIT || (l->options & QTEA_OPT_RESIDUAL_FP8)) return false;
+  if (l->format != QTEA_FMT_2BIT) return false;
   return l->group_size == 128 || !(l->options & QTEA_OPT_BIAS);
 }
 

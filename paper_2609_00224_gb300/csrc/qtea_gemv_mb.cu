@@ -147,10 +147,24 @@ __device__ __forceinline__ UnitPos unit_pos(const MbProblemArgs* tab, int n_prob
 // come from the staged tile: rv [64 groups][rvs] fp16, ri [64][ris] position bytes (entry e of a
 // group in bits 2(e % 4) of byte e / 4), xr [16 batch rows][xrs] fp16 (zero past the valid
 // entries); only entries below ne count.
-template <int NB>
-__device__ __forceinline__ void res_step(const uint16_t* rv, int rvs, const uint8_t* ri, int ris, const uint16_t* xr,
+// FP8 E4M3 (bias 7, subnormals m * 2^-9, NaN at S.1111.111, no infinity) as fp16 bits; every value
+// is exactly representable in fp16.
+__device__ __forceinline__ uint32_t e4m3_to_f16_bits(uint32_t b) {
+  const uint32_t e = (b >> 3) & 15u, m = b & 7u;
+  uint32_t mag;
+  if (e == 0u) mag = __half_as_ushort(__float2half_rn((float)m * 0.001953125f));  // m * 2^-9, exact
+  else if (e == 15u && m == 7u) mag = 0x7e00u;
+  else mag = ((e + 8u) << 10) | (m << 7);
+  return ((b & 0x80u) << 8) | mag;
+}
+
+// FP8: rv holds one E4M3 byte per entry (row stride rvs bytes), converted to fp16 exactly.
+template <int NB, bool FP8 = false>
+__device__ __forceinline__ void res_step(const void* rv_, int rvs, const uint8_t* ri, int ris, const uint16_t* xr,
                                          int xrs, int ne, int step, int tr, int g, int q, int mt, bool quad_loads,
                                          float (&res)[NB][2][4]) {
+  const uint16_t* rv = static_cast<const uint16_t*>(rv_);
+  const uint8_t* rv8 = static_cast<const uint8_t*>(rv_);
   const int e0 = step * 16 + 4 * q;
   const uint32_t pos = (uint32_t)(g & 3);  // row & 3 for every row of the thread
   uint2 xb[2];
@@ -167,7 +181,17 @@ __device__ __forceinline__ void res_step(const uint16_t* rv, int rvs, const uint
       const uint32_t d = (uint32_t)ri[gl * ris + (e0 >> 2)] ^ (pos * 0x55u);
       const uint32_t nz = (d | (d >> 1)) & 0x55u;
       uint32_t lo, hi;
-      if (quad_loads) {  // the four values in one 8-byte load (rvs % 4 == 0, e0 + 3 < ne or zero)
+      if (FP8) {
+        uint32_t q4 = 0;  // the four E4M3 bytes
+        if (quad_loads) {  // one 4-byte load (rvs % 4 == 0)
+          if (e0 < ne) q4 = *reinterpret_cast<const uint32_t*>(rv8 + gl * rvs + e0);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) q4 |= (e0 + k < ne ? (uint32_t)rv8[gl * rvs + e0 + k] : 0u) << (8 * k);
+        }
+        lo = e4m3_to_f16_bits(q4 & 0xffu) | (e4m3_to_f16_bits((q4 >> 8) & 0xffu) << 16);
+        hi = e4m3_to_f16_bits((q4 >> 16) & 0xffu) | (e4m3_to_f16_bits(q4 >> 24) << 16);
+      } else if (quad_loads) {  // the four values in one 8-byte load (rvs % 4 == 0, e0 + 3 < ne or zero)
         uint2 v = make_uint2(0, 0);
         if (e0 < ne) v = *reinterpret_cast<const uint2*>(rv + gl * rvs + e0);
         lo = v.x;
@@ -482,8 +506,9 @@ __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u
       const int s = a.s, rs = (s + 3) >> 2, s16 = a.s16;
       const int passes = a.res_passes, gpp = (kMbTileRows / 4) / passes;
       const int g0 = c.t * (kMbTileRows / 4), ng_tile = min(kMbTileRows / 4, a.N / 4 - g0);
-      uint16_t* rv = reinterpret_cast<uint16_t*>(rstage);
-      uint8_t* ri = rstage + (((size_t)gpp * s * 2 + 15) & ~(size_t)15);
+      const int es = a.fp8 ? 1 : 2;  // bytes per residual value
+      uint8_t* rv = rstage;
+      uint8_t* ri = rstage + (((size_t)gpp * s * es + 15) & ~(size_t)15);
       uint16_t* xr = reinterpret_cast<uint16_t*>(ri + (((size_t)gpp * rs + 15) & ~(size_t)15));
       float* out = rslot + (size_t)slot * 256 * 8 * MT;
       if (k >= 2 && !mbar_wait(smem_u32(&res_empty[slot]), (uint32_t)(((k >> 1) - 1) & 1), status)) failed = true;
@@ -492,8 +517,9 @@ __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u
         const int G0 = pass * gpp;
         const int ng = max(0, min(gpp, ng_tile - G0));
         helpers_sync();  // every helper is done with the staging buffer
-        const size_t vb = (size_t)ng * s * 2, ib = (size_t)ng * rs;
-        const size_t vsrc = (size_t)(g0 + G0) * s, isrc = (size_t)(g0 + G0) * rs;
+        const size_t vb = (size_t)ng * s * es, ib = (size_t)ng * rs;
+        const size_t vsrc = (size_t)(g0 + G0) * s * es, isrc = (size_t)(g0 + G0) * rs;  // bytes
+        const uint8_t* rvals = reinterpret_cast<const uint8_t*>(a.rvals);
         if (htid == 0) {
           const uint32_t vbb = (uint32_t)(vb & ~(size_t)15), ibb = (uint32_t)(ib & ~(size_t)15);
           const uint32_t xbb = pass == 0 ? (uint32_t)(32 * s16) : 0u;
@@ -501,14 +527,14 @@ __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u
           // the helpers' reads of the previous pass (generic proxy) before the copies (async proxy)
           asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
           mbar_arrive_expect_tx(bar, vbb + ibb + xbb);
-          if (vbb) bulk_load(smem_u32(rv), a.rvals + vsrc, vbb, bar);
+          if (vbb) bulk_load(smem_u32(rv), rvals + vsrc, vbb, bar);
           if (ibb) bulk_load(smem_u32(ri), a.ridx + isrc, ibb, bar);
           if (xbb) bulk_load(smem_u32(xr), a.xs, xbb, bar);
         }
         {
-          const int vt = (int)((vb & 15) >> 1), it = (int)(ib & 15);
-          const size_t v0 = (vb & ~(size_t)15) >> 1, i0 = ib & ~(size_t)15;
-          if (htid < vt) rv[v0 + htid] = __ldg(a.rvals + vsrc + v0 + htid);
+          const int vt = (int)(vb & 15), it = (int)(ib & 15);  // tail bytes
+          const size_t v0 = vb & ~(size_t)15, i0 = ib & ~(size_t)15;
+          if (htid < vt) rv[v0 + htid] = __ldg(rvals + vsrc + v0 + htid);
           if (htid >= 32 && htid - 32 < it) ri[i0 + htid - 32] = __ldg(a.ridx + isrc + i0 + htid - 32);
         }
         if (!mbar_wait(smem_u32(staged), (uint32_t)(sphase & 1), status)) failed = true;
@@ -523,7 +549,10 @@ __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u
 #pragma unroll
             for (int e = 0; e < 4; ++e) res[0][j][e] = 0.f;
           const int tr = 16 * (rb - G0 / 4);  // first row of the block within the pass
-          if (quad) {
+          if (a.fp8) {
+            for (int step = 0; step * 16 < s; ++step)
+              res_step<1, true>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, quad, res);
+          } else if (quad) {
             for (int step = 0; step * 16 < s; ++step) res_step<1>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, true, res);
           } else {
             for (int step = 0; step * 16 < s; ++step) res_step<1>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, false, res);

@@ -163,6 +163,7 @@ struct MbProblemArgs {
   int N, n_tiles, n_chunks, s, s16, res_mode;
   int res_passes;           // kMbResHelpers: a tile's row groups are staged in 1, 2 or 4 passes
   int bias;                 // scale groups: row_scale holds (alpha, beta) pairs
+  int fp8;                  // kMbResHelpers: residual values in FP8 E4M3 (one byte each)
   long long unit_begin;
 };
 
@@ -180,11 +181,11 @@ constexpr size_t kMbPartFloatsPerCta = 2 * 256 * 16;
 // Residual of one 256-row tile in accumulator order: [256 threads][16] floats.
 constexpr size_t kMbResFloatsPerTile = 256 * 16;
 
-// Helpers' staging of one pass over a tile's residual: the values and position bytes of 64 / passes
-// row groups as stored, and x at the salient columns [16][s16].
-__host__ __device__ inline size_t mb_res_stage_bytes(int s, int passes) {
+// Helpers' staging of one pass over a tile's residual: the values (2 bytes each, or 1 in FP8) and
+// position bytes of 64 / passes row groups as stored, and x at the salient columns [16][s16].
+__host__ __device__ inline size_t mb_res_stage_bytes(int s, int passes, bool fp8) {
   const size_t g = (size_t)(kMbTileRows / 4 / passes), rs = (size_t)((s + 3) / 4), s16 = (size_t)((s + 15) / 16 * 16);
-  return ((g * s * 2 + 15) & ~(size_t)15) + ((g * rs + 15) & ~(size_t)15) + 16 * s16 * 2;
+  return ((g * s * (fp8 ? 1 : 2) + 15) & ~(size_t)15) + ((g * rs + 15) & ~(size_t)15) + 16 * s16 * 2;
 }
 
 // Shared memory of the low-batch kernel (offsets from the 1024-byte aligned base).

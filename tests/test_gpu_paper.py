@@ -129,18 +129,29 @@ def test_paper_storage_llama3_8b_layer(qt, matrix, M):
     assert_within(y[:, rows], y_ref, b, p.name)
 
 
+@pytest.mark.parametrize("fp8", [0, 1])
 @pytest.mark.parametrize("bias", [0, 1])
 @pytest.mark.parametrize("N,K,s", [(512, 2048, 24), (516, 3072, 40), (1024, 1024, 0), (260, 1536, 7)])
-def test_group_scales_through_the_tensor_core_kernel(qt, N, K, s, bias):
-    """2-bit codes with alpha (and beta) per 128-column group, row_scale rows a multiple of 16 bytes
-    (the shapes the tensor-core kernel takes): batch 1, 5 and 16, several tiles, ragged N, s not a
-    multiple of 4."""
-    p = synth.make_problem("t", N, K, 16, s, seed=N + K + s + 7 * bias, group_size=128,
-                           beta_std=0.002 if bias else 0.0)
+def test_group_scales_through_the_tensor_core_kernel(qt, N, K, s, bias, fp8):
+    """2-bit codes with alpha (and beta) per 128-column group, fp16 or FP8 residual values, row_scale
+    rows a multiple of 16 bytes (the shapes the tensor-core kernel takes): batch 1, 5 and 16, several
+    tiles, ragged N, s not a multiple of 4 (byte-wise residual loads and tails)."""
+    p = synth.make_problem("t", N, K, 16, s, seed=N + K + s + 7 * bias + 13 * fp8, group_size=128,
+                           beta_std=0.002 if bias else 0.0, residual_fp8=bool(fp8))
     for M in (1, 5, 16):
         y, _ = run_paper(qt, p, qt.QTEA_FMT_2BIT, bias, M=M)
         y_ref, b = reference(p, bias, M=M)
-        assert_within(y, y_ref, b, f"N {N} K {K} s {s} bias {bias} M {M}")
+        assert_within(y, y_ref, b, f"N {N} K {K} s {s} bias {bias} fp8 {fp8} M {M}")
+
+
+@pytest.mark.parametrize("M", [1, 4, 16])
+def test_fp8_residual_one_alpha_per_row_tensor_core_kernel(qt, M):
+    """FP8 E4M3 residual with one alpha per row (the tensor-core kernel's helpers convert every E4M3
+    value exactly), dense salient set, ragged N."""
+    p = synth.make_problem("t", 1028, 2048, 16, 200, seed=77 + M, residual_fp8=True)
+    y, _ = run_paper(qt, p, qt.QTEA_FMT_2BIT, False, M=M)
+    y_ref, b = reference(p, False, M=M)
+    assert_within(y, y_ref, b, f"fp8 M {M}")
 
 
 def test_group_scales_llama3_8b_layer_2bit(qt):
