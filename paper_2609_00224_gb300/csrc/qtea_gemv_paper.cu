@@ -102,17 +102,33 @@ __global__ void __launch_bounds__(kPaperWarps * 32) qtea_gemv_paper_kernel(const
     for (int m = 0; m < MB; ++m) acc[m] += al * tvx[m] + be * sx[m];
   }
   if (p.s > 0) {
+    // lane takes entries lane, lane + 32, ...; four at a time, with the position bytes, salient
+    // columns and values of all four loaded before any is used, then their x
     const int q = o >> 2, pos = o & 3, rs = (p.s + 3) / 4;
-    for (int c = lane; c < p.s; c += 32) {
-      if (((p.ridx[(size_t)q * rs + (c >> 2)] >> (2 * (c & 3))) & 3) != pos) continue;
-      int j = p.sal[c];
-      j = j < 0 ? 0 : (j >= p.K ? p.K - 1 : j);
-      const size_t e = (size_t)q * p.s + c;
-      const float r = p.residual_fp8 ? e4m3_to_float(reinterpret_cast<const uint8_t*>(p.rvals)[e])
-                                     : h2f(reinterpret_cast<const uint16_t*>(p.rvals)[e]);
+    for (int c0 = lane; c0 < p.s; c0 += 128) {
+      uint32_t pb[4];
+      int jj[4];
+      float r[4];
 #pragma unroll
-      for (int m = 0; m < MB; ++m)
-        if (m < M) res[m] += r * h2f(p.x[(size_t)m * p.K + j]);
+      for (int k = 0; k < 4; ++k) {
+        const int c = c0 + 32 * k;
+        const bool in = c < p.s;
+        pb[k] = in ? __ldg(p.ridx + (size_t)q * rs + (c >> 2)) : 0u;
+        jj[k] = in ? __ldg(p.sal + c) : 0;
+        const size_t e = (size_t)q * p.s + c;
+        r[k] = !in ? 0.f
+                   : p.residual_fp8 ? e4m3_to_float(__ldg(reinterpret_cast<const uint8_t*>(p.rvals) + e))
+                                    : h2f(__ldg(reinterpret_cast<const uint16_t*>(p.rvals) + e));
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int c = c0 + 32 * k;
+        if (c >= p.s || ((pb[k] >> (2 * (c & 3))) & 3u) != (uint32_t)pos) continue;
+        const int j = jj[k] < 0 ? 0 : (jj[k] >= p.K ? p.K - 1 : jj[k]);
+#pragma unroll
+        for (int m = 0; m < MB; ++m)
+          if (m < M) res[m] += r[k] * h2f(__ldg(p.x + (size_t)m * p.K + j));
+      }
     }
   }
 #pragma unroll
