@@ -177,3 +177,32 @@ def test_group_scales_llama3_8b_layer_2bit(qt):
         rows = np.sort(np.random.default_rng(m).choice(p.N, size=32, replace=False)).astype(np.int32)
         y_ref, b = reference(p, True, rows=rows)
         assert_within(y.cpu().numpy().astype(np.float64)[:, rows], y_ref, b, f"{p.N}x{p.K}")
+
+
+@pytest.mark.parametrize("M", [1, 3, 16])
+def test_grouped_call_mixing_storage_formats(qt, M):
+    """One grouped call over the library's own layouts, 2-bit layouts with scale groups (one kernel
+    variant per launch, so the call splits), an FP8 residual and a base-3 layout (the general
+    kernel): every y against the oracle."""
+    specs = [  # (N, K, s, fmt, group, bias, fp8)
+        (512, 2048, 24, 0, 0, 0, 0), (516, 2048, 16, 0, 128, 1, 0), (256, 1024, 8, 0, 0, 0, 0),
+        (260, 3072, 12, 0, 128, 0, 1), (128, 1024, 8, 1, 128, 1, 1), (64, 300, 4, 0, 0, 0, 1)]
+    probs, items = [], []
+    for i, (N, K, s, fmt, group, bias, fp8) in enumerate(specs):
+        p = synth.make_problem("mix", N, K, 16, s, seed=500 + 11 * i + M, group_size=group,
+                               beta_std=0.002 if bias else 0.0, residual_fp8=bool(fp8))
+        lay = qt.qtea_pack_layout(dev(p.T), n_salient=p.s, group_size=group or K, fmt=fmt)
+        lay.set_options((qt.QTEA_OPT_BIAS if bias else 0) | (qt.QTEA_OPT_RESIDUAL_FP8 if fp8 else 0))
+        rv = dev(p.residual_vals) if fp8 else dev(p.residual_vals.view(np.int16), torch.float16)
+        items.append(dict(x=dev(p.x[:M].view(np.int16), torch.float16), layout=lay,
+                          row_scale=dev(scales(p, bias).view(np.int16), torch.float16),
+                          col_scale=dev(p.v.view(np.int16), torch.float16), salient_idx=dev(p.salient_idx),
+                          residual_vals=rv, residual_idx=dev(p.residual_idx)))
+        probs.append((p, bias))
+    ys = qt.qtea_gemv_grouped(items)
+    torch.cuda.synchronize()
+    for it in items:
+        assert qt.qtea_device_status(it["layout"]) == 0
+    for (p, bias), y in zip(probs, ys):
+        y_ref, b = reference(p, bias, M=M)
+        assert_within(y.cpu().numpy().astype(np.float64), y_ref, b, f"{p.N}x{p.K} M {M}")
