@@ -40,6 +40,7 @@ void release(qtea_layout* l) {
   if (l->counters) cudaFree(l->counters);
   if (l->status) cudaFree(l->status);
   if (l->mb_ws) cudaFree(l->mb_ws);
+  if (l->mb_gbar) cudaFree(l->mb_gbar);
   if (l->mb_part) cudaFree(l->mb_part);
   if (l->mb_counters) cudaFree(l->mb_counters);
   delete l;
@@ -93,6 +94,9 @@ int plan_m1(qtea_layout* l, const cudaDeviceProp& prop) {
           cudaMalloc(&l->mb_counters, ctr) != cudaSuccess)
         return QTEA_ERR_ALLOC;
       if (cudaMemset(l->mb_counters, 0, ctr) != cudaSuccess) return QTEA_ERR_CUDA;
+      if (cudaMalloc(&l->mb_gbar, sizeof(unsigned long long)) != cudaSuccess) return QTEA_ERR_ALLOC;
+      if (cudaMemset(l->mb_gbar, 0, sizeof(unsigned long long)) != cudaSuccess) return QTEA_ERR_CUDA;
+      l->mb_gbar_next = 0;
     }
   }
   if (cudaMalloc(&l->workspace, (size_t)l->sm_count * 2 * kTileRows * sizeof(float)) != cudaSuccess)
@@ -301,6 +305,15 @@ bool mb_group_plan(MbGroup& g, int sm_count, size_t smem_optin) {
   g.grid = (int)(g.gp.total_units < sm_count ? g.gp.total_units : sm_count);
   if (g.grid > kMaxGrid) g.grid = kMaxGrid;
   for (int b = 0; b <= g.grid; ++b) g.gp.cta_u0[b] = (int)unit_begin_of(b, g.gp.total_units, g.grid);
+  // no residual left to the prep kernel: its other work moves into the main kernel (one launch)
+  g.gp.fused = 1;
+  for (int k = 0; k < g.gp.n_problems; ++k)
+    if (g.gp.prob[k].res_mode == kMbResPrep) g.gp.fused = 0;
+  if (g.gp.fused) {
+    g.gp.prep = g.pg;
+    const int scratch = 16 * kChunkCols * 2 + kChunkCols * 2;  // prep_chunk's
+    if (g.gp.res_stage_bytes < scratch) g.gp.res_stage_bytes = scratch;
+  }
   for (int S = kMaxStagesMb; S >= kMinStagesMb; --S) {
     const size_t bytes = mb_smem_bytes(S, g.gp.M, g.grp, g.gp.res_stage_bytes);
     if (bytes <= smem_optin) {
@@ -312,8 +325,15 @@ bool mb_group_plan(MbGroup& g, int sm_count, size_t smem_optin) {
   return false;
 }
 
-int mb_group_launch(MbGroup& g, cudaStream_t st) {
-  if (launch_mb_prep(g.pg, st) != cudaSuccess) return QTEA_ERR_CUDA;
+int mb_group_launch(MbGroup& g, const qtea_layout* l0, cudaStream_t st) {
+  if (g.gp.fused) {
+    // the barrier counter only grows: this launch's CTAs wait for it to reach the value after them
+    g.gp.gbar = l0->mb_gbar;
+    l0->mb_gbar_next += (unsigned long long)g.grid;
+    g.gp.gbar_target = l0->mb_gbar_next;
+  } else if (launch_mb_prep(g.pg, st) != cudaSuccess) {
+    return QTEA_ERR_CUDA;
+  }
   return launch_mb(g.maps, g.ab_maps, g.gp, g.grp, g.grid, g.smem, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
 }
 
@@ -351,7 +371,7 @@ int run_mb(const qtea_gemv_problem* qs, const int* idx, int n, int M, cudaStream
       ++i;
       continue;
     }
-    int rc = mb_group_launch(g, st);
+    int rc = mb_group_launch(g, l0, st);
     if (rc) return rc;
     i += taken;
   }

@@ -214,13 +214,73 @@ __device__ __forceinline__ void res_step(const void* rv_, int rvs, const uint8_t
   }
 }
 
+// v and x of chunk ch of problem p in fragment order, and the group sums of x: 256 threads (tid),
+// sm holds 17,408 bytes of scratch, sync() is a barrier over the 256 threads. Entry (step s, quad
+// lane q) of the v block holds the pairs (v[16W + i], v[16W + i + 8]) for i = 2(s & 3) and i + 1,
+// W = 4(s >> 2) + q; entry (step s, lane 4g + q) of x block j holds the same two pairs of x[8j + g].
+// Columns >= K and batch rows >= M are zero. Steps 8k .. 8k + 7 cover columns 128k .. 128k + 127.
+template <typename Sync>
+__device__ __forceinline__ void prep_chunk(const MbPrepProblem& p, int M, int mt, int ch, int tid, uint8_t* sm,
+                                           Sync sync) {
+  uint16_t(*xsm)[kChunkCols] = reinterpret_cast<uint16_t(*)[kChunkCols]>(sm);
+  uint16_t* vsm = reinterpret_cast<uint16_t*>(sm + 16 * kChunkCols * 2);
+  const int col0 = ch * kChunkCols;
+#pragma unroll 2
+  for (int i = tid; i < kChunkCols; i += 256) {
+    const int col = col0 + i;
+    const bool in = col < p.K;
+    vsm[i] = in ? __ldg(p.v + col) : (uint16_t)0;
+    uint16_t xv[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) xv[m] = (in && m < M) ? __ldg(p.x + (size_t)m * p.K + col) : (uint16_t)0;
+#pragma unroll
+    for (int m = 0; m < 16; ++m) xsm[m][i] = xv[m];
+  }
+  sync();
+  uint8_t* out = p.ws + (size_t)ch * kMbChunkWsBytes;
+  auto pair = [](const uint16_t* row, int c) { return (uint32_t)row[c] | ((uint32_t)row[c + 8] << 16); };
+  if (tid < 128) {
+    const int s = tid >> 2, q = tid & 3;
+    const int base = 16 * (4 * (s >> 2) + q), i0 = 2 * (s & 3);
+    reinterpret_cast<uint2*>(out)[tid] = make_uint2(pair(vsm, base + i0), pair(vsm, base + i0 + 1));
+  }
+  for (int e = tid; e < mt * 1024; e += 256) {
+    const int j = e >> 10, s = (e >> 5) & 31, lane = e & 31, g = lane >> 2, q = lane & 3;
+    const int base = 16 * (4 * (s >> 2) + q), i0 = 2 * (s & 3);
+    const uint16_t* row = xsm[8 * j + g];
+    reinterpret_cast<uint2*>(out + kMbChunkHead)[e] = make_uint2(pair(row, base + i0), pair(row, base + i0 + 1));
+  }
+  {
+    // sum of x over each 128-column group k of the chunk for batch row m (the beta term of Eq. 10):
+    // four lanes per (k, m) add 32 columns each, then a fixed butterfly
+    const int k = tid >> 6, m = (tid >> 2) & 15, part = tid & 3;
+    float sxv = 0.f;
+#pragma unroll 8
+    for (int c = 0; c < 32; ++c) sxv += __half2float(__ushort_as_half(xsm[m][128 * k + 32 * part + c]));
+    sxv += __shfl_xor_sync(0xffffffffu, sxv, 1);
+    sxv += __shfl_xor_sync(0xffffffffu, sxv, 2);
+    if (part == 0) reinterpret_cast<float*>(out + kMbVBytes)[16 * k + m] = sxv;
+  }
+}
+
+// x at salient columns 256 blk .. 256 blk + 255 of problem p, all 16 batch rows (xs[m][c], zero
+// beyond s or M); one column per thread.
+__device__ __forceinline__ void prep_gather(const MbPrepProblem& p, int M, int blk, int tid) {
+  const int c = blk * 256 + tid;
+  if (c < p.s16) {
+    int col = c < p.s ? __ldg(p.sal + c) : 0;
+    col = col < 0 ? 0 : (col >= p.K ? p.K - 1 : col);
+    uint16_t xv[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) xv[m] = (c < p.s && m < M) ? __ldg(p.x + (size_t)m * p.K + col) : (uint16_t)0;
+#pragma unroll
+    for (int m = 0; m < 16; ++m) p.xs[(size_t)m * p.s16 + c] = xv[m];
+  }
+}
+
 // Blocks of a problem: its chunks; then, for a residual left to the prep kernel, its 256-row tiles;
 // or, for a residual of the main kernel's helpers, blocks that gather x at the salient columns
 // (xs[m][c], zero beyond s or M), 256 columns each.
-// Chunk ch's 512 columns: entry (step s, quad lane q) of the v block holds the pairs
-// (v[16W + i], v[16W + i + 8]) for i = 2(s & 3) and i + 1, W = 4(s >> 2) + q; entry (step s,
-// lane 4g + q) of x block j holds the same two pairs of x[8j + g]. Columns >= K and batch rows >= M
-// are zero. Steps 8k .. 8k + 7 cover columns 128k .. 128k + 127 (words 8k .. 8k + 7) only.
 // Tile t: the residual of its 256 rows for every batch row, computed with the main kernel's thread
 // mapping (thread tid holds rows tr + 16b + g and + 8, batch rows 8j + 2q and + 1) and stored in
 // that order, so that each main-kernel thread reads its part with vector loads. The tile's values
@@ -244,17 +304,7 @@ __global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant
   const int local = (int)blockIdx.x - p.block_begin;
   const int tid = threadIdx.x;
   if (local >= p.n_chunks && p.res_mode == kMbResHelpers) {
-    // ---- x at 256 salient columns, all 16 batch rows
-    const int c = (local - p.n_chunks) * 256 + tid;
-    if (c < p.s16) {
-      int col = c < p.s ? __ldg(p.sal + c) : 0;
-      col = col < 0 ? 0 : (col >= p.K ? p.K - 1 : col);
-      uint16_t xv[16];
-#pragma unroll
-      for (int m = 0; m < 16; ++m) xv[m] = (c < p.s && m < M) ? __ldg(p.x + (size_t)m * p.K + col) : (uint16_t)0;
-#pragma unroll
-      for (int m = 0; m < 16; ++m) p.xs[(size_t)m * p.s16 + c] = xv[m];
-    }
+    prep_gather(p, M, local - p.n_chunks, tid);
     return;
   }
   if (local >= p.n_chunks) {
@@ -350,46 +400,7 @@ __global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant
         if (j < gr.mt) dst[b * gr.mt + j] = make_float4(res[b][j][0], res[b][j][1], res[b][j][2], res[b][j][3]);
     return;
   }
-  // ---- v and x of chunk ch in fragment order
-  uint16_t(*xsm)[kChunkCols] = reinterpret_cast<uint16_t(*)[kChunkCols]>(sm);
-  uint16_t* vsm = reinterpret_cast<uint16_t*>(sm + 16 * kChunkCols * 2);
-  const int ch = local, col0 = ch * kChunkCols;
-#pragma unroll 2
-  for (int i = tid; i < kChunkCols; i += 256) {
-    const int col = col0 + i;
-    const bool in = col < p.K;
-    vsm[i] = in ? __ldg(p.v + col) : (uint16_t)0;
-    uint16_t xv[16];
-#pragma unroll
-    for (int m = 0; m < 16; ++m) xv[m] = (in && m < M) ? __ldg(p.x + (size_t)m * p.K + col) : (uint16_t)0;
-#pragma unroll
-    for (int m = 0; m < 16; ++m) xsm[m][i] = xv[m];
-  }
-  __syncthreads();
-  uint8_t* out = p.ws + (size_t)ch * kMbChunkWsBytes;
-  auto pair = [](const uint16_t* row, int c) { return (uint32_t)row[c] | ((uint32_t)row[c + 8] << 16); };
-  if (tid < 128) {
-    const int s = tid >> 2, q = tid & 3;
-    const int base = 16 * (4 * (s >> 2) + q), i0 = 2 * (s & 3);
-    reinterpret_cast<uint2*>(out)[tid] = make_uint2(pair(vsm, base + i0), pair(vsm, base + i0 + 1));
-  }
-  for (int e = tid; e < gr.mt * 1024; e += 256) {
-    const int j = e >> 10, s = (e >> 5) & 31, lane = e & 31, g = lane >> 2, q = lane & 3;
-    const int base = 16 * (4 * (s >> 2) + q), i0 = 2 * (s & 3);
-    const uint16_t* row = xsm[8 * j + g];
-    reinterpret_cast<uint2*>(out + kMbChunkHead)[e] = make_uint2(pair(row, base + i0), pair(row, base + i0 + 1));
-  }
-  {
-    // sum of x over each 128-column group k of the chunk for batch row m (the beta term of Eq. 10):
-    // four lanes per (k, m) add 32 columns each, then a fixed butterfly
-    const int k = tid >> 6, m = (tid >> 2) & 15, part = tid & 3;
-    float sxv = 0.f;
-#pragma unroll 8
-    for (int c = 0; c < 32; ++c) sxv += __half2float(__ushort_as_half(xsm[m][128 * k + 32 * part + c]));
-    sxv += __shfl_xor_sync(0xffffffffu, sxv, 1);
-    sxv += __shfl_xor_sync(0xffffffffu, sxv, 2);
-    if (part == 0) reinterpret_cast<float*>(out + kMbVBytes)[16 * k + m] = sxv;
-  }
+  prep_chunk(p, M, gr.mt, local, tid, sm, [] { __syncthreads(); });
 }
 
 // ---------------------------------------------------------------- decode of one unit
@@ -481,6 +492,31 @@ __device__ __forceinline__ void decode_unit(const uint8_t* sb, int tr, int g, in
 // ---------------------------------------------------------------- helper warps (residual)
 
 __device__ __forceinline__ void helpers_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kMbHelperWarps * 32) : "memory"); }
+__device__ __forceinline__ void consumers_sync() {
+  asm volatile("bar.sync 2, %0;" ::"n"(kMbConsumerWarps * 32) : "memory");
+}
+
+// Grid-wide barrier of a cooperative launch: every CTA adds one to a monotonic counter (release at
+// GPU scope, after its threads' writes) and waits until it reaches `target` (acquire); bounded, a
+// timeout is recorded in the status word.
+__device__ __forceinline__ void grid_sync(unsigned long long* bar, unsigned long long target, int* status) {
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    asm volatile("fence.acq_rel.gpu;" ::: "memory");
+    asm volatile("red.release.gpu.global.add.u64 [%0], 1;" ::"l"(bar) : "memory");
+    const unsigned long long t0 = global_ns();
+    for (;;) {
+      unsigned long long v;
+      asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(bar) : "memory");
+      if (v >= target) break;
+      if (global_ns() - t0 > kWaitLimitNs) {
+        atomicExch(status, (int)QTEA_ERR_TIMEOUT);
+        break;
+      }
+    }
+  }
+  __syncthreads();
+}
 
 // The residual (Eq. 11) of every tile whose first chunk this CTA decodes, in the order the consumers
 // reach those tiles, into a ring of two result slots laid out in the consumers' accumulator order
@@ -496,6 +532,9 @@ __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u
                                          int hw, int lane, int* status) {
   const int g = lane >> 2, q = lane & 3;
   const int htid = hw * 32 + lane;
+  // x at the salient columns was written by other threads' generic stores; the bulk copies read it
+  // through the async proxy
+  asm volatile("fence.proxy.async.global;" ::: "memory");
   UnitPos c = unit_pos(tab, NP, u0);
   int k = 0, sphase = 0;
   bool failed = false;
@@ -650,12 +689,32 @@ __global__ void __launch_bounds__(kMbThreads, 1)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
+  if (gp.fused) {
+    // the prep work (fragment-order v and x of every chunk, x at the salient columns) spread over the
+    // CTAs, done by the consumer threads while the first code stages stream in; then a grid barrier
+    if (warp < kMbConsumerWarps) {
+      for (int item = blockIdx.x; item < gp.prep.n_blocks; item += gridDim.x) {
+        int pi = 0;
+        while (pi + 1 < gp.prep.n_problems && item >= gp.prep.prob[pi + 1].block_begin) ++pi;
+        const MbPrepProblem pp = gp.prep.prob[pi];
+        const int local = item - pp.block_begin;
+        if (local < pp.n_chunks) prep_chunk(pp, gp.M, MT, local, (int)threadIdx.x, rstage, [] { consumers_sync(); });
+        else prep_gather(pp, gp.M, local - pp.n_chunks, (int)threadIdx.x);
+        consumers_sync();  // the scratch is free again
+      }
+    }
+    grid_sync(gp.gbar, gp.gbar_target, gp.status);
+  }
+
   if (warp > kMbConsumerWarps) {
     helper_role<MT>(tab, NP, u0, n_units, rslot, rstage, res_full, res_empty, staged, warp - kMbConsumerWarps - 1,
                     lane, gp.status);
   } else if (warp == kMbConsumerWarps) {
     // ---------------------------------------------------------------- producer lane
     if (lane == 0) {
+      // the chunks' fragment-order v and x were written by generic stores (this or another CTA, or
+      // the prep kernel); the bulk copies read them through the async proxy
+      asm volatile("fence.proxy.async.global;" ::: "memory");
       for (int i = 0; i < n_units; ++i) {
         const int st = i % S, ph = i / S;
         const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
@@ -945,11 +1004,13 @@ cudaError_t launch_mb(const TensorMaps& maps, const TensorMaps& ab_maps, const M
   cfg.blockDim = dim3(kMbThreads);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeCooperative;  // fused: the CTAs wait on one another (grid barrier)
+  attr[1].val.cooperative = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = p.fused ? 2 : 1;
   if (grp) {
     if (p.M <= 8) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, true>, maps, ab_maps, p);
     return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2, true>, maps, ab_maps, p);

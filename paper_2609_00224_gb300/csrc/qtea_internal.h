@@ -169,8 +169,12 @@ struct MbProblemArgs {
 
 struct MbGroupParams {
   MbProblemArgs prob[kMaxProblems];
+  MbPrepGroup prep;         // fused: the prep work, done by the main kernel's CTAs before a grid barrier
+  int fused;
+  unsigned long long* gbar; // fused: grid barrier counter (monotonic), target below
+  unsigned long long gbar_target;
   int n_problems, n_stages, M;
-  int res_stage_bytes;      // the helpers' staging buffer
+  int res_stage_bytes;      // the helpers' staging buffer (and the fused prep's scratch)
   int* status;              // device status word (the first layout's)
   long long total_units;
   int cta_u0[kMaxGrid + 1];
@@ -271,6 +275,8 @@ struct qtea_layout {
   bool mb_ok;
   size_t mb_smem_optin;
   size_t prep_smem_optin;  // dynamic shared memory the prep kernel may use
+  unsigned long long* mb_gbar;                // grid barrier counter of fused low-batch launches
+  mutable unsigned long long mb_gbar_next;    // its value after the last launch issued (host side)
   uint8_t* mb_ws;        // [n_chunks][kMbChunkWsBytes] v and x in fragment order, then the residual
                          // of every 256-row tile [n_tiles][kMbResFloatsPerTile]
   float* mb_part;        // [sm_count][kMbPartFloatsPerCta] partial rows of split tiles
