@@ -214,14 +214,15 @@ __device__ __forceinline__ void res_step(const void* rv_, int rvs, const uint8_t
   }
 }
 
-// v and x of chunk ch of problem p in fragment order, and the group sums of x: 256 threads (tid),
-// sm holds 17,408 bytes of scratch, sync() is a barrier over the 256 threads. Entry (step s, quad
+// v and x of chunk ch of problem p in fragment order, and the group sums of x, to out (global
+// memory or a stage): 256 threads (tid), sm holds 17,408 bytes of scratch, sync() is a barrier over
+// the 256 threads. Entry (step s, quad
 // lane q) of the v block holds the pairs (v[16W + i], v[16W + i + 8]) for i = 2(s & 3) and i + 1,
 // W = 4(s >> 2) + q; entry (step s, lane 4g + q) of x block j holds the same two pairs of x[8j + g].
 // Columns >= K and batch rows >= M are zero. Steps 8k .. 8k + 7 cover columns 128k .. 128k + 127.
 template <typename Sync>
 __device__ __forceinline__ void prep_chunk(const MbPrepProblem& p, int M, int mt, int ch, int tid, uint8_t* sm,
-                                           Sync sync) {
+                                           uint8_t* out, Sync sync) {
   uint16_t(*xsm)[kChunkCols] = reinterpret_cast<uint16_t(*)[kChunkCols]>(sm);
   uint16_t* vsm = reinterpret_cast<uint16_t*>(sm + 16 * kChunkCols * 2);
   const int col0 = ch * kChunkCols;
@@ -237,7 +238,6 @@ __device__ __forceinline__ void prep_chunk(const MbPrepProblem& p, int M, int mt
     for (int m = 0; m < 16; ++m) xsm[m][i] = xv[m];
   }
   sync();
-  uint8_t* out = p.ws + (size_t)ch * kMbChunkWsBytes;
   auto pair = [](const uint16_t* row, int c) { return (uint32_t)row[c] | ((uint32_t)row[c + 8] << 16); };
   if (tid < 128) {
     const int s = tid >> 2, q = tid & 3;
@@ -400,7 +400,7 @@ __global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant
         if (j < gr.mt) dst[b * gr.mt + j] = make_float4(res[b][j][0], res[b][j][1], res[b][j][2], res[b][j][3]);
     return;
   }
-  prep_chunk(p, M, gr.mt, local, tid, sm, [] { __syncthreads(); });
+  prep_chunk(p, M, gr.mt, local, tid, sm, p.ws + (size_t)local * kMbChunkWsBytes, [] { __syncthreads(); });
 }
 
 // ---------------------------------------------------------------- decode of one unit
@@ -496,26 +496,27 @@ __device__ __forceinline__ void consumers_sync() {
   asm volatile("bar.sync 2, %0;" ::"n"(kMbConsumerWarps * 32) : "memory");
 }
 
-// Grid-wide barrier of a cooperative launch: every CTA adds one to a monotonic counter (release at
-// GPU scope, after its threads' writes) and waits until it reaches `target` (acquire); bounded, a
-// timeout is recorded in the status word.
-__device__ __forceinline__ void grid_sync(unsigned long long* bar, unsigned long long target, int* status) {
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    asm volatile("fence.acq_rel.gpu;" ::: "memory");
-    asm volatile("red.release.gpu.global.add.u64 [%0], 1;" ::"l"(bar) : "memory");
-    const unsigned long long t0 = global_ns();
-    for (;;) {
-      unsigned long long v;
-      asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(bar) : "memory");
-      if (v >= target) break;
-      if (global_ns() - t0 > kWaitLimitNs) {
-        atomicExch(status, (int)QTEA_ERR_TIMEOUT);
-        break;
-      }
+// Arrival at the grid-wide barrier of a cooperative launch: one thread adds one to a monotonic
+// counter, release at GPU scope (after a barrier over the threads whose writes it publishes).
+__device__ __forceinline__ void grid_arrive(unsigned long long* bar) {
+  asm volatile("fence.acq_rel.gpu;" ::: "memory");
+  asm volatile("red.release.gpu.global.add.u64 [%0], 1;" ::"l"(bar) : "memory");
+}
+
+// One thread waits until every CTA arrived (acquire at GPU scope); bounded, a timeout is recorded in
+// the status word. Data the other CTAs wrote is then read by bulk copies (async proxy).
+__device__ __forceinline__ void grid_wait(const unsigned long long* bar, unsigned long long target, int* status) {
+  const unsigned long long t0 = global_ns();
+  for (;;) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(bar) : "memory");
+    if (v >= target) break;
+    if (global_ns() - t0 > kWaitLimitNs) {
+      atomicExch(status, (int)QTEA_ERR_TIMEOUT);
+      break;
     }
   }
-  __syncthreads();
+  asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
 // The residual (Eq. 11) of every tile whose first chunk this CTA decodes, in the order the consumers
@@ -529,11 +530,11 @@ __device__ __forceinline__ void grid_sync(unsigned long long* bar, unsigned long
 template <int MT>
 __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u0, int n_units, float* rslot,
                                          uint8_t* rstage, uint64_t* res_full, uint64_t* res_empty, uint64_t* staged,
-                                         int hw, int lane, int* status) {
+                                         const MbGroupParams& gp, int hw, int lane, int* status) {
   const int g = lane >> 2, q = lane & 3;
   const int htid = hw * 32 + lane;
-  // x at the salient columns was written by other threads' generic stores; the bulk copies read it
-  // through the async proxy
+  // x at the salient columns is gathered by the CTAs before the grid barrier (with fused prep work)
+  if (gp.fused) grid_wait(gp.gbar, gp.gbar_target, status);
   asm volatile("fence.proxy.async.global;" ::: "memory");
   UnitPos c = unit_pos(tab, NP, u0);
   int k = 0, sphase = 0;
@@ -680,7 +681,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
     for (int i = 0; i < S && i < n_units; ++i) {
       const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
       const uint32_t bar = smem_u32(&full[i]);
-      mbar_arrive_expect_tx(bar, kFill);
+      mbar_arrive_expect_tx(bar, (gp.fused && i == 0) ? kFill - (kMbChunkHead + MT * kMbXTileBytes) : kFill);
       tma_load_2d(smem_u32(stages + (size_t)i * kStage), &maps.m[up.p], up.ch * kChunkRowBytes, up.t * kMbTileRows,
                   bar);
       last_fill[i] = 1;
@@ -689,32 +690,44 @@ __global__ void __launch_bounds__(kMbThreads, 1)
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
 
-  if (gp.fused) {
-    // the prep work (fragment-order v and x of every chunk, x at the salient columns) spread over the
-    // CTAs, done by the consumer threads while the first code stages stream in; then a grid barrier
-    if (warp < kMbConsumerWarps) {
+  if (gp.fused && warp < kMbConsumerWarps) {
+    // the prep work, done by the consumer threads while the first code stages stream in: this CTA's
+    // first unit's v and x straight into stage 0, then its share of every chunk's fragment-order v and
+    // x and of x at the salient columns (global memory, for the later units of all CTAs), then an
+    // arrival at the grid barrier that the producer and the helpers wait on before their bulk copies
+    {
+      const UnitPos up = unit_pos(tab, NP, u0);
+      const MbPrepProblem pp = gp.prep.prob[up.p];
+      prep_chunk(pp, gp.M, MT, up.ch, (int)threadIdx.x, rstage, stages + kMbCodeBytes, [] { consumers_sync(); });
+      consumers_sync();
+    }
+    {
       for (int item = blockIdx.x; item < gp.prep.n_blocks; item += gridDim.x) {
         int pi = 0;
         while (pi + 1 < gp.prep.n_problems && item >= gp.prep.prob[pi + 1].block_begin) ++pi;
         const MbPrepProblem pp = gp.prep.prob[pi];
         const int local = item - pp.block_begin;
-        if (local < pp.n_chunks) prep_chunk(pp, gp.M, MT, local, (int)threadIdx.x, rstage, [] { consumers_sync(); });
-        else prep_gather(pp, gp.M, local - pp.n_chunks, (int)threadIdx.x);
+        if (local < pp.n_chunks)
+          prep_chunk(pp, gp.M, MT, local, (int)threadIdx.x, rstage, pp.ws + (size_t)local * kMbChunkWsBytes,
+                     [] { consumers_sync(); });
+        else
+          prep_gather(pp, gp.M, local - pp.n_chunks, (int)threadIdx.x);
         consumers_sync();  // the scratch is free again
       }
     }
-    grid_sync(gp.gbar, gp.gbar_target, gp.status);
+    if (threadIdx.x == 0) grid_arrive(gp.gbar);
   }
 
   if (warp > kMbConsumerWarps) {
-    helper_role<MT>(tab, NP, u0, n_units, rslot, rstage, res_full, res_empty, staged, warp - kMbConsumerWarps - 1,
+    helper_role<MT>(tab, NP, u0, n_units, rslot, rstage, res_full, res_empty, staged, gp, warp - kMbConsumerWarps - 1,
                     lane, gp.status);
   } else if (warp == kMbConsumerWarps) {
     // ---------------------------------------------------------------- producer lane
     if (lane == 0) {
-      // the chunks' fragment-order v and x were written by generic stores (this or another CTA, or
-      // the prep kernel); the bulk copies read them through the async proxy
+      // the chunks' fragment-order v and x were written by generic stores (the CTAs before the grid
+      // barrier, or the prep kernel); the bulk copies read them through the async proxy
       asm volatile("fence.proxy.async.global;" ::: "memory");
+      bool barrier_passed = !gp.fused;
       for (int i = 0; i < n_units; ++i) {
         const int st = i % S, ph = i / S;
         const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
@@ -726,8 +739,16 @@ __global__ void __launch_bounds__(kMbThreads, 1)
           tma_load_2d(smem_u32(sb), &maps.m[up.p], up.ch * kChunkRowBytes, up.t * kMbTileRows, bar);
           last_fill[st] = ph + 1;
         }
-        bulk_load(smem_u32(sb + kMbCodeBytes), tab[up.p].ws + (size_t)up.ch * kMbChunkWsBytes,
-                  (uint32_t)(kMbChunkHead + MT * kMbXTileBytes), bar);
+        if (!(gp.fused && i == 0)) {  // fused: unit 0's v and x were written by this CTA's consumers
+          if (!barrier_passed) {
+            grid_wait(gp.gbar, gp.gbar_target, gp.status);
+            barrier_passed = true;
+          }
+          // stage 0 held generic stores of unit 0 before this copy overwrites it
+          if (st == 0) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+          bulk_load(smem_u32(sb + kMbCodeBytes), tab[up.p].ws + (size_t)up.ch * kMbChunkWsBytes,
+                    (uint32_t)(kMbChunkHead + MT * kMbXTileBytes), bar);
+        }
         if (GRP) {
           // the unit's alpha (and beta): 8 fp16 per row from column 8 ch (pairs) or 8 (ch / 2)
           const int xa = tab[up.p].bias ? 8 * up.ch : 8 * (up.ch >> 1);
