@@ -99,7 +99,8 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
 
 /*
  * y = x * W^T for the layout's N x K ternary weights plus the 1:4 salient residual
- * (Eq. 10 and Eq. 11 with beta = 0 and one alpha per row).
+ * (Eq. 10 and Eq. 11: one alpha per row, or alpha and optionally beta per row and group of 128
+ * columns as the layout's group_size and options say).
  *
  *   x              device fp16 [M][K], activations
  *   packed_ternary layout from qtea_pack_layout
@@ -124,10 +125,13 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
  * workspace. Results are bitwise reproducible for a given (layout, inputs, device); a grouped
  * call (qtea_gemv_grouped) is reproducible for the same group, but its rounding may differ
  * from separate calls because the split of work over the CTAs differs.
- * Numerics: the ternary sum is accumulated exactly in integers over 512-column blocks,
- * with v*x represented in fixed point relative to the block's largest |v*x| (24-bit unless
- * qtea_set_activation_precision selects 16-bit); block sums, alpha and the residual are
- * combined in fp32.
+ * Numerics: at M = 1 (the library's own storage) the ternary sum is accumulated exactly in
+ * integers over 512-column blocks, with v*x represented in fixed point relative to the block's
+ * largest |v*x| (24-bit unless qtea_set_activation_precision selects 16-bit); block sums, alpha
+ * and the residual are combined in fp32. At 2 <= M <= 16, and for 2-bit layouts in the paper's
+ * storage at any M, the tensor cores take 2T*v and x in fp16 (both exact, which needs |v| < 32768)
+ * with exact fp32 products and fp32 sums; alpha, beta and the residual are applied in fp32.
+ * Base-3 layouts use a general kernel (fp32 throughout).
  */
 int qtea_gemv(const uint16_t* x, const qtea_layout* packed_ternary, const uint16_t* row_scale,
               const uint16_t* col_scale, const int32_t* salient_idx, const uint16_t* residual_vals,
@@ -147,9 +151,10 @@ typedef struct qtea_gemv_problem {
 
 /*
  * Several independent GEMVs with the same batch M, as if qtea_gemv were called for each in
- * order, but with M = 1 problems sharing launches: up to 8 problems whose activation staging
- * fits shared memory run in one persistent kernel, which removes per-launch ramp-up and tail
- * time when the problems are small (e.g. the q/k/v/o/gate/up/down GEMVs of one decoder layer).
+ * order, but sharing launches: up to 8 consecutive problems that the same kernel variant serves
+ * (batch 1; low batch with one alpha per row; low batch with scale groups) run in one persistent
+ * launch, which removes per-launch ramp-up and tail time when the problems are small (e.g. the
+ * q/k/v/o/gate/up/down GEMVs of one decoder layer).
  * Every problem is validated before anything is launched; a failing check returns its status
  * and launches nothing. No two problems may write overlapping y, and problems must not share
  * a layout. QTEA_ERR_TIMEOUT from a grouped launch is recorded in the layout of the first
