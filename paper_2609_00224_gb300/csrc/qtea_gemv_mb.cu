@@ -1,35 +1,36 @@
-// Low-batch QTEA GEMV for sm_103a (2 <= M <= 16): y[m] = alpha * (T . (v * x[m])) + residual,
-// on the tensor cores.
+// Tensor-core QTEA GEMV for sm_103a: y[m] = x[m] * W^T for 2 <= M <= 16 batch rows, and for
+// 2-bit layouts in the paper's storage at any M.
 //
-// Computes Eq. 10 (one alpha per row, beta = 0) plus Eq. 11 of the QTEA paper (Sec. 3.5) for a
-// batch of M activation rows. With M rows the product is a skinny dense contraction, so it runs
-// on mma.sync m16n8k16 (fp16 operands, fp32 accumulation), exactly:
+// Computes Eq. 10 (one alpha per row, or alpha and beta per row and 128-column group) plus Eq. 11
+// of the QTEA paper (Sec. 3.5). With M rows the product is a skinny dense contraction, so it runs on
+// mma.sync m16n8k16 (fp16 operands, fp32 accumulation), exactly:
 //  * A = 2T * v. A 32-bit code word holds the codes c = T + 1 of 16 consecutive columns; shifting
 //    it left by 14 - 2i puts the codes of columns i and i + 8 at bits 14-15 and 30-31, and one
 //    LOP3 (~w & 0xC000C000) turns each into the fp16 value -2, -0 or +2 (sign bit and the top
 //    exponent bit). One multiply by the pair (v_i, v_{i+8}) gives 2T * v exactly (a power-of-two
-//    multiple of an fp16 value). The accumulator is halved once at the end.
+//    multiple of an fp16 value). The accumulator is halved once (per group with scale groups).
 //  * B = x, the fp16 activations, unchanged; each product is exact in fp32 and the sums
 //    accumulate in fp32. The contraction index runs over the columns in the order that pairing
-//    gives (columns i and i + 8 of a word side by side), so a prep kernel writes, once per call and
-//    512-column chunk, v and x in exactly the register order the fragments need ("fragment
-//    order"): one 8-byte shared load per thread and step.
-//  * The residual of Eq. 11 is an exact contraction too: over "virtual columns", one per
-//    salient column, A holds the fp16 residual value of the row's group where the stored
-//    position is the row and 0 elsewhere, and B holds x at the salient column. The prep kernel
-//    computes it per 256-row tile (its loads are scattered and would stall the decode) and the
-//    main kernel adds it, unscaled by alpha, at the tile's end.
-// Work: a unit is 256 rows x 512 columns of one problem; the units of every problem of a group
-// form one sequence that is split evenly over persistent CTAs (one launch for all the GEMVs of a
-// group). Each of eight consumer warps owns two 16-row blocks of a unit, so every B fragment it
-// loads feeds two MMAs; two accumulator sets alternate between steps so that consecutive MMAs do
-// not wait on each other. A tile whose units span several
-// CTAs is finished by the last of them (per warp, counted with an acq_rel atomic): it adds the
-// partial rows in CTA order, so results do not depend on timing. A producer lane streams the
-// CTA's units through a ring of shared-memory stages: 256 rows x 128 bytes of codes by TMA
-// (128-byte swizzle) and the chunk's v and x in fragment order by bulk copy.
-// |v| must stay below 32768 (2v is formed in fp16). Every wait on an mbarrier is bounded (~2 s,
-// then QTEA_ERR_TIMEOUT in the status word).
+//    gives (columns i and i + 8 of a word side by side), so v and x of each 512-column chunk are
+//    written once per call in exactly the register order the fragments need ("fragment order"):
+//    one 8-byte shared load per thread and step. Each MMA step stays inside one 128-column group.
+//  * The residual of Eq. 11 is an exact contraction too: over "virtual columns", one per salient
+//    column, A holds the residual value (fp16, or FP8 E4M3 converted exactly) of the row's group
+//    where the stored position is the row and 0 elsewhere, and B holds x at the salient column.
+//    Helper warps compute it per 256-row tile from bulk-copied residual rows, off the decode's
+//    path; it is added, unscaled by alpha, at the tile's end.
+// Work: a unit is 256 rows x 512 columns of one problem; the units of every problem of a group form
+// one sequence split evenly over persistent CTAs (one cooperative launch for all the GEMVs of a
+// group). The consumer threads first build the fragment-order chunks (spread over the CTAs; each
+// CTA's own first chunk straight into its first stage), then decode. Each of eight consumer warps
+// owns two 16-row blocks of a unit, so every B fragment it loads feeds two MMAs; two accumulator
+// sets alternate between steps. A tile whose units span several CTAs is finished by the last of
+// them (per warp, counted with an acq_rel atomic), which adds the partial rows in CTA order, so
+// results do not depend on timing. A producer lane streams the CTA's units through a ring of
+// shared-memory stages: 256 rows x 128 bytes of codes by TMA (128-byte swizzle), the chunk's v and
+// x in fragment order by bulk copy, and with scale groups the unit's alpha (and beta) by TMA.
+// |v| must stay below 32768 (2v is formed in fp16). Every wait is bounded (~2 s, then
+// QTEA_ERR_TIMEOUT in the status word).
 #include <cuda_fp16.h>
 
 #include "qtea_internal.h"
