@@ -246,3 +246,14 @@ def paper_problem(config: int, matrix: int, M: Optional[int] = None, layer: int 
 
 def config_shapes(config: int) -> List[Tuple[str, int, int]]:
     return list(CONFIGS[config]["shapes"])
+
+
+def quant_problem(seed: int, N: int, K: int, std: float = 0.02):
+    """Inputs of the quantizer for one linear layer: full-precision weights W [N][K] (float32, drawn
+    N(0, std) and rounded to binary16, so the same bytes feed every consumer) and a positive
+    curvature diagonal h [K] standing in for diag(H) of a calibration set (float32,
+    exp(N(0, 1)) rounded to binary16): the heavy-tailed spread that calibration Hessians show."""
+    W = normal_f16(seed, 40, (N, K), 0.0, std).view(np.float16).astype(np.float32)
+    z = normal_f16(seed, 41, (K,), 0.0, 1.0).view(np.float16).astype(np.float64)
+    h = np.array([f16_from_double(float(np.exp(t))) for t in z], np.uint16).view(np.float16).astype(np.float32)
+    return W, h
