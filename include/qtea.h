@@ -166,6 +166,34 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
  * last qtea_gemv that uses the layout has completed; it synchronizes nothing itself. */
 void qtea_free(qtea_layout* layout);
 
+/*
+ * The quantizer's per-layer steps (Sec. 3.1-3.3 and the 1:4 residual of Sec. 3.2 / 3.5; not the
+ * error propagation of Sec. 3.4), from full-precision weights to this library's inputs:
+ *
+ *   W              device fp32 [N][K], the full-precision weights (row = output feature)
+ *   hdiag          device fp32 [K], diag(H) of the calibration Hessian (Sec. 3.2)
+ *   group_size     K (one alpha per row) or 128 (alpha, and beta with QTEA_OPT_BIAS, per group)
+ *   n_salient      s, 0 <= s <= K; N % 4 == 0 when s > 0
+ *   options        0 or QTEA_OPT_BIAS (beta = the group mean; without it beta = 0)
+ *   fit_iters      refits of alpha as the mean |W - beta| over the nonzero codes (0 .. 64)
+ *   rescale_iters  rounds of the column rescale v_j and reassignment (0 .. 64; the paper uses a
+ *                  small number, e.g. 2)
+ *   codes          out: device int8 [N][K], T in {-1, 0, +1} (the input of qtea_pack_layout)
+ *   row_scale      out: device fp16 [N][G] alpha, or [N][G][2] (alpha, beta) with QTEA_OPT_BIAS
+ *   col_scale      out: device fp16 [K] v
+ *   salient_idx    out: device int32 [s], ascending: the s columns with the largest
+ *                  max_i W_ij^2 hdiag_j^2 (ties: lower column)
+ *   residual_vals  out: device fp16 [N/4][s], residual_idx out: device uint8 [N/4][ceil(s/4)]: per
+ *                  group of four rows and salient column, the largest W - W^ and its position
+ *
+ * Decisions are taken in fp32 with every sum in index order, so the outputs are reproducible bit
+ * for bit. Asynchronous on `stream`; scratch comes from the stream-ordered allocator.
+ * Returns QTEA_ERR_INVALID_ARG or QTEA_ERR_UNSUPPORTED for arguments outside the above.
+ */
+int qtea_quantize(const float* W, const float* hdiag, int N, int K, int group_size, int n_salient, int options,
+                  int fit_iters, int rescale_iters, int8_t* codes, uint16_t* row_scale, uint16_t* col_scale,
+                  int32_t* salient_idx, uint16_t* residual_vals, uint8_t* residual_idx, qtea_stream_t stream);
+
 /* Static English description of a status code. Never NULL. */
 const char* qtea_status_string(int status);
 

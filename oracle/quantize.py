@@ -74,7 +74,8 @@ def group_fit(W: np.ndarray, group: int, bias: bool, fit_iters: int):
             t = _assign(d, (a * F(0.5)).astype(F)[:, None])
             num = _seq_sum(np.where(t != 0, ad, F(0)), 1)
             cnt = (t != 0).sum(axis=1)
-            a = np.where(cnt > 0, (num / cnt.astype(F)).astype(F), a).astype(F)
+            with np.errstate(divide="ignore", invalid="ignore"):  # all-zero groups keep alpha
+                a = np.where(cnt > 0, (num / cnt.astype(F)).astype(F), a).astype(F)
         T[:, gi * group:gi * group + cols.shape[1]] = _assign(d, (a * F(0.5)).astype(F)[:, None])
         alpha[:, gi] = a
         beta[:, gi] = b
@@ -104,7 +105,8 @@ def column_rescale(W: np.ndarray, alpha: np.ndarray, beta: np.ndarray, T: np.nda
             nz = T[i] != 0
             acc = np.where(nz, (acc + term[i]).astype(F), acc).astype(F)
             cnt += nz
-        v = np.where(cnt > 0, (acc / cnt.astype(F)).astype(F), v).astype(F)
+        with np.errstate(divide="ignore", invalid="ignore"):  # columns without nonzero codes keep v
+            v = np.where(cnt > 0, (acc / cnt.astype(F)).astype(F), v).astype(F)
         half = ((v[None, :] * a).astype(F) * F(0.5)).astype(F)
         T = _assign(d, half)
     return v, T

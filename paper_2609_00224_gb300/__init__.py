@@ -85,6 +85,8 @@ def load(build_if_missing: bool = True):
     lib.qtea_layout_copy_packed.argtypes = [P, P, ctypes.c_size_t, P]
     lib.qtea_gemv_m1_static.restype = i32
     lib.qtea_gemv_m1_static.argtypes = [P, P, i32, i32, i32, P, P, P, P, P, P, P]
+    lib.qtea_quantize.restype = i32
+    lib.qtea_quantize.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, P, P, P, P, P, P, P]
     _lib = lib
     return lib
 
@@ -260,3 +262,36 @@ def packed_bytes(layout: Layout):
     if rc:
         raise QteaError(rc, "qtea_layout_copy_packed")
     return out[:n]
+
+
+def qtea_quantize(W, hdiag, group_size: Optional[int] = None, n_salient: int = 0, bias: bool = False,
+                  fit_iters: int = 4, rescale_iters: int = 2, stream=None) -> dict:
+    """The quantizer's per-layer steps on the GPU: fp32 weights W [N][K] and diag(H) [K] (CUDA
+    tensors) to the GEMV's inputs. Returns a dict of CUDA tensors: codes int8 [N][K], row_scale
+    int16 (fp16 bits) [N][G] or [N][2G] with bias, col_scale [K], salient_idx int32 [s],
+    residual_vals [N/4][s] and residual_idx uint8 [N/4][ceil(s/4)]."""
+    import torch
+    if W.dim() != 2:
+        raise ValueError("W must be [N][K]")
+    N, K = W.shape
+    g = K if group_size is None else int(group_size)
+    G = (K + g - 1) // g if g > 0 else 1
+    s = int(n_salient)
+    dev = W.device
+    out = dict(
+        codes=torch.empty((N, K), dtype=torch.int8, device=dev),
+        row_scale=torch.empty((N, G * (2 if bias else 1)), dtype=torch.int16, device=dev),
+        col_scale=torch.empty((K,), dtype=torch.int16, device=dev),
+        salient_idx=torch.empty((s,), dtype=torch.int32, device=dev),
+        residual_vals=torch.empty((N // 4, s), dtype=torch.int16, device=dev),
+        residual_idx=torch.empty((N // 4, (s + 3) // 4), dtype=torch.uint8, device=dev),
+    )
+    rc = load().qtea_quantize(
+        _ptr(W, (torch.float32,), "W"), _ptr(hdiag, (torch.float32,), "hdiag", (K,)), N, K, g, s,
+        QTEA_OPT_BIAS if bias else 0, int(fit_iters), int(rescale_iters), out["codes"].data_ptr(),
+        out["row_scale"].data_ptr(), out["col_scale"].data_ptr(), out["salient_idx"].data_ptr() if s else None,
+        out["residual_vals"].data_ptr() if s else None, out["residual_idx"].data_ptr() if s else None,
+        _stream(stream))
+    if rc:
+        raise QteaError(rc, "qtea_quantize")
+    return out

@@ -680,6 +680,42 @@ int qtea_layout_describe(const qtea_layout* l, qtea_layout_desc* out) {
   return QTEA_OK;
 }
 
+int qtea_quantize(const float* W, const float* hdiag, int N, int K, int group_size, int n_salient, int options,
+                  int fit_iters, int rescale_iters, int8_t* codes, uint16_t* row_scale, uint16_t* col_scale,
+                  int32_t* salient_idx, uint16_t* residual_vals, uint8_t* residual_idx, qtea_stream_t stream) {
+  if (N <= 0 || K <= 0 || N > (1 << 20) || K > 65536 || n_salient < 0 || n_salient > K) return QTEA_ERR_INVALID_ARG;
+  if (group_size != K && group_size != 128) return QTEA_ERR_UNSUPPORTED;
+  if (n_salient > 0 && N % 4 != 0) return QTEA_ERR_INVALID_ARG;
+  if (options & ~QTEA_OPT_BIAS) return QTEA_ERR_INVALID_ARG;
+  if (fit_iters < 0 || fit_iters > 64 || rescale_iters < 0 || rescale_iters > 64) return QTEA_ERR_INVALID_ARG;
+  if (!W || !hdiag || !codes || !row_scale || !col_scale) return QTEA_ERR_INVALID_ARG;
+  if (n_salient > 0 && (!salient_idx || !residual_vals || !residual_idx)) return QTEA_ERR_INVALID_ARG;
+  if (!aligned(W, 4) || !aligned(hdiag, 4) || !aligned(row_scale, 2) || !aligned(col_scale, 2) ||
+      (n_salient > 0 && (!aligned(salient_idx, 4) || !aligned(residual_vals, 2))))
+    return QTEA_ERR_INVALID_ARG;
+  QuantArgs a;
+  a.W = W;
+  a.h = hdiag;
+  a.N = N;
+  a.K = K;
+  a.group = group_size;
+  a.s = n_salient;
+  a.bias = (options & QTEA_OPT_BIAS) ? 1 : 0;
+  a.fit_iters = fit_iters;
+  a.rescale_iters = rescale_iters;
+  a.codes = codes;
+  a.row_scale = row_scale;
+  a.col_scale = col_scale;
+  a.sal = salient_idx;
+  a.rvals = residual_vals;
+  a.ridx = residual_idx;
+  if (launch_quantize(a, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_ERR_CUDA;
+  }
+  return QTEA_OK;
+}
+
 int qtea_set_layout_options(qtea_layout* l, int options) {
   if (!l || (options & ~(QTEA_OPT_BIAS | QTEA_OPT_RESIDUAL_FP8)) != 0) return QTEA_ERR_INVALID_ARG;
   l->options = options;

@@ -244,6 +244,20 @@ struct PaperParams {
   int M, N, K, s, G, group_size, row_bytes, format, bias, residual_fp8;
 };
 
+// The quantizer's per-layer steps (qtea_quant.cu).
+struct QuantArgs {
+  const float* W;           // [N][K]
+  const float* h;           // [K] diag(H)
+  int N, K, group, s, bias, fit_iters, rescale_iters;
+  int8_t* codes;            // [N][K]
+  uint16_t* row_scale;      // [N][G] alpha, or [N][G][2] (alpha, beta)
+  uint16_t* col_scale;      // [K] v
+  int32_t* sal;             // [s]
+  uint16_t* rvals;          // [N/4][s]
+  uint8_t* ridx;            // [N/4][ceil(s/4)]
+};
+
+cudaError_t launch_quantize(const QuantArgs& a, cudaStream_t st);
 cudaError_t launch_paper(const PaperParams& p, cudaStream_t st);
 cudaError_t launch_pack_base3(const int8_t* codes, int N, int K, uint8_t* packed, int* bad_flag, cudaStream_t st);
 cudaError_t launch_m1(const TensorMaps& maps, const GroupParams& p, int grid, size_t smem, cudaStream_t st);

@@ -48,6 +48,15 @@ def test_host_side_argument_checks_need_no_gpu():
                                 ctypes.byref(out)) == qt.QTEA_ERR_UNSUPPORTED  # groups other than K or 128
     assert lib.qtea_set_layout_options(None, qt.QTEA_OPT_BIAS) == qt.QTEA_ERR_INVALID_ARG
     assert lib.qtea_gemv(None, None, None, None, None, None, None, None, 1, None) == qt.QTEA_ERR_INVALID_ARG
+    q = lib.qtea_quantize
+    P = ctypes.c_void_p(16)
+    assert q(None, P, 4, 8, 8, 0, 0, 2, 2, P, P, P, None, None, None, None) == qt.QTEA_ERR_INVALID_ARG  # no W
+    assert q(P, P, 6, 8, 8, 4, 0, 2, 2, P, P, P, P, P, P, None) == qt.QTEA_ERR_INVALID_ARG  # N % 4 with s > 0
+    assert q(P, P, 4, 8, 8, 9, 0, 2, 2, P, P, P, P, P, P, None) == qt.QTEA_ERR_INVALID_ARG  # s > K
+    assert q(P, P, 4, 8, 8, 2, 0, 2, 2, P, P, P, None, P, P, None) == qt.QTEA_ERR_INVALID_ARG  # no salient list
+    assert q(P, P, 4, 256, 64, 0, 0, 2, 2, P, P, P, None, None, None, None) == qt.QTEA_ERR_UNSUPPORTED  # group
+    assert q(P, P, 4, 8, 8, 0, 4, 2, 2, P, P, P, None, None, None, None) == qt.QTEA_ERR_INVALID_ARG  # option
+    assert q(P, P, 4, 8, 8, 0, 0, -1, 2, P, P, P, None, None, None, None) == qt.QTEA_ERR_INVALID_ARG  # iters
     lib.qtea_free(None)
 
 
