@@ -626,6 +626,45 @@ def qtea_arm(args):
                  "2bit_fp16_residual": dict(paper_leg(qt.QTEA_FMT_2BIT, False),
                                             kernel="qtea_gemv_mb_kernel (tensor cores, scale groups)")}
 
+    # ---- the quantizer's per-layer steps (scores, top-s, group fit, column rescale, binary16 scales,
+    #      1:4 residual) on the Llama3-8B layer's seven fp32 weight matrices: 128-column groups with
+    #      beta, 4 alpha refits, 2 rescale rounds, the GEMV's salient count
+    def quant_leg():
+        shapes = synth.config_shapes(1)
+        gen = torch.Generator(device="cuda").manual_seed(1234)
+        mats = []
+        for _, N, K in shapes:
+            W = (torch.randn(N, K, device="cuda", generator=gen) * 0.02).half().float()
+            h = torch.exp(torch.randn(K, device="cuda", generator=gen)).half().float()
+            mats.append((W, h, synth.salient_count(K)))
+        stream.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(stream):
+            for W, h, s in mats:  # warm-up (allocator pool, caches)
+                qt.qtea_quantize(W, h, group_size=128, n_salient=s, bias=True, stream=stream)
+        stream.synchronize()
+        reps = 3
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        with torch.cuda.stream(stream):
+            for _ in range(reps):
+                for W, h, s in mats:
+                    qt.qtea_quantize(W, h, group_size=128, n_salient=s, bias=True, stream=stream)
+        e1.record(stream)
+        stream.synchronize()
+        ms = e0.elapsed_time(e1) / reps
+        w = sum(N * K for _, N, K in shapes)
+        del mats
+        torch.cuda.empty_cache()
+        return {"workload": "llama3_8b_layer_fp32_weights", "ms_per_layer": round(ms, 3),
+                "Mweights_per_s": round(w / (ms * 1e-3) / 1e6, 1),
+                "W_read_GBps_once": round(4 * w / (ms * 1e-3) / 1e9, 1),
+                "settings": {"group": 128, "bias": True, "fit_iters": 4, "rescale_iters": 2},
+                "bit_identical_to": "oracle/quantize.py (tests/test_gpu_quantize.py)"}
+
+    quant = None
+    if not args.no_quant:
+        quant = quant_leg()
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         probs = [g["host"] for g in layers[0]]
@@ -654,7 +693,7 @@ def qtea_arm(args):
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
                          "us_per_launch": round(1e3 * total_ms / args.steps, 3),
                          "us_per_launch_isolated": None if iso_us is None else round(iso_us, 3)},
-            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
+            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "quantizer": quant, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
             "setup_s": round(t_gen, 1),
         }
         print(json.dumps(line), flush=True)
@@ -701,6 +740,7 @@ def main():
     ap.add_argument("--no-dense", action="store_true", help="skip the dense fp16 cuBLAS baseline")
     ap.add_argument("--no-m-sweep", action="store_true", help="skip the Qwen3-14B batch sweep (M = 1 .. 16)")
     ap.add_argument("--no-paper", action="store_true", help="skip the layer in the paper's own storage")
+    ap.add_argument("--no-quant", action="store_true", help="skip the quantizer timing")
     ap.add_argument("--layers", type=int, default=32,
                     help="independent resident layers the steps rotate over (32 = the whole Llama3-8B stack)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
