@@ -194,6 +194,70 @@ def oracle_sample_seconds(problems, rows_stride, budget_s):
     return done_bytes, t_total, n_rows_total
 
 
+def _oracle_rows_worker(w, workers, stride, cmd_q, done_q):
+    """One host core of the parallel oracle timing: generate the layer-0 problems once, then for
+    each step compute the step's sampled rows (every stride-th row, offset by the step) that fall to
+    this worker, reporting (bytes, rows, seconds)."""
+    import oracle
+    import synth
+    probs = [synth.config_problem(CONFIG_ID, mi, layer=0) for mi in range(7)]
+    done_q.put(("ready", w))
+    while True:
+        cmd = cmd_q.get()
+        if cmd is None:
+            return
+        step = cmd
+        t0 = time.perf_counter()
+        b, n = 0.0, 0
+        for p in probs:
+            rows = np.arange(step % stride, p.N, stride, dtype=np.int32)[w::workers]
+            if len(rows):
+                oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx, rows=rows,
+                            want_bound=False)
+            b += algorithmic_bytes(p.N, p.K, p.s) * len(rows) / p.N
+            n += len(rows)
+        done_q.put(("step", w, b, n, time.perf_counter() - t0))
+
+
+class ParallelOracle:
+    """The oracle as it stands, one process per host core (spawned, so no CUDA state is inherited),
+    each taking a disjoint share of a step's sampled output rows."""
+
+    def __init__(self, stride, workers=None):
+        import multiprocessing as mp
+        ctx = mp.get_context("spawn")
+        self.workers = workers or len(os.sched_getaffinity(0))
+        self.stride = stride
+        self.done_q = ctx.Queue()
+        self.cmd_qs = [ctx.Queue() for _ in range(self.workers)]
+        self.procs = [ctx.Process(target=_oracle_rows_worker, args=(w, self.workers, stride, self.cmd_qs[w],
+                                                                   self.done_q), daemon=True)
+                      for w in range(self.workers)]
+        for pr in self.procs:
+            pr.start()
+        for _ in range(self.workers):
+            tag, _w = self.done_q.get(timeout=600)
+            assert tag == "ready"
+
+    def step(self, step):
+        """One step on all workers; returns (bytes, rows, wall seconds)."""
+        t0 = time.perf_counter()
+        for q in self.cmd_qs:
+            q.put(step)
+        b, n = 0.0, 0
+        for _ in range(self.workers):
+            _tag, _w, bw, nw, _t = self.done_q.get(timeout=600)
+            b += bw
+            n += nw
+        return b, n, time.perf_counter() - t0
+
+    def close(self):
+        for q in self.cmd_qs:
+            q.put(None)
+        for pr in self.procs:
+            pr.join(timeout=60)
+
+
 # ---------------------------------------------------------------------------- arms
 
 def max_over_ranks(ms, world, device):
@@ -228,28 +292,28 @@ def reference_arm(args):
     import synth
     oracle.build()
     synth.build()
-    problems = [synth.config_problem(CONFIG_ID, mi, layer=0) for mi in range(7)]
-    rows_stride = 64  # every 64th output row of each of the 7 GEMVs per step
-    for _ in range(args.warmup):
-        oracle_sample_seconds(problems[1:2], rows_stride * 4, 0.0)
-    tot_b, tot_t, tot_rows = 0.0, 0.0, 0
-    for step in range(args.steps):
-        for p in problems:
-            rows = np.arange(step % rows_stride, p.N, rows_stride, dtype=np.int32)
-            t0 = time.perf_counter()
-            oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx, rows=rows,
-                        want_bound=False)
-            tot_t += time.perf_counter() - t0
-            tot_b += algorithmic_bytes(p.N, p.K, p.s) * len(rows) / p.N
-            tot_rows += len(rows)
+    rows_stride = 16  # every 16th output row of each of the 7 GEMVs per step
+    pool = ParallelOracle(rows_stride)
+    try:
+        for w in range(args.warmup):
+            pool.step(w)
+        tot_b, tot_t, tot_rows = 0.0, 0.0, 0
+        for step in range(args.steps):
+            b, n, t = pool.step(step)
+            tot_b += b
+            tot_rows += n
+            tot_t += t
+    finally:
+        pool.close()
     value = tot_b / tot_t / 1e9
     sample = (f"each step: every {rows_stride}th output row of the 7 Llama3-8B layer GEMVs "
-              f"({tot_rows // max(args.steps, 1)} rows/step), fp64 oracle, 1 thread")
+              f"({tot_rows // max(args.steps, 1)} rows/step), fp64 oracle, {pool.workers} processes "
+              f"(one per host core) on disjoint rows")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / max(args.steps, 1),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {"workload": WORKLOAD, "M": 1, "note": "bounded row sample per step"},
-            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": pool.workers, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
     return 0
@@ -626,6 +690,54 @@ def qtea_arm(args):
                  "2bit_fp16_residual": dict(paper_leg(qt.QTEA_FMT_2BIT, False),
                                             kernel="qtea_gemv_mb_kernel (tensor cores, scale groups)")}
 
+    # ---- the Llama3-70B layer (8192-wide, 28672-row MLP: the large-K shapes) at M = 1, the seven
+    #      GEMVs per step as one grouped call, rotating over resident layers whose codes exceed L2
+    def llama70b_leg():
+        cfg, n_res, nsteps = 3, 3, 24
+        shapes = synth.config_shapes(cfg)
+        players, pbytes = [], []
+        for li in range(n_res):
+            L, b = [], 0
+            for mi, (_, N, K) in enumerate(shapes):
+                pp = synth.config_problem(cfg, mi, layer=li)
+                f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
+                T = torch.from_numpy(pp.T).cuda()
+                lay = qt.qtea_pack_layout(T, n_salient=pp.s)
+                lay.set_activation_precision(args.act_bits)
+                del T
+                L.append(dict(x=f16(pp.x), layout=lay, row_scale=f16(pp.alpha.reshape(-1)), col_scale=f16(pp.v),
+                              salient_idx=torch.from_numpy(pp.salient_idx).cuda(), residual_vals=f16(pp.residual_vals),
+                              residual_idx=torch.from_numpy(pp.residual_idx).cuda(),
+                              y=torch.empty((1, N), dtype=torch.float32, device="cuda")))
+                b += algorithmic_bytes(N, K, pp.s)
+            players.append(L)
+            pbytes.append(b)
+        codes = sum(g["layout"].describe()["packed_bytes"] for L in players for g in L)
+        with torch.cuda.stream(stream):
+            qt.qtea_gemv_grouped(players[0], stream=stream)
+        gp = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gp, stream=stream):
+            for st in range(nsteps):
+                qt.qtea_gemv_grouped(players[st % n_res], stream=stream)
+        ms = timed_replay(gp)
+        del gp
+        status = max(qt.qtea_device_status(g["layout"]) for L in players for g in L)
+        if status:
+            raise RuntimeError(f"device status {status} in the Llama3-70B steps")
+        tb = sum(pbytes[st % n_res] for st in range(nsteps))
+        gbs = tb / (ms * 1e-3) / 1e9
+        res = {"workload": "llama3_70b_layer_gemvs", "M": 1, "us_per_step": round(ms * 1e3 / nsteps, 2),
+               "GBps": round(gbs, 1), "frac_of_measured_hbm": round(gbs / peak, 3),
+               "bytes_per_step": round(tb / nsteps), "layers_resident": n_res, "resident_code_bytes": codes,
+               "act_bits": args.act_bits, "kernel": "qtea_gemv_m1_kernel (one grouped launch per step)"}
+        del players
+        torch.cuda.empty_cache()
+        return res
+
+    l70 = None
+    if not args.no_70b:
+        l70 = llama70b_leg()
+
     # ---- the quantizer's per-layer steps (scores, top-s, group fit, column rescale, binary16 scales,
     #      1:4 residual) on the Llama3-8B layer's seven fp32 weight matrices: 128-column groups with
     #      beta, 4 alpha refits, 2 rescale rounds, the GEMV's salient count
@@ -672,6 +784,19 @@ def qtea_arm(args):
         cpu = {"value": round(b / t / 1e9, 4), "unit": "GB/s", "cores": 1, "kind": "oracle",
                "sample": f"{rows} output rows (every 16th row, cycling over the 7 layer-0 GEMVs) for "
                          f"{t:.1f} s, fp64, 1 thread"}
+        if not args.no_cpu_all_cores:
+            pool = ParallelOracle(16)
+            try:
+                pb, pn, pt, st = 0.0, 0, 0.0, 0
+                while pt < args.cpu_seconds:
+                    b_, n_, t_ = pool.step(st)
+                    pb, pn, pt, st = pb + b_, pn + n_, pt + t_, st + 1
+            finally:
+                pool.close()
+            cpu["all_cores"] = {"value": round(pb / pt / 1e9, 4), "unit": "GB/s", "cores": pool.workers,
+                                "kind": "oracle",
+                                "sample": f"{pn} output rows ({st} steps of every 16th row of the 7 layer-0 "
+                                          f"GEMVs) in {pt:.1f} s, fp64, one process per core on disjoint rows"}
 
     traffic = profiled_traffic()
 
@@ -693,7 +818,7 @@ def qtea_arm(args):
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
                          "us_per_launch": round(1e3 * total_ms / args.steps, 3),
                          "us_per_launch_isolated": None if iso_us is None else round(iso_us, 3)},
-            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "quantizer": quant, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
+            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "llama3_70b_layer": l70, "quantizer": quant, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
             "setup_s": round(t_gen, 1),
         }
         print(json.dumps(line), flush=True)
@@ -741,10 +866,12 @@ def main():
     ap.add_argument("--no-m-sweep", action="store_true", help="skip the Qwen3-14B batch sweep (M = 1 .. 16)")
     ap.add_argument("--no-paper", action="store_true", help="skip the layer in the paper's own storage")
     ap.add_argument("--no-quant", action="store_true", help="skip the quantizer timing")
+    ap.add_argument("--no-70b", action="store_true", help="skip the Llama3-70B layer steps")
     ap.add_argument("--layers", type=int, default=32,
                     help="independent resident layers the steps rotate over (32 = the whole Llama3-8B stack)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-cpu-all-cores", action="store_true", help="skip the oracle timing on all host cores")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-per-shape", action="store_true")
     ap.add_argument("--act-bits", type=int, choices=[16, 24], default=24,
