@@ -150,6 +150,10 @@ int launch_paper_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
   p.format = l->format;
   p.bias = (l->options & QTEA_OPT_BIAS) ? 1 : 0;
   p.residual_fp8 = (l->options & QTEA_OPT_RESIDUAL_FP8) ? 1 : 0;
+  p.staged_ok = l->paper_staged_ok ? 1 : 0;
+  p.sm_count = l->sm_count > 0 ? l->sm_count : 1;
+  p.smem_optin = l->smem_optin;
+  p.smem_per_sm = l->smem_per_sm;
   return launch_paper(p, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
 }
 
@@ -575,6 +579,11 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
   l->row_bytes = format == QTEA_FMT_BASE3 ? l->K_pad / 128 * 26 : l->K_pad / 4;
   l->device = dev;
   l->act_bits = 24;
+  l->sm_count = prop.multiProcessorCount;
+  l->smem_optin = prop.sharedMemPerBlockOptin;
+  l->smem_per_sm = prop.sharedMemPerMultiprocessor;
+  l->paper_staged_ok = paper_configure(prop.sharedMemPerBlockOptin) == cudaSuccess;
+  if (!l->paper_staged_ok) cudaGetLastError();
   l->packed_bytes = (size_t)N * (size_t)l->row_bytes;
   if (cudaMalloc(&l->packed, l->packed_bytes > 0 ? l->packed_bytes : 16) != cudaSuccess ||
       cudaMalloc(&l->status, 2 * sizeof(int)) != cudaSuccess) {

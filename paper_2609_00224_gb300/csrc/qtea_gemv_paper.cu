@@ -16,6 +16,8 @@
 // of four.
 #include <cuda_fp16.h>
 
+#include <algorithm>
+
 #include "qtea_internal.h"
 
 namespace qtea {
@@ -143,6 +145,410 @@ __global__ void __launch_bounds__(kPaperWarps * 32) qtea_gemv_paper_kernel(const
   }
 }
 
+// The same product with the activations staged once per CTA (M <= 4, when v*x of every batch row,
+// the per-group sums of x and the base-3 table fit in shared memory): each CTA writes
+// x~[m][j] = v_j * x[m][j] (exact in fp32) and, with beta, sum_{j in g} x[m][j] (partial sums of
+// eight columns, then a fixed order), then its warps walk rows. A warp loads 26 code bytes per
+// lane (832 consecutive bytes of the row) before decoding any; lane l takes bytes l, l + 32, ...,
+// so the columns of a load instruction are 4 or 5 apart and their x~ lie in distinct banks. Each
+// byte adds alpha_g * sum T x~ over its columns; beta * sum x is added once per group.
+constexpr int kStagedWarps = 16;
+constexpr int kStagedBatch = 26;
+
+size_t staged_smem_bytes(int M, int K, int G, bool bias) {
+  return (size_t)M * K * sizeof(float) + (bias ? (size_t)M * G * sizeof(float) : 0) +
+         (size_t)M * ((K + 7) / 8) * sizeof(float) + 256 * sizeof(uint16_t);
+}
+
+template <int MB, bool B3>
+__global__ void __launch_bounds__(kStagedWarps * 32) qtea_gemv_paper_staged_kernel(const PaperParams p) {
+  extern __shared__ __align__(16) float smf[];
+  const int K = p.K, G = p.G, M = p.M;
+  const int K8 = (K + 7) / 8;
+  float* xt = smf;                                     // [M][K]
+  float* sx = xt + (size_t)M * K;                      // [M][G], with beta
+  float* s8 = sx + (p.bias ? (size_t)M * G : 0);       // [M][K8] sums of x over eight columns
+  uint16_t* lut = reinterpret_cast<uint16_t*>(s8 + (size_t)M * K8);  // [243]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (B3)
+    for (int i = threadIdx.x; i < 243; i += blockDim.x) {
+      int b = i;
+      uint32_t v = 0;
+      for (int d = 0; d < 5; ++d) {
+        v |= (uint32_t)(b % 3) << (2 * d);
+        b /= 3;
+      }
+      lut[i] = (uint16_t)v;
+    }
+  // x~ and eight-column sums of x: 16-byte loads where x and v are 16-byte aligned and K % 8 == 0
+  const bool vec = (K & 7) == 0 && ((reinterpret_cast<uintptr_t>(p.x) | reinterpret_cast<uintptr_t>(p.v)) & 15) == 0;
+  if (vec) {
+    constexpr int kU = 4;
+    for (int t0 = threadIdx.x; t0 < M * K8; t0 += kU * blockDim.x) {
+      uint4 xv[kU], vv[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int t = t0 + u * blockDim.x;
+        if (t < M * K8) {
+          const int m = t / K8, j8 = t - m * K8;
+          xv[u] = __ldg(reinterpret_cast<const uint4*>(p.x + (size_t)m * K) + j8);
+          vv[u] = __ldg(reinterpret_cast<const uint4*>(p.v) + j8);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int t = t0 + u * blockDim.x;
+        if (t >= M * K8) continue;
+        const int m = t / K8, j8 = t - m * K8;
+        const uint32_t xw[4] = {xv[u].x, xv[u].y, xv[u].z, xv[u].w}, vw[4] = {vv[u].x, vv[u].y, vv[u].z, vv[u].w};
+        float sum8 = 0.f;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+          const float xe = h2f((uint16_t)(xw[e >> 1] >> (16 * (e & 1))));
+          const float ve = h2f((uint16_t)(vw[e >> 1] >> (16 * (e & 1))));
+          xt[(size_t)m * K + 8 * j8 + e] = ve * xe;
+          sum8 += xe;
+        }
+        s8[t] = sum8;
+      }
+    }
+  } else {
+    for (int t = threadIdx.x; t < M * K8; t += blockDim.x) {
+      const int m = t / K8, j8 = t - m * K8;
+      float sum8 = 0.f;
+      for (int e = 0; e < 8; ++e) {
+        const int j = 8 * j8 + e;
+        if (j >= K) break;
+        const float xe = h2f(__ldg(p.x + (size_t)m * K + j));
+        xt[(size_t)m * K + j] = h2f(__ldg(p.v + j)) * xe;
+        sum8 += xe;
+      }
+      s8[t] = sum8;
+    }
+  }
+  __syncthreads();
+  if (p.bias)  // groups are K or 128 columns: whole eight-column blocks, summed in order
+    for (int t = threadIdx.x; t < M * G; t += blockDim.x) {
+      const int m = t / G, g = t - m * G;
+      const int b0 = g * p.group_size / 8, b1 = min(K8, (g * p.group_size + p.group_size + 7) / 8);
+      float a = 0.f;
+      for (int b8 = b0; b8 < b1; ++b8) a += s8[(size_t)m * K8 + b8];
+      sx[t] = a;
+    }
+  __syncthreads();
+
+  const int per = B3 ? 5 : 4, bytes = B3 ? 26 : 32;
+  const int sc_stride = p.bias ? 2 : 1;
+  for (int o = blockIdx.x * kStagedWarps + warp; o < p.N; o += gridDim.x * kStagedWarps) {
+    const uint8_t* row = p.packed + (size_t)o * p.row_bytes;
+    const uint16_t* sc = p.scales + (size_t)o * G * sc_stride;
+    // bring the row's scales into L1 ahead of the per-byte lookups
+    float warm = 0.f;
+    for (int e = 2 * lane; e < G * sc_stride; e += 64) warm += h2f(__ldg(sc + e));
+    float acc[MB];
+#pragma unroll
+    for (int m = 0; m < MB; ++m) acc[m] = 0.f;
+    for (int i0 = 0; i0 < p.row_bytes; i0 += 32 * kStagedBatch) {
+      uint32_t byte[kStagedBatch];
+#pragma unroll
+      for (int k = 0; k < kStagedBatch; ++k) {
+        const int i = i0 + lane + 32 * k;
+        byte[k] = i < p.row_bytes ? (uint32_t)__ldg(row + i) : 0xFFFFFFFFu;
+      }
+#pragma unroll
+      for (int k = 0; k < kStagedBatch; ++k) {
+        if (byte[k] == 0xFFFFFFFFu) continue;
+        const int i = i0 + lane + 32 * k;
+        const int blk = i / bytes, q = i - blk * bytes;
+        const int c0 = blk * 128 + per * q;
+        if (c0 >= K) continue;
+        const float al = h2f(__ldg(sc + (size_t)((blk * 128) / p.group_size) * sc_stride));
+        const uint32_t codes = B3 ? (uint32_t)lut[min(byte[k], 242u)] : byte[k];
+        float part[MB];
+#pragma unroll
+        for (int m = 0; m < MB; ++m) part[m] = 0.f;
+#pragma unroll
+        for (int d = 0; d < per; ++d) {
+          const int col = c0 + d;
+          if ((B3 && per * q + d >= 128) || col >= K) continue;
+          const uint32_t c = (codes >> (2 * d)) & 3u;
+#pragma unroll
+          for (int m = 0; m < MB; ++m) {
+            if (m < M) {
+              const float xv = xt[(size_t)m * K + col];
+              part[m] += c == 2u ? xv : (c == 0u ? -xv : 0.f);
+            }
+          }
+        }
+#pragma unroll
+        for (int m = 0; m < MB; ++m) acc[m] += al * part[m];
+      }
+    }
+    acc[0] += warm * 0.f;  // keeps the warming loads (adds zero)
+    if (p.bias)
+      for (int g = lane; g < G; g += 32) {
+        const float be = h2f(__ldg(sc + (size_t)g * 2 + 1));
+#pragma unroll
+        for (int m = 0; m < MB; ++m)
+          if (m < M) acc[m] += be * sx[(size_t)m * G + g];
+      }
+    float res[MB];
+#pragma unroll
+    for (int m = 0; m < MB; ++m) res[m] = 0.f;
+    if (p.s > 0) {
+      const int q4 = o >> 2, pos = o & 3, rs = (p.s + 3) / 4;
+      for (int c0 = lane; c0 < p.s; c0 += 128) {
+        uint32_t pb[4];
+        int jj[4];
+        float r[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int c = c0 + 32 * k;
+          const bool in = c < p.s;
+          pb[k] = in ? __ldg(p.ridx + (size_t)q4 * rs + (c >> 2)) : 0u;
+          jj[k] = in ? __ldg(p.sal + c) : 0;
+          const size_t e = (size_t)q4 * p.s + c;
+          r[k] = !in ? 0.f
+                     : p.residual_fp8 ? e4m3_to_float(__ldg(reinterpret_cast<const uint8_t*>(p.rvals) + e))
+                                      : h2f(__ldg(reinterpret_cast<const uint16_t*>(p.rvals) + e));
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int c = c0 + 32 * k;
+          if (c >= p.s || ((pb[k] >> (2 * (c & 3))) & 3u) != (uint32_t)pos) continue;
+          const int j = jj[k] < 0 ? 0 : (jj[k] >= K ? K - 1 : jj[k]);
+#pragma unroll
+          for (int m = 0; m < MB; ++m)
+            if (m < M) res[m] += r[k] * h2f(__ldg(p.x + (size_t)m * K + j));
+        }
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < MB; ++m) {
+      float a = acc[m], r = res[m];
+#pragma unroll
+      for (int off = 16; off; off >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, off);
+        r += __shfl_xor_sync(0xffffffffu, r, off);
+      }
+      if (lane == 0 && m < M) p.y[(size_t)m * p.N + o] = a + r;
+    }
+  }
+}
+
+// Base-3 layouts with staged activations in fixed point (M <= 4): per batch row and 128-column block
+// the CTA scales x~ = v*x by a power of two so that |X| < 2^22 (X = round(x~ * 2^e), e from the
+// block's largest |x~|), splits X into three byte planes (low and middle unsigned, top signed) and
+// stores, per five-column group q of the block, one 32-byte record: the planes of columns 5q..5q+3
+// (one word each), of column 5q+4 (one word each, other lanes zero), and S = sum of the group's X.
+// A 243-entry table turns a code byte into the same two words of codes c = T + 1. Per byte,
+// sum_d c_d X_d is six dp4a, exact in int32; sum_d T_d X_d = that - S; it is scaled once by
+// alpha * 2^-e. The rounding of X is the only approximation: |x~ - X 2^-e| <= 2^-e / 2 with
+// 2^-e <= 2^-21 * max|x~| of the block.
+constexpr int kB3Rec = 8;          // words per five-column record
+constexpr int kB3BlockWords = 212;  // records of one block (26 x 8 words) plus 4 words: lanes that
+                                    // read different blocks' records hit distinct banks
+
+size_t b3_smem_bytes(int M, int K, int G, bool bias) {
+  const size_t n_blocks = (size_t)(K + 127) / 128;
+  return (size_t)M * n_blocks * kB3BlockWords * sizeof(uint32_t) + 2 * (size_t)M * n_blocks * sizeof(float) +
+         (bias ? (size_t)M * G * sizeof(float) : 0) + 243 * sizeof(uint2) + 16;
+}
+
+template <int MB>
+__global__ void __launch_bounds__(kStagedWarps * 32) qtea_gemv_paper_b3_kernel(const PaperParams p) {
+  extern __shared__ __align__(16) uint32_t smw[];
+  const int K = p.K, G = p.G, M = p.M;
+  const int n_blocks = (K + 127) / 128;
+  uint32_t* rec = smw;                                                    // [M][n_blocks][212]
+  float* inv = reinterpret_cast<float*>(rec + (size_t)M * n_blocks * kB3BlockWords);  // [M][n_blocks] 2^-e
+  float* sx = inv + (size_t)M * n_blocks;                                 // [M][G] sum of x, with beta
+  uint2* lut = reinterpret_cast<uint2*>(sx + (p.bias ? (size_t)M * G : 0) + (size_t)M * n_blocks + 2);  // [243]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (reinterpret_cast<uintptr_t>(lut) & 7) lut = reinterpret_cast<uint2*>(reinterpret_cast<uintptr_t>(lut) + 4);
+  for (int i = threadIdx.x; i < 243; i += blockDim.x) {
+    int b = i;
+    uint32_t w1 = 0, w2 = 0;
+    for (int d = 0; d < 5; ++d) {
+      const uint32_t c = (uint32_t)(b % 3);
+      b /= 3;
+      if (d < 4) w1 |= c << (8 * d);
+      else w2 = c;
+    }
+    lut[i] = make_uint2(w1, w2);
+  }
+  // one warp per (batch row, block), two tasks' loads in flight: lane q < 26 owns columns
+  // 5q .. 5q+4 of the block; the warp also sums the block's x for the beta term
+  float* bx = sx + (p.bias ? (size_t)M * G : 0);  // [M][n_blocks], in the slack before the table
+  for (int t0 = warp; t0 < M * n_blocks; t0 += 2 * kStagedWarps) {
+    float xv[2][5], vv[2][5];
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int t = t0 + u * kStagedWarps;
+      const int m = t / n_blocks, blk = t - m * n_blocks;
+#pragma unroll
+      for (int d = 0; d < 5; ++d) {
+        const int cb = 5 * lane + d, col = blk * 128 + cb;
+        const bool in = t < M * n_blocks && lane < 26 && cb < 128 && col < K;
+        xv[u][d] = in ? h2f(__ldg(p.x + (size_t)m * K + col)) : 0.f;
+        vv[u][d] = in ? h2f(__ldg(p.v + col)) : 0.f;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int t = t0 + u * kStagedWarps;
+      if (t >= M * n_blocks) break;  // warp-uniform
+      float xt[5];
+      float amax = 0.f, xs = 0.f;
+#pragma unroll
+      for (int d = 0; d < 5; ++d) {
+        xt[d] = vv[u][d] * xv[u][d];
+        amax = fmaxf(amax, fabsf(xt[d]));
+        xs += xv[u][d];
+      }
+#pragma unroll
+      for (int off = 16; off; off >>= 1) {
+        amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
+        xs += __shfl_xor_sync(0xffffffffu, xs, off);
+      }
+      int ex = 0;
+      if (amax > 0.f) frexpf(amax, &ex);  // amax < 2^ex
+      const int e = 22 - ex;              // |X| <= 2^22 * amax / 2^ex < 2^22
+      if (lane < 26) {
+        uint32_t a0 = 0, a1 = 0, a2 = 0, b0 = 0, b1 = 0, b2 = 0;
+        int sum = 0;
+#pragma unroll
+        for (int d = 0; d < 5; ++d) {
+          const int X = amax > 0.f ? __float2int_rn(ldexpf(xt[d], e)) : 0;
+          sum += X;
+          const uint32_t u0 = (uint32_t)X & 0xFFu, u1 = ((uint32_t)X >> 8) & 0xFFu, u2 = ((uint32_t)X >> 16) & 0xFFu;
+          if (d < 4) {
+            a0 |= u0 << (8 * d);
+            a1 |= u1 << (8 * d);
+            a2 |= u2 << (8 * d);
+          } else {
+            b0 = u0;
+            b1 = u1;
+            b2 = u2;
+          }
+        }
+        uint32_t* r = rec + (size_t)t * kB3BlockWords + lane * kB3Rec;
+        reinterpret_cast<uint4*>(r)[0] = make_uint4(a0, b0, a1, b1);
+        reinterpret_cast<uint4*>(r)[1] = make_uint4(a2, b2, (uint32_t)sum, 0u);
+      }
+      if (lane == 0) {
+        inv[t] = amax > 0.f ? ldexpf(1.f, -e) : 0.f;
+        bx[t] = xs;
+      }
+    }
+  }
+  __syncthreads();
+  if (p.bias)  // groups of 128 columns are the blocks; a whole-row group sums the blocks in order
+    for (int t = threadIdx.x; t < M * G; t += blockDim.x) {
+      const int m = t / G, g = t - m * G;
+      float a = 0.f;
+      if (p.group_size >= K)
+        for (int blk = 0; blk < n_blocks; ++blk) a += bx[m * n_blocks + blk];
+      else
+        a = bx[m * n_blocks + g];
+      sx[t] = a;
+    }
+  __syncthreads();
+
+  const bool row_group = p.group_size >= K;  // one scale group per row
+  const int sc_stride = p.bias ? 2 : 1;
+  for (int o = blockIdx.x * kStagedWarps + warp; o < p.N; o += gridDim.x * kStagedWarps) {
+    const uint8_t* row = p.packed + (size_t)o * p.row_bytes;
+    const uint16_t* sc = p.scales + (size_t)o * G * sc_stride;
+    float acc[MB];
+#pragma unroll
+    for (int m = 0; m < MB; ++m) acc[m] = 0.f;
+    // lane l takes block b0 + l of the row: its 26 code bytes (13 two-byte loads), one alpha, and
+    // an int32 sum over the block (|sum_j T_j X_j| < 128 * 2^22), converted once
+    for (int b0 = 0; b0 < n_blocks; b0 += 32) {
+      const int blk = b0 + lane;
+      const bool on = blk < n_blocks;
+      const uint16_t* cb = reinterpret_cast<const uint16_t*>(row + (size_t)(on ? blk : 0) * 26);
+      uint32_t h[13];
+#pragma unroll
+      for (int k = 0; k < 13; ++k) h[k] = on ? (uint32_t)__ldg(cb + k) : 0x7979u;  // 121 = five T = 0 digits
+      const float al = on ? h2f(__ldg(sc + (row_group ? 0 : (size_t)blk * sc_stride))) : 0.f;
+      int isum[MB];
+#pragma unroll
+      for (int m = 0; m < MB; ++m) isum[m] = 0;
+#pragma unroll
+      for (int j = 0; j < 26; ++j) {
+        const uint32_t byte = (h[j >> 1] >> (8 * (j & 1))) & 0xFFu;
+        const uint2 cw = lut[min(byte, 242u)];
+#pragma unroll
+        for (int m = 0; m < MB; ++m) {
+          if (m < M) {
+            const uint32_t* r = rec + (size_t)(m * n_blocks + (on ? blk : 0)) * kB3BlockWords + j * kB3Rec;
+            const uint4 r0 = reinterpret_cast<const uint4*>(r)[0];
+            const uint4 r1 = reinterpret_cast<const uint4*>(r)[1];
+            const int s0 = __dp4a(cw.x, r0.x, __dp4a(cw.y, r0.y, 0u));
+            const int s1 = __dp4a(cw.x, r0.z, __dp4a(cw.y, r0.w, 0u));
+            const int s2 = __dp4a((int)cw.x, (int)r1.x, __dp4a((int)cw.y, (int)r1.y, 0));
+            isum[m] += s2 * 65536 + s1 * 256 + s0 - (int)r1.z;
+          }
+        }
+      }
+      if (on)
+#pragma unroll
+        for (int m = 0; m < MB; ++m)
+          if (m < M) acc[m] += (al * inv[m * n_blocks + blk]) * (float)isum[m];
+    }
+    if (p.bias)
+      for (int g = lane; g < G; g += 32) {
+        const float be = h2f(__ldg(sc + (size_t)g * 2 + 1));
+#pragma unroll
+        for (int m = 0; m < MB; ++m)
+          if (m < M) acc[m] += be * sx[(size_t)m * G + g];
+      }
+    float res[MB];
+#pragma unroll
+    for (int m = 0; m < MB; ++m) res[m] = 0.f;
+    if (p.s > 0) {
+      const int q4 = o >> 2, pos = o & 3, rs = (p.s + 3) / 4;
+      for (int c0 = lane; c0 < p.s; c0 += 128) {
+        uint32_t pb[4];
+        int jj[4];
+        float r[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int c = c0 + 32 * k;
+          const bool in = c < p.s;
+          pb[k] = in ? __ldg(p.ridx + (size_t)q4 * rs + (c >> 2)) : 0u;
+          jj[k] = in ? __ldg(p.sal + c) : 0;
+          const size_t e = (size_t)q4 * p.s + c;
+          r[k] = !in ? 0.f
+                     : p.residual_fp8 ? e4m3_to_float(__ldg(reinterpret_cast<const uint8_t*>(p.rvals) + e))
+                                      : h2f(__ldg(reinterpret_cast<const uint16_t*>(p.rvals) + e));
+        }
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int c = c0 + 32 * k;
+          if (c >= p.s || ((pb[k] >> (2 * (c & 3))) & 3u) != (uint32_t)pos) continue;
+          const int j = jj[k] < 0 ? 0 : (jj[k] >= K ? K - 1 : jj[k]);
+#pragma unroll
+          for (int m = 0; m < MB; ++m)
+            if (m < M) res[m] += r[k] * h2f(__ldg(p.x + (size_t)m * K + j));
+        }
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < MB; ++m) {
+      float a = acc[m], r = res[m];
+#pragma unroll
+      for (int off = 16; off; off >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, off);
+        r += __shfl_xor_sync(0xffffffffu, r, off);
+      }
+      if (lane == 0 && m < M) p.y[(size_t)m * p.N + o] = a + r;
+    }
+  }
+}
+
 // Base-3 packing (Sec. 3.5): per row, K_pad3 / 128 groups of 26 bytes; byte q of a group holds
 // columns 5q .. 5q+4 of the group as sum_d (T + 1) 3^d, the lowest column in the least significant
 // digit. Byte 25 holds columns 125-127 and two pad digits; pad digits and columns >= K are digit 1
@@ -176,9 +582,70 @@ __global__ void qtea_pack_base3_kernel(const int8_t* __restrict__ codes, int N, 
 
 }  // namespace
 
+template <int MB, bool B3>
+cudaError_t launch_staged(const PaperParams& p, size_t smem, cudaStream_t st) {
+  int per_sm = 1;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, qtea_gemv_paper_staged_kernel<MB, B3>, kStagedWarps * 32,
+                                                    smem) != cudaSuccess)
+    return cudaGetLastError();
+  const int want = (p.N + kStagedWarps - 1) / kStagedWarps;
+  const int grid = std::max(1, std::min(want, p.sm_count * std::max(per_sm, 1)));
+  qtea_gemv_paper_staged_kernel<MB, B3><<<grid, kStagedWarps * 32, smem, st>>>(p);
+  return cudaGetLastError();
+}
+
+template <int MB>
+cudaError_t launch_b3(const PaperParams& p, size_t smem, cudaStream_t st) {
+  int per_sm = 1;  // resident CTAs per SM: the grid is persistent, so each CTA stages once
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, qtea_gemv_paper_b3_kernel<MB>, kStagedWarps * 32, smem) !=
+      cudaSuccess)
+    return cudaGetLastError();
+  const int want = (p.N + kStagedWarps - 1) / kStagedWarps;
+  const int grid = std::max(1, std::min(want, p.sm_count * std::max(per_sm, 1)));
+  qtea_gemv_paper_b3_kernel<MB><<<grid, kStagedWarps * 32, smem, st>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t paper_configure(size_t smem_optin) {
+  const int dyn = (int)smem_optin;
+  cudaError_t e;
+#define QTEA_STAGED_ATTR(MB, B3)                                                                              \
+  if ((e = cudaFuncSetAttribute(qtea_gemv_paper_staged_kernel<MB, B3>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                                dyn)) != cudaSuccess)                                                          \
+    return e;
+  if ((e = cudaFuncSetAttribute(qtea_gemv_paper_b3_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn)) !=
+      cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(qtea_gemv_paper_b3_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn)) !=
+      cudaSuccess)
+    return e;
+  if ((e = cudaFuncSetAttribute(qtea_gemv_paper_b3_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, dyn)) !=
+      cudaSuccess)
+    return e;
+  QTEA_STAGED_ATTR(1, false)
+  QTEA_STAGED_ATTR(2, false)
+  QTEA_STAGED_ATTR(4, false)
+#undef QTEA_STAGED_ATTR
+  return cudaSuccess;
+}
+
 cudaError_t launch_paper(const PaperParams& p, cudaStream_t st) {
   const int grid = (p.N + kPaperWarps - 1) / kPaperWarps;
   if (grid == 0) return cudaSuccess;
+  if (p.staged_ok && p.M <= 4 && p.format == QTEA_FMT_BASE3) {
+    const size_t smem = b3_smem_bytes(p.M, p.K, p.G, p.bias != 0);
+    if (smem <= p.smem_optin) {
+      if (p.M <= 1) return launch_b3<1>(p, smem, st);
+      if (p.M <= 2) return launch_b3<2>(p, smem, st);
+      return launch_b3<4>(p, smem, st);
+    }
+  }
+  const size_t smem = staged_smem_bytes(p.M, p.K, p.G, p.bias != 0);
+  if (p.staged_ok && p.M <= 4 && p.format != QTEA_FMT_BASE3 && smem <= p.smem_optin) {
+    if (p.M <= 1) return launch_staged<1, false>(p, smem, st);
+    if (p.M <= 2) return launch_staged<2, false>(p, smem, st);
+    return launch_staged<4, false>(p, smem, st);
+  }
   const int threads = kPaperWarps * 32;
   if (p.M <= 1) qtea_gemv_paper_kernel<1><<<grid, threads, 0, st>>>(p);
   else if (p.M <= 2) qtea_gemv_paper_kernel<2><<<grid, threads, 0, st>>>(p);

@@ -242,6 +242,8 @@ struct PaperParams {
   const uint8_t* ridx;      // [N/4][ceil(s/4)]
   float* y;                 // [M][N]
   int M, N, K, s, G, group_size, row_bytes, format, bias, residual_fp8;
+  int staged_ok, sm_count;   // the staged-activation kernel is configured; SMs of the device
+  size_t smem_optin, smem_per_sm;
 };
 
 // The quantizer's per-layer steps (qtea_quant.cu).
@@ -259,6 +261,7 @@ struct QuantArgs {
 
 cudaError_t launch_quantize(const QuantArgs& a, cudaStream_t st);
 cudaError_t launch_paper(const PaperParams& p, cudaStream_t st);
+cudaError_t paper_configure(size_t smem_optin);
 cudaError_t launch_pack_base3(const int8_t* codes, int N, int K, uint8_t* packed, int* bad_flag, cudaStream_t st);
 cudaError_t launch_m1(const TensorMaps& maps, const GroupParams& p, int grid, size_t smem, cudaStream_t st);
 cudaError_t m1_configure(size_t smem_optin, size_t* dyn_max);
@@ -277,6 +280,8 @@ struct qtea_layout {
   int device;
   int sm_count;
   size_t smem_optin;
+  size_t smem_per_sm;
+  bool paper_staged_ok;  // the paper-storage kernel with staged activations is configured
   // batch-1 kernel resources
   bool m1_ok;
   int act_bits;          // activation precision of batch-1 calls: 24 (default) or 16
