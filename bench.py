@@ -686,7 +686,7 @@ def qtea_arm(args):
     if not args.no_paper:
         paper = {"workload": "llama3_8b_layer_paper_storage", "M": 1,
                  "base3_fp8": dict(paper_leg(qt.QTEA_FMT_BASE3, True),
-                                   kernel="qtea_gemv_paper_kernel (general, one warp per row)"),
+                                   kernel="qtea_gemv_paper_b3_kernel (staged fixed-point activations, dp4a)"),
                  "2bit_fp16_residual": dict(paper_leg(qt.QTEA_FMT_2BIT, False),
                                             kernel="qtea_gemv_mb_kernel (tensor cores, scale groups)")}
 
