@@ -129,7 +129,7 @@ int check_problem(const qtea_gemv_problem& q, int M) {
 // The paper's own storage: base-3 codes, groups of 128 columns, beta or FP8 residual values.
 bool is_paper(const qtea_layout* l) { return l->format != QTEA_FMT_2BIT || l->group_size != l->K || l->options != 0; }
 
-int launch_paper_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
+PaperParams paper_params(const qtea_gemv_problem& q, int M) {
   const qtea_layout* l = q.packed_ternary;
   PaperParams p;
   p.x = q.x;
@@ -154,7 +154,26 @@ int launch_paper_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
   p.sm_count = l->sm_count > 0 ? l->sm_count : 1;
   p.smem_optin = l->smem_optin;
   p.smem_per_sm = l->smem_per_sm;
-  return launch_paper(p, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+  return p;
+}
+
+int launch_paper_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
+  return launch_paper(paper_params(q, M), st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+}
+
+// Base-3 problems with staged activations: up to eight per launch.
+int run_b3(const qtea_gemv_problem* qs, const int* idx, int n, int M, cudaStream_t st) {
+  for (int i = 0; i < n; i += 8) {
+    B3Group g;
+    g.n = n - i < 8 ? n - i : 8;
+    g.work[0] = 0;
+    for (int k = 0; k < g.n; ++k) {
+      g.prob[k] = paper_params(qs[idx[i + k]], M);
+      g.work[k + 1] = g.work[k] + (long long)g.prob[k].N * ((g.prob[k].K + 127) / 128);
+    }
+    if (launch_b3(g, st) != cudaSuccess) return QTEA_ERR_CUDA;
+  }
+  return QTEA_OK;
 }
 
 int launch_generic_problem(const qtea_gemv_problem& q, int M, cudaStream_t st) {
@@ -631,7 +650,8 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
   int* m1_idx = n_problems > 0 ? static_cast<int*>(std::malloc(sizeof(int) * 2 * (size_t)n_problems)) : nullptr;
   if (n_problems > 0 && !m1_idx) return QTEA_ERR_ALLOC;
   int* mb_idx = m1_idx + n_problems;
-  int n_m1 = 0, n_mb = 0, rc = QTEA_OK;
+  int b3_idx[8];
+  int n_m1 = 0, n_mb = 0, n_b3 = 0, rc = QTEA_OK;
   for (int i = 0; i < n_problems && rc == QTEA_OK; ++i) {
     const qtea_gemv_problem& q = problems[i];
     const qtea_layout* l = q.packed_ternary;
@@ -645,11 +665,20 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
     } else if (mb_capable(l, M)) {
       mb_idx[n_mb++] = i;
     } else if (is_paper(l)) {
-      rc = launch_paper_problem(q, M, st);
+      if (b3_eligible(paper_params(q, M))) {
+        b3_idx[n_b3++] = i;
+        if (n_b3 == 8) {
+          rc = run_b3(problems, b3_idx, n_b3, M, st);
+          n_b3 = 0;
+        }
+      } else {
+        rc = launch_paper_problem(q, M, st);
+      }
     } else {
       rc = launch_generic_problem(q, M, st);
     }
   }
+  if (rc == QTEA_OK && n_b3 > 0) rc = run_b3(problems, b3_idx, n_b3, M, st);
   if (rc == QTEA_OK && n_m1 > 0) rc = run_m1(problems, m1_idx, n_m1, st);
   if (rc == QTEA_OK && n_mb > 0) rc = run_mb(problems, mb_idx, n_mb, M, st);
   std::free(m1_idx);

@@ -349,34 +349,22 @@ constexpr int kB3Rec = 8;          // words per five-column record
 constexpr int kB3BlockWords = 212;  // records of one block (26 x 8 words) plus 4 words: lanes that
                                     // read different blocks' records hit distinct banks
 
-size_t b3_smem_bytes(int M, int K, int G, bool bias) {
+// Shared memory of one base-3 problem after the 256-entry table: records, 2^-e and block sums of x
+// per batch row and block, and the per-group sums of x with beta.
+size_t b3_region_bytes(int M, int K, int G, bool bias) {
   const size_t n_blocks = (size_t)(K + 127) / 128;
   return (size_t)M * n_blocks * kB3BlockWords * sizeof(uint32_t) + 2 * (size_t)M * n_blocks * sizeof(float) +
-         (bias ? (size_t)M * G * sizeof(float) : 0) + 243 * sizeof(uint2) + 16;
+         (bias ? (size_t)M * G * sizeof(float) : 0);
 }
 
 template <int MB>
-__global__ void __launch_bounds__(kStagedWarps * 32) qtea_gemv_paper_b3_kernel(const PaperParams p) {
-  extern __shared__ __align__(16) uint32_t smw[];
+__device__ void b3_problem(const PaperParams& p, int row_lo, int row_hi, uint32_t* smw, const uint2* lut) {
   const int K = p.K, G = p.G, M = p.M;
   const int n_blocks = (K + 127) / 128;
   uint32_t* rec = smw;                                                    // [M][n_blocks][212]
   float* inv = reinterpret_cast<float*>(rec + (size_t)M * n_blocks * kB3BlockWords);  // [M][n_blocks] 2^-e
   float* sx = inv + (size_t)M * n_blocks;                                 // [M][G] sum of x, with beta
-  uint2* lut = reinterpret_cast<uint2*>(sx + (p.bias ? (size_t)M * G : 0) + (size_t)M * n_blocks + 2);  // [243]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (reinterpret_cast<uintptr_t>(lut) & 7) lut = reinterpret_cast<uint2*>(reinterpret_cast<uintptr_t>(lut) + 4);
-  for (int i = threadIdx.x; i < 243; i += blockDim.x) {
-    int b = i;
-    uint32_t w1 = 0, w2 = 0;
-    for (int d = 0; d < 5; ++d) {
-      const uint32_t c = (uint32_t)(b % 3);
-      b /= 3;
-      if (d < 4) w1 |= c << (8 * d);
-      else w2 = c;
-    }
-    lut[i] = make_uint2(w1, w2);
-  }
   // one warp per (batch row, block), two tasks' loads in flight: lane q < 26 owns columns
   // 5q .. 5q+4 of the block; the warp also sums the block's x for the beta term
   float* bx = sx + (p.bias ? (size_t)M * G : 0);  // [M][n_blocks], in the slack before the table
@@ -457,7 +445,7 @@ __global__ void __launch_bounds__(kStagedWarps * 32) qtea_gemv_paper_b3_kernel(c
 
   const bool row_group = p.group_size >= K;  // one scale group per row
   const int sc_stride = p.bias ? 2 : 1;
-  for (int o = blockIdx.x * kStagedWarps + warp; o < p.N; o += gridDim.x * kStagedWarps) {
+  for (int o = row_lo + warp; o < row_hi; o += kStagedWarps) {
     const uint8_t* row = p.packed + (size_t)o * p.row_bytes;
     const uint16_t* sc = p.scales + (size_t)o * G * sc_stride;
     float acc[MB];
@@ -549,6 +537,39 @@ __global__ void __launch_bounds__(kStagedWarps * 32) qtea_gemv_paper_b3_kernel(c
   }
 }
 
+// The base-3 problems of a grouped call in one launch. The rows of all problems, each weighted by
+// its blocks, are split evenly over the persistent CTAs; a CTA stages a problem once for the rows
+// of it that fall in its share (one or two problems for most CTAs).
+template <int MB>
+__global__ void __launch_bounds__(kStagedWarps * 32) qtea_gemv_paper_b3_kernel(const B3Group g) {
+  extern __shared__ __align__(16) uint32_t smw[];
+  uint2* lut = reinterpret_cast<uint2*>(smw);  // [256]
+  for (int i = threadIdx.x; i < 256; i += blockDim.x) {  // bytes above 242 never occur; T = 0 there
+    int b = i < 243 ? i : 121;
+    uint32_t w1 = 0, w2 = 0;
+    for (int d = 0; d < 5; ++d) {
+      const uint32_t c = (uint32_t)(b % 3);
+      b /= 3;
+      if (d < 4) w1 |= c << (8 * d);
+      else w2 = c;
+    }
+    lut[i] = make_uint2(w1, w2);
+  }
+  const long long total = g.work[g.n];
+  const long long lo = total * blockIdx.x / gridDim.x, hi = total * (blockIdx.x + 1) / gridDim.x;
+  for (int q = 0; q < g.n; ++q) {
+    const long long w0 = g.work[q], w1 = g.work[q + 1];
+    const long long a = lo > w0 ? lo : w0, b = hi < w1 ? hi : w1;
+    if (a >= b) continue;
+    const int nb = (g.prob[q].K + 127) / 128;
+    // row r belongs to the CTA whose share holds its first block
+    const int row_lo = (int)((a - w0 + nb - 1) / nb), row_hi = (int)((b - w0 + nb - 1) / nb);
+    if (row_lo >= row_hi) continue;
+    __syncthreads();  // the previous problem's rows are done with the staged data
+    b3_problem<MB>(g.prob[q], row_lo, row_hi, smw + 512, lut);
+  }
+}
+
 // Base-3 packing (Sec. 3.5): per row, K_pad3 / 128 groups of 26 bytes; byte q of a group holds
 // columns 5q .. 5q+4 of the group as sum_d (T + 1) 3^d, the lowest column in the least significant
 // digit. Byte 25 holds columns 125-127 and two pad digits; pad digits and columns >= K are digit 1
@@ -595,15 +616,36 @@ cudaError_t launch_staged(const PaperParams& p, size_t smem, cudaStream_t st) {
 }
 
 template <int MB>
-cudaError_t launch_b3(const PaperParams& p, size_t smem, cudaStream_t st) {
-  int per_sm = 1;  // resident CTAs per SM: the grid is persistent, so each CTA stages once
+cudaError_t launch_b3_group(const B3Group& g, size_t smem, int sm_count, cudaStream_t st) {
+  int per_sm = 1;  // resident CTAs per SM: the grid is persistent, so each CTA stages once per problem
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, qtea_gemv_paper_b3_kernel<MB>, kStagedWarps * 32, smem) !=
       cudaSuccess)
     return cudaGetLastError();
-  const int want = (p.N + kStagedWarps - 1) / kStagedWarps;
-  const int grid = std::max(1, std::min(want, p.sm_count * std::max(per_sm, 1)));
-  qtea_gemv_paper_b3_kernel<MB><<<grid, kStagedWarps * 32, smem, st>>>(p);
+  long long rows = 0;
+  for (int q = 0; q < g.n; ++q) rows += g.prob[q].N;
+  const long long want = (rows + kStagedWarps - 1) / kStagedWarps;
+  const int grid = (int)std::max<long long>(1, std::min<long long>(want, (long long)sm_count * std::max(per_sm, 1)));
+  qtea_gemv_paper_b3_kernel<MB><<<grid, kStagedWarps * 32, smem, st>>>(g);
   return cudaGetLastError();
+}
+
+size_t b3_smem_bytes(int M, int K, int G, bool bias) { return 2048 + b3_region_bytes(M, K, G, bias) + 16; }
+
+cudaError_t launch_b3(const B3Group& g, cudaStream_t st) {
+  size_t smem = 0;
+  for (int q = 0; q < g.n; ++q) {
+    const PaperParams& p = g.prob[q];
+    smem = std::max(smem, b3_smem_bytes(p.M, p.K, p.G, p.bias != 0));
+  }
+  const int M = g.n > 0 ? g.prob[0].M : 1, sm = g.n > 0 ? g.prob[0].sm_count : 1;
+  if (M <= 1) return launch_b3_group<1>(g, smem, sm, st);
+  if (M <= 2) return launch_b3_group<2>(g, smem, sm, st);
+  return launch_b3_group<4>(g, smem, sm, st);
+}
+
+bool b3_eligible(const PaperParams& p) {
+  return p.staged_ok && p.format == QTEA_FMT_BASE3 && p.M >= 1 && p.M <= 4 &&
+         b3_smem_bytes(p.M, p.K, p.G, p.bias != 0) <= p.smem_optin;
 }
 
 cudaError_t paper_configure(size_t smem_optin) {
@@ -632,13 +674,13 @@ cudaError_t paper_configure(size_t smem_optin) {
 cudaError_t launch_paper(const PaperParams& p, cudaStream_t st) {
   const int grid = (p.N + kPaperWarps - 1) / kPaperWarps;
   if (grid == 0) return cudaSuccess;
-  if (p.staged_ok && p.M <= 4 && p.format == QTEA_FMT_BASE3) {
-    const size_t smem = b3_smem_bytes(p.M, p.K, p.G, p.bias != 0);
-    if (smem <= p.smem_optin) {
-      if (p.M <= 1) return launch_b3<1>(p, smem, st);
-      if (p.M <= 2) return launch_b3<2>(p, smem, st);
-      return launch_b3<4>(p, smem, st);
-    }
+  if (b3_eligible(p)) {
+    B3Group g;
+    g.prob[0] = p;
+    g.n = 1;
+    g.work[0] = 0;
+    g.work[1] = (long long)p.N * ((p.K + 127) / 128);
+    return launch_b3(g, st);
   }
   const size_t smem = staged_smem_bytes(p.M, p.K, p.G, p.bias != 0);
   if (p.staged_ok && p.M <= 4 && p.format != QTEA_FMT_BASE3 && smem <= p.smem_optin) {

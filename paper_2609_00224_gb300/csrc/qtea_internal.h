@@ -260,7 +260,17 @@ struct QuantArgs {
 };
 
 cudaError_t launch_quantize(const QuantArgs& a, cudaStream_t st);
+// Up to eight base-3 problems of one batch size in one launch; work[q] = sum over earlier problems of
+// rows x 128-column blocks.
+struct B3Group {
+  PaperParams prob[8];
+  long long work[9];
+  int n;
+};
+
 cudaError_t launch_paper(const PaperParams& p, cudaStream_t st);
+cudaError_t launch_b3(const B3Group& g, cudaStream_t st);
+bool b3_eligible(const PaperParams& p);
 cudaError_t paper_configure(size_t smem_optin);
 cudaError_t launch_pack_base3(const int8_t* codes, int N, int K, uint8_t* packed, int* bad_flag, cudaStream_t st);
 cudaError_t launch_m1(const TensorMaps& maps, const GroupParams& p, int grid, size_t smem, cudaStream_t st);
