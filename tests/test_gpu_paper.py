@@ -206,3 +206,38 @@ def test_grouped_call_mixing_storage_formats(qt, M):
     for (p, bias), y in zip(probs, ys):
         y_ref, b = reference(p, bias, M=M)
         assert_within(y.cpu().numpy().astype(np.float64), y_ref, b, f"{p.N}x{p.K} M {M}")
+
+
+@pytest.mark.parametrize("M", [1, 2, 4, 5])
+def test_grouped_base3_calls(qt, M):
+    """Eleven base-3 layouts in one grouped call (two launches of the staged fixed-point kernel at
+    M <= 4, the general kernel at M = 5): ragged K against the 128-column blocks, groups of 128 or
+    the whole row, with and without beta, FP8 or fp16 residual values, no residual with N not a
+    multiple of 4, and a 2-bit layout in between that takes another kernel."""
+    specs = [  # (N, K, s, fmt, group, bias, fp8)
+        (256, 1024, 8, 1, 128, 1, 1), (64, 300, 4, 1, 0, 0, 0), (130, 700, 0, 1, 128, 1, 0),
+        (512, 2048, 24, 1, 128, 0, 1), (36, 128, 4, 1, 0, 1, 1), (100, 257, 0, 1, 0, 0, 0),
+        (64, 1024, 8, 0, 0, 1, 0), (128, 4096, 40, 1, 128, 1, 1), (260, 640, 12, 1, 128, 1, 0),
+        (8, 1, 0, 1, 0, 0, 0), (1024, 512, 16, 1, 128, 1, 1), (68, 1920, 8, 1, 0, 1, 1)]
+    probs, items = [], []
+    for i, (N, K, s, fmt, group, bias, fp8) in enumerate(specs):
+        p = synth.make_problem("b3", N, K, 16, s, seed=900 + 13 * i + M, group_size=group,
+                               beta_std=0.002 if bias else 0.0, residual_fp8=bool(fp8))
+        lay = qt.qtea_pack_layout(dev(p.T), n_salient=p.s, group_size=group or K, fmt=fmt)
+        lay.set_options((qt.QTEA_OPT_BIAS if bias else 0) | (qt.QTEA_OPT_RESIDUAL_FP8 if fp8 else 0))
+        rv = dev(p.residual_vals) if fp8 else dev(p.residual_vals.view(np.int16), torch.float16)
+        items.append(dict(x=dev(p.x[:M].view(np.int16), torch.float16), layout=lay,
+                          row_scale=dev(scales(p, bias).view(np.int16), torch.float16),
+                          col_scale=dev(p.v.view(np.int16), torch.float16),
+                          salient_idx=dev(p.salient_idx) if s else None, residual_vals=rv if s else None,
+                          residual_idx=dev(p.residual_idx) if s else None))
+        probs.append((p, bias))
+    ys = qt.qtea_gemv_grouped(items)
+    ys2 = qt.qtea_gemv_grouped(items)
+    torch.cuda.synchronize()
+    for it in items:
+        assert qt.qtea_device_status(it["layout"]) == 0
+    for (p, bias), y, y2 in zip(probs, ys, ys2):
+        y_ref, b = reference(p, bias, M=M)
+        assert_within(y.cpu().numpy().astype(np.float64), y_ref, b, f"{p.N}x{p.K} M {M}")
+        assert torch.equal(y, y2), "repeated grouped calls differ"
