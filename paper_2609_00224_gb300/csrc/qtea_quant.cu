@@ -289,6 +289,103 @@ __global__ void __launch_bounds__(kQSumWarps * 32) quant_colsum_kernel(const flo
   if (warp == 0 && jin && cnt > 0) v[j] = __fdiv_rn(acc, (float)cnt);
 }
 
+// The same column sums with the tiles streamed: 16-byte rows (K % 16 == 0), so W, the codes and
+// alpha, beta of a 128-row tile reach shared memory by cp.async, four tiles in flight. Warps 1..7
+// turn a landed tile into terms (the marker where T_ij = 0) while warp 0 adds the previous tile's
+// terms in row order.
+constexpr int kCsStages = 4;
+
+struct CsSmem {
+  float w[kCsStages][kQSumRows][32];
+  int8_t t[kCsStages][kQSumRows][32];
+  float ab[kCsStages][kQSumRows][2];
+  unsigned term[2][kQSumRows][32];
+};
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async4(void* dst, const void* src) {
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"((uint32_t)__cvta_generic_to_shared(dst)), "l"(src)
+               : "memory");
+}
+
+__global__ void __launch_bounds__(kQSumWarps * 32) quant_colsum_async_kernel(const float* __restrict__ W,
+                                                                            const float* __restrict__ alpha,
+                                                                            const float* __restrict__ beta,
+                                                                            const int8_t* __restrict__ T, int N,
+                                                                            int K, int group, int G,
+                                                                            float* __restrict__ v) {
+  extern __shared__ __align__(16) unsigned char cs_raw[];
+  CsSmem& sm = *reinterpret_cast<CsSmem*>(cs_raw);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int j0 = blockIdx.x * 32;  // 32 columns of one scale group (groups are K or 128 columns)
+  const int g = j0 / group;
+  const int n_tiles = (N + kQSumRows - 1) / kQSumRows;
+  const int pt = threadIdx.x - 32, n_pt = (kQSumWarps - 1) * 32;
+  auto issue = [&](int k) {
+    if (k < n_tiles) {
+      const int st = k % kCsStages, i0 = k * kQSumRows;
+      for (int c = pt; c < kQSumRows * 8; c += n_pt) {
+        const int r = c >> 3, q = c & 7;
+        // K % 16 == 0: a 16-byte chunk lies wholly inside or wholly past the row's end
+        if (i0 + r < N && j0 + 4 * q < K) cp_async16(&sm.w[st][r][4 * q], W + (size_t)(i0 + r) * K + j0 + 4 * q);
+      }
+      for (int c = pt; c < kQSumRows * 2; c += n_pt) {
+        const int r = c >> 1, q = c & 1;
+        if (i0 + r < N && j0 + 16 * q < K) cp_async16(&sm.t[st][r][16 * q], T + (size_t)(i0 + r) * K + j0 + 16 * q);
+      }
+      for (int r = pt; r < kQSumRows; r += n_pt)
+        if (i0 + r < N) {
+          cp_async4(&sm.ab[st][r][0], alpha + (size_t)(i0 + r) * G + g);
+          cp_async4(&sm.ab[st][r][1], beta + (size_t)(i0 + r) * G + g);
+        }
+    }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  if (warp > 0)
+    for (int k = 0; k < kCsStages - 1; ++k) issue(k);
+  float acc = 0.f;
+  int cnt = 0;
+  for (int k = 0; k <= n_tiles; ++k) {
+    if (warp > 0) {
+      if (k < n_tiles) {
+        issue(k + kCsStages - 1);
+        asm volatile("cp.async.wait_group %0;" ::"n"(kCsStages - 1) : "memory");
+        asm volatile("bar.sync 1, %0;" ::"r"(n_pt) : "memory");  // every producer's copies of tile k
+        const int st = k % kCsStages, i0 = k * kQSumRows;
+        unsigned(*tb)[32] = sm.term[k & 1];
+        for (int e = pt; e < kQSumRows * 32; e += n_pt) {
+          const int r = e >> 5, c = e & 31;
+          unsigned u = kQNoTerm;
+          if (i0 + r < N && j0 + c < K && sm.t[st][r][c] != 0)
+            u = __float_as_uint(__fdiv_rn(fabsf(__fsub_rn(sm.w[st][r][c], sm.ab[st][r][1])), sm.ab[st][r][0]));
+          tb[r][c] = u;
+        }
+      }
+    } else if (k > 0) {
+      const unsigned(*tb)[32] = sm.term[(k - 1) & 1];
+      const int rows = min(kQSumRows, N - (k - 1) * kQSumRows);  // rows past N hold the marker
+      for (int r0 = 0; r0 < rows; r0 += 8) {
+        unsigned u[8];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) u[q] = tb[r0 + q][lane];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          if (u[q] != kQNoTerm) {
+            acc = __fadd_rn(acc, __uint_as_float(u[q]));
+            ++cnt;
+          }
+        }
+      }
+    }
+    __syncthreads();
+  }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  if (warp == 0 && j0 + lane < K && cnt > 0) v[j0 + lane] = __fdiv_rn(acc, (float)cnt);
+}
+
 // T_ij = nearest of {-v_j alpha, 0, +v_j alpha} to W_ij - beta (threshold (v_j alpha) / 2), every entry.
 // With K % 4 == 0 a thread takes four columns of one row (one 16-byte load of W, one 4-byte store of
 // codes; the four columns share a scale group); otherwise one entry.
@@ -378,6 +475,18 @@ __global__ void __launch_bounds__(kQThreads) quant_residual_kernel(const float* 
 
 inline unsigned blocks(long long n, int per) { return (unsigned)((n + per - 1) / per); }
 
+// The streamed column-sum kernel's shared memory is above the default 48 KB: opt in once.
+bool cs_async_ready() {
+  static int state = 0;  // 0 unknown, 1 ready, 2 unavailable
+  if (state == 0)
+    state = cudaFuncSetAttribute(quant_colsum_async_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)sizeof(CsSmem)) == cudaSuccess
+                ? 1
+                : 2;
+  if (state == 2) cudaGetLastError();
+  return state == 1;
+}
+
 }  // namespace
 
 cudaError_t launch_quantize(const QuantArgs& a, cudaStream_t st) {
@@ -417,9 +526,16 @@ cudaError_t launch_quantize(const QuantArgs& a, cudaStream_t st) {
     const bool vec = a.K % 4 == 0 && (reinterpret_cast<uintptr_t>(a.W) & 15) == 0 &&
                      (reinterpret_cast<uintptr_t>(a.codes) & 3) == 0;
     const dim3 rgrid(blocks(vec ? a.K / 4 : a.K, kQThreads), (unsigned)std::min(a.N, 65535));
+    // streamed column sums where every row of W and of the codes is 16-byte aligned
+    const bool cs_async = a.K % 16 == 0 && (reinterpret_cast<uintptr_t>(a.W) & 15) == 0 &&
+                          (reinterpret_cast<uintptr_t>(a.codes) & 15) == 0 && cs_async_ready();
     for (int it = 0; it < a.rescale_iters; ++it) {
-      quant_colsum_kernel<<<blocks(a.K, 32), kQSumWarps * 32, 0, st>>>(a.W, alpha, beta, a.codes, a.N, a.K, a.group,
-                                                                        G, v);
+      if (cs_async)
+        quant_colsum_async_kernel<<<blocks(a.K, 32), kQSumWarps * 32, sizeof(CsSmem), st>>>(
+            a.W, alpha, beta, a.codes, a.N, a.K, a.group, G, v);
+      else
+        quant_colsum_kernel<<<blocks(a.K, 32), kQSumWarps * 32, 0, st>>>(a.W, alpha, beta, a.codes, a.N, a.K,
+                                                                          a.group, G, v);
       if (vec)
         quant_reassign_kernel<true><<<rgrid, kQThreads, 0, st>>>(a.W, alpha, beta, v, a.N, a.K, a.group, G, a.codes);
       else

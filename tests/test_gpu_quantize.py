@@ -49,6 +49,9 @@ CASES = [
     (16, 40, None, 40, True),   # every column salient
     (12, 513, 128, 0, True),    # no salient columns
     (32, 5000, 128, 520, False),  # the compaction's segments several columns long
+    (20, 272, 128, 8, True),    # K % 32 == 16: the last 32-column block ends past the row (streamed sums)
+    (36, 144, None, 8, False),  # the same with one group per row
+    (300, 1056, 128, 12, True),  # 128-row tiles with a ragged last tile
 ]
 
 
