@@ -86,9 +86,11 @@ typedef enum qtea_option {
  * bytes; byte q of group h holds columns 128h + 5q + d, d = 0..4, as sum_d (T+1) 3^d (lowest
  * column in the least significant digit); byte 25 holds three columns and two pad digits; pad
  * digits and columns >= K are digit 1.
- * Layouts other than 2-bit with group_size = K and no options (the paper's storage) run on a
- * general kernel for every M; the TMA batch-1 and tensor-core low-batch kernels serve the
- * 2-bit, one-scale-per-row layout.
+ * Which kernel serves a call: the TMA batch-1 kernel takes 2-bit, one-scale-per-row layouts
+ * without options at M = 1; the tensor-core low-batch kernel takes those at M >= 2 and 2-bit
+ * layouts in the paper's storage (groups of 128 columns, or beta absent) at any M; base-3 layouts
+ * at M <= 4 run on a kernel that stages v*x once per CTA in fixed point (the base-3 problems of a
+ * grouped call share one launch); the rest run on general kernels.
  *
  * The call validates every code on the device and synchronizes `stream` once to read the
  * result; invalid codes give QTEA_ERR_BAD_CODES and no layout. It allocates the packed
@@ -131,7 +133,10 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
  * and the residual are combined in fp32. At 2 <= M <= 16, and for 2-bit layouts in the paper's
  * storage at any M, the tensor cores take 2T*v and x in fp16 (both exact, which needs |v| < 32768)
  * with exact fp32 products and fp32 sums; alpha, beta and the residual are applied in fp32.
- * Base-3 layouts use a general kernel (fp32 throughout).
+ * Base-3 layouts at M <= 4 (when v*x of the call fits in shared memory): the ternary sum is
+ * accumulated exactly in integers over 128-column blocks, with v*x in fixed point relative to the
+ * block's largest |v*x| (|X| < 2^22); block sums, alpha, beta and the residual are combined in
+ * fp32. Other layouts and batch sizes: fp32 throughout.
  */
 int qtea_gemv(const uint16_t* x, const qtea_layout* packed_ternary, const uint16_t* row_scale,
               const uint16_t* col_scale, const int32_t* salient_idx, const uint16_t* residual_vals,
@@ -228,9 +233,9 @@ int qtea_set_activation_precision(qtea_layout* layout, int bits);
 /*
  * Storage options of the scales and residual values qtea_gemv reads with this layout: any
  * combination of QTEA_OPT_BIAS and QTEA_OPT_RESIDUAL_FP8 (0 restores fp16 alpha only and fp16
- * residual values). Other bits -> QTEA_ERR_INVALID_ARG. With any option set, calls run on the
- * general kernel (see qtea_pack_layout). Set it before the calls that use it; it takes effect
- * for calls made afterwards.
+ * residual values). Other bits -> QTEA_ERR_INVALID_ARG. With any option set, calls leave the
+ * batch-1 kernel (see qtea_pack_layout for which kernel serves which storage). Set it before the
+ * calls that use it; it takes effect for calls made afterwards.
  */
 int qtea_set_layout_options(qtea_layout* layout, int options);
 

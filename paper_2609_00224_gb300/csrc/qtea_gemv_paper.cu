@@ -8,12 +8,17 @@
 // paper's base-3 layout (five codes per byte, 26 bytes per 128 columns), and residual values in
 // fp16 or in the paper's FP8 E4M3.
 //
-// One warp per output row, walking the row's 128-column blocks; a block lies in one scale group
-// (groups are 128 columns or the whole row). Lane l takes code byte l of the block and adds
-// alpha * sum T v x + beta * sum x over its columns for every batch row; the lanes' sums are added
-// once at the end. Base-3 bytes are expanded to five 2-bit codes through a 243-entry table in shared
-// memory. v*x is exact in fp32; sums are fp32. The same warp adds the residual of the row's group
-// of four.
+// Three kernels:
+//  * qtea_gemv_paper_b3_kernel (base-3, M <= 4): v*x staged once per CTA as fixed point per
+//    128-column block, decoded with dp4a through a byte table; several problems per launch.
+//  * qtea_gemv_paper_staged_kernel (2-bit, M <= 4): v*x staged once per CTA in fp32.
+//  * qtea_gemv_paper_kernel (any layout, any M): one warp per output row reading x and v from
+//    global memory. A block lies in one scale group (groups are 128 columns or the whole row);
+//    lane l takes code byte l of the block and adds alpha * sum T v x + beta * sum x over its
+//    columns for every batch row; the lanes' sums are added once at the end. Base-3 bytes are
+//    expanded to five 2-bit codes through a 243-entry table in shared memory. v*x is exact in fp32;
+//    sums are fp32.
+// In each, the warp of a row adds the residual of the row's group of four.
 #include <cuda_fp16.h>
 
 #include <algorithm>
