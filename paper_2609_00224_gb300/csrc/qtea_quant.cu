@@ -477,14 +477,13 @@ inline unsigned blocks(long long n, int per) { return (unsigned)((n + per - 1) /
 
 // The streamed column-sum kernel's shared memory is above the default 48 KB: opt in once.
 bool cs_async_ready() {
-  static int state = 0;  // 0 unknown, 1 ready, 2 unavailable
-  if (state == 0)
-    state = cudaFuncSetAttribute(quant_colsum_async_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)sizeof(CsSmem)) == cudaSuccess
-                ? 1
-                : 2;
-  if (state == 2) cudaGetLastError();
-  return state == 1;
+  static const bool ready = [] {  // initialised once, thread-safe
+    const bool ok = cudaFuncSetAttribute(quant_colsum_async_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)sizeof(CsSmem)) == cudaSuccess;
+    if (!ok) cudaGetLastError();
+    return ok;
+  }();
+  return ready;
 }
 
 }  // namespace
