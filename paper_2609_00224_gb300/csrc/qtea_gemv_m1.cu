@@ -26,8 +26,9 @@
 //  * Split tiles are reduced by the last-arriving CTA (atomic counter, no spin-wait) in a
 //    fixed CTA order, so results are bitwise reproducible.
 //  * Programmatic dependent launch: before griddepcontrol.wait a CTA only initialises its
-//    barriers and starts the TMA of its first units' codes, which the library owns and no other
-//    kernel writes. Everything the caller owns (x, v, alpha, the residual, y) and the split-tile
+//    barriers, starts the TMA of its first units' codes, which the library owns and no other
+//    kernel writes, and prefetches into L2 the lines of x and v those units read (a prefetch
+//    reads no value). Everything the caller owns (x, v, alpha, the residual, y) and the split-tile
 //    workspace is touched after the wait. Each CTA lets the next launch start once it is running.
 // Every wait on an mbarrier is bounded: after ~2 s the waiting thread records
 // QTEA_ERR_TIMEOUT in the status word and its role stops.
@@ -671,6 +672,19 @@ __global__ void __launch_bounds__(kThreads, 1)
       const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
       issue_unit(&maps.m[up.p], up.t, up.ch, smem_u32(r.codes + (size_t)i * kStageBytes), smem_u32(&r.full_c[i]));
       r.last_fill[i] = 1;
+    }
+  }
+  // warm L2 with the lines of x and v that the first six units read (eight 128-byte lines of each
+  // per 512-column chunk, one per helper lane): a prefetch reads no value into the SM, so the data
+  // the units use is still read after the wait, from L2, where a preceding kernel's writes land
+  if (warp >= kConsumerWarps && warp < kProducerWarp) {
+    const int hl = (warp - kConsumerWarps) * 32 + lane, i = hl >> 4, l16 = hl & 15;
+    if (i < n_units) {
+      const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
+      const ProblemArgs& pa = tab[up.p];
+      const int col = up.ch * kChunkCols + (l16 & 7) * 64;  // 64 fp16 values per line
+      if (col < pa.K)
+        asm volatile("prefetch.global.L2 [%0];" ::"l"((l16 < 8 ? pa.x : pa.v) + col) : "memory");
     }
   }
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
