@@ -52,6 +52,7 @@ CASES = [
     (20, 272, 128, 8, True),    # K % 32 == 16: the last 32-column block ends past the row (streamed sums)
     (36, 144, None, 8, False),  # the same with one group per row
     (300, 1056, 128, 12, True),  # 128-row tiles with a ragged last tile
+    (6, 50, None, 0, True),     # no residual: N need not be a multiple of 4
 ]
 
 
