@@ -459,6 +459,33 @@ def qtea_arm(args):
                                      "gbs": round(bts / (us * 1e-6) / 1e9, 1),
                                      "eff_bits_per_weight": round(8 * (bts - 2 * K - 4 * N) / (N * K), 3)}
 
+    # ---- the 32-layer stack in a decoder's dependency order: per layer four grouped calls
+    #      (q, k, v | o | gate, up | down), every layer of the stack once per token, the tokens
+    #      back to back in one graph (x per GEMV synthetic, not chained)
+    stack = None
+    if not args.no_stack and len(layers) >= 2:
+        order = [[0, 1, 2], [3], [4, 5], [6]]
+        n_tok = max(2, min(8, args.steps // len(layers)))
+        gs_ = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            for L in group_args:
+                for grp in order:
+                    qt.qtea_gemv_grouped([L[j] for j in grp], stream=stream)
+        barrier()
+        with torch.cuda.graph(gs_, stream=stream):
+            for _ in range(n_tok):
+                for L in group_args:
+                    for grp in order:
+                        qt.qtea_gemv_grouped([L[j] for j in grp], stream=stream)
+        ms_s = timed_replay(gs_)
+        del gs_
+        tok_b = sum(step_bytes)
+        stack = {"workload": f"llama3_8b_stack_{len(layers)}_layers_dependency_order", "tokens": n_tok,
+                 "launches_per_token": 4 * len(layers), "us_per_token": round(ms_s * 1e3 / n_tok, 1),
+                 "linear_tokens_per_s": round(n_tok / (ms_s * 1e-3), 1),
+                 "GBps": round(tok_b * n_tok / (ms_s * 1e-3) / 1e9, 1),
+                 "frac_of_measured_hbm": round(tok_b * n_tok / (ms_s * 1e-3) / 1e9 / peak, 3)}
+
     # ---- the other activation precision, same steps (reported beside the headline mode)
     alt = {}
     other = 16 if args.act_bits == 24 else 24
@@ -845,7 +872,7 @@ def qtea_arm(args):
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
                          "us_per_launch": round(1e3 * total_ms / args.steps, 3),
                          "us_per_launch_isolated": None if iso_us is None else round(iso_us, 3)},
-            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "llama3_70b_layer": l70, "quantizer": quant, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
+            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "decode_stack": stack, "llama3_70b_layer": l70, "quantizer": quant, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
             "setup_s": round(t_gen, 1),
         }
         print(json.dumps(line), flush=True)
@@ -894,6 +921,7 @@ def main():
     ap.add_argument("--no-paper", action="store_true", help="skip the layer in the paper's own storage")
     ap.add_argument("--no-quant", action="store_true", help="skip the quantizer timing")
     ap.add_argument("--no-70b", action="store_true", help="skip the Llama3-70B layer steps")
+    ap.add_argument("--no-stack", action="store_true", help="skip the stack in dependency order")
     ap.add_argument("--layers", type=int, default=32,
                     help="independent resident layers the steps rotate over (32 = the whole Llama3-8B stack)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
