@@ -290,10 +290,11 @@ __global__ void __launch_bounds__(kQSumWarps * 32) quant_colsum_kernel(const flo
 }
 
 // The same column sums with the tiles streamed: 16-byte rows (K % 16 == 0), so W, the codes and
-// alpha, beta of a 128-row tile reach shared memory by cp.async, four tiles in flight. Warps 1..7
+// alpha, beta of a 128-row tile reach shared memory by cp.async, four tiles in flight. Warps 1..31
 // turn a landed tile into terms (the marker where T_ij = 0) while warp 0 adds the previous tile's
 // terms in row order.
 constexpr int kCsStages = 4;
+constexpr int kCsWarps = 32;  // warp 0 adds; 31 warps form the terms (the divisions bound them)
 
 struct CsSmem {
   float w[kCsStages][kQSumRows][32];
@@ -311,7 +312,7 @@ __device__ __forceinline__ void cp_async4(void* dst, const void* src) {
                : "memory");
 }
 
-__global__ void __launch_bounds__(kQSumWarps * 32) quant_colsum_async_kernel(const float* __restrict__ W,
+__global__ void __launch_bounds__(kCsWarps * 32) quant_colsum_async_kernel(const float* __restrict__ W,
                                                                             const float* __restrict__ alpha,
                                                                             const float* __restrict__ beta,
                                                                             const int8_t* __restrict__ T, int N,
@@ -323,7 +324,7 @@ __global__ void __launch_bounds__(kQSumWarps * 32) quant_colsum_async_kernel(con
   const int j0 = blockIdx.x * 32;  // 32 columns of one scale group (groups are K or 128 columns)
   const int g = j0 / group;
   const int n_tiles = (N + kQSumRows - 1) / kQSumRows;
-  const int pt = threadIdx.x - 32, n_pt = (kQSumWarps - 1) * 32;
+  const int pt = threadIdx.x - 32, n_pt = (kCsWarps - 1) * 32;
   auto issue = [&](int k) {
     if (k < n_tiles) {
       const int st = k % kCsStages, i0 = k * kQSumRows;
@@ -530,7 +531,7 @@ cudaError_t launch_quantize(const QuantArgs& a, cudaStream_t st) {
                           (reinterpret_cast<uintptr_t>(a.codes) & 15) == 0 && cs_async_ready();
     for (int it = 0; it < a.rescale_iters; ++it) {
       if (cs_async)
-        quant_colsum_async_kernel<<<blocks(a.K, 32), kQSumWarps * 32, sizeof(CsSmem), st>>>(
+        quant_colsum_async_kernel<<<blocks(a.K, 32), kCsWarps * 32, sizeof(CsSmem), st>>>(
             a.W, alpha, beta, a.codes, a.N, a.K, a.group, G, v);
       else
         quant_colsum_kernel<<<blocks(a.K, 32), kQSumWarps * 32, 0, st>>>(a.W, alpha, beta, a.codes, a.N, a.K,
