@@ -343,16 +343,19 @@ __global__ void __launch_bounds__(kStagedWarps * 32) qtea_gemv_paper_staged_kern
 
 // Base-3 layouts with staged activations in fixed point (M <= 4): per batch row and 128-column block
 // the CTA scales x~ = v*x by a power of two so that |X| < 2^22 (X = round(x~ * 2^e), e from the
-// block's largest |x~|), splits X into three byte planes (low and middle unsigned, top signed) and
-// stores, per five-column group q of the block, one 32-byte record: the planes of columns 5q..5q+3
-// (one word each), of column 5q+4 (one word each, other lanes zero), and S = sum of the group's X.
-// A 243-entry table turns a code byte into the same two words of codes c = T + 1. Per byte,
-// sum_d c_d X_d is six dp4a, exact in int32; sum_d T_d X_d = that - S; it is scaled once by
-// alpha * 2^-e. The rounding of X is the only approximation: |x~ - X 2^-e| <= 2^-e / 2 with
+// block's largest |x~|) and splits X into three byte planes (low and middle unsigned, top signed).
+// The block's 26 code bytes are taken four at a time (seven groups, the last two bytes of the
+// seventh standing for columns past the block, X = 0 there). Per group one 64-byte record: for each
+// plane, the four bytes' first four columns (one word per byte), then the four bytes' fifth
+// columns in one word per plane, and S = sum of the group's X. A 243-entry table turns a code byte
+// into a word of its first four codes c = T + 1 and its fifth code. Per group, sum c X is fifteen
+// dp4a, exact in int32; sum T X = that - S, summed over the block and scaled once by alpha * 2^-e.
+// The rounding of X is the only approximation: |x~ - X 2^-e| <= 2^-e / 2 with
 // 2^-e <= 2^-21 * max|x~| of the block.
-constexpr int kB3Rec = 8;          // words per five-column record
-constexpr int kB3BlockWords = 212;  // records of one block (26 x 8 words) plus 4 words: lanes that
-                                    // read different blocks' records hit distinct banks
+constexpr int kB3Groups = 7;        // groups of four code bytes per block
+constexpr int kB3GroupWords = 16;   // words per group record
+constexpr int kB3BlockWords = 116;  // 7 x 16 words plus 4: lanes that read different blocks'
+                                    // records hit distinct banks
 
 // Shared memory of one base-3 problem after the 256-entry table: records, 2^-e and block sums of x
 // per batch row and block, and the per-group sums of x with beta.
@@ -407,27 +410,43 @@ __device__ void b3_problem(const PaperParams& p, int row_lo, int row_hi, uint32_
       int ex = 0;
       if (amax > 0.f) frexpf(amax, &ex);  // amax < 2^ex
       const int e = 22 - ex;              // |X| <= 2^22 * amax / 2^ex < 2^22
-      if (lane < 26) {
-        uint32_t a0 = 0, a1 = 0, a2 = 0, b0 = 0, b1 = 0, b2 = 0;
-        int sum = 0;
+      // lane q owns code byte q of the block (columns 5q .. 5q+4; lanes 26 and 27 stand for the two
+      // padding bytes of the seventh group and hold X = 0)
+      uint32_t a0 = 0, a1 = 0, a2 = 0, f0 = 0, f1 = 0, f2 = 0;
+      int sum = 0;
 #pragma unroll
-        for (int d = 0; d < 5; ++d) {
-          const int X = amax > 0.f ? __float2int_rn(ldexpf(xt[d], e)) : 0;
-          sum += X;
-          const uint32_t u0 = (uint32_t)X & 0xFFu, u1 = ((uint32_t)X >> 8) & 0xFFu, u2 = ((uint32_t)X >> 16) & 0xFFu;
-          if (d < 4) {
-            a0 |= u0 << (8 * d);
-            a1 |= u1 << (8 * d);
-            a2 |= u2 << (8 * d);
-          } else {
-            b0 = u0;
-            b1 = u1;
-            b2 = u2;
-          }
+      for (int d = 0; d < 5; ++d) {
+        const int X = amax > 0.f ? __float2int_rn(ldexpf(xt[d], e)) : 0;
+        sum += X;
+        const uint32_t u0 = (uint32_t)X & 0xFFu, u1 = ((uint32_t)X >> 8) & 0xFFu, u2 = ((uint32_t)X >> 16) & 0xFFu;
+        if (d < 4) {
+          a0 |= u0 << (8 * d);
+          a1 |= u1 << (8 * d);
+          a2 |= u2 << (8 * d);
+        } else {
+          f0 = u0;
+          f1 = u1;
+          f2 = u2;
         }
-        uint32_t* r = rec + (size_t)t * kB3BlockWords + lane * kB3Rec;
-        reinterpret_cast<uint4*>(r)[0] = make_uint4(a0, b0, a1, b1);
-        reinterpret_cast<uint4*>(r)[1] = make_uint4(a2, b2, (uint32_t)sum, 0u);
+      }
+      // the group's fifth columns, byte i from lane 4 (q / 4) + i, and the group's sum of X
+      uint32_t w0 = 0, w1 = 0, w2 = 0;
+      int gsum = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const int src = (lane & ~3) + i;
+        w0 |= __shfl_sync(0xffffffffu, f0, src) << (8 * i);
+        w1 |= __shfl_sync(0xffffffffu, f1, src) << (8 * i);
+        w2 |= __shfl_sync(0xffffffffu, f2, src) << (8 * i);
+        gsum += __shfl_sync(0xffffffffu, sum, src);
+      }
+      if (lane < 4 * kB3Groups) {
+        uint32_t* r = rec + (size_t)t * kB3BlockWords + (lane >> 2) * kB3GroupWords;
+        const int b = lane & 3;
+        r[b] = a0;
+        r[4 + b] = a1;
+        r[8 + b] = a2;
+        if (b == 0) *reinterpret_cast<uint4*>(r + 12) = make_uint4(w0, w1, w2, (uint32_t)gsum);
       }
       if (lane == 0) {
         inv[t] = amax > 0.f ? ldexpf(1.f, -e) : 0.f;
@@ -470,19 +489,29 @@ __device__ void b3_problem(const PaperParams& p, int row_lo, int row_hi, uint32_
 #pragma unroll
       for (int m = 0; m < MB; ++m) isum[m] = 0;
 #pragma unroll
-      for (int j = 0; j < 26; ++j) {
-        const uint32_t byte = (h[j >> 1] >> (8 * (j & 1))) & 0xFFu;
-        const uint2 cw = lut[min(byte, 242u)];
+      for (int gq = 0; gq < kB3Groups; ++gq) {
+        uint2 cw[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const int j = 4 * gq + i;  // bytes 26 and 27 stand for columns past the block: T = 0
+          const uint32_t byte = j < 26 ? (h[j >> 1] >> (8 * (j & 1))) & 0xFFu : 121u;
+          cw[i] = lut[byte];
+        }
+        const uint32_t c4 = cw[0].y | (cw[1].y << 8) | (cw[2].y << 16) | (cw[3].y << 24);
 #pragma unroll
         for (int m = 0; m < MB; ++m) {
           if (m < M) {
-            const uint32_t* r = rec + (size_t)(m * n_blocks + (on ? blk : 0)) * kB3BlockWords + j * kB3Rec;
-            const uint4 r0 = reinterpret_cast<const uint4*>(r)[0];
-            const uint4 r1 = reinterpret_cast<const uint4*>(r)[1];
-            const int s0 = __dp4a(cw.x, r0.x, __dp4a(cw.y, r0.y, 0u));
-            const int s1 = __dp4a(cw.x, r0.z, __dp4a(cw.y, r0.w, 0u));
-            const int s2 = __dp4a((int)cw.x, (int)r1.x, __dp4a((int)cw.y, (int)r1.y, 0));
-            isum[m] += s2 * 65536 + s1 * 256 + s0 - (int)r1.z;
+            const uint4* r = reinterpret_cast<const uint4*>(
+                rec + (size_t)(m * n_blocks + (on ? blk : 0)) * kB3BlockWords + gq * kB3GroupWords);
+            const uint4 p0 = r[0], p1 = r[1], p2 = r[2], ft = r[3];
+            int s0 = __dp4a(cw[0].x, p0.x, __dp4a(cw[1].x, p0.y, __dp4a(cw[2].x, p0.z, __dp4a(cw[3].x, p0.w, 0u))));
+            int s1 = __dp4a(cw[0].x, p1.x, __dp4a(cw[1].x, p1.y, __dp4a(cw[2].x, p1.z, __dp4a(cw[3].x, p1.w, 0u))));
+            int s2 = __dp4a((int)cw[0].x, (int)p2.x,
+                            __dp4a((int)cw[1].x, (int)p2.y, __dp4a((int)cw[2].x, (int)p2.z, __dp4a((int)cw[3].x, (int)p2.w, 0))));
+            s0 = __dp4a(c4, ft.x, (unsigned)s0);
+            s1 = __dp4a(c4, ft.y, (unsigned)s1);
+            s2 = __dp4a((int)c4, (int)ft.z, s2);
+            isum[m] += s2 * 65536 + s1 * 256 + s0 - (int)ft.w;
           }
         }
       }
