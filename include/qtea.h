@@ -192,8 +192,12 @@ void qtea_free(qtea_layout* layout);
  *                  group of four rows and salient column, the largest W - W^ and its position
  *
  * Decisions are taken in fp32 with every sum in index order, so the outputs are reproducible bit
- * for bit. Asynchronous on `stream`; scratch comes from the stream-ordered allocator.
- * Returns QTEA_ERR_INVALID_ARG or QTEA_ERR_UNSUPPORTED for arguments outside the above.
+ * for bit. Asynchronous on `stream`; scratch (about 16 K + 8 N G bytes) comes from the
+ * stream-ordered allocator.
+ * Limits: 1 <= N <= 2^20, 1 <= K <= 65536; W and hdiag 4-byte aligned, row_scale, col_scale and
+ * residual_vals 2-byte aligned, salient_idx 4-byte aligned. Returns QTEA_ERR_INVALID_ARG or
+ * QTEA_ERR_UNSUPPORTED for arguments outside the above, QTEA_ERR_CUDA when a launch or the
+ * scratch allocation fails.
  */
 int qtea_quantize(const float* W, const float* hdiag, int N, int K, int group_size, int n_salient, int options,
                   int fit_iters, int rescale_iters, int8_t* codes, uint16_t* row_scale, uint16_t* col_scale,
