@@ -94,6 +94,13 @@ def test_llama_shape_sample(qt):
     assert_same(run(qt, W, h, 128, 41, True), oq.quantize(W, h, 128, 41, True), 41)
 
 
+def test_down_proj_width(qt):
+    """The widest Llama3-8B input (K = 14336, down_proj) on a 1024-row slice: 448 column blocks in
+    the streamed column sums, 112 groups per row, 8 row tiles, the GEMV's salient count."""
+    W, h = synth.quant_problem(33, 1024, 14336)
+    assert_same(run(qt, W, h, 128, 432, True), oq.quantize(W, h, 128, 432, True), 432)
+
+
 @pytest.mark.parametrize("bias", [False, True])
 def test_quantized_layer_through_the_gemv(qt, bias):
     """qtea_quantize's outputs go straight into qtea_pack_layout + qtea_gemv; the result matches the
