@@ -31,7 +31,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "µs/call and achieved HBM GB/s (% of GB300 peak) for batch-1 ternary+1:4 GEMV"
 WORKLOAD = "llama3_8b_layer_gemvs_m1"
-CONFIG_ID = 1
+LAYER_WORKLOAD = "llama3_8b_layer"  # the seven GEMVs of one Llama3-8B decoder layer
 
 
 def algorithmic_bytes(N, K, s, M=1):
@@ -155,8 +155,8 @@ class ExternalEvents:
 def make_layer(layer, torch, qt, synth, keep_host=False):
     """Generate one layer's seven problems, pack them on the device, keep device operands."""
     out = []
-    for mi, (name, N, K) in enumerate(synth.config_shapes(CONFIG_ID)):
-        p = synth.config_problem(CONFIG_ID, mi, layer=layer)
+    for mi, (name, N, K) in enumerate(synth.workload_shapes(LAYER_WORKLOAD)):
+        p = synth.workload_problem(LAYER_WORKLOAD, mi, layer=layer)
         f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
         T = torch.from_numpy(p.T).cuda()
         lay = qt.qtea_pack_layout(T, n_salient=p.s)
@@ -200,7 +200,7 @@ def _oracle_rows_worker(w, workers, stride, cmd_q, done_q):
     this worker, reporting (bytes, rows, seconds)."""
     import oracle
     import synth
-    probs = [synth.config_problem(CONFIG_ID, mi, layer=0) for mi in range(7)]
+    probs = [synth.workload_problem(LAYER_WORKLOAD, mi, layer=0) for mi in range(7)]
     done_q.put(("ready", w))
     while True:
         cmd = cmd_q.get()
@@ -631,8 +631,8 @@ def qtea_arm(args):
         qlayers = []
         for li in range(4):
             L = []
-            for mi, (name, N, K) in enumerate(synth.config_shapes(2)):
-                pq = synth.config_problem(2, mi, M=16, layer=li)
+            for mi, (name, N, K) in enumerate(synth.workload_shapes("qwen3_14b_layer")):
+                pq = synth.workload_problem("qwen3_14b_layer", mi, M=16, layer=li)
                 f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
                 T = torch.from_numpy(pq.T).cuda()
                 lay = qt.qtea_pack_layout(T, n_salient=pq.s)
@@ -695,7 +695,7 @@ def qtea_arm(args):
         for li in range(n_res):
             L = []
             for mi in range(7):
-                pp = synth.paper_problem(1, mi, layer=li, residual_fp8=fp8)
+                pp = synth.paper_problem("llama3_8b_layer", mi, layer=li, residual_fp8=fp8)
                 f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
                 T = torch.from_numpy(pp.T).cuda()
                 lay = qt.qtea_pack_layout(T, n_salient=pp.s, group_size=128, fmt=fmt)
@@ -708,7 +708,7 @@ def qtea_arm(args):
                               residual_idx=torch.from_numpy(pp.residual_idx).cuda(),
                               y=torch.empty((1, pp.N), dtype=torch.float32, device="cuda")))
             players.append(L)
-        shapes = synth.config_shapes(1)
+        shapes = synth.workload_shapes("llama3_8b_layer")
         if fmt == qt.QTEA_FMT_BASE3 and fp8:
             pbytes = sum(paper_algorithmic_bytes(N, K, synth.salient_count(K)) for _, N, K in shapes)
         else:
@@ -747,13 +747,13 @@ def qtea_arm(args):
     # ---- the Llama3-70B layer (8192-wide, 28672-row MLP: the large-K shapes) at M = 1, the seven
     #      GEMVs per step as one grouped call, rotating over resident layers whose codes exceed L2
     def llama70b_leg():
-        cfg, n_res, nsteps = 3, 3, 24
-        shapes = synth.config_shapes(cfg)
+        wl, n_res, nsteps = "llama3_70b_layer", 3, 24
+        shapes = synth.workload_shapes(wl)
         players, pbytes = [], []
         for li in range(n_res):
             L, b = [], 0
             for mi, (_, N, K) in enumerate(shapes):
-                pp = synth.config_problem(cfg, mi, layer=li)
+                pp = synth.workload_problem(wl, mi, layer=li)
                 f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
                 T = torch.from_numpy(pp.T).cuda()
                 lay = qt.qtea_pack_layout(T, n_salient=pp.s)
@@ -796,7 +796,7 @@ def qtea_arm(args):
     #      1:4 residual) on the Llama3-8B layer's seven fp32 weight matrices: 128-column groups with
     #      beta, 4 alpha refits, 2 rescale rounds, the GEMV's salient count
     def quant_leg():
-        shapes = synth.config_shapes(1)
+        shapes = synth.workload_shapes("llama3_8b_layer")
         gen = torch.Generator(device="cuda").manual_seed(1234)
         mats = []
         for _, N, K in shapes:
@@ -896,7 +896,7 @@ def profile_case(args):
     M = args.m
     probs = []
     for mi in range(7):
-        p = synth.config_problem(2, mi, M=M)
+        p = synth.workload_problem("qwen3_14b_layer", mi, M=M)
         lay = qt.qtea_pack_layout(torch.from_numpy(p.T).cuda(), n_salient=p.s)
         probs.append(dict(x=f16(p.x), layout=lay, row_scale=f16(p.alpha.reshape(-1)), col_scale=f16(p.v),
                           salient_idx=torch.from_numpy(p.salient_idx).cuda(), residual_vals=f16(p.residual_vals),

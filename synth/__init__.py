@@ -7,7 +7,7 @@ library both consume exactly the bytes produced here.
 
 The workload shapes stand in for real model weights (which are not available): the layer
 shapes of Llama3-8B, Qwen3-14B and Llama3-70B, with random ternary codes and the value
-distributions listed in ``CONFIGS``.
+distributions listed in ``WORKLOADS``.
 """
 from __future__ import annotations
 
@@ -196,31 +196,33 @@ LLAMA3_70B = [("q_proj", 8192, 8192), ("k_proj", 1024, 8192), ("v_proj", 1024, 8
               ("o_proj", 8192, 8192), ("gate_proj", 28672, 8192), ("up_proj", 28672, 8192),
               ("down_proj", 8192, 28672)]
 
-CONFIGS: Dict[int, dict] = {
-    0: dict(name="tiny_1024", shapes=[("tiny", 1024, 1024)], M=[1], p=(0.3, 0.4), residual="normal",
-            residual_scale=0.02, fixed_s=32),
-    1: dict(name="llama3_8b_layer", shapes=LLAMA3_8B, M=[1], p=(0.3, 0.4), residual="normal",
-            residual_scale=0.02),
-    2: dict(name="qwen3_14b_layer", shapes=QWEN3_14B, M=[1, 2, 4, 8, 16], p=(0.25, 0.5), residual="normal",
-            residual_scale=0.02),
-    3: dict(name="llama3_70b_layer", shapes=LLAMA3_70B, M=[1], p=(0.3, 0.4), residual="laplace",
-            residual_scale=0.01),
-    4: dict(name="llama3_8b_32layer_stack", shapes=LLAMA3_8B, M=[1], p=(0.3, 0.4), residual="normal",
-            residual_scale=0.02, layers=32),
+# The workloads, by name. seed_base is the first seed of the workload: the operands of matrix j of
+# layer l are drawn with seed seed_base + 16 l + j.
+WORKLOADS: Dict[str, dict] = {
+    "tiny_1024": dict(seed_base=0, shapes=[("tiny", 1024, 1024)], M=[1], p=(0.3, 0.4), residual="normal",
+                      residual_scale=0.02, fixed_s=32),
+    "llama3_8b_layer": dict(seed_base=1000, shapes=LLAMA3_8B, M=[1], p=(0.3, 0.4), residual="normal",
+                            residual_scale=0.02),
+    "qwen3_14b_layer": dict(seed_base=2000, shapes=QWEN3_14B, M=[1, 2, 4, 8, 16], p=(0.25, 0.5),
+                            residual="normal", residual_scale=0.02),
+    "llama3_70b_layer": dict(seed_base=3000, shapes=LLAMA3_70B, M=[1], p=(0.3, 0.4), residual="laplace",
+                             residual_scale=0.01),
+    "llama3_8b_32layer_stack": dict(seed_base=4000, shapes=LLAMA3_8B, M=[1], p=(0.3, 0.4), residual="normal",
+                                    residual_scale=0.02, layers=32),
 }
 
 
-def config_seed(config: int, layer: int, matrix: int) -> int:
-    return 1000 * config + 16 * layer + matrix
+def workload_seed(workload: str, layer: int, matrix: int) -> int:
+    return WORKLOADS[workload]["seed_base"] + 16 * layer + matrix
 
 
-def config_problem(config: int, matrix: int, M: Optional[int] = None, layer: int = 0) -> Problem:
-    cfg = CONFIGS[config]
+def workload_problem(workload: str, matrix: int, M: Optional[int] = None, layer: int = 0) -> Problem:
+    cfg = WORKLOADS[workload]
     name, N, K = cfg["shapes"][matrix]
     s = cfg.get("fixed_s") or salient_count(K)
     M = cfg["M"][0] if M is None else M
     p_neg, p_zero = cfg["p"]
-    return make_problem(f"{cfg['name']}/{name}", N, K, M, s, config_seed(config, layer, matrix), p_neg, p_zero,
+    return make_problem(f"{workload}/{name}", N, K, M, s, workload_seed(workload, layer, matrix), p_neg, p_zero,
                         cfg["residual"], cfg["residual_scale"])
 
 
@@ -230,22 +232,22 @@ def config_problem(config: int, matrix: int, M: Optional[int] = None, layer: int
 PAPER_FORMAT = dict(group_size=128, beta_std=0.002, residual_fp8=True)
 
 
-def paper_problem(config: int, matrix: int, M: Optional[int] = None, layer: int = 0,
+def paper_problem(workload: str, matrix: int, M: Optional[int] = None, layer: int = 0,
                   residual_fp8: bool = True) -> Problem:
-    """config_problem's operands in the paper's storage (same seed, hence the same codes, x and v);
-    residual_fp8=False keeps fp16 residual values with the paper's scale groups."""
-    cfg = CONFIGS[config]
+    """workload_problem's operands in the paper's storage (same seed, hence the same codes, x and
+    v); residual_fp8=False keeps fp16 residual values with the paper's scale groups."""
+    cfg = WORKLOADS[workload]
     name, N, K = cfg["shapes"][matrix]
     s = cfg.get("fixed_s") or salient_count(K)
     M = cfg["M"][0] if M is None else M
     p_neg, p_zero = cfg["p"]
     fmt = dict(PAPER_FORMAT, residual_fp8=residual_fp8)
-    return make_problem(f"{cfg['name']}/{name}/paper_format", N, K, M, s, config_seed(config, layer, matrix), p_neg,
+    return make_problem(f"{workload}/{name}/paper_format", N, K, M, s, workload_seed(workload, layer, matrix), p_neg,
                         p_zero, "normal", cfg["residual_scale"], **fmt)
 
 
-def config_shapes(config: int) -> List[Tuple[str, int, int]]:
-    return list(CONFIGS[config]["shapes"])
+def workload_shapes(workload: str) -> List[Tuple[str, int, int]]:
+    return list(WORKLOADS[workload]["shapes"])
 
 
 def quant_problem(seed: int, N: int, K: int, std: float = 0.02):

@@ -122,7 +122,7 @@ def test_options_switch_a_default_layout_to_the_paper_path(qt):
 def test_paper_storage_llama3_8b_layer(qt, matrix, M):
     """The Llama3-8B layer GEMVs in the paper's storage (base-3, 128-column groups with beta, FP8
     residual), on 48 sampled output rows."""
-    p = synth.paper_problem(1, matrix, M=M)
+    p = synth.paper_problem("llama3_8b_layer", matrix, M=M)
     y, _ = run_paper(qt, p, qt.QTEA_FMT_BASE3, True)
     rows = np.sort(np.random.default_rng(matrix).choice(p.N, size=48, replace=False)).astype(np.int32)
     y_ref, b = reference(p, True, rows=rows)

@@ -77,10 +77,12 @@ def test_pack_is_bit_identical_to_oracle(qt, N, K):
     assert lay.describe()["K_pad"] == -(-K // 64) * 64
 
 
-@pytest.mark.parametrize("config,matrix", [(0, 0), (1, 0), (1, 1), (1, 6), (3, 4), (3, 6)])
-def test_batch1_kernel_serves_workload_shapes(qt, config, matrix):
-    """The configured shapes must run on the TMA stream-K kernel, not the general fallback."""
-    p = synth.config_problem(config, matrix)
+@pytest.mark.parametrize("workload,matrix", [("tiny_1024", 0), ("llama3_8b_layer", 0), ("llama3_8b_layer", 1),
+                                              ("llama3_8b_layer", 6), ("llama3_70b_layer", 4),
+                                              ("llama3_70b_layer", 6)])
+def test_batch1_kernel_serves_workload_shapes(qt, workload, matrix):
+    """The workload shapes must run on the TMA stream-K kernel, not the general fallback."""
+    p = synth.workload_problem(workload, matrix)
     lay = qt.qtea_pack_layout(dev(p.T), n_salient=p.s)
     assert lay.describe()["batch1_kernel"] == 1
 
@@ -152,12 +154,12 @@ def test_low_batch_unaligned_operands(qt, M):
     assert_within(y.cpu().numpy().astype(np.float64), y_ref, b, f"unaligned M={M}")
 
 
-def test_config0_tiny(qt):
-    p = synth.config_problem(0, 0)
+def test_tiny_1024(qt):
+    p = synth.workload_problem("tiny_1024", 0)
     d = Dev(qt, p)
     y = d.run(qt)
     y_ref, b = oracle_ref(p)
-    worst = assert_within(y, y_ref, b, "config 0")
+    worst = assert_within(y, y_ref, b, "tiny_1024")
     assert worst < 0.25  # keep a 4x margin on the tolerance
 
 
@@ -254,9 +256,10 @@ def sample_rows(N, n=48, seed=0):
     return np.array(rows, np.int32)
 
 
-@pytest.mark.parametrize("config,matrix", [(1, m) for m in range(7)] + [(3, m) for m in range(7)])
-def test_full_size_layers_m1(qt, config, matrix):
-    p = synth.config_problem(config, matrix)
+@pytest.mark.parametrize("workload,matrix",
+                         [("llama3_8b_layer", m) for m in range(7)] + [("llama3_70b_layer", m) for m in range(7)])
+def test_full_size_layers_m1(qt, workload, matrix):
+    p = synth.workload_problem(workload, matrix)
     d = Dev(qt, p)
     y = d.run(qt)
     rows = sample_rows(p.N, seed=matrix)
@@ -267,7 +270,7 @@ def test_full_size_layers_m1(qt, config, matrix):
 @pytest.mark.parametrize("matrix", range(7))
 @pytest.mark.parametrize("M", [1, 2, 4, 8, 16])
 def test_full_size_qwen3_14b_batch_sweep(qt, matrix, M):
-    p = synth.config_problem(2, matrix, M=M)
+    p = synth.workload_problem("qwen3_14b_layer", matrix, M=M)
     d = Dev(qt, p)
     y = d.run(qt)
     rows = sample_rows(p.N, n=16, seed=matrix + M)
@@ -297,7 +300,7 @@ def test_grouped_matches_oracle(qt, n):
 
 
 def test_grouped_llama3_8b_layer(qt):
-    ps = [synth.config_problem(1, m) for m in range(7)]
+    ps = [synth.workload_problem("llama3_8b_layer", m) for m in range(7)]
     ds = [Dev(qt, p) for p in ps]
     ys = qt.qtea_gemv_grouped([problem_dict(d) for d in ds])
     torch.cuda.synchronize()
@@ -316,7 +319,7 @@ def test_grouped_llama3_8b_layer(qt):
 @pytest.mark.parametrize("layer", [0, 17, 31])
 def test_grouped_llama3_8b_stack_layers(qt, layer):
     """Layers of the 32-layer stack (independent seeds per layer), as the benchmark launches them."""
-    ps = [synth.config_problem(4, m, layer=layer) for m in range(7)]
+    ps = [synth.workload_problem("llama3_8b_32layer_stack", m, layer=layer) for m in range(7)]
     ds = [Dev(qt, p) for p in ps]
     ys = qt.qtea_gemv_grouped([problem_dict(d) for d in ds])
     torch.cuda.synchronize()
@@ -350,12 +353,14 @@ def test_grouped_batch2_uses_general_path(qt):
 
 # ---------------------------------------------------------------- 16-bit activation mode
 
-@pytest.mark.parametrize("config,matrix", [(0, 0), (1, 1), (1, 4), (1, 6), (2, 0), (2, 6), (3, 1), (3, 6)])
-def test_fast_mode_keeps_a_4x_margin(qt, config, matrix):
-    p = synth.config_problem(config, matrix)
+@pytest.mark.parametrize("workload,matrix", [("tiny_1024", 0), ("llama3_8b_layer", 1), ("llama3_8b_layer", 4),
+                                              ("llama3_8b_layer", 6), ("qwen3_14b_layer", 0), ("qwen3_14b_layer", 6),
+                                              ("llama3_70b_layer", 1), ("llama3_70b_layer", 6)])
+def test_fast_mode_keeps_a_4x_margin(qt, workload, matrix):
+    p = synth.workload_problem(workload, matrix)
     d = Dev(qt, p, act_bits=16)
     y = d.run(qt)
-    rows = sample_rows(p.N, n=64, seed=config * 10 + matrix)
+    rows = sample_rows(p.N, n=64, seed=synth.WORKLOADS[workload]["seed_base"] // 100 + matrix)
     y_ref, b = oracle_ref(p, rows=rows)
     worst = assert_within(y[:, rows], y_ref, b, f"16-bit {p.name}")
     assert worst < 0.25

@@ -147,7 +147,7 @@ def test_fp8_residual_equals_the_same_values_in_fp16():
 def test_paper_storage_matches_dense():
     """The paper's own storage end to end: alpha and beta per (row, 128-column group), FP8 E4M3
     residual values; brute-force dense W^ (E4M3 decoded by the pinned routine) times x."""
-    p = synth.paper_problem(0, 0)
+    p = synth.paper_problem("tiny_1024", 0)
     p.T, p.x = p.T[:64, :300], p.x[:, :300]  # a ragged last group
     N, K = p.T.shape
     G = -(-K // 128)
@@ -388,7 +388,7 @@ def test_asic_latency_model_reproduces_paper_table():
 # ---------------------------------------------------------------- generated inputs
 
 def test_generated_inputs_invariants():
-    p = synth.config_problem(1, 1)  # k_proj 1024 x 4096
+    p = synth.workload_problem("llama3_8b_layer", 1)  # k_proj 1024 x 4096
     assert p.T.dtype == np.int8 and set(np.unique(p.T).tolist()) <= {-1, 0, 1}
     n = p.T.size
     for val, prob in [(-1, 0.3), (0, 0.4), (1, 0.3)]:

@@ -47,10 +47,10 @@ def _dev(a, dtype=None):
 
 
 CASES = [
-    ("tiny 1024x1024", lambda: synth.config_problem(0, 0)),
+    ("tiny 1024x1024", lambda: synth.workload_problem("tiny_1024", 0)),
     ("ragged 1000x1000", lambda: synth.make_problem("r", 1000, 1000, 1, 24, seed=11)),
-    ("llama3-8b down_proj 4096x14336", lambda: synth.config_problem(1, 6)),
-    ("llama3-8b gate_proj 14336x4096", lambda: synth.config_problem(1, 4)),
+    ("llama3-8b down_proj 4096x14336", lambda: synth.workload_problem("llama3_8b_layer", 6)),
+    ("llama3-8b gate_proj 14336x4096", lambda: synth.workload_problem("llama3_8b_layer", 4)),
     ("no residual 2048x3000", lambda: synth.make_problem("n", 2048, 3000, 1, 0, seed=12)),
 ]
 
