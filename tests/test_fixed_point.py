@@ -51,8 +51,9 @@ def test_plane_dot_products_give_the_exact_sum():
 
 
 def test_block_sum_headroom():
-    """A 128-column block's sum_j T_j X_j is at most 128 * 2^22 = 2^29 in magnitude; the batch-1
-    kernel's 24-bit planes over 512 columns stay below 2^31 as well."""
+    """A 128-column block's sum_j T_j X_j is at most 128 * 2^22 = 2^29 in magnitude (int32 in the
+    base-3 kernel); the batch-1 kernel's sum c X over 512 columns of 24-bit X stays below 2^33 and is
+    formed in int64."""
     assert 128 * ((1 << 22) - 1) < 2 ** 29
     assert 2 * 512 * ((1 << 23) - 1) < 2 ** 33  # sum c X before the sum X correction, in int64 there
 
