@@ -25,7 +25,7 @@ _LIB_PATH = os.path.join(_HERE, "libqtea_synth.so")
 _lib = None
 
 # stream ids, one per tensor kind
-S_CODES, S_ALPHA, S_V, S_X, S_SALIENT, S_RVALS, S_RIDX, S_BETA = 1, 2, 3, 4, 5, 6, 7, 8
+S_CODES, S_ALPHA, S_V, S_X, S_SALIENT, S_RVALS, S_RIDX, S_BETA, S_MASSIVE = 1, 2, 3, 4, 5, 6, 7, 8, 9
 
 
 def build(force: bool = False) -> str:
@@ -155,8 +155,8 @@ class Problem:
 def make_problem(name: str, N: int, K: int, M: int, s: int, seed: int, p_neg: float = 0.3,
                  p_zero: float = 0.4, residual: str = "normal", residual_scale: float = 0.02,
                  alpha_range=(0.01, 0.05), v_range=(0.8, 1.2), group_size: int = 0, beta_std: float = 0.0,
-                 residual_fp8: bool = False) -> Problem:
-    """Seeded operands. group_size > 0 gives one alpha per (row, group of group_size columns),
+                 residual_fp8: bool = False, x_std: float = 1.0) -> Problem:
+    """Seeded operands (x drawn N(0, x_std)). group_size > 0 gives one alpha per (row, group of group_size columns),
     beta_std > 0 a per-(row, group) beta drawn N(0, beta_std), and residual_fp8 residual values
     rounded to FP8 E4M3 instead of fp16: the paper's own storage (Sec. 3.3, Eq. 4; Sec. 4.1)."""
     if s > 0 and N % 4:
@@ -166,7 +166,7 @@ def make_problem(name: str, N: int, K: int, M: int, s: int, seed: int, p_neg: fl
     T = codes(seed, S_CODES, (N, K), p_neg, p_zero)
     alpha = uniform_f16(seed, S_ALPHA, (N, G), *alpha_range)
     v = uniform_f16(seed, S_V, (K,), *v_range)
-    x = normal_f16(seed, S_X, (M, K), 0.0, 1.0)
+    x = normal_f16(seed, S_X, (M, K), 0.0, x_std)
     sal = salient(seed, S_SALIENT, K, s)
     if residual_fp8:
         if residual != "normal":
@@ -244,6 +244,19 @@ def paper_problem(workload: str, matrix: int, M: Optional[int] = None, layer: in
     fmt = dict(PAPER_FORMAT, residual_fp8=residual_fp8)
     return make_problem(f"{workload}/{name}/paper_format", N, K, M, s, workload_seed(workload, layer, matrix), p_neg,
                         p_zero, "normal", cfg["residual_scale"], **fmt)
+
+
+def plant_massive(x: np.ndarray, seed: int, magnitudes, lo: int = 0, hi: Optional[int] = None) -> np.ndarray:
+    """Activations with a few "massive" values, as LLM hidden states show at some channels: a copy of
+    x (fp16 bits [M][K]) in which len(magnitudes) distinct columns of [lo, hi), drawn with the seed,
+    hold +-magnitude (alternating signs, every batch row), rounded to binary16. Returns the columns."""
+    K = x.shape[-1]
+    hi = K if hi is None else min(hi, K)
+    n = len(magnitudes)
+    cols = np.sort(salient(seed, S_MASSIVE, hi - lo, n) + lo)
+    for i, (c, m) in enumerate(zip(cols, magnitudes)):
+        x[..., c] = f16_from_double(float(m) if i % 2 == 0 else -float(m))
+    return cols
 
 
 def workload_shapes(workload: str) -> List[Tuple[str, int, int]]:
