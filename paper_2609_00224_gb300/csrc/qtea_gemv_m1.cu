@@ -251,7 +251,22 @@ __device__ __forceinline__ void load_chunk(const ProblemArgs& a, int ch, int lan
   }
 }
 
-// The chunk's v*x as fixed point: byte planes of this lane's word, and (lane 0) the metadata.
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// The chunk's v*x as fixed point: byte planes of this lane's word, and the metadata.
+//  * Outliers: in up to kOutlierRounds rounds, the elements above 1/16 of the largest |v*x| not yet
+//    taken are taken, as long as at most kMaxOutliers are taken in all. A round of ordinary values
+//    has hundreds above that threshold and ends the search, so only values at least 16 times above
+//    the rest are ever taken. They get X = 0 in the planes and are listed in the metadata with
+//    their exact v*x, which the consumers add per row in fp32.
+//  * The remaining values set the quantum: their largest magnitude amax in [2^e, 2^(e+1)) gives
+//    q = 2^(e-22) for 24 bits (|X| < 2^23) or q = 2^(e-14) for 16 bits (|X| < 2^15). 16 bits are
+//    taken where the caller allows it and amax is within 8 times the root mean square of the
+//    remaining values (no heavy tail that would coarsen the quantum of the others).
 __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLoads& L, uint8_t* ax, int lane) {
   float xt[16];
 #pragma unroll
@@ -259,29 +274,61 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
     xt[2 * i] = h2f((uint16_t)(L.v[i] & 0xffffu)) * h2f((uint16_t)(L.x[i] & 0xffffu));
     xt[2 * i + 1] = h2f((uint16_t)(L.v[i] >> 16)) * h2f((uint16_t)(L.x[i] >> 16));
   }
-  float amax = 0.f, ssq = 0.f;
+  float lmax = 0.f;
 #pragma unroll
-  for (int i = 0; i < 16; ++i) {
-    amax = fmaxf(amax, fabsf(xt[i]));
-    ssq = fmaf(xt[i], xt[i], ssq);
-  }
+  for (int i = 0; i < 16; ++i) lmax = fmaxf(lmax, fabsf(xt[i]));
+  float amax = warp_max(lmax);
+  uint32_t outm = 0;  // bit i: xt[i] is an outlier
+  int n_out = 0;
+#pragma unroll 1
+  for (int round = 0; round < kOutlierRounds && amax > 0.f; ++round) {
+    const float thr = amax * 0.0625f;
+    uint32_t m = 0;
 #pragma unroll
-  for (int o = 16; o; o >>= 1) {
-    amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
-    ssq += __shfl_xor_sync(0xffffffffu, ssq, o);
+    for (int i = 0; i < 16; ++i) m |= (fabsf(xt[i]) > thr ? 1u : 0u) << i;
+    m &= ~outm;
+    const int c = (int)__reduce_add_sync(0xffffffffu, (unsigned)__popc(m));
+    if (c > kMaxOutliers - n_out) break;
+    outm |= m;
+    n_out += c;
+    lmax = 0.f;
+#pragma unroll
+    for (int i = 0; i < 16; ++i) lmax = fmaxf(lmax, ((outm >> i) & 1u) ? 0.f : fabsf(xt[i]));
+    amax = warp_max(lmax);
   }
-  // 16-bit fixed point only where the chunk's largest |v*x| is within 8x its root mean square
-  // (no outliers that would coarsen the quantum of the others); otherwise 24-bit
-  const bool two = a.act_bits == 16 && amax * amax <= 64.f * (ssq / (float)kChunkCols);
-  // amax in [2^e, 2^(e+1)) -> q = 2^(e-21), |X| <= 2^22 (24-bit) or q = 2^(e-13), |X| <= 2^14
+  ChunkMeta* meta = reinterpret_cast<ChunkMeta*>(ax + kAuxMeta);
+  if (n_out > 0) {  // list them: lane order, then element order
+    const int mine = __popc(outm);
+    int off = mine;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int t = __shfl_up_sync(0xffffffffu, off, o);
+      if (lane >= o) off += t;
+    }
+    off -= mine;
+#pragma unroll
+    for (int i = 0; i < 16; ++i)
+      if ((outm >> i) & 1u) {
+        meta->out_col[off] = (uint16_t)(lane * 16 + i);
+        meta->out_val[off] = xt[i];
+        ++off;
+      }
+  }
+  float ssq = 0.f;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) ssq = ((outm >> i) & 1u) ? ssq : fmaf(xt[i], xt[i], ssq);
+#pragma unroll
+  for (int o = 16; o; o >>= 1) ssq += __shfl_xor_sync(0xffffffffu, ssq, o);
+  const bool two = a.act_bits == 16 && amax * amax <= 64.f * (ssq / (float)(kChunkCols - n_out));
   const int e = amax > 0.f ? (int)((__float_as_uint(amax) >> 23) & 0xff) - 127 : 0;
-  const int qsh = two ? 13 : 21;
+  const int qsh = two ? 14 : 22;
+  const int xmax = two ? 32767 : 8388607;  // a value of amax rounds to at most 2^(qsh+1): clamp
   const float inv_q = __uint_as_float((uint32_t)(127 + qsh - e) << 23);
   int X[16];
   long long sx = 0;
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
-    X[i] = __float2int_rn(xt[i] * inv_q);
+    X[i] = ((outm >> i) & 1u) ? 0 : min(__float2int_rn(xt[i] * inv_q), xmax);
     sx += X[i];
   }
   uint4* dst = reinterpret_cast<uint4*>(ax + (size_t)lane * kPlaneBytesPerWord);
@@ -318,12 +365,10 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
 #pragma unroll
   for (int o = 16; o; o >>= 1) sx += __shfl_xor_sync(0xffffffffu, sx, o);
   if (lane == 0) {
-    ChunkMeta mm;
-    mm.scale4 = __uint_as_float((uint32_t)(127 + e - qsh - 2) << 23);  // q / 4
-    mm.planes = two ? 2 : 3;
-    mm.sum_x = sx;
-    mm.pad[0] = mm.pad[1] = 0;
-    *reinterpret_cast<ChunkMeta*>(ax + kAuxMeta) = mm;
+    meta->scale4 = __uint_as_float((uint32_t)(127 + e - qsh - 2) << 23);  // q / 4
+    meta->planes = two ? 2 : 3;
+    meta->sum_x = sx;
+    meta->n_out = n_out;
   }
 }
 
@@ -523,22 +568,41 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
     if (!__all_sync(0xffffffffu, ok)) break;
 
     const uint8_t* ax = r.aux + (size_t)slot * kAuxBytes;
-    const ChunkMeta m = *reinterpret_cast<const ChunkMeta*>(ax + kAuxMeta);
+    const ChunkMeta* mp = reinterpret_cast<const ChunkMeta*>(ax + kAuxMeta);
+    const float scale4 = mp->scale4;
+    const int planes = mp->planes, n_out = mp->n_out;
+    const long long sum_x = mp->sum_x;
     const uint4* row0 =
         reinterpret_cast<const uint4*>(r.codes + (size_t)st * kStageBytes + (size_t)ra * kChunkRowBytes);
     const uint4* row1 = row0 + 32 * (kChunkRowBytes / 16);
     const uint4* pl = reinterpret_cast<const uint4*>(ax);
     long long d0, d1;
-    if (m.planes == 2) {
+    if (planes == 2) {
       RowAcc<2> a0, a1;
       decode_unit<2>(row0, row1, pl, sw, a0, a1);
-      d0 = finish_chunk<2>(a0, m.sum_x);
-      d1 = finish_chunk<2>(a1, m.sum_x);
+      d0 = finish_chunk<2>(a0, sum_x);
+      d1 = finish_chunk<2>(a1, sum_x);
     } else {
       RowAcc<3> a0, a1;
       decode_unit<3>(row0, row1, pl, sw, a0, a1);
-      d0 = finish_chunk<3>(a0, m.sum_x);
-      d1 = finish_chunk<3>(a1, m.sum_x);
+      d0 = finish_chunk<3>(a0, sum_x);
+      d1 = finish_chunk<3>(a1, sum_x);
+    }
+    // outliers: T * v*x in fp32, the code of both rows read from the staged tile (byte col / 4 of
+    // the row, in 16-byte granule (col / 64) ^ (row % 8) of the 128-byte swizzle; rows ra and ra + 32
+    // share the swizzle phase)
+    float o0 = 0.f, o1 = 0.f;
+    if (n_out > 0) {
+      const uint8_t* cb0 = reinterpret_cast<const uint8_t*>(row0);
+      const uint8_t* cb1 = reinterpret_cast<const uint8_t*>(row1);
+#pragma unroll 1
+      for (int k = 0; k < n_out; ++k) {
+        const int col = mp->out_col[k];
+        const float xv = mp->out_val[k];
+        const int off = ((((col >> 6) ^ sw) << 4) | ((col >> 2) & 15)), sh = 2 * (col & 3);
+        o0 = fmaf((float)(int)((cb0[off] >> sh) & 3u) - 1.f, xv, o0);
+        o1 = fmaf((float)(int)((cb1[off] >> sh) & 3u) - 1.f, xv, o1);
+      }
     }
     ok = mbar_wait(smem_u32(&r.full_a[slot]), (uint32_t)((i / kAuxSlots) & 1), status);
     if (!__all_sync(0xffffffffu, ok)) break;
@@ -550,8 +614,8 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
       mbar_arrive(smem_u32(&r.empty_c[st]));
       mbar_arrive(smem_u32(&r.empty_a[slot]));
     }
-    yacc0 += (float)d0 * m.scale4;
-    yacc1 += (float)d1 * m.scale4;
+    yacc0 += fmaf((float)d0, scale4, o0);
+    yacc1 += fmaf((float)d1, scale4, o1);
 
     // ---- tile epilogue once this CTA's part of tile t is done
     if (c.ch == n_chunks - 1 || u == u1 - 1) {

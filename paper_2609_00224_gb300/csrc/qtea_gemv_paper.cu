@@ -350,12 +350,17 @@ __global__ void __launch_bounds__(kStagedWarps * 32) qtea_gemv_paper_staged_kern
 // columns in one word per plane, and S = sum of the group's X. A 243-entry table turns a code byte
 // into a word of its first four codes c = T + 1 and its fifth code. Per group, sum c X is fifteen
 // dp4a, exact in int32; sum T X = that - S, summed over the block and scaled once by alpha * 2^-e.
+// Outliers: values of x~ at least 16 times above the rest of the block (found in rounds, as in the
+// batch-1 kernel) are taken out of the planes, up to kB3MaxOut per block, and added exactly in fp32:
+// T x~ with T read from the row's code byte. The rest set the scale: |X| < 2^23.
 // The rounding of X is the only approximation: |x~ - X 2^-e| <= 2^-e / 2 with
-// 2^-e <= 2^-21 * max|x~| of the block.
+// 2^-e <= 2^-22 * max|x~| over the block's values that are not outliers.
 constexpr int kB3Groups = 7;        // groups of four code bytes per block
 constexpr int kB3GroupWords = 16;   // words per group record
-constexpr int kB3BlockWords = 116;  // 7 x 16 words plus 4: lanes that read different blocks'
-                                    // records hit distinct banks
+constexpr int kB3BlockWords = 116;  // 7 x 16 words plus 4 (outliers: count and columns, then up to
+                                    // three values); lanes that read different blocks' records hit
+                                    // distinct banks
+constexpr int kB3MaxOut = 3;
 
 // Shared memory of one base-3 problem after the 256-entry table: records, 2^-e and block sums of x
 // per batch row and block, and the per-group sums of x with beta.
@@ -407,16 +412,36 @@ __device__ void b3_problem(const PaperParams& p, int row_lo, int row_hi, uint32_
         amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, off));
         xs += __shfl_xor_sync(0xffffffffu, xs, off);
       }
+      uint32_t outm = 0;  // bit d: xt[d] is an outlier
+      int n_out = 0;
+#pragma unroll 1
+      for (int round = 0; round < kB3MaxOut && amax > 0.f; ++round) {
+        const float thr = amax * 0.0625f;
+        uint32_t m = 0;
+#pragma unroll
+        for (int d = 0; d < 5; ++d) m |= (fabsf(xt[d]) > thr ? 1u : 0u) << d;
+        m &= ~outm;
+        const int c = (int)__reduce_add_sync(0xffffffffu, (unsigned)__popc(m));
+        if (c > kB3MaxOut - n_out) break;
+        outm |= m;
+        n_out += c;
+        float lm = 0.f;
+#pragma unroll
+        for (int d = 0; d < 5; ++d) lm = fmaxf(lm, ((outm >> d) & 1u) ? 0.f : fabsf(xt[d]));
+#pragma unroll
+        for (int off = 16; off; off >>= 1) lm = fmaxf(lm, __shfl_xor_sync(0xffffffffu, lm, off));
+        amax = lm;
+      }
       int ex = 0;
       if (amax > 0.f) frexpf(amax, &ex);  // amax < 2^ex
-      const int e = 22 - ex;              // |X| <= 2^22 * amax / 2^ex < 2^22
+      const int e = 23 - ex;              // |X| <= 2^23 * amax / 2^ex: at most 2^23 - 1 after the clamp
       // lane q owns code byte q of the block (columns 5q .. 5q+4; lanes 26 and 27 stand for the two
       // padding bytes of the seventh group and hold X = 0)
       uint32_t a0 = 0, a1 = 0, a2 = 0, f0 = 0, f1 = 0, f2 = 0;
       int sum = 0;
 #pragma unroll
       for (int d = 0; d < 5; ++d) {
-        const int X = amax > 0.f ? __float2int_rn(ldexpf(xt[d], e)) : 0;
+        const int X = (amax > 0.f && !((outm >> d) & 1u)) ? min(__float2int_rn(ldexpf(xt[d], e)), 8388607) : 0;
         sum += X;
         const uint32_t u0 = (uint32_t)X & 0xFFu, u1 = ((uint32_t)X >> 8) & 0xFFu, u2 = ((uint32_t)X >> 16) & 0xFFu;
         if (d < 4) {
@@ -447,6 +472,27 @@ __device__ void b3_problem(const PaperParams& p, int row_lo, int row_hi, uint32_
         r[4 + b] = a1;
         r[8 + b] = a2;
         if (b == 0) *reinterpret_cast<uint4*>(r + 12) = make_uint4(w0, w1, w2, (uint32_t)gsum);
+      }
+      {  // the outlier list in the record's last four words: count and columns, then the values
+        uint32_t* ol = rec + (size_t)t * kB3BlockWords + kB3Groups * kB3GroupWords;
+        const int mine = __popc(outm);
+        int off = mine;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+          const int v = __shfl_up_sync(0xffffffffu, off, o);
+          if (lane >= o) off += v;
+        }
+        off -= mine;  // earlier lanes' outliers
+        uint32_t cols = 0;
+#pragma unroll
+        for (int d = 0; d < 5; ++d)
+          if ((outm >> d) & 1u) {
+            ol[1 + off] = __float_as_uint(xt[d]);
+            cols |= (uint32_t)(5 * lane + d) << (8 * (1 + off));
+            ++off;
+          }
+        cols = __reduce_or_sync(0xffffffffu, cols);
+        if (lane == 0) ol[0] = cols | (uint32_t)n_out;
       }
       if (lane == 0) {
         inv[t] = amax > 0.f ? ldexpf(1.f, -e) : 0.f;
@@ -518,7 +564,21 @@ __device__ void b3_problem(const PaperParams& p, int row_lo, int row_hi, uint32_
       if (on)
 #pragma unroll
         for (int m = 0; m < MB; ++m)
-          if (m < M) acc[m] += (al * inv[m * n_blocks + blk]) * (float)isum[m];
+          if (m < M) {
+            // the block's outliers: T x~ in fp32, T from the code byte (reloaded: a register array
+            // indexed by a loop value would go to local memory)
+            const uint32_t* ol = rec + (size_t)(m * n_blocks + blk) * kB3BlockWords + kB3Groups * kB3GroupWords;
+            const uint32_t head = ol[0];
+            float ov = 0.f;
+            for (int k = 0; k < (int)(head & 0xFFu); ++k) {
+              const int c = (int)((head >> (8 * (1 + k))) & 0xFFu);
+              const uint2 cw = lut[__ldg(row + (size_t)blk * 26 + c / 5)];
+              const int d = c % 5;
+              const int code = d < 4 ? (int)((cw.x >> (8 * d)) & 0xFFu) : (int)cw.y;
+              ov = fmaf((float)(code - 1), __uint_as_float(ol[1 + k]), ov);
+            }
+            acc[m] += al * fmaf(inv[m * n_blocks + blk], (float)isum[m], ov);
+          }
     }
     if (p.bias)
       for (int g = lane; g < G; g += 32) {

@@ -38,17 +38,26 @@ constexpr int kMinStages = 2;
 constexpr int kAuxSlots = 2 * kHelperWarps;                    // each helper owns two slots
 constexpr int kResBlock = 8;                                   // salient entries per residual block
 
-struct ChunkMeta {
+// Elements of a chunk's v*x at least 16 times larger than every other element (found in up to
+// kOutlierRounds rounds) are taken out of the fixed-point planes, up to kMaxOutliers of them, and
+// added exactly in fp32 (T * v*x per row, the code read from the staged tile).
+constexpr int kMaxOutliers = 16;
+constexpr int kOutlierRounds = 4;
+
+struct ChunkMeta {  // 128 bytes
   float scale4;      // q / 4, q the fixed-point quantum of v*x in this chunk (a power of two)
   int planes;        // byte planes of the chunk's fixed-point v*x: 3 (24-bit) or 2 (16-bit)
-  long long sum_x;   // sum of the chunk's fixed-point v*x values
-  long long pad[2];
+  long long sum_x;   // sum of the chunk's fixed-point v*x values (outliers excluded)
+  int n_out;         // outliers of the chunk (0 .. kMaxOutliers)
+  int pad[3];
+  uint16_t out_col[kMaxOutliers];  // their columns within the chunk
+  float out_val[kMaxOutliers];     // their v*x, exact
 };
 
 // Auxiliary slot: planes [32 words][48 bytes], metadata, residual sums [512 rows].
 constexpr int kAuxMeta = kPlaneBytesPerChunk;
 constexpr int kAuxRes = kAuxMeta + (int)sizeof(ChunkMeta);
-constexpr int kAuxBytes = kAuxRes + kTileRows * (int)sizeof(float);  // 3616
+constexpr int kAuxBytes = kAuxRes + kTileRows * (int)sizeof(float);  // 3712
 // Per helper: x at one residual block's 8 entries spread over the 4 positions of a group,
 // T[entry][position] = x * one-hot(position), so that an entry adds with 4 FMAs and no selects.
 constexpr int kOneHotBytes = kResBlock * 4 * 16;               // 512
