@@ -929,7 +929,7 @@ def main():
     ap.add_argument("--no-cpu-all-cores", action="store_true", help="skip the oracle timing on all host cores")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-per-shape", action="store_true")
-    ap.add_argument("--act-bits", type=int, choices=[16, 24], default=24,
+    ap.add_argument("--act-bits", type=int, choices=[16, 24], default=16,
                     help="activation precision of the timed region (24 = exact default, 16 = fast mode)")
     ap.add_argument("--profile-case", choices=["qwen3_14b_layer"], default=None,
                     help="run a small fixed workload for profilers instead of the benchmark")

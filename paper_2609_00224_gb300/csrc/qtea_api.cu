@@ -597,7 +597,7 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
   l->options = 0;
   l->row_bytes = format == QTEA_FMT_BASE3 ? l->K_pad / 128 * 26 : l->K_pad / 4;
   l->device = dev;
-  l->act_bits = 24;
+  l->act_bits = 16;
   l->sm_count = prop.multiProcessorCount;
   l->smem_optin = prop.sharedMemPerBlockOptin;
   l->smem_per_sm = prop.sharedMemPerMultiprocessor;
@@ -832,7 +832,7 @@ int qtea_gemv_m1_static(const uint16_t* x, const uint8_t* packed, int N, int K, 
   l.device = dev;
   l.sm_count = d.sm_count;
   l.smem_optin = d.smem_optin;
-  l.act_bits = 24;
+  l.act_bits = 16;
   l.n_tiles = (N + kTileRows - 1) / kTileRows;
   l.n_chunks = (l.K_pad + kChunkCols - 1) / kChunkCols;
   l.workspace = reinterpret_cast<float*>(d.scratch);

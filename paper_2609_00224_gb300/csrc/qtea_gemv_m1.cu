@@ -126,62 +126,74 @@ __device__ __forceinline__ void issue_unit(const CUtensorMap* map, int t, int ch
 
 // ---------------------------------------------------------------- decode (consumers)
 
-// Accumulators of one row for one chunk: [plane][scale set]; scale set 0 holds codes of
-// column groups 0 and 2 (weight 1), set 1 codes of groups 1 and 3 (weight 4).
+// Accumulators of one row for one chunk: [plane][column group]. A code word masked with
+// 0x03030303 << 2k holds the codes of column group k in its byte lanes, scaled by 4^k (no shift).
 template <int P>
 struct RowAcc {
-  int a[P][2];
+  int a[P][4];
 };
 
+// dp4a of unsigned code bytes with a signed plane (the top byte plane of X).
+__device__ __forceinline__ int dp4a_us(uint32_t a, uint32_t b, int c) {
+  int d;
+  asm("dp4a.u32.s32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+
 // One 32-bit word = 16 codes of one row. Plane registers of the word, in the order
-// [group k][plane q] (k = columns {k, 4+k, 8+k, 12+k} in byte lanes 0..3): for P = 3,
+// [group k][plane q] (group k = columns {k, 4+k, 8+k, 12+k} in byte lanes 0..3): for P = 3,
 // P0 = {g0p0, g0p1, g0p2, g1p0}, P1 = {g1p1, g1p2, g2p0, g2p1}, P2 = {g2p2, g3p0, g3p1, g3p2};
 // for P = 2, P0 = {g0p0, g0p1, g1p0, g1p1}, P1 = {g2p0, g2p1, g3p0, g3p1}. The top plane is
 // signed, the others unsigned.
 __device__ __forceinline__ void decode_word3(uint32_t w, const uint4& P0, const uint4& P1, const uint4& P2,
                                              RowAcc<3>& r) {
-  const uint32_t w4 = w >> 4;
-  const uint32_t g0 = w & 0x03030303u;   // columns 0,4,8,12 -> byte lanes, values 0..2
-  const uint32_t g1 = w & 0x0C0C0C0Cu;   // columns 1,5,9,13, values 0,4,8
-  const uint32_t g2 = w4 & 0x03030303u;  // columns 2,6,10,14
-  const uint32_t g3 = w4 & 0x0C0C0C0Cu;  // columns 3,7,11,15
+  const uint32_t g0 = w & 0x03030303u;  // columns 0,4,8,12 -> byte lanes, values c
+  const uint32_t g1 = w & 0x0C0C0C0Cu;  // columns 1,5,9,13, values 4c
+  const uint32_t g2 = w & 0x30303030u;  // columns 2,6,10,14, values 16c
+  const uint32_t g3 = w & 0xC0C0C0C0u;  // columns 3,7,11,15, values 64c
   r.a[0][0] = (int)__dp4a(g0, P0.x, (unsigned)r.a[0][0]);
   r.a[1][0] = (int)__dp4a(g0, P0.y, (unsigned)r.a[1][0]);
-  r.a[2][0] = __dp4a((int)g0, (int)P0.z, r.a[2][0]);
+  r.a[2][0] = dp4a_us(g0, P0.z, r.a[2][0]);
   r.a[0][1] = (int)__dp4a(g1, P0.w, (unsigned)r.a[0][1]);
   r.a[1][1] = (int)__dp4a(g1, P1.x, (unsigned)r.a[1][1]);
-  r.a[2][1] = __dp4a((int)g1, (int)P1.y, r.a[2][1]);
-  r.a[0][0] = (int)__dp4a(g2, P1.z, (unsigned)r.a[0][0]);
-  r.a[1][0] = (int)__dp4a(g2, P1.w, (unsigned)r.a[1][0]);
-  r.a[2][0] = __dp4a((int)g2, (int)P2.x, r.a[2][0]);
-  r.a[0][1] = (int)__dp4a(g3, P2.y, (unsigned)r.a[0][1]);
-  r.a[1][1] = (int)__dp4a(g3, P2.z, (unsigned)r.a[1][1]);
-  r.a[2][1] = __dp4a((int)g3, (int)P2.w, r.a[2][1]);
+  r.a[2][1] = dp4a_us(g1, P1.y, r.a[2][1]);
+  r.a[0][2] = (int)__dp4a(g2, P1.z, (unsigned)r.a[0][2]);
+  r.a[1][2] = (int)__dp4a(g2, P1.w, (unsigned)r.a[1][2]);
+  r.a[2][2] = dp4a_us(g2, P2.x, r.a[2][2]);
+  r.a[0][3] = (int)__dp4a(g3, P2.y, (unsigned)r.a[0][3]);
+  r.a[1][3] = (int)__dp4a(g3, P2.z, (unsigned)r.a[1][3]);
+  r.a[2][3] = dp4a_us(g3, P2.w, r.a[2][3]);
 }
 
 __device__ __forceinline__ void decode_word2(uint32_t w, const uint4& P0, const uint4& P1, RowAcc<2>& r) {
-  const uint32_t w4 = w >> 4;
   const uint32_t g0 = w & 0x03030303u;
   const uint32_t g1 = w & 0x0C0C0C0Cu;
-  const uint32_t g2 = w4 & 0x03030303u;
-  const uint32_t g3 = w4 & 0x0C0C0C0Cu;
+  const uint32_t g2 = w & 0x30303030u;
+  const uint32_t g3 = w & 0xC0C0C0C0u;
   r.a[0][0] = (int)__dp4a(g0, P0.x, (unsigned)r.a[0][0]);
-  r.a[1][0] = __dp4a((int)g0, (int)P0.y, r.a[1][0]);
+  r.a[1][0] = dp4a_us(g0, P0.y, r.a[1][0]);
   r.a[0][1] = (int)__dp4a(g1, P0.z, (unsigned)r.a[0][1]);
-  r.a[1][1] = __dp4a((int)g1, (int)P0.w, r.a[1][1]);
-  r.a[0][0] = (int)__dp4a(g2, P1.x, (unsigned)r.a[0][0]);
-  r.a[1][0] = __dp4a((int)g2, (int)P1.y, r.a[1][0]);
-  r.a[0][1] = (int)__dp4a(g3, P1.z, (unsigned)r.a[0][1]);
-  r.a[1][1] = __dp4a((int)g3, (int)P1.w, r.a[1][1]);
+  r.a[1][1] = dp4a_us(g1, P0.w, r.a[1][1]);
+  r.a[0][2] = (int)__dp4a(g2, P1.x, (unsigned)r.a[0][2]);
+  r.a[1][2] = dp4a_us(g2, P1.y, r.a[1][2]);
+  r.a[0][3] = (int)__dp4a(g3, P1.z, (unsigned)r.a[0][3]);
+  r.a[1][3] = dp4a_us(g3, P1.w, r.a[1][3]);
 }
 
-// 4 * sum_j (c_j - 1) X_j over the chunk, exact, as int64.
+// sum_j c_j X_j of plane q: group k's accumulator is 4^k times its share, exactly divisible.
 template <int P>
-__device__ __forceinline__ long long finish_chunk(const RowAcc<P>& r, long long sum_x) {
-  long long v = 0;
-#pragma unroll
-  for (int q = 0; q < P; ++q) v += (4ll * r.a[q][0] + r.a[q][1]) * (1ll << (8 * q));
-  return v - 4ll * sum_x;
+__device__ __forceinline__ int plane_sum(const RowAcc<P>& r, int q) {
+  return r.a[q][0] + (r.a[q][1] >> 2) + (r.a[q][2] >> 4) + (r.a[q][3] >> 6);
+}
+
+// sum_j (c_j - 1) X_j over the chunk, exact: in int32 with two planes (|sum| < 2^25), in int64
+// with three.
+__device__ __forceinline__ float finish_chunk2(const RowAcc<2>& r, int sum_x) {
+  return (float)(plane_sum<2>(r, 0) + (plane_sum<2>(r, 1) << 8) - sum_x);
+}
+__device__ __forceinline__ float finish_chunk3(const RowAcc<3>& r, long long sum_x) {
+  return (float)((long long)plane_sum<3>(r, 0) + ((long long)plane_sum<3>(r, 1) << 8) +
+                 ((long long)plane_sum<3>(r, 2) << 16) - sum_x);
 }
 
 // Decode one unit (two rows per lane, 32 words each) against the chunk's P byte planes.
@@ -192,7 +204,9 @@ __device__ __forceinline__ void decode_unit(const uint4* row0, const uint4* row1
                                             RowAcc<P>& a0, RowAcc<P>& a1) {
   constexpr int kW = (P == 3) ? 3 : 2;  // uint4 of planes per word (stride 3 in the slot)
 #pragma unroll
-  for (int k = 0; k < P; ++k) { a0.a[k][0] = a0.a[k][1] = 0; a1.a[k][0] = a1.a[k][1] = 0; }
+  for (int k = 0; k < P; ++k)
+#pragma unroll
+    for (int g = 0; g < 4; ++g) a0.a[k][g] = a1.a[k][g] = 0;
   uint4 P0 = pl[0], P1 = pl[1], P2 = kW == 3 ? pl[2] : make_uint4(0, 0, 0, 0);
   uint4 c0 = row0[0 ^ sw], c1 = row1[0 ^ sw];
 #pragma unroll 2  // two chunks per iteration: the code and plane registers alternate without copies
@@ -365,7 +379,7 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
 #pragma unroll
   for (int o = 16; o; o >>= 1) sx += __shfl_xor_sync(0xffffffffu, sx, o);
   if (lane == 0) {
-    meta->scale4 = __uint_as_float((uint32_t)(127 + e - qsh - 2) << 23);  // q / 4
+    meta->scale = __uint_as_float((uint32_t)(127 + e - qsh) << 23);  // q
     meta->planes = two ? 2 : 3;
     meta->sum_x = sx;
     meta->n_out = n_out;
@@ -541,6 +555,23 @@ __device__ __noinline__ void helper_role(const Ring r, int u0, int n_units, int 
   }
 }
 
+// Residual sums of the auxiliary slot: wait until the helper has written them, add the lane's two
+// rows, release the slot.
+__device__ __forceinline__ bool take_residual(const Ring& r, int slot, uint32_t parity, int ra, int lane,
+                                              float& racc0, float& racc1, int* status) {
+  const bool ok = mbar_wait(smem_u32(&r.full_a[slot]), parity, status);
+  if (!__all_sync(0xffffffffu, ok)) return false;
+  const float* res = reinterpret_cast<const float*>(r.aux + (size_t)slot * kAuxBytes + kAuxRes);
+  racc0 += res[ra];
+  racc1 += res[ra + 32];
+  __syncwarp();
+  if (lane == 0) mbar_arrive(smem_u32(&r.empty_a[slot]));
+  return true;
+}
+
+// The consumers take the units in order. A unit's residual sums are added one unit later (or at
+// the tile's end), so the helpers' residual work is not waited for right after each decode; the
+// sums are still added in unit order, so results stay bitwise reproducible.
 __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, long long total, int u0, int u1,
                                            int warp, int lane, int* status) {
   const int n_units = u1 - u0;
@@ -551,10 +582,13 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
   uint16_t al0 = 0, al1 = 0;  // raw fp16 bits: converted at the tile's end, so no wait on the load here
   bool need_alpha = true;
   UnitPos c = unit_pos(r.tab, r.n_problems, u0);
+  int st = 0, slot = 0;             // code stage and auxiliary slot of unit i
+  uint32_t ph_c = 0, ph_a = 0;      // parity of their current fill
+  int pend = -1;                    // auxiliary slot whose residual sums are still to be added
+  uint32_t pend_ph = 0;
 
   for (int i = 0; i < n_units; ++i) {
     const int u = u0 + i;
-    const int st = i % r.S, slot = i % kAuxSlots;
     const ProblemArgs& a = r.tab[c.p];
     const int n_chunks = a.n_chunks, N = a.N;
     const int row0g = c.t * kTileRows + ra, row1g = row0g + 32;
@@ -563,30 +597,30 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
       al1 = row1g < N ? __ldg(a.alpha + row1g) : (uint16_t)0;
       need_alpha = false;
     }
-    bool ok = mbar_wait(smem_u32(&r.full_c[st]), (uint32_t)((i / r.S) & 1), status);
-    ok = ok && mbar_wait(smem_u32(&r.planes_a[slot]), (uint32_t)((i / kAuxSlots) & 1), status);
+    bool ok = mbar_wait(smem_u32(&r.full_c[st]), ph_c, status);
+    ok = ok && mbar_wait(smem_u32(&r.planes_a[slot]), ph_a, status);
     if (!__all_sync(0xffffffffu, ok)) break;
 
     const uint8_t* ax = r.aux + (size_t)slot * kAuxBytes;
     const ChunkMeta* mp = reinterpret_cast<const ChunkMeta*>(ax + kAuxMeta);
-    const float scale4 = mp->scale4;
+    const float scale = mp->scale;
     const int planes = mp->planes, n_out = mp->n_out;
     const long long sum_x = mp->sum_x;
     const uint4* row0 =
         reinterpret_cast<const uint4*>(r.codes + (size_t)st * kStageBytes + (size_t)ra * kChunkRowBytes);
     const uint4* row1 = row0 + 32 * (kChunkRowBytes / 16);
     const uint4* pl = reinterpret_cast<const uint4*>(ax);
-    long long d0, d1;
+    float d0, d1;
     if (planes == 2) {
       RowAcc<2> a0, a1;
       decode_unit<2>(row0, row1, pl, sw, a0, a1);
-      d0 = finish_chunk<2>(a0, sum_x);
-      d1 = finish_chunk<2>(a1, sum_x);
+      d0 = finish_chunk2(a0, (int)sum_x);
+      d1 = finish_chunk2(a1, (int)sum_x);
     } else {
       RowAcc<3> a0, a1;
       decode_unit<3>(row0, row1, pl, sw, a0, a1);
-      d0 = finish_chunk<3>(a0, sum_x);
-      d1 = finish_chunk<3>(a1, sum_x);
+      d0 = finish_chunk3(a0, sum_x);
+      d1 = finish_chunk3(a1, sum_x);
     }
     // outliers: T * v*x in fp32, the code of both rows read from the staged tile (byte col / 4 of
     // the row, in 16-byte granule (col / 64) ^ (row % 8) of the 128-byte swizzle; rows ra and ra + 32
@@ -604,21 +638,23 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
         o1 = fmaf((float)(int)((cb1[off] >> sh) & 3u) - 1.f, xv, o1);
       }
     }
-    ok = mbar_wait(smem_u32(&r.full_a[slot]), (uint32_t)((i / kAuxSlots) & 1), status);
-    if (!__all_sync(0xffffffffu, ok)) break;
-    const float* res = reinterpret_cast<const float*>(ax + kAuxRes);
-    racc0 += res[ra];
-    racc1 += res[ra + 32];
     __syncwarp();
-    if (lane == 0) {  // release the code stage and the auxiliary slot
-      mbar_arrive(smem_u32(&r.empty_c[st]));
-      mbar_arrive(smem_u32(&r.empty_a[slot]));
-    }
-    yacc0 += fmaf((float)d0, scale4, o0);
-    yacc1 += fmaf((float)d1, scale4, o1);
+    if (lane == 0) mbar_arrive(smem_u32(&r.empty_c[st]));  // codes and metadata no longer read
+    yacc0 += fmaf(d0, scale, o0);
+    yacc1 += fmaf(d1, scale, o1);
 
-    // ---- tile epilogue once this CTA's part of tile t is done
-    if (c.ch == n_chunks - 1 || u == u1 - 1) {
+    // residual sums: the previous unit's now, this unit's at the tile's end or with the next unit
+    if (pend >= 0) {
+      if (!take_residual(r, pend, pend_ph, ra, lane, racc0, racc1, status)) break;
+      pend = -1;
+    }
+    const bool tile_end = c.ch == n_chunks - 1 || u == u1 - 1;
+    if (!tile_end) {
+      pend = slot;
+      pend_ph = ph_a;
+    } else {
+      if (!take_residual(r, slot, ph_a, ra, lane, racc0, racc1, status)) break;
+      // ---- tile epilogue: this CTA's part of tile t is done
       const int t = c.t;
       const long long A = a.unit_begin + (long long)t * n_chunks, B = A + n_chunks;
       const float val0 = h2f(al0) * yacc0 + racc0;
@@ -664,6 +700,14 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
       }
       yacc0 = yacc1 = racc0 = racc1 = 0.f;
       need_alpha = true;
+    }
+    if (++st == r.S) {
+      st = 0;
+      ph_c ^= 1u;
+    }
+    if (++slot == kAuxSlots) {
+      slot = 0;
+      ph_a ^= 1u;
     }
     if (++c.ch == n_chunks) {
       c.ch = 0;

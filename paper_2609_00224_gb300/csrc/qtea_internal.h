@@ -45,7 +45,7 @@ constexpr int kMaxOutliers = 16;
 constexpr int kOutlierRounds = 4;
 
 struct ChunkMeta {  // 128 bytes
-  float scale4;      // q / 4, q the fixed-point quantum of v*x in this chunk (a power of two)
+  float scale;       // q, the fixed-point quantum of v*x in this chunk (a power of two)
   int planes;        // byte planes of the chunk's fixed-point v*x: 3 (24-bit) or 2 (16-bit)
   long long sum_x;   // sum of the chunk's fixed-point v*x values (outliers excluded)
   int n_out;         // outliers of the chunk (0 .. kMaxOutliers)
