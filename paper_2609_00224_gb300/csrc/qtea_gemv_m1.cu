@@ -265,10 +265,10 @@ __device__ __forceinline__ void load_chunk(const ProblemArgs& a, int ch, int lan
   }
 }
 
+// Largest of the lanes' non-negative values: their bit patterns order as unsigned integers, so one
+// warp reduction instruction serves.
 __device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
+  return __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(v)));
 }
 
 // The chunk's v*x as fixed point: byte planes of this lane's word, and the metadata.
@@ -339,7 +339,7 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
   const int xmax = two ? 32767 : 8388607;  // a value of amax rounds to at most 2^(qsh+1): clamp
   const float inv_q = __uint_as_float((uint32_t)(127 + qsh - e) << 23);
   int X[16];
-  long long sx = 0;
+  int sx = 0;  // |sx| < 16 * 2^23 per lane
 #pragma unroll
   for (int i = 0; i < 16; ++i) {
     X[i] = ((outm >> i) & 1u) ? 0 : min(__float2int_rn(xt[i] * inv_q), xmax);
@@ -376,12 +376,14 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
     dst[1] = make_uint4(reg[4], reg[5], reg[6], reg[7]);
     dst[2] = make_uint4(reg[8], reg[9], reg[10], reg[11]);
   }
-#pragma unroll
-  for (int o = 16; o; o >>= 1) sx += __shfl_xor_sync(0xffffffffu, sx, o);
+  // the chunk's sum of X, exact: the lanes' sums split into 16-bit halves, each summed by one warp
+  // reduction instruction (|sum| < 2^32 in 24-bit mode)
+  const unsigned s_lo = __reduce_add_sync(0xffffffffu, (unsigned)sx & 0xFFFFu);
+  const int s_hi = (int)__reduce_add_sync(0xffffffffu, (unsigned)(sx >> 16));
   if (lane == 0) {
     meta->scale = __uint_as_float((uint32_t)(127 + e - qsh) << 23);  // q
     meta->planes = two ? 2 : 3;
-    meta->sum_x = sx;
+    meta->sum_x = (long long)s_hi * 65536 + (long long)s_lo;
     meta->n_out = n_out;
   }
 }
@@ -436,9 +438,9 @@ __device__ __forceinline__ void load_block(const ProblemArgs& a, int q, int b, u
 
 // Stage unit (t, ch) of problem *pa into auxiliary slot ax. First the planes and metadata, which
 // need x and v only, then (after the arrival on planes_bar) the residual sums of the tile's 512
-// rows over the unit's salient blocks: the consumers wait for those only after the decode. The
-// residual loads go out after the planes are published, so they never delay them (a unit's first
-// planes are on the critical path of the launch). Lane owns residual groups lane + 32k.
+// rows over the unit's salient blocks: the consumers add those one unit later. The residual loads
+// go out after the planes are published: issued earlier, they queue in front of the x and v loads
+// behind the code stream and delay the planes. Lane owns residual groups lane + 32k.
 __device__ __noinline__ void stage_unit(const ProblemArgs* pa, int t, int ch, uint8_t* ax, int lane,
                                         uint32_t planes_bar, float4* onehot) {
   const ProblemArgs a = *pa;
@@ -592,9 +594,9 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
     const ProblemArgs& a = r.tab[c.p];
     const int n_chunks = a.n_chunks, N = a.N;
     const int row0g = c.t * kTileRows + ra, row1g = row0g + 32;
-    if (need_alpha) {  // used at the tile's end; the loads complete during the decode
-      al0 = row0g < N ? __ldg(a.alpha + row0g) : (uint16_t)0;
-      al1 = row1g < N ? __ldg(a.alpha + row1g) : (uint16_t)0;
+    if (need_alpha) {  // used at the tile's end: unconditional loads (rows clamped), so nothing waits here
+      al0 = __ldg(a.alpha + min(row0g, N - 1));
+      al1 = __ldg(a.alpha + min(row1g, N - 1));
       need_alpha = false;
     }
     bool ok = mbar_wait(smem_u32(&r.full_c[st]), ph_c, status);
