@@ -557,51 +557,111 @@ __device__ __noinline__ void helper_role(const Ring r, int u0, int n_units, int 
   }
 }
 
-// Residual sums of the auxiliary slot: wait until the helper has written them, add the lane's two
-// rows, release the slot.
+// Residual sums of the auxiliary slot: wait until the helper has written them, return the lane's
+// two rows, release the slot.
 __device__ __forceinline__ bool take_residual(const Ring& r, int slot, uint32_t parity, int ra, int lane,
-                                              float& racc0, float& racc1, int* status) {
+                                              float& res0, float& res1, int* status) {
   const bool ok = mbar_wait(smem_u32(&r.full_a[slot]), parity, status);
   if (!__all_sync(0xffffffffu, ok)) return false;
   const float* res = reinterpret_cast<const float*>(r.aux + (size_t)slot * kAuxBytes + kAuxRes);
-  racc0 += res[ra];
-  racc1 += res[ra + 32];
+  res0 = res[ra];
+  res1 = res[ra + 32];
   __syncwarp();
   if (lane == 0) mbar_arrive(smem_u32(&r.empty_a[slot]));
   return true;
 }
 
-// The consumers take the units in order. A unit's residual sums are added one unit later (or at
-// the tile's end), so the helpers' residual work is not waited for right after each decode; the
-// sums are still added in unit order, so results stay bitwise reproducible.
+// A tile whose last unit this CTA has decoded: its lane rows' ternary sums, residual sums so far and
+// alpha bits, held until the residual of that last unit is in.
+struct DoneTile {
+  float y0, y1, r0, r1;
+  uint16_t al0, al1;
+  int p, t;
+};
+
+// Write the tile's rows: directly when this CTA holds all of the tile's units, else through the
+// split-tile workspace, the last of the tile's contributors summing all parts in CTA order.
+__device__ __forceinline__ void tile_epilogue(const ProblemArgs& a, const DoneTile& d, const int* cta_u0,
+                                              long long total, int u0, int u1, int warp, int lane, int ra) {
+  const int N = a.N, t = d.t;
+  const int row0g = t * kTileRows + ra, row1g = row0g + 32;
+  const float val0 = h2f(d.al0) * d.y0 + d.r0;
+  const float val1 = h2f(d.al1) * d.y1 + d.r1;
+  const long long A = a.unit_begin + (long long)t * a.n_chunks, B = A + a.n_chunks;
+  float* y = a.y;
+  if (A >= u0 && B <= u1) {
+    if (row0g < N) y[row0g] = val0;
+    if (row1g < N) y[row1g] = val1;
+    return;
+  }
+  // partial tile: publish this warp's 64 rows, then the last of the tile's contributors (per warp:
+  // counter t * kConsumerWarps + warp) sums all partials in CTA order. Slot 0 of a CTA holds the
+  // tile its range starts in, slot 1 the tile its range ends in.
+  const int grid = gridDim.x;
+  float* ws = a.ws;
+  const int my_slot = (u0 >= A) ? 0 : 1;
+  float* wsp = ws + ((size_t)blockIdx.x * 2 + my_slot) * kTileRows;
+  wsp[ra] = val0;
+  wsp[ra + 32] = val1;
+  __syncwarp();
+  const int bf = unit_owner(A, total, grid), bl = unit_owner(B - 1, total, grid);
+  int last = 0;
+  if (lane == 0) {
+    // acq_rel at gpu scope: the warp's partials (ordered before by __syncwarp) are published with
+    // the increment, and the last arriver sees every other contributor's partials
+    unsigned* ctr = a.counters + (size_t)t * kConsumerWarps + warp;
+    unsigned prev;
+    asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], 1;" : "=r"(prev) : "l"(ctr) : "memory");
+    last = (prev == (unsigned)(bl - bf));  // every CTA in [bf, bl] holds units of this tile
+    if (last) *ctr = 0u;                   // self-reset for the next call
+  }
+  last = __shfl_sync(0xffffffffu, last, 0);
+  __syncwarp();
+  if (last) {
+    float s0 = 0.f, s1 = 0.f;
+    for (int cb = bf; cb <= bl; ++cb) {
+      const int cslot = (cta_u0[cb] >= A) ? 0 : 1;
+      const float* src = ws + ((size_t)cb * 2 + cslot) * kTileRows;
+      s0 += __ldcg(src + ra);
+      s1 += __ldcg(src + ra + 32);
+    }
+    if (row0g < N) y[row0g] = s0;
+    if (row1g < N) y[row1g] = s1;
+  }
+}
+
+// The consumers take the units in order. A unit's residual sums, and for the last unit of a tile
+// the tile's epilogue, wait until the next unit has been decoded, so the helpers' residual work is
+// not waited for right after each decode; the sums are still added in unit order, so results stay
+// bitwise reproducible.
 __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, long long total, int u0, int u1,
                                            int warp, int lane, int* status) {
   const int n_units = u1 - u0;
   const int ra = warp * 64 + lane;  // tile rows owned by this lane: ra and ra + 32
   const int sw = lane & 7;          // 128-byte swizzle phase of both rows
-  const int grid = gridDim.x;
   float yacc0 = 0.f, yacc1 = 0.f, racc0 = 0.f, racc1 = 0.f;
   uint16_t al0 = 0, al1 = 0;  // raw fp16 bits: converted at the tile's end, so no wait on the load here
   bool need_alpha = true;
   UnitPos c = unit_pos(r.tab, r.n_problems, u0);
   int st = 0, slot = 0;             // code stage and auxiliary slot of unit i
   uint32_t ph_c = 0, ph_a = 0;      // parity of their current fill
-  int pend = -1;                    // auxiliary slot whose residual sums are still to be added
+  int pend = -1;                    // auxiliary slot of the previous unit (residual not yet added)
   uint32_t pend_ph = 0;
+  bool done = false;                // the previous unit ended a tile: its epilogue is pending
+  DoneTile dt;
 
   for (int i = 0; i < n_units; ++i) {
     const int u = u0 + i;
     const ProblemArgs& a = r.tab[c.p];
     const int n_chunks = a.n_chunks, N = a.N;
-    const int row0g = c.t * kTileRows + ra, row1g = row0g + 32;
     if (need_alpha) {  // used at the tile's end: unconditional loads (rows clamped), so nothing waits here
-      al0 = __ldg(a.alpha + min(row0g, N - 1));
-      al1 = __ldg(a.alpha + min(row1g, N - 1));
+      al0 = __ldg(a.alpha + min(c.t * kTileRows + ra, N - 1));
+      al1 = __ldg(a.alpha + min(c.t * kTileRows + ra + 32, N - 1));
       need_alpha = false;
     }
     bool ok = mbar_wait(smem_u32(&r.full_c[st]), ph_c, status);
     ok = ok && mbar_wait(smem_u32(&r.planes_a[slot]), ph_a, status);
-    if (!__all_sync(0xffffffffu, ok)) break;
+    if (!__all_sync(0xffffffffu, ok)) return;
 
     const uint8_t* ax = r.aux + (size_t)slot * kAuxBytes;
     const ChunkMeta* mp = reinterpret_cast<const ChunkMeta*>(ax + kAuxMeta);
@@ -645,61 +705,32 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
     yacc0 += fmaf(d0, scale, o0);
     yacc1 += fmaf(d1, scale, o1);
 
-    // residual sums: the previous unit's now, this unit's at the tile's end or with the next unit
+    // the previous unit's residual sums (into the tile they belong to), then its tile's epilogue
     if (pend >= 0) {
-      if (!take_residual(r, pend, pend_ph, ra, lane, racc0, racc1, status)) break;
-      pend = -1;
-    }
-    const bool tile_end = c.ch == n_chunks - 1 || u == u1 - 1;
-    if (!tile_end) {
-      pend = slot;
-      pend_ph = ph_a;
-    } else {
-      if (!take_residual(r, slot, ph_a, ra, lane, racc0, racc1, status)) break;
-      // ---- tile epilogue: this CTA's part of tile t is done
-      const int t = c.t;
-      const long long A = a.unit_begin + (long long)t * n_chunks, B = A + n_chunks;
-      const float val0 = h2f(al0) * yacc0 + racc0;
-      const float val1 = h2f(al1) * yacc1 + racc1;
-      float* y = a.y;
-      if (A >= u0 && B <= u1) {
-        if (row0g < N) y[row0g] = val0;
-        if (row1g < N) y[row1g] = val1;
+      float q0, q1;
+      if (!take_residual(r, pend, pend_ph, ra, lane, q0, q1, status)) return;
+      if (done) {
+        dt.r0 += q0;
+        dt.r1 += q1;
+        tile_epilogue(r.tab[dt.p], dt, cta_u0, total, u0, u1, warp, lane, ra);
+        done = false;
       } else {
-        // partial tile: publish this warp's 64 rows, then the last of the tile's contributors
-        // (per warp: counter t * kConsumerWarps + warp) sums all partials in CTA order. Slot 0
-        // of a CTA holds the tile its range starts in, slot 1 the tile its range ends in.
-        float* ws = a.ws;
-        const int my_slot = (u0 >= A) ? 0 : 1;
-        float* wsp = ws + ((size_t)blockIdx.x * 2 + my_slot) * kTileRows;
-        wsp[ra] = val0;
-        wsp[ra + 32] = val1;
-        __syncwarp();
-        const int bf = unit_owner(A, total, grid), bl = unit_owner(B - 1, total, grid);
-        int last = 0;
-        if (lane == 0) {
-          // acq_rel at gpu scope: the warp's partials (ordered before by __syncwarp) are published
-          // with the increment, and the last arriver sees every other contributor's partials
-          unsigned* ctr = a.counters + (size_t)t * kConsumerWarps + warp;
-          unsigned prev;
-          asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], 1;" : "=r"(prev) : "l"(ctr) : "memory");
-          last = (prev == (unsigned)(bl - bf));  // every CTA in [bf, bl] holds units of this tile
-          if (last) *ctr = 0u;                   // self-reset for the next call
-        }
-        last = __shfl_sync(0xffffffffu, last, 0);
-        __syncwarp();
-        if (last) {
-          float s0 = 0.f, s1 = 0.f;
-          for (int cb = bf; cb <= bl; ++cb) {
-            const int cslot = (cta_u0[cb] >= A) ? 0 : 1;
-            const float* src = ws + ((size_t)cb * 2 + cslot) * kTileRows;
-            s0 += __ldcg(src + ra);
-            s1 += __ldcg(src + ra + 32);
-          }
-          if (row0g < N) y[row0g] = s0;
-          if (row1g < N) y[row1g] = s1;
-        }
+        racc0 += q0;
+        racc1 += q1;
       }
+    }
+    pend = slot;
+    pend_ph = ph_a;
+    if (c.ch == n_chunks - 1 || u == u1 - 1) {  // this CTA's part of tile c.t is decoded
+      dt.y0 = yacc0;
+      dt.y1 = yacc1;
+      dt.r0 = racc0;
+      dt.r1 = racc1;
+      dt.al0 = al0;
+      dt.al1 = al1;
+      dt.p = c.p;
+      dt.t = c.t;
+      done = true;
       yacc0 = yacc1 = racc0 = racc1 = 0.f;
       need_alpha = true;
     }
@@ -717,6 +748,16 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
         c.t = 0;
         ++c.p;
       }
+    }
+  }
+  // the last unit always ends a tile
+  if (pend >= 0) {
+    float q0, q1;
+    if (!take_residual(r, pend, pend_ph, ra, lane, q0, q1, status)) return;
+    if (done) {
+      dt.r0 += q0;
+      dt.r1 += q1;
+      tile_epilogue(r.tab[dt.p], dt, cta_u0, total, u0, u1, warp, lane, ra);
     }
   }
 }
