@@ -47,7 +47,9 @@ typedef enum qtea_status {
   QTEA_ERR_CUDA = 4,        /* a CUDA runtime error (no device, launch failure, ...) */
   QTEA_ERR_ALLOC = 5,       /* device memory allocation failed */
   QTEA_ERR_TIMEOUT = 6,     /* a bounded wait inside a kernel gave up (see qtea_device_status) */
-  QTEA_ERR_SCRATCH_LIMIT = 7 /* larger than the static scratch of qtea_gemv_m1_static allows */
+  QTEA_ERR_SCRATCH_LIMIT = 7, /* larger than the static scratch of qtea_gemv_m1_static allows */
+  QTEA_ERR_STATE = 8          /* the static scratch of qtea_gemv_m1_static is not in its start state
+                                 (see qtea_gemv_m1_static_status) */
 } qtea_status;
 
 typedef enum qtea_format {
@@ -128,15 +130,16 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
  * call (qtea_gemv_grouped) is reproducible for the same group, but its rounding may differ
  * from separate calls because the split of work over the CTAs differs.
  * Numerics: at M = 1 (the library's own storage) the ternary sum is accumulated exactly in
- * integers over 512-column blocks, with v*x represented in fixed point relative to the block's
- * largest |v*x| (24-bit unless qtea_set_activation_precision selects 16-bit); block sums, alpha
- * and the residual are combined in fp32. At 2 <= M <= 16, and for 2-bit layouts in the paper's
+ * integers over 512-column blocks, with v*x represented in 16-bit or 24-bit fixed point relative
+ * to the block's largest |v*x| after its massive values are taken out and added exactly in fp32
+ * (qtea_set_activation_precision); block sums, alpha and the residual are combined in fp32. At 2 <= M <= 16, and for 2-bit layouts in the paper's
  * storage at any M, the tensor cores take 2T*v and x in fp16 (both exact, which needs |v| < 32768)
  * with exact fp32 products and fp32 sums; alpha, beta and the residual are applied in fp32.
  * Base-3 layouts at M <= 4 (when v*x of the call fits in shared memory): the ternary sum is
  * accumulated exactly in integers over 128-column blocks, with v*x in fixed point relative to the
- * block's largest |v*x| (|X| < 2^22); block sums, alpha, beta and the residual are combined in
- * fp32. Other layouts and batch sizes: fp32 throughout.
+ * block's largest |v*x| (|X| < 2^23) after up to 3 massive values per block are taken out and
+ * added exactly in fp32; block sums, alpha, beta and the residual are combined in fp32. Other
+ * layouts and batch sizes: fp32 throughout.
  */
 int qtea_gemv(const uint16_t* x, const qtea_layout* packed_ternary, const uint16_t* row_scale,
               const uint16_t* col_scale, const int32_t* salient_idx, const uint16_t* residual_vals,
@@ -225,11 +228,14 @@ int qtea_layout_copy_packed(const qtea_layout* layout, void* dst, size_t bytes, 
 /*
  * Activation precision of batch-1 (M = 1) calls on this layout. The ternary sum is always
  * accumulated exactly in integers over 512-column blocks; what changes is how finely v*x is
- * represented in fixed point relative to the block's largest |v*x|:
- *   bits = 24 (default): 24-bit, three byte planes per column.
- *   bits = 16: 16-bit (two byte planes, a third fewer dot-product instructions per weight)
- *              for every block whose largest |v*x| is at most 8 times the block's root mean
- *              square; blocks with outliers, and layouts with K < 1024, keep 24 bits.
+ * represented in fixed point. In each block, values at least 16 times larger than all the others
+ * (up to 16 of them, e.g. an LLM's massive activations) are taken out and added exactly in fp32;
+ * the rest are held relative to their largest magnitude:
+ *   bits = 16 (default): 16-bit (|X| < 2^15, two byte planes) for every block whose remaining
+ *              largest |v*x| is at most 8 times their root mean square; other blocks, and
+ *              layouts with K < 1024, use 24 bits.
+ *   bits = 24: 24-bit (|X| < 2^23, three byte planes, half again as many dot-product
+ *              instructions per weight) for every block.
  * Returns QTEA_ERR_INVALID_ARG for other values. Batch sizes M > 1 are not affected.
  */
 int qtea_set_activation_precision(qtea_layout* layout, int bits);
@@ -261,36 +267,53 @@ int qtea_device_status(const qtea_layout* layout, qtea_stream_t stream);
  * caller owns and takes its split-tile scratch from a fixed array in the library's static device
  * memory. It calls no cudaMalloc, cudaFree or other allocating routine.
  *
- * Computes, for M = 1, what qtea_gemv computes (Eq. 10 and Eq. 11, one alpha per row, beta = 0),
- * with the default 24-bit activation precision.
+ * Computes what qtea_gemv computes for M = 1 on a layout with one alpha per row, no beta and fp16
+ * residual values, with the default activation precision (qtea_set_activation_precision).
  *   x, row_scale, col_scale, salient_idx, residual_vals, residual_idx, y
  *                  as for qtea_gemv, with M = 1
  *   packed         device, 16-byte aligned, caller-owned: the 2-bit layout qtea_pack_layout
  *                  writes, N rows of K_pad/4 bytes (K_pad = K rounded up to a multiple of 64),
  *                  code T+1 four per byte, least significant first, pad columns code 1 (for
  *                  instance a copy made once with qtea_layout_copy_packed). Codes are not
- *                  validated: code 3 decodes as T = 2.
+ *                  validated: code 3 decodes as T = 2. The call's kernel reads them only after the
+ *                  preceding work on `stream` has completed, so a kernel that writes them just
+ *                  before the call on the same stream is seen.
  *   N, K, n_salient  sizes as for qtea_pack_layout (N % 4 == 0 when n_salient > 0)
  * Limits of the static scratch (663,808 bytes of device memory per device): N <= 131072 (at most
  * 256 tiles of 512 rows); a larger N returns QTEA_ERR_SCRATCH_LIMIT. At most 160 CTAs are used.
  * Set-up: the first call on each device, with that device current, looks the scratch up with
  * cudaGetSymbolAddress and sets the kernel's shared-memory attribute. Make that first call before
  * any stream capture on the device. Later calls encode a tensor map on the host and launch.
- * Start state: the split-tile counters in the scratch must be zero when a call starts. Static
- * device memory is zero when the library's module loads, and every completed call leaves the
- * counters at zero.
+ * Start state: the split-tile counters and the status word in the scratch must be zero when a call
+ * starts. Static device memory is zero when the library's module loads, and every completed call
+ * leaves them at zero. A call whose kernel gave up a bounded wait (QTEA_ERR_TIMEOUT) can leave
+ * counters set: qtea_gemv_m1_static_status reports that and restores the start state.
  * Concurrency: every call on a device shares the one scratch. Calls that may overlap on the
  * device (different streams without ordering, several host threads) race and give wrong results:
  * order them, e.g. on one stream.
- * A bounded wait that times out inside the kernel is recorded in the scratch's status word and is
- * not reported by this call (qtea_device_status reads layouts only).
  * Returns QTEA_OK, QTEA_ERR_INVALID_ARG, QTEA_ERR_SCRATCH_LIMIT, QTEA_ERR_UNSUPPORTED (device
- * ordinal >= 64) or QTEA_ERR_CUDA.
+ * ordinal >= 64) or QTEA_ERR_CUDA. A timeout inside the kernel is not reported by this call (it
+ * is asynchronous): qtea_gemv_m1_static_status reads it.
  */
 int qtea_gemv_m1_static(const uint16_t* x, const uint8_t* packed, int N, int K, int n_salient,
                         const uint16_t* row_scale, const uint16_t* col_scale, const int32_t* salient_idx,
                         const uint16_t* residual_vals, const uint8_t* residual_idx, float* y,
                         qtea_stream_t stream);
+
+/*
+ * State of the static scratch of qtea_gemv_m1_static on the current device (no counterpart in the
+ * paper; it serves the allocation-free entry point). Synchronizes `stream`, then reads the
+ * scratch's status word and split-tile counters:
+ *   QTEA_OK           both at zero: the start state every call needs;
+ *   QTEA_ERR_TIMEOUT  a kernel of an earlier call gave up a bounded wait (its y is unspecified);
+ *   QTEA_ERR_STATE    counters left set without a recorded timeout (e.g. calls that overlapped).
+ * With clear != 0, a non-OK state is reset to zero afterwards (cudaMemsetAsync on the static
+ * array, then a synchronization of `stream`), so the next call starts correctly. Order this call
+ * after the calls it inspects, e.g. on the same stream. It allocates nothing (the counters are
+ * copied to an 8 KB array on the calling thread's stack). Returns the state above, or
+ * QTEA_ERR_UNSUPPORTED (device ordinal >= 64) or QTEA_ERR_CUDA.
+ */
+int qtea_gemv_m1_static_status(int clear, qtea_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -22,6 +22,7 @@ QTEA_ERR_CUDA = 4
 QTEA_ERR_ALLOC = 5
 QTEA_ERR_TIMEOUT = 6
 QTEA_ERR_SCRATCH_LIMIT = 7
+QTEA_ERR_STATE = 8
 QTEA_FMT_2BIT = 0
 QTEA_FMT_BASE3 = 1
 QTEA_OPT_BIAS = 1
@@ -85,6 +86,8 @@ def load(build_if_missing: bool = True):
     lib.qtea_layout_copy_packed.argtypes = [P, P, ctypes.c_size_t, P]
     lib.qtea_gemv_m1_static.restype = i32
     lib.qtea_gemv_m1_static.argtypes = [P, P, i32, i32, i32, P, P, P, P, P, P, P]
+    lib.qtea_gemv_m1_static_status.restype = i32
+    lib.qtea_gemv_m1_static_status.argtypes = [i32, P]
     lib.qtea_quantize.restype = i32
     lib.qtea_quantize.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, P, P, P, P, P, P, P]
     _lib = lib

@@ -466,13 +466,15 @@ int group_launch(M1Group& g, cudaStream_t st) {
   return launch_m1(g.maps, g.gp, g.grid, g.smem, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
 }
 
-// Batch-1 dispatch: pack as many consecutive problems as fit into each launch.
-int run_m1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st) {
+// Batch-1 dispatch: pack as many consecutive problems as fit into each launch. caller_codes: the
+// packed codes belong to the caller, so the kernel reads them only after the grid dependency wait.
+int run_m1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st, bool caller_codes = false) {
   int i = 0;
   while (i < n) {
     const qtea_layout* l0 = qs[idx[i]].packed_ternary;
     M1Group g;
     group_reset(g);
+    g.gp.codes_after_wait = caller_codes ? 1 : 0;
     int taken = 0;
     while (i + taken < n) {
       M1Group trial = g;
@@ -564,6 +566,7 @@ const char* qtea_status_string(int status) {
     case QTEA_ERR_ALLOC: return "device allocation failed";
     case QTEA_ERR_TIMEOUT: return "bounded wait in a kernel timed out";
     case QTEA_ERR_SCRATCH_LIMIT: return "problem larger than the static scratch of qtea_gemv_m1_static";
+    case QTEA_ERR_STATE: return "static scratch of qtea_gemv_m1_static not in its start state (overlapping calls?)";
     default: return "unknown status";
   }
 }
@@ -861,8 +864,43 @@ int qtea_gemv_m1_static(const uint16_t* x, const uint8_t* packed, int N, int K, 
   rc = check_problem(q, 1);
   if (rc) return rc;
   const int idx0 = 0;
-  rc = l.m1_ok ? run_m1(&q, &idx0, 1, st) : launch_generic_problem(q, 1, st);
+  rc = l.m1_ok ? run_m1(&q, &idx0, 1, st, true) : launch_generic_problem(q, 1, st);
   if (rc != QTEA_OK) cudaGetLastError();
+  return rc;
+}
+
+int qtea_gemv_m1_static_status(int clear, qtea_stream_t stream) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= kStaticMaxDevices) return QTEA_ERR_UNSUPPORTED;
+  StaticDevice d;
+  int rc = static_setup(dev, &d);
+  if (rc) return rc;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  unsigned char* ctr = d.scratch + kStaticWsBytes;  // counters, then the status word
+  int* word = reinterpret_cast<int*>(d.scratch + kStaticWsBytes + kStaticCtrBytes);
+  // host copies on this thread's stack (8 KB of counters): no allocation
+  unsigned host_ctr[kStaticCtrBytes / sizeof(unsigned)];
+  int host_word = 0;
+  if (cudaMemcpyAsync(host_ctr, ctr, kStaticCtrBytes, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaMemcpyAsync(&host_word, word, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_ERR_CUDA;
+  }
+  bool dirty = false;
+  for (size_t k = 0; k < kStaticCtrBytes / sizeof(unsigned); ++k) dirty = dirty || host_ctr[k] != 0u;
+  rc = host_word != 0 ? host_word : dirty ? QTEA_ERR_STATE : QTEA_OK;
+  if (clear && rc != QTEA_OK) {  // counters and status word back to zero: the start state of a call
+    if (cudaMemsetAsync(ctr, 0, kStaticCtrBytes + sizeof(int), st) != cudaSuccess ||
+        cudaStreamSynchronize(st) != cudaSuccess) {
+      cudaGetLastError();
+      return QTEA_ERR_CUDA;
+    }
+  }
   return rc;
 }
 

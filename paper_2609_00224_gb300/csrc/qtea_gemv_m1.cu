@@ -26,9 +26,10 @@
 //  * Split tiles are reduced by the last-arriving CTA (atomic counter, no spin-wait) in a
 //    fixed CTA order, so results are bitwise reproducible.
 //  * Programmatic dependent launch: before griddepcontrol.wait a CTA only initialises its
-//    barriers, starts the TMA of its first units' codes, which the library owns and no other
-//    kernel writes, and prefetches into L2 the lines of x and v those units read (a prefetch
-//    reads no value). Everything the caller owns (x, v, alpha, the residual, y) and the split-tile
+//    barriers, starts the TMA of its first units' codes when the library owns them (a layout's
+//    packed codes, which no kernel writes after packing; caller-owned codes are fetched after the
+//    wait), and prefetches into L2 the lines of x and v those units read (a prefetch reads no
+//    value). Everything else the caller owns (x, v, alpha, the residual, y) and the split-tile
 //    workspace is touched after the wait. Each CTA lets the next launch start once it is running.
 // Every wait on an mbarrier is bounded: after ~2 s the waiting thread records
 // QTEA_ERR_TIMEOUT in the status word and its role stops.
@@ -528,6 +529,15 @@ struct Ring {
   int S, n_problems;
 };
 
+// The first fill of every code stage.
+__device__ __forceinline__ void first_fills(const TensorMaps& maps, const Ring& r, int u0, int n_units) {
+  for (int i = 0; i < r.S && i < n_units; ++i) {
+    const UnitPos up = unit_pos(r.tab, r.n_problems, (long long)u0 + i);
+    issue_unit(&maps.m[up.p], up.t, up.ch, smem_u32(r.codes + (size_t)i * kStageBytes), smem_u32(&r.full_c[i]));
+    r.last_fill[i] = 1;
+  }
+}
+
 // The producer lane: keeps the code stages filled. Fills 0 .. S-1 were issued before the grid
 // dependency wait.
 __device__ __noinline__ void producer_role(const TensorMaps& maps, const Ring r, int u0, int n_units, int* status) {
@@ -817,14 +827,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&maps.m[lane])) : "memory");
   __syncthreads();
 
-  // the first fill of every code stage: library-owned codes only, so it may start before the wait
-  if (warp == kProducerWarp && lane == 0) {
-    for (int i = 0; i < S && i < n_units; ++i) {
-      const UnitPos up = unit_pos(tab, NP, (long long)u0 + i);
-      issue_unit(&maps.m[up.p], up.t, up.ch, smem_u32(r.codes + (size_t)i * kStageBytes), smem_u32(&r.full_c[i]));
-      r.last_fill[i] = 1;
-    }
-  }
+  // the first fill of every code stage: before the wait when the library owns the codes (no kernel
+  // writes them after the layout is packed), after it when the caller does
+  const bool pre_fill = gp.codes_after_wait == 0;
+  if (pre_fill && warp == kProducerWarp && lane == 0) first_fills(maps, r, u0, n_units);
   // warm L2 with the lines of x and v that the first six units read (eight 128-byte lines of each
   // per 512-column chunk, one per helper lane): a prefetch reads no value into the SM, so the data
   // the units use is still read after the wait, from L2, where a preceding kernel's writes land
@@ -840,6 +846,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (!pre_fill && warp == kProducerWarp && lane == 0) first_fills(maps, r, u0, n_units);
 
   if (warp < kConsumerWarps) consumer_role(r, gp.cta_u0, gp.total_units, u0, u1, warp, lane, gp.status);
   else if (warp < kProducerWarp) helper_role(r, u0, n_units, warp - kConsumerWarps, lane, gp.status);

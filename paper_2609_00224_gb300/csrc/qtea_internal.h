@@ -86,6 +86,7 @@ struct TensorMaps {
 struct GroupParams {
   ProblemArgs prob[kMaxProblems];
   int n_problems, n_stages;
+  int codes_after_wait;     // the codes belong to the caller: no code fill before the grid dependency wait
   int* status;              // device status word (the first layout's)
   long long total_units;
   int cta_u0[kMaxGrid + 1]; // first unit of every CTA (balanced split), cta_u0[grid] = total

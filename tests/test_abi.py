@@ -30,7 +30,7 @@ def test_library_exports_every_declared_symbol():
 
 
 def test_status_strings():
-    for code in range(7):
+    for code in range(9):
         assert qt.status_string(code) and qt.status_string(code) != "unknown status"
     assert qt.status_string(99) == "unknown status"
 
@@ -66,3 +66,5 @@ def test_compute_entry_points_fail_without_gpu():
     out = ctypes.c_void_p()
     rc = lib.qtea_pack_layout(ctypes.c_void_p(16), 4, 8, 8, 0, 0, None, ctypes.byref(out))
     assert rc == qt.QTEA_ERR_CUDA and not out.value
+    # the allocation-free entry's state query needs the device too, and reports it
+    assert lib.qtea_gemv_m1_static_status(1, None) == qt.QTEA_ERR_CUDA
