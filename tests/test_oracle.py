@@ -304,6 +304,38 @@ def test_rejects_bad_inputs():
 
 # ---------------------------------------------------------------- packed layouts
 
+def residual_golden_case():
+    """Two groups of four rows, five salient columns, no ternary part: y = x * R placed by the
+    positions. The position bytes are written by hand from the layout rule (entry c of group q at
+    bits 2 (c % 4) of byte q * ceil(s/4) + c / 4): group 0 positions [1, 3, 0, 2 | 2] are bytes
+    0x8D (1 + 3*4 + 0*16 + 2*64) and 0x02; group 1 positions [3, 2, 1, 0 | 1] are 0x1B and 0x01."""
+    N, K, s = 8, 8, 5
+    sal = np.array([1, 2, 4, 6, 7], np.int32)
+    ridx = np.array([[0x8D, 0x02], [0x1B, 0x01]], np.uint8)
+    one = synth.f16_from_double(1.0)
+    R = np.array([[0.5, 0.25, -1.0, 2.0, 0.125], [-0.5, 4.0, 0.75, -2.0, 1.5]])
+    rv = np.array([[synth.f16_from_double(r) for r in row] for row in R], np.uint16)
+    T = np.zeros((N, K), np.int8)
+    alpha = np.full((N, 1), one, np.uint16)
+    v = np.full(K, one, np.uint16)
+    return N, K, sal, ridx, R, rv, T, alpha, v
+
+
+def test_residual_positions_hand_written_bytes():
+    N, K, sal, ridx, R, rv, T, alpha, v = residual_golden_case()
+    # expected rows of every entry, read off the hand-written positions above
+    rows = {(0, 0): 1, (0, 1): 3, (0, 2): 0, (0, 3): 2, (0, 4): 2,
+            (1, 0): 7, (1, 1): 6, (1, 2): 5, (1, 3): 4, (1, 4): 5}
+    for c, col in enumerate(sal):
+        x = np.zeros((1, K), np.uint16)
+        x[0, col] = synth.f16_from_double(1.0)
+        y, _ = oracle.gemv(x, T, alpha, v, sal, rv, ridx)
+        want = np.zeros(N)
+        want[rows[(0, c)]] += R[0, c]
+        want[rows[(1, c)]] += R[1, c]
+        assert np.array_equal(y[0], want), (c, y[0], want)
+
+
 def test_pack_2bit_known_bytes_and_padding():
     for t, byte in [(-1, 0x00), (0, 0x55), (1, 0xAA)]:
         T = np.full((3, 8), t, np.int8)

@@ -13,6 +13,7 @@ import pytest
 
 import oracle
 import synth
+from test_oracle import residual_golden_case
 
 F16 = np.float16
 SRC = os.path.join(os.path.dirname(oracle.__file__), "qtea_oracle.c")
@@ -92,6 +93,23 @@ def pin_failures(lib):
             for c in range(p.s):
                 W[4 * q + pos[q, c], p.salient_idx[c]] += dec[int(p.residual_vals[q, c])]
         check("fp8_residual", np.allclose(y, f(p.x) @ W.T, rtol=1e-12, atol=1e-13))
+    # residual positions from hand-written bytes (test_oracle.residual_golden_case)
+    N, K, sal, ridx, R, rv, T, alpha, v = residual_golden_case()
+    rows = [[1, 3, 0, 2, 2], [7, 6, 5, 4, 5]]
+    ok = True
+    for c, col in enumerate(sal):
+        x = np.zeros((1, K), np.uint16)
+        x[0, col] = synth.f16_from_double(1.0)
+        try:
+            y, _ = oracle.gemv(x, T, alpha, v, sal, rv, ridx, lib=lib)
+        except oracle.OracleError:
+            ok = False
+            break
+        want = np.zeros(N)
+        want[rows[0][c]] += R[0, c]
+        want[rows[1][c]] += R[1, c]
+        ok = ok and np.array_equal(y[0], want)
+    check("residual_golden", ok)
     # LUT symmetry and single-digit entries
     xs = np.array([0.3, -1.25, 2.0, 0.125, -0.5])
     lut = oracle.lut5(xs, lib=lib)
@@ -117,6 +135,8 @@ MUTANTS = {
     "half_subnormal_scale": [("ldexp((double)frac, -24)", "ldexp((double)frac, -23)")],
     "base3_digit_order": [("int value = 0, weight = 1;", "int value = 0, weight = 81;"), ("weight *= 3;", "weight /= 3;")],
     "lut_digit_offset": [("(double)(rest % 3 - 1) * xs[d]", "(double)(rest % 3) * xs[d]")],
+    "residual_position_msb_first": [(">> (2 * (c % 4))) & 3;", ">> (6 - 2 * (c % 4))) & 3;")],
+    "residual_position_byte_stride": [("ridx[(size_t)q * residual_stride(s) + c / 4]", "ridx[(size_t)q * (s / 4) + c / 4]")],
 }
 
 
