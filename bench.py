@@ -744,6 +744,59 @@ def qtea_arm(args):
                  "2bit_fp16_residual": dict(paper_leg(qt.QTEA_FMT_2BIT, False),
                                             kernel="qtea_gemv_mb_kernel (tensor cores, scale groups)")}
 
+    # ---- the paper's decode against the fixed-point one: the Llama3-8B layer in base-3 codes (one
+    #      alpha per row, fp16 residual values), the same resident layouts decoded by the sign-symmetric
+    #      lookup table (Sec. 3.5, Appendix A) and by the fixed-point dot-product kernel
+    def lut_leg():
+        n_res, nsteps = 4, 16
+        shapes = synth.workload_shapes(LAYER_WORKLOAD)
+        players = []
+        for li in range(n_res):
+            L = []
+            for mi in range(7):
+                pp = synth.workload_problem(LAYER_WORKLOAD, mi, layer=li)
+                f16 = lambda a: torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
+                T = torch.from_numpy(pp.T).cuda()
+                lay = qt.qtea_pack_layout(T, n_salient=pp.s, fmt=qt.QTEA_FMT_BASE3)
+                del T
+                L.append(dict(x=f16(pp.x), layout=lay, row_scale=f16(pp.alpha.reshape(-1)), col_scale=f16(pp.v),
+                              salient_idx=torch.from_numpy(pp.salient_idx).cuda(), residual_vals=f16(pp.residual_vals),
+                              residual_idx=torch.from_numpy(pp.residual_idx).cuda(),
+                              y=torch.empty((1, pp.N), dtype=torch.float32, device="cuda")))
+            players.append(L)
+        # base-3 codes, one alpha per row, fp16 residual values
+        pbytes = sum(algorithmic_bytes(N, K, synth.salient_count(K)) - N * (-(-K // 64) * 64) // 4
+                     + N * (-(-K // 128)) * 26 for _, N, K in shapes)
+        out = {}
+        for name, opt in (("lut", 0), ("fixed_point_dp4a", qt.QTEA_OPT_FIXED_POINT)):
+            for L in players:
+                for g in L:
+                    g["layout"].set_options(opt)
+            with torch.cuda.stream(stream):
+                qt.qtea_gemv_grouped(players[0], stream=stream)
+            gp = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gp, stream=stream):
+                for st in range(nsteps):
+                    qt.qtea_gemv_grouped(players[st % n_res], stream=stream)
+            tp = timed_replay(gp) * 1e3 / nsteps
+            del gp
+            status = max(qt.qtea_device_status(g["layout"]) for L in players for g in L)
+            if status:
+                raise RuntimeError(f"device status {status} in the {name} steps")
+            out[name] = {"us_per_step": round(tp, 2), "GBps": round(pbytes / (tp * 1e-6) / 1e9, 1),
+                         "frac_of_measured_hbm": round(pbytes / (tp * 1e-6) / 1e9 / peak, 3)}
+        out["lut"]["kernel"] = "qtea_gemv_lut_kernel (half-LUT of 122 fp32 entries per code byte)"
+        out["fixed_point_dp4a"]["kernel"] = "qtea_gemv_paper_b3_kernel (22/23-bit planes, dp4a)"
+        out["bytes_per_step"] = pbytes
+        out["layers_resident"] = n_res
+        del players
+        torch.cuda.empty_cache()
+        return out
+
+    lut = None
+    if not args.no_paper:
+        lut = {"workload": "llama3_8b_layer_base3_one_alpha_per_row", "M": 1, **lut_leg()}
+
     # ---- the Llama3-70B layer (8192-wide, 28672-row MLP: the large-K shapes) at M = 1, the seven
     #      GEMVs per step as one grouped call, rotating over resident layers whose codes exceed L2
     def llama70b_leg():
@@ -872,7 +925,7 @@ def qtea_arm(args):
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,
                          "us_per_launch": round(1e3 * total_ms / args.steps, 3),
                          "us_per_launch_isolated": None if iso_us is None else round(iso_us, 3)},
-            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "decode_stack": stack, "llama3_70b_layer": l70, "quantizer": quant, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
+            "cpu_baseline": cpu, "dense_fp16_cublas": dense, "batch_sweep": msweep, "paper_storage": paper, "lut_vs_fixed_point": lut, "decode_stack": stack, "llama3_70b_layer": l70, "quantizer": quant, "e2e": e2e, "clocks": clk, "act_bits": args.act_bits, "other_precision": alt, "gpu_launches": args.steps, "launch": "one grouped launch per step (7 GEMVs)", "graphs": True,
             "setup_s": round(t_gen, 1),
         }
         print(json.dumps(line), flush=True)

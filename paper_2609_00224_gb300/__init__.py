@@ -27,6 +27,7 @@ QTEA_FMT_2BIT = 0
 QTEA_FMT_BASE3 = 1
 QTEA_OPT_BIAS = 1
 QTEA_OPT_RESIDUAL_FP8 = 2
+QTEA_OPT_FIXED_POINT = 4
 QTEA_MAX_M = 16
 
 _lib = None

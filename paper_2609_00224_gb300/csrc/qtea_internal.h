@@ -227,6 +227,50 @@ cudaError_t launch_mb_prep(const MbPrepGroup& g, cudaStream_t st);
 cudaError_t launch_mb(const TensorMaps& maps, const TensorMaps& ab_maps, const MbGroupParams& p, bool grp, int grid,
                       size_t smem, cudaStream_t st);
 
+// ---------------------------------------------------------------- table-lookup kernel (base-3, M = 1)
+// The paper's decode (Sec. 3.5, Appendix A): per chunk of 8 blocks of 128 columns (208 code bytes
+// per row) a sign-symmetric table of 122 fp32 dot products per code byte, in shared memory; 16 warps
+// of 32 rows each make a 512-row tile.
+constexpr int kLutWarps = 16;
+constexpr int kLutThreads = kLutWarps * 32;
+constexpr int kLutTileRows = kLutWarps * 32;                   // 512
+constexpr int kLutBlocks = 8;                                  // 128-column blocks per chunk
+constexpr int kLutCols = kLutBlocks * 128;                     // 1024
+constexpr int kLutPacks = kLutBlocks * 26;                     // 208 code bytes per row and chunk
+constexpr int kLutLanes = kLutPacks / 8;                       // 26 lanes of 8 code bytes
+constexpr int kLutHalf = 122;                                  // entries of a half table
+constexpr int kLutStride = 224;                                // floats per table row (7 x 32 banks)
+constexpr int kLutMaxEntries = 1040;                           // salient entries a chunk may take
+constexpr int kLutResBatch = 32;                               // salient entries per residual batch
+constexpr size_t kLutSmemBytes = (size_t)(kLutHalf * kLutStride + kLutCols + kLutMaxEntries) * sizeof(float);
+
+struct LutProblem {
+  const uint16_t* x;        // [K]
+  const uint8_t* packed;    // [N][row_bytes] base-3
+  const uint16_t* alpha;    // [N]
+  const uint16_t* v;        // [K]
+  const int32_t* sal;       // [s]
+  const void* rvals;        // [N/4][s] fp16, or FP8 E4M3 bytes
+  const uint8_t* ridx;      // [N/4][ceil(s/4)]
+  float* y;                 // [N]
+  float* ws;                // [grid][2][kLutTileRows] partial rows of split tiles
+  unsigned* counters;       // [n_tiles][kLutWarps], zero between calls
+  int N, K, s, row_bytes, n_blocks, n_tiles, n_chunks;
+  int fp8;                  // residual values in FP8 E4M3
+  int aligned8;             // rows start on 8-byte boundaries (8-byte code loads)
+  long long unit_begin;     // first unit of this problem in the launch
+};
+
+struct LutParams {
+  LutProblem prob[kMaxProblems];
+  int n_problems;
+  long long total_units;
+  int cta_u0[kMaxGrid + 1];
+};
+
+cudaError_t lut_configure(size_t smem_optin);
+cudaError_t launch_lut(const LutParams& p, int grid, cudaStream_t st);
+
 // ---------------------------------------------------------------- generic kernel (any M)
 struct GenericParams {
   const uint16_t* x;        // [M][K]
@@ -320,4 +364,8 @@ struct qtea_layout {
                          // of every 256-row tile [n_tiles][kMbResFloatsPerTile]
   float* mb_part;        // [sm_count][kMbPartFloatsPerCta] partial rows of split tiles
   unsigned* mb_counters; // [n_tiles of 256 rows][kMbConsumerWarps]
+  // table-lookup kernel resources (base-3 layouts)
+  bool lut_ok;
+  float* lut_ws;         // [sm_count][2][kLutTileRows]
+  unsigned* lut_counters;  // [n_tiles of 512 rows][kLutWarps]
 };

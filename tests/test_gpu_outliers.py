@@ -114,12 +114,15 @@ def test_low_batch_massive_activations(qt, name, mags, sd, M):
 
 
 @pytest.mark.parametrize("name,mags,sd", CASES, ids=[c[0] for c in CASES])
-@pytest.mark.parametrize("M", [1, 3])
-def test_base3_kernel_massive_activations(qt, name, mags, sd, M):
-    """The paper's base-3 codes (one alpha per row here, so only the code format differs)."""
+@pytest.mark.parametrize("M,fixed", [(1, True), (1, False), (3, True)])
+def test_base3_kernel_massive_activations(qt, name, mags, sd, M, fixed):
+    """The paper's base-3 codes (one alpha per row here, so only the code format differs), through the
+    fixed-point kernel and, at M = 1, the table-lookup decode."""
     p, cols = problem(name, mags, sd, M=M)
     layout = qt.qtea_pack_layout(dev(p.T), n_salient=p.s, fmt=qt.QTEA_FMT_BASE3)
-    check(run(qt, layout, args(p)), p, cols, f"base-3 M={M} {name}")
+    if fixed:
+        layout.set_options(qt.QTEA_OPT_FIXED_POINT)
+    check(run(qt, layout, args(p)), p, cols, f"base-3 M={M} fixed={fixed} {name}")
 
 
 @pytest.mark.parametrize("name,mags,sd", CASES, ids=[c[0] for c in CASES])

@@ -113,8 +113,10 @@ def test_options_switch_a_default_layout_to_the_paper_path(qt):
     assert_within(y, y_ref, b, "2-bit with beta")
     layout.set_options(0)
     assert layout.describe()["batch1_kernel"] == 1
+    layout.set_options(qt.QTEA_OPT_FIXED_POINT)  # a base-3 choice: a 2-bit layout stays on the batch-1 kernel
+    assert layout.describe()["batch1_kernel"] == 1
     with pytest.raises(qt.QteaError):
-        layout.set_options(4)
+        layout.set_options(8)
 
 
 @pytest.mark.parametrize("matrix", range(7))
