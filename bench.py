@@ -935,31 +935,107 @@ def qtea_arm(args):
 
 
 def profile_case(args):
-    """A small fixed workload for ncu captures: the Qwen3-14B layer's seven GEMVs at batch M as one
-    grouped call, `--calls` times, then a status check. Prints one line; times nothing."""
+    """Small fixed workloads for ncu captures, one per kernel path; each runs `--calls` calls over
+    `--profile-layers` resident layers (their codes exceed L2 with the default 4), then checks the
+    device status. Prints one line; times nothing.
+
+      qwen3_14b_layer        the Qwen3-14B layer's seven GEMVs at batch --m, grouped (low-batch
+                             kernel; batch-1 kernel at --m 1)
+      llama3_8b_layer        the Llama3-8B layer's seven GEMVs at batch 1, grouped (batch-1 kernel)
+      llama3_8b_base3        the same in base-3 codes, one alpha per row (table-lookup kernel;
+                             --fixed-point: the fixed-point base-3 kernel)
+      llama3_8b_paper        the paper's storage (base-3, alpha and beta per 128 columns, FP8
+                             residual) at batch --m (fixed-point base-3 kernel for --m <= 4, the
+                             general paper kernel above)
+      llama3_8b_paper_2bit   2-bit codes with one (alpha, beta) per row at batch --m (staged paper
+                             kernel for --m <= 4)
+      unaligned_residual     Qwen3-14B q_proj at batch --m with residual arrays off 16-byte
+                             boundaries (low-batch prep kernel, then the main kernel)
+      pack                   packing of the Llama3-8B layer's codes, 2-bit and base-3
+      quantize               the quantizer on the Llama3-8B layer's seven weight matrices
+    """
     import numpy as np
     import torch
     import paper_2609_00224_gb300 as qt
     import synth
     qt.load()
+    case, M, n_layers = args.profile_case, args.m, args.profile_layers
 
     def f16(a):
         return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).cuda().view(torch.float16)
 
-    M = args.m
-    probs = []
-    for mi in range(7):
-        p = synth.workload_problem("qwen3_14b_layer", mi, M=M)
-        lay = qt.qtea_pack_layout(torch.from_numpy(p.T).cuda(), n_salient=p.s)
-        probs.append(dict(x=f16(p.x), layout=lay, row_scale=f16(p.alpha.reshape(-1)), col_scale=f16(p.v),
-                          salient_idx=torch.from_numpy(p.salient_idx).cuda(), residual_vals=f16(p.residual_vals),
-                          residual_idx=torch.from_numpy(p.residual_idx).cuda(),
-                          y=torch.empty((M, p.N), dtype=torch.float32, device="cuda")))
-    for _ in range(args.calls):
-        qt.qtea_gemv_grouped(probs)
+    def layer(wl, li, make, fmt=qt.QTEA_FMT_2BIT, group=None, opts=0, M_=1):
+        out = []
+        for mi in range(7):
+            p = make(wl, mi, li, M_)
+            lay = qt.qtea_pack_layout(torch.from_numpy(p.T).cuda(), n_salient=p.s, group_size=group or p.K, fmt=fmt)
+            lay.set_options(opts)
+            if p.beta is not None:
+                sc = np.stack([p.alpha.reshape(p.N, -1), p.beta.reshape(p.N, -1)], axis=-1).reshape(-1)
+            else:
+                sc = p.alpha.reshape(-1)
+            rv = torch.from_numpy(p.residual_vals).cuda() if p.residual_fp8 else f16(p.residual_vals)
+            out.append(dict(x=f16(p.x), layout=lay, row_scale=f16(sc), col_scale=f16(p.v),
+                            salient_idx=torch.from_numpy(p.salient_idx).cuda(), residual_vals=rv,
+                            residual_idx=torch.from_numpy(p.residual_idx).cuda(),
+                            y=torch.empty((M_, p.N), dtype=torch.float32, device="cuda")))
+        return out
+
+    work = lambda wl, mi, li, M_: synth.workload_problem(wl, mi, M=M_, layer=li)
+    layers = []
+    if case == "qwen3_14b_layer":
+        layers = [layer("qwen3_14b_layer", li, work, M_=M) for li in range(n_layers)]
+    elif case == "llama3_8b_layer":
+        layers = [layer("llama3_8b_layer", li, work) for li in range(n_layers)]
+    elif case == "llama3_8b_base3":
+        opts = qt.QTEA_OPT_FIXED_POINT if args.fixed_point else 0
+        layers = [layer("llama3_8b_layer", li, work, fmt=qt.QTEA_FMT_BASE3, opts=opts) for li in range(n_layers)]
+    elif case == "llama3_8b_paper":
+        paper = lambda wl, mi, li, M_: synth.paper_problem(wl, mi, M=M_, layer=li)
+        layers = [layer("llama3_8b_layer", li, paper, fmt=qt.QTEA_FMT_BASE3, group=128,
+                        opts=qt.QTEA_OPT_BIAS | qt.QTEA_OPT_RESIDUAL_FP8, M_=M) for li in range(n_layers)]
+    elif case == "llama3_8b_paper_2bit":
+        bias_row = lambda wl, mi, li, M_: synth.make_problem(
+            "bias", *synth.workload_shapes(wl)[mi][1:], M_, synth.salient_count(synth.workload_shapes(wl)[mi][2]),
+            synth.workload_seed(wl, li, mi), beta_std=0.002)
+        layers = [layer("llama3_8b_layer", li, bias_row, opts=qt.QTEA_OPT_BIAS, M_=M) for li in range(n_layers)]
+    elif case == "unaligned_residual":
+        for li in range(n_layers):
+            p = synth.workload_problem("qwen3_14b_layer", 0, M=M, layer=li)
+            lay = qt.qtea_pack_layout(torch.from_numpy(p.T).cuda(), n_salient=p.s)
+            rvb = torch.zeros(p.residual_vals.size + 1, dtype=torch.float16, device="cuda")
+            rvb[1:] = f16(p.residual_vals).reshape(-1)
+            layers.append([dict(x=f16(p.x), layout=lay, row_scale=f16(p.alpha.reshape(-1)), col_scale=f16(p.v),
+                                salient_idx=torch.from_numpy(p.salient_idx).cuda(),
+                                residual_vals=rvb[1:].view(p.residual_vals.shape),
+                                residual_idx=torch.from_numpy(p.residual_idx).cuda(),
+                                y=torch.empty((M, p.N), dtype=torch.float32, device="cuda"))])
+    elif case == "pack":
+        for li in range(args.calls):
+            for mi in range(7):
+                p = synth.workload_problem("llama3_8b_layer", mi, layer=li)
+                T = torch.from_numpy(p.T).cuda()
+                for fmt in (qt.QTEA_FMT_2BIT, qt.QTEA_FMT_BASE3):
+                    qt.qtea_pack_layout(T, n_salient=p.s, fmt=fmt)
+        torch.cuda.synchronize()
+        print(json.dumps({"profile_case": case, "calls": args.calls, "status": 0}))
+        return 0
+    elif case == "quantize":
+        mats = []
+        for mi, (_, N, K) in enumerate(synth.workload_shapes("llama3_8b_layer")):
+            W, h = synth.quant_problem(1000 + mi, N, K)
+            mats.append((torch.from_numpy(W).cuda(), torch.from_numpy(h).cuda(), synth.salient_count(K)))
+        for _ in range(args.calls):
+            for W, h, s_ in mats:
+                qt.qtea_quantize(W, h, group_size=128, n_salient=s_, bias=True)
+        torch.cuda.synchronize()
+        print(json.dumps({"profile_case": case, "calls": args.calls, "status": 0}))
+        return 0
+    for c in range(args.calls):
+        qt.qtea_gemv_grouped(layers[c % len(layers)])
     torch.cuda.synchronize()
-    status = qt.qtea_device_status(probs[0]["layout"])
-    print(json.dumps({"profile_case": args.profile_case, "M": M, "calls": args.calls, "status": status}))
+    status = max(qt.qtea_device_status(g["layout"]) for L in layers for g in L)
+    print(json.dumps({"profile_case": case, "M": M, "calls": args.calls, "status": status}))
     return 1 if status else 0
 
 
@@ -984,9 +1060,13 @@ def main():
     ap.add_argument("--no-per-shape", action="store_true")
     ap.add_argument("--act-bits", type=int, choices=[16, 24], default=16,
                     help="activation precision of the timed region (24 = exact default, 16 = fast mode)")
-    ap.add_argument("--profile-case", choices=["qwen3_14b_layer"], default=None,
+    ap.add_argument("--profile-case", choices=["qwen3_14b_layer", "llama3_8b_layer", "llama3_8b_base3",
+                                               "llama3_8b_paper", "llama3_8b_paper_2bit", "unaligned_residual",
+                                               "pack", "quantize"], default=None,
                     help="run a small fixed workload for profilers instead of the benchmark")
     ap.add_argument("--m", type=int, default=2, help="batch of --profile-case")
+    ap.add_argument("--profile-layers", type=int, default=4, help="resident layers of --profile-case")
+    ap.add_argument("--fixed-point", action="store_true", help="--profile-case llama3_8b_base3: fixed-point kernel")
     ap.add_argument("--calls", type=int, default=3, help="grouped calls of --profile-case")
     args = ap.parse_args()
     if args.profile_case:
