@@ -740,7 +740,8 @@ def qtea_arm(args):
     if not args.no_paper:
         paper = {"workload": "llama3_8b_layer_paper_storage", "M": 1,
                  "base3_fp8": dict(paper_leg(qt.QTEA_FMT_BASE3, True),
-                                   kernel="qtea_gemv_paper_b3_kernel (staged fixed-point activations, dp4a)"),
+                                   kernel="qtea_gemv_lut_kernel<grouped> (the paper's table decode, alpha and "
+                                          "beta per 128 columns staged per tile)"),
                  "2bit_fp16_residual": dict(paper_leg(qt.QTEA_FMT_2BIT, False),
                                             kernel="qtea_gemv_mb_kernel (tensor cores, scale groups)")}
 

@@ -62,9 +62,9 @@ typedef enum qtea_option {
   QTEA_OPT_BIAS = 1,         /* row_scale holds (alpha, beta) pairs: fp16 [N][G][2] (Eq. 4's beta) */
   QTEA_OPT_RESIDUAL_FP8 = 2, /* residual_vals holds FP8 E4M3 bytes [N/4][s] (Sec. 4.1), passed
                                 through the same pointer argument */
-  QTEA_OPT_FIXED_POINT = 4   /* base-3 layouts with one alpha per row and no beta: batch-1 calls
-                                decode by the fixed-point dot-product kernel instead of the paper's
-                                sign-symmetric lookup table (Sec. 3.5, Appendix A), the default */
+  QTEA_OPT_FIXED_POINT = 4   /* base-3 layouts: batch-1 calls decode by the fixed-point
+                                dot-product kernel instead of the paper's sign-symmetric lookup
+                                table (Sec. 3.5, Appendix A), the default */
 } qtea_option;
 
 /* Largest batch (rows of x) one qtea_gemv call accepts. */
@@ -94,9 +94,10 @@ typedef enum qtea_option {
  * Which kernel serves a call: the TMA batch-1 kernel takes 2-bit, one-scale-per-row layouts
  * without options at M = 1; the tensor-core low-batch kernel takes those at M >= 2 and 2-bit
  * layouts in the paper's storage (groups of 128 columns, or beta absent) at any M; base-3 layouts
- * with one alpha per row and no beta at M = 1 run on the paper's table-lookup decode (Sec. 3.5,
- * Appendix A); other base-3 layouts at M <= 4 run on a kernel that stages v*x once per CTA in fixed
- * point (the base-3 problems of a grouped call share one launch); the rest run on general kernels.
+ * at M = 1 run on the paper's table-lookup decode (Sec. 3.5, Appendix A); base-3 layouts at
+ * 2 <= M <= 4 (or at M = 1 with QTEA_OPT_FIXED_POINT) run on a kernel that stages v*x once per CTA
+ * in fixed point (the base-3 problems of a grouped call share one launch); the rest run on general
+ * kernels.
  *
  * The call validates every code on the device and synchronizes `stream` once to read the
  * result; invalid codes give QTEA_ERR_BAD_CODES and no layout. It allocates the packed
@@ -247,9 +248,9 @@ int qtea_set_activation_precision(qtea_layout* layout, int bits);
 /*
  * Storage options of the scales and residual values qtea_gemv reads with this layout: any
  * combination of QTEA_OPT_BIAS and QTEA_OPT_RESIDUAL_FP8 (0 restores fp16 alpha only and fp16
- * residual values), and QTEA_OPT_FIXED_POINT for base-3 layouts (at M = 1, base-3 layouts with
- * one alpha per row and no beta decode by table lookup unless this option asks for the fixed-point
- * kernel; other base-3 calls always use the fixed-point kernel). Other bits -> QTEA_ERR_INVALID_ARG.
+ * residual values), and QTEA_OPT_FIXED_POINT for base-3 layouts (at M = 1 base-3 layouts decode by
+ * table lookup unless this option asks for the fixed-point kernel; at 2 <= M <= 4 they always use
+ * the fixed-point kernel). Other bits -> QTEA_ERR_INVALID_ARG.
  * With QTEA_OPT_BIAS or QTEA_OPT_RESIDUAL_FP8 set, calls leave the batch-1 kernel (see
  * qtea_pack_layout for which kernel serves which storage); QTEA_OPT_FIXED_POINT changes nothing for
  * 2-bit layouts. Set it before the calls that use it; it takes effect for calls made afterwards.

@@ -129,32 +129,37 @@ int plan_lut(qtea_layout* l, const cudaDeviceProp& prop) {
   return QTEA_OK;
 }
 
-// The table-lookup kernel takes this batch-1 problem: base-3 codes, one alpha per row, no beta,
-// the fixed-point kernel not asked for, and a chunk's share of the salient entries within its
-// staging. (Measured on the Llama3-8B layer in base-3 codes: 63 us per step by table, 97 us by the
-// fixed-point kernel.)
+// The table-lookup kernel takes this batch-1 problem: base-3 codes (alpha per row or per group of
+// 128 columns, with or without beta), the fixed-point kernel not asked for, and a chunk's share of
+// the salient entries within its staging. (Measured on the Llama3-8B
+// layer in base-3 codes: 63 us per step by table, 97 us by the fixed-point kernel.)
 bool lut_eligible(const qtea_layout* l, int M) {
   if (M != 1 || !l->lut_ok || l->format != QTEA_FMT_BASE3 || (l->options & QTEA_OPT_FIXED_POINT)) return false;
-  if (l->group_size != l->K || (l->options & QTEA_OPT_BIAS)) return false;
   const int n_blocks = l->K_pad / 128, n_chunks = (n_blocks + kLutBlocks - 1) / kLutBlocks;
   const int nb = (l->n_salient + 7) / 8;
   return ((nb + n_chunks - 1) / n_chunks) * 8 <= kLutMaxEntries;
 }
 
-// Table-lookup problems, up to kMaxProblems per launch.
+// Scale groups for the table-lookup kernel: alpha (and beta) staged per 128-column block, each
+// block reading its group's pair; a layout with one alpha per row and no beta needs none.
+bool lut_grouped(const qtea_layout* l) { return l->group_size != l->K || (l->options & QTEA_OPT_BIAS); }
+
+// Table-lookup problems: consecutive problems of one variant (with or without scale groups), up to
+// kMaxProblems, share a launch.
 int run_lut(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st) {
-  for (int i = 0; i < n; i += kMaxProblems) {
+  int i = 0;
+  while (i < n) {
     LutParams P;
     std::memset(&P, 0, sizeof(P));
-    const int k = n - i < kMaxProblems ? n - i : kMaxProblems;
-    int sm_count = 1;
-    for (int j = 0; j < k; ++j) {
-      const qtea_gemv_problem& q = qs[idx[i + j]];
+    const bool grouped = lut_grouped(qs[idx[i]].packed_ternary);
+    int k = 0, sm_count = 1;
+    while (i + k < n && k < kMaxProblems && lut_grouped(qs[idx[i + k]].packed_ternary) == grouped) {
+      const qtea_gemv_problem& q = qs[idx[i + k]];
       const qtea_layout* l = q.packed_ternary;
-      LutProblem& a = P.prob[j];
+      LutProblem& a = P.prob[k];
       a.x = q.x;
       a.packed = l->packed;
-      a.alpha = q.row_scale;
+      a.scales = q.row_scale;
       a.v = q.col_scale;
       a.sal = q.salient_idx;
       a.rvals = q.residual_vals;
@@ -171,16 +176,20 @@ int run_lut(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st)
       a.n_chunks = (a.n_blocks + kLutBlocks - 1) / kLutBlocks;
       a.fp8 = (l->options & QTEA_OPT_RESIDUAL_FP8) ? 1 : 0;
       a.aligned8 = (l->row_bytes % 8 == 0 && aligned(l->packed, 8)) ? 1 : 0;
+      a.G = (l->K + l->group_size - 1) / l->group_size;
+      a.bias = (l->options & QTEA_OPT_BIAS) ? 1 : 0;
+      a.gdiv = l->group_size == l->K ? a.n_blocks : 1;
       a.unit_begin = P.total_units;
       P.total_units += (long long)a.n_tiles * a.n_chunks;
-      sm_count = l->sm_count;  // every layout of the group records the device's SM count
+      sm_count = l->sm_count;  // every layout records the device's SM count (its workspace's CTA slots)
+      ++k;
     }
     P.n_problems = k;
     int grid = (int)(P.total_units < sm_count ? P.total_units : sm_count);
     if (grid > kMaxGrid) grid = kMaxGrid;
-    // the split-tile workspace of each layout has sm_count CTA slots
     for (int b = 0; b <= grid; ++b) P.cta_u0[b] = (int)unit_begin_of(b, P.total_units, grid);
-    if (launch_lut(P, grid, st) != cudaSuccess) return QTEA_ERR_CUDA;
+    if (launch_lut(P, grouped, grid, st) != cudaSuccess) return QTEA_ERR_CUDA;
+    i += k;
   }
   return QTEA_OK;
 }

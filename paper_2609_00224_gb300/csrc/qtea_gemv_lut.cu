@@ -5,7 +5,8 @@
 // code 121 (five zeros) has value 0, so 122 entries per pack hold it: entry k = the value of code
 // 121 + k, and code c < 121 reads entry 121 - c with the sign flipped (the half-LUT).
 //
-// Serves base-3 layouts with one alpha per row and no beta at M = 1, fp16 or FP8 residual values.
+// Serves base-3 layouts at M = 1: one alpha per row, or the paper's storage with alpha and beta per
+// row and group of 128 columns (Eq. 10), fp16 or FP8 residual values.
 // Design for sm_103a:
 //  * Work: a unit is (problem, 512-row tile, chunk of 8 blocks of 128 columns = 208 code bytes per
 //    row). The units of all problems form one sequence split evenly over persistent CTAs (one per
@@ -14,12 +15,15 @@
 //  * Per unit the CTA builds the chunk's half-LUTs in shared memory: 208 packs x 122 fp32 entries,
 //    each entry ((((t4 x4 + t3 x3) + t2 x2) + t1 x1) + t0 x0) in that fixed order (t = digit - 1,
 //    x = v*x exact in fp32), so an entry's value does not depend on who builds it.
-//  * Lookup: a warp takes 32 rows. Lane l < 26 owns the chunk's code bytes 8l .. 8l+7 of every row
-//    (one 8-byte load per row); entry k of pack 8l + j sits at table column 26 j + l of a 224-float
-//    table row, so the 26 lanes always read 26 distinct banks (no conflicts whatever the codes).
-//    Per byte: |c - 121| -> shared load -> sign flip -> add. Each lane accumulates its 8 packs for
-//    each of the 32 rows; a transposed butterfly (31 shuffles) then leaves row r0 + l's chunk sum in
-//    lane l, in a fixed order.
+//  * Lookup: a warp takes 32 rows, 8 at a time. Lane l < 26 owns the chunk's code bytes 8l .. 8l+7
+//    of every row (one 8-byte load per row); entry k of pack 8l + j sits at table column 26 j + l of
+//    a 224-float table row, so the 26 lanes always read 26 distinct banks (no conflicts whatever the
+//    codes). Per byte: |c - 121| -> shared load -> sign flip -> add. Each lane sums its 8 packs of
+//    each row; two shuffle rounds and a transposed butterfly over the rest leave each of the 8 rows'
+//    chunk sums in fixed lanes, in a fixed order.
+//  * Scale groups of 128 columns: a lane's 8 packs lie in at most two blocks; their table values
+//    are scaled by those blocks' alpha (staged with beta for the tile's rows and the chunk's blocks)
+//    before the lanes are summed, and each row adds beta times the blocks' sums of x.
 //  * Residual (Eq. 11): the chunk's share of the salient entries (blocks of 8 entries split over the
 //    chunks by index, as in the dp4a kernel), x at their columns staged with the table; each lane
 //    adds its row's entries (loads issued before the lookups, used after). Never scaled by alpha.
@@ -120,20 +124,43 @@ __device__ __forceinline__ uint2 load_codes(const LutProblem& a, int row, int ch
   return w;
 }
 
-// acc[r] += the lane's 8 packs of row r (codes w).
+// The lane's 8 packs of one row (codes w): plain sum, or with scale groups each value times the
+// alpha of its block (fa[j], the lo or hi block's alpha).
 __device__ __forceinline__ float row_packs(const float* colp, uint2 w) {
-  float s = 0.f;
+  float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-  for (int j = 0; j < 4; ++j) s += lookup(colp + 26 * j, (w.x >> (8 * j)) & 0xFFu);
+  for (int j = 0; j < 4; j += 2) {
+    s0 += lookup(colp + 26 * j, (w.x >> (8 * j)) & 0xFFu);
+    s1 += lookup(colp + 26 * (j + 1), (w.x >> (8 * (j + 1))) & 0xFFu);
+  }
 #pragma unroll
-  for (int j = 0; j < 4; ++j) s += lookup(colp + 26 * (4 + j), (w.y >> (8 * j)) & 0xFFu);
-  return s;
+  for (int j = 0; j < 4; j += 2) {
+    s0 += lookup(colp + 26 * (4 + j), (w.y >> (8 * j)) & 0xFFu);
+    s1 += lookup(colp + 26 * (5 + j), (w.y >> (8 * (j + 1))) & 0xFFu);
+  }
+  return s0 + s1;
 }
 
-// After it, lane l holds sum over the warp's lanes of v[l] (v[r] = lane's value for row r).
-__device__ __forceinline__ float transpose_reduce(float (&v)[32], int lane) {
+__device__ __forceinline__ float row_packs_grouped(const float* colp, uint2 w, int jb, float a_lo, float a_hi) {
+  float s0 = 0.f, s1 = 0.f;
 #pragma unroll
-  for (int s = 16; s >= 1; s >>= 1) {
+  for (int j = 0; j < 8; ++j) {
+    const uint32_t c = ((j < 4 ? w.x : w.y) >> (8 * (j & 3))) & 0xFFu;
+    const float v = lookup(colp + 26 * j, c);
+    if (j & 1) s1 = fmaf(j < jb ? a_lo : a_hi, v, s1);
+    else s0 = fmaf(j < jb ? a_lo : a_hi, v, s0);
+  }
+  return s0 + s1;
+}
+
+// Sum of the 8 rows' values over the warp's 32 lanes: lanes l with l % 8 == r end with row r's sum.
+__device__ __forceinline__ float reduce8(float (&v)[8], int lane) {
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] += __shfl_xor_sync(0xffffffffu, v[i], 16);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] += __shfl_xor_sync(0xffffffffu, v[i], 8);
+#pragma unroll
+  for (int s = 4; s >= 1; s >>= 1) {
     const bool up = (lane & s) != 0;
 #pragma unroll
     for (int i = 0; i < s; ++i) {
@@ -145,12 +172,17 @@ __device__ __forceinline__ float transpose_reduce(float (&v)[32], int lane) {
   return v[0];
 }
 
+template <bool GROUPED>
 __global__ void __launch_bounds__(kLutThreads, 1) qtea_gemv_lut_kernel(const __grid_constant__ LutParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   LutSmem sm;
   sm.table = reinterpret_cast<float*>(smem);
   sm.xt = sm.table + kLutHalf * kLutStride;
   sm.xs = sm.xt + kLutCols;
+  float* bsx = sm.xs + kLutMaxEntries;                                // [kLutBlocks] sums of x per block
+  uint32_t* sab = reinterpret_cast<uint32_t*>(bsx + kLutBlocks);      // [kLutTileRows][kLutBlocks] (alpha, beta)
+  // a lane's packs 8l .. 8l+7 lie in blocks b_lo and b_lo + 1; packs j < jb in b_lo
+  const int b_lo = (8 * (threadIdx.x & 31)) / 26, jb = 26 * (b_lo + 1) - 8 * (threadIdx.x & 31);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int u0 = P.cta_u0[blockIdx.x], u1 = P.cta_u0[blockIdx.x + 1];
   const long long total = P.total_units;
@@ -184,6 +216,30 @@ __global__ void __launch_bounds__(kLutThreads, 1) qtea_gemv_lut_kernel(const __g
     for (int i = threadIdx.x; i < kLutCols; i += kLutThreads) {
       const int col = ch * kLutCols + i;
       sm.xt[i] = col < a.K ? h2f(__ldg(a.v + col)) * h2f(__ldg(a.x + col)) : 0.f;  // exact in fp32
+    }
+    if (GROUPED) {
+      // alpha and beta (0 without the bias option) of the tile's rows and the chunk's blocks, and the
+      // blocks' sums of x (in column order, by one warp per block)
+      for (int i = threadIdx.x; i < kLutTileRows * kLutBlocks; i += kLutThreads) {
+        const int r = i / kLutBlocks, b = i - r * kLutBlocks, rg = t * kLutTileRows + r;
+        const int g = (ch * kLutBlocks + b) / a.gdiv;  // the block's scale group
+        uint32_t ab = 0;
+        if (rg < a.N && b < nbk) {
+          const uint16_t* sc = a.scales + (size_t)rg * a.G * (a.bias ? 2 : 1) + (size_t)g * (a.bias ? 2 : 1);
+          ab = (uint32_t)__ldg(sc) | (a.bias ? (uint32_t)__ldg(sc + 1) << 16 : 0u);
+        }
+        sab[i] = ab;
+      }
+      if (warp < kLutBlocks) {
+        float sx = 0.f;
+        for (int c = lane; c < 128; c += 32) {
+          const int col = ch * kLutCols + warp * 128 + c;
+          sx += col < a.K ? h2f(__ldg(a.x + col)) : 0.f;
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) sx += __shfl_xor_sync(0xffffffffu, sx, o);
+        if (lane == 0) bsx[warp] = sx;
+      }
     }
     for (int e = e0 + threadIdx.x; e < e1; e += kLutThreads) {
       int col = __ldg(a.sal + e);
@@ -223,21 +279,37 @@ __global__ void __launch_bounds__(kLutThreads, 1) qtea_gemv_lut_kernel(const __g
 
     // lookups: 32 rows of the warp, 8 rows per batch, the next batch's codes loaded ahead
     const float* colp = sm.table + lane;  // + 26 j + k * kLutStride
-    float acc[32];
-#pragma unroll
+    float chunk_sum = 0.f;                // row `row` over the chunk (alpha applied with scale groups)
+#pragma unroll 1
     for (int bt = 0; bt < 4; ++bt) {
       if (bt < 3) {
 #pragma unroll
         for (int r = 0; r < 8; ++r) nw[r] = load_codes(a, rbase + 8 * (bt + 1) + r, ch, lane, valid_packs);
       }
+      float acc[8];
 #pragma unroll
-      for (int r = 0; r < 8; ++r) acc[8 * bt + r] = lane < kLutLanes ? row_packs(colp, cw[r]) : 0.f;
-      if (bt < 3) {
-#pragma unroll
-        for (int r = 0; r < 8; ++r) cw[r] = nw[r];
+      for (int r = 0; r < 8; ++r) {
+        if (lane >= kLutLanes) {
+          acc[r] = 0.f;
+        } else if (GROUPED) {
+          const uint32_t* ab = sab + (warp * 32 + 8 * bt + r) * kLutBlocks;
+          const float a_lo = h2f((uint16_t)(ab[b_lo] & 0xFFFFu));
+          const float a_hi = jb < 8 ? h2f((uint16_t)(ab[b_lo + 1] & 0xFFFFu)) : 0.f;
+          acc[r] = row_packs_grouped(colp, cw[r], jb, a_lo, a_hi);
+        } else {
+          acc[r] = row_packs(colp, cw[r]);
+        }
       }
+      const float s8 = reduce8(acc, lane);  // row rbase + 8 bt + lane % 8
+      if ((lane >> 3) == bt) chunk_sum = s8;
+#pragma unroll
+      for (int r = 0; r < 8; ++r) cw[r] = nw[r];
     }
-    const float chunk_sum = transpose_reduce(acc, lane);  // row `row` over the chunk
+    if (GROUPED) {  // beta times the blocks' sums of x
+      const uint32_t* ab = sab + (warp * 32 + lane) * kLutBlocks;
+#pragma unroll
+      for (int b = 0; b < kLutBlocks; ++b) chunk_sum = fmaf(h2f((uint16_t)(ab[b] >> 16)), bsx[b], chunk_sum);
+    }
 
     for (int eb = e0; eb < e1; eb += kLutResBatch) {
       if (eb > e0) load_res(eb);
@@ -258,7 +330,7 @@ __global__ void __launch_bounds__(kLutThreads, 1) qtea_gemv_lut_kernel(const __g
     // tile epilogue once this CTA's part of tile t is done
     if (ch == a.n_chunks - 1 || u == u1 - 1) {
       const long long A = a.unit_begin + (long long)t * a.n_chunks, B = A + a.n_chunks;
-      const float al = row_ok ? h2f(__ldg(a.alpha + row)) : 0.f;
+      const float al = GROUPED ? 1.f : (row_ok ? h2f(__ldg(a.scales + row)) : 0.f);
       const float val = fmaf(al, tacc, racc);
       const int tr = warp * 32 + lane;  // row within the tile
       if (A >= u0 && B <= u1) {
@@ -295,10 +367,14 @@ __global__ void __launch_bounds__(kLutThreads, 1) qtea_gemv_lut_kernel(const __g
 
 cudaError_t lut_configure(size_t smem_optin) {
   if (kLutSmemBytes > smem_optin) return cudaErrorInvalidValue;
-  return cudaFuncSetAttribute(qtea_gemv_lut_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kLutSmemBytes);
+  cudaError_t e = cudaFuncSetAttribute(qtea_gemv_lut_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kLutSmemBytes);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(qtea_gemv_lut_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              (int)kLutSmemBytes);
 }
 
-cudaError_t launch_lut(const LutParams& p, int grid, cudaStream_t st) {
+cudaError_t launch_lut(const LutParams& p, bool grouped, int grid, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)grid);
   cfg.blockDim = dim3(kLutThreads);
@@ -309,7 +385,8 @@ cudaError_t launch_lut(const LutParams& p, int grid, cudaStream_t st) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, qtea_gemv_lut_kernel, p);
+  return grouped ? cudaLaunchKernelEx(&cfg, qtea_gemv_lut_kernel<true>, p)
+                 : cudaLaunchKernelEx(&cfg, qtea_gemv_lut_kernel<false>, p);
 }
 
 }  // namespace qtea

@@ -242,12 +242,15 @@ constexpr int kLutHalf = 122;                                  // entries of a h
 constexpr int kLutStride = 224;                                // floats per table row (7 x 32 banks)
 constexpr int kLutMaxEntries = 1040;                           // salient entries a chunk may take
 constexpr int kLutResBatch = 32;                               // salient entries per residual batch
-constexpr size_t kLutSmemBytes = (size_t)(kLutHalf * kLutStride + kLutCols + kLutMaxEntries) * sizeof(float);
+// table, v*x of the chunk, x at the chunk's salient columns, the blocks' sums of x, (alpha, beta) of
+// the tile's rows and the chunk's blocks (scale groups)
+constexpr size_t kLutSmemBytes =
+    (size_t)(kLutHalf * kLutStride + kLutCols + kLutMaxEntries + kLutBlocks + kLutTileRows * kLutBlocks) * 4;
 
 struct LutProblem {
   const uint16_t* x;        // [K]
   const uint8_t* packed;    // [N][row_bytes] base-3
-  const uint16_t* alpha;    // [N]
+  const uint16_t* scales;   // [N] alpha, or with groups [N][G] alpha or [N][G][2] (alpha, beta)
   const uint16_t* v;        // [K]
   const int32_t* sal;       // [s]
   const void* rvals;        // [N/4][s] fp16, or FP8 E4M3 bytes
@@ -258,6 +261,8 @@ struct LutProblem {
   int N, K, s, row_bytes, n_blocks, n_tiles, n_chunks;
   int fp8;                  // residual values in FP8 E4M3
   int aligned8;             // rows start on 8-byte boundaries (8-byte code loads)
+  int G, bias;              // scale groups per row (the launch's variant when grouped), beta present
+  int gdiv;                 // 128-column blocks per scale group (1, or all of them with one group)
   long long unit_begin;     // first unit of this problem in the launch
 };
 
@@ -269,7 +274,7 @@ struct LutParams {
 };
 
 cudaError_t lut_configure(size_t smem_optin);
-cudaError_t launch_lut(const LutParams& p, int grid, cudaStream_t st);
+cudaError_t launch_lut(const LutParams& p, bool grouped, int grid, cudaStream_t st);
 
 // ---------------------------------------------------------------- generic kernel (any M)
 struct GenericParams {

@@ -138,3 +138,86 @@ def test_lut_matches_fixed_point_kernel_within_tolerance(qt):
     y_ref, bound = oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx)
     lim = REL * bound + ABS
     assert np.all(np.abs(y_lut.cpu().numpy() - y_dp4a.cpu().numpy()) <= 2 * lim)
+
+
+def paper_args(p, bias):
+    f16 = lambda a: dev(np.ascontiguousarray(a).view(np.int16), torch.float16)
+    if bias:
+        sc = np.stack([p.alpha.reshape(p.N, -1), p.beta.reshape(p.N, -1)], axis=-1).reshape(-1)
+    else:
+        sc = p.alpha.reshape(-1)
+    a = args(p)
+    a["row_scale"] = f16(sc)
+    return a
+
+
+def run_grouped(qt, p, bias, fixed=False):
+    layout = qt.qtea_pack_layout(dev(p.T), n_salient=p.s, group_size=p.group_size or p.K, fmt=qt.QTEA_FMT_BASE3)
+    opts = (qt.QTEA_OPT_BIAS if bias else 0) | (qt.QTEA_OPT_RESIDUAL_FP8 if p.residual_fp8 else 0)
+    layout.set_options(opts | (qt.QTEA_OPT_FIXED_POINT if fixed else 0))
+    a = paper_args(p, bias)
+    y = qt.qtea_gemv(a["x"], layout, a["row_scale"], a["col_scale"], a["salient_idx"], a["residual_vals"],
+                     a["residual_idx"])
+    torch.cuda.synchronize()
+    assert qt.qtea_device_status(layout) == 0
+    return y
+
+
+def check_grouped(y, p, bias, what, rows=None):
+    y_ref, bound = oracle.gemv(p.x, p.T, p.alpha, p.v, p.salient_idx, p.residual_vals, p.residual_idx,
+                               beta=p.beta if bias else None, group_size=p.group_size or p.K, rows=rows,
+                               residual_fp8=p.residual_fp8)
+    yy = y.cpu().numpy().astype(np.float64)
+    if rows is not None:
+        yy = yy[:, rows]
+    err = np.abs(yy - y_ref)
+    lim = REL * bound + ABS
+    assert np.all(err <= lim), f"{what}: worst normalised error {(err / lim).max():.3g}"
+    return float((err / lim).max())
+
+
+@pytest.mark.parametrize("N,K,s", [(4, 128, 4), (12, 300, 16), (516, 1000, 32), (1024, 1100, 40), (2048, 4096, 120)])
+@pytest.mark.parametrize("group,bias,fp8", [(128, True, True), (128, False, False), (128, True, False), (0, True, True)])
+def test_lut_scale_groups(qt, N, K, s, group, bias, fp8):
+    """The paper's storage through the table: alpha (and beta) per 128-column group, or one (alpha,
+    beta) pair per row (group 0 = K); K = 1100 leaves a last chunk of one block."""
+    p = synth.make_problem("lutg", N, K, 1, s, seed=N + K + s + group + 2 * bias + fp8, group_size=group,
+                           beta_std=0.002 if bias else 0.0, residual_fp8=fp8)
+    y = run_grouped(qt, p, bias)
+    check_grouped(y, p, bias, f"N={N} K={K} s={s} group={group} bias={bias} fp8={fp8}")
+
+
+@pytest.mark.parametrize("matrix", range(7))
+def test_lut_paper_storage_llama3_8b_layer(qt, matrix):
+    """The Llama3-8B layer in the paper's storage (base-3, alpha and beta per 128 columns, FP8
+    residual): the table decode, and within tolerance of the fixed-point kernel on the same layout."""
+    p = synth.paper_problem("llama3_8b_layer", matrix)
+    y = run_grouped(qt, p, True)
+    rows = np.sort(np.random.default_rng(matrix).choice(p.N, size=48, replace=False)).astype(np.int32)
+    assert check_grouped(y, p, True, p.name, rows=rows) < 0.25
+    y_fixed = run_grouped(qt, p, True, fixed=True)
+    check_grouped(y_fixed, p, True, p.name + " fixed point", rows=rows)
+
+
+def test_lut_grouped_call_mixes_variants(qt):
+    """One grouped call with base-3 problems with and without scale groups (two launches) and a
+    2-bit problem: each result matches the oracle."""
+    ps = [synth.paper_problem("llama3_8b_layer", 1), synth.workload_problem("llama3_8b_layer", 2),
+          synth.make_problem("g", 1024, 2048, 1, 64, seed=3, group_size=128, beta_std=0.002)]
+    bias = [True, False, True]
+    fmts = [qt.QTEA_FMT_BASE3, qt.QTEA_FMT_BASE3, qt.QTEA_FMT_BASE3]
+    probs, lays = [], []
+    for p, b, f in zip(ps, bias, fmts):
+        lay = qt.qtea_pack_layout(dev(p.T), n_salient=p.s, group_size=p.group_size or p.K, fmt=f)
+        lay.set_options((qt.QTEA_OPT_BIAS if b else 0) | (qt.QTEA_OPT_RESIDUAL_FP8 if p.residual_fp8 else 0))
+        lays.append(lay)
+        probs.append(dict(layout=lay, **paper_args(p, b)))
+    q2 = synth.workload_problem("llama3_8b_layer", 0)
+    lay2 = qt.qtea_pack_layout(dev(q2.T), n_salient=q2.s)
+    probs.append(dict(layout=lay2, **args(q2)))
+    ys = qt.qtea_gemv_grouped(probs)
+    torch.cuda.synchronize()
+    for p, b, y in zip(ps, bias, ys):
+        rows = np.arange(0, p.N, 37, dtype=np.int32)
+        check_grouped(y, p, b, "mixed " + p.name, rows=rows)
+    check(ys[3], q2, "mixed 2-bit", rows=np.arange(0, q2.N, 37, dtype=np.int32))
