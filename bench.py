@@ -743,7 +743,8 @@ def qtea_arm(args):
                                    kernel="qtea_gemv_lut_kernel<grouped> (the paper's table decode, alpha and "
                                           "beta per 128 columns staged per tile)"),
                  "2bit_fp16_residual": dict(paper_leg(qt.QTEA_FMT_2BIT, False),
-                                            kernel="qtea_gemv_mb_kernel (tensor cores, scale groups)")}
+                                            kernel="qtea_gemv_m1_kernel, grouped variant (alpha and beta "
+                                                   "applied per 128-column group in the decode)")}
 
     # ---- the paper's decode against the fixed-point one: the Llama3-8B layer in base-3 codes (one
     #      alpha per row, fp16 residual values), the same resident layouts decoded by the sign-symmetric
@@ -948,8 +949,8 @@ def profile_case(args):
       llama3_8b_paper        the paper's storage (base-3, alpha and beta per 128 columns, FP8
                              residual) at batch --m (fixed-point base-3 kernel for --m <= 4, the
                              general paper kernel above)
-      llama3_8b_paper_2bit   2-bit codes with one (alpha, beta) per row at batch --m (staged paper
-                             kernel for --m <= 4)
+      llama3_8b_paper_2bit   2-bit codes with one (alpha, beta) per row and FP8 residual values at
+                             batch --m (staged paper kernel for --m <= 4)
       unaligned_residual     Qwen3-14B q_proj at batch --m with residual arrays off 16-byte
                              boundaries (low-batch prep kernel, then the main kernel)
       pack                   packing of the Llama3-8B layer's codes, 2-bit and base-3
@@ -998,8 +999,9 @@ def profile_case(args):
     elif case == "llama3_8b_paper_2bit":
         bias_row = lambda wl, mi, li, M_: synth.make_problem(
             "bias", *synth.workload_shapes(wl)[mi][1:], M_, synth.salient_count(synth.workload_shapes(wl)[mi][2]),
-            synth.workload_seed(wl, li, mi), beta_std=0.002)
-        layers = [layer("llama3_8b_layer", li, bias_row, opts=qt.QTEA_OPT_BIAS, M_=M) for li in range(n_layers)]
+            synth.workload_seed(wl, li, mi), beta_std=0.002, residual_fp8=True)
+        layers = [layer("llama3_8b_layer", li, bias_row, opts=qt.QTEA_OPT_BIAS | qt.QTEA_OPT_RESIDUAL_FP8, M_=M)
+                  for li in range(n_layers)]
     elif case == "unaligned_residual":
         for li in range(n_layers):
             p = synth.workload_problem("qwen3_14b_layer", 0, M=M, layer=li)

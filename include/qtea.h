@@ -91,9 +91,10 @@ typedef enum qtea_option {
  * bytes; byte q of group h holds columns 128h + 5q + d, d = 0..4, as sum_d (T+1) 3^d (lowest
  * column in the least significant digit); byte 25 holds three columns and two pad digits; pad
  * digits and columns >= K are digit 1.
- * Which kernel serves a call: the TMA batch-1 kernel takes 2-bit, one-scale-per-row layouts
- * without options at M = 1; the tensor-core low-batch kernel takes those at M >= 2 and 2-bit
- * layouts in the paper's storage (groups of 128 columns, or beta absent) at any M; base-3 layouts
+ * Which kernel serves a call: the TMA batch-1 kernel takes 2-bit layouts with fp16 residual values
+ * at M = 1 (one alpha per row, or alpha and beta per row or per 128-column group); the tensor-core
+ * low-batch kernel takes those at M >= 2 and 2-bit layouts with FP8 residual values (groups of 128
+ * columns, or beta absent) at any M; base-3 layouts
  * at M = 1 run on the paper's table-lookup decode (Sec. 3.5, Appendix A); base-3 layouts at
  * 2 <= M <= 4 (or at M = 1 with QTEA_OPT_FIXED_POINT) run on a kernel that stages v*x once per CTA
  * in fixed point (the base-3 problems of a grouped call share one launch); the rest run on general
@@ -219,8 +220,8 @@ typedef struct qtea_layout_desc {
   int N, K, K_pad, group_size, n_salient, format;
   size_t packed_bytes;      /* size of the packed ternary weights */
   const void* packed_data;  /* device pointer to the packed ternary weights */
-  int batch1_kernel;        /* 1 if M = 1 calls run the TMA stream-K batch-1 kernel, 0 if they
-                               fall back to the general kernel (e.g. no tensor-map support) */
+  int batch1_kernel;        /* 1 if M = 1 calls run the TMA stream-K batch-1 kernel (2-bit codes,
+                               fp16 residual values), 0 otherwise */
   int options;              /* QTEA_OPT_* flags */
 } qtea_layout_desc;
 

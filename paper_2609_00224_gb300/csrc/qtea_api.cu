@@ -211,6 +211,13 @@ int check_problem(const qtea_gemv_problem& q, int M) {
   return QTEA_OK;
 }
 
+// The batch-1 kernel serves 2-bit layouts with fp16 residual values: one alpha per row, or alpha
+// (and beta) per group of 128 columns or per row (its grouped variant).
+bool m1_capable(const qtea_layout* l) {
+  return l->format == QTEA_FMT_2BIT && !(l->options & QTEA_OPT_RESIDUAL_FP8) &&
+         (l->group_size == l->K || l->group_size == 128);
+}
+
 // The paper's own storage: base-3 codes, groups of 128 columns, beta or FP8 residual values.
 bool is_paper(const qtea_layout* l) {
   return l->format != QTEA_FMT_2BIT || l->group_size != l->K ||
@@ -523,6 +530,11 @@ bool group_add(M1Group& g, const qtea_gemv_problem& q) {
   a.n_tiles = l->n_tiles;
   a.n_chunks = l->n_chunks;
   a.act_bits = (l->act_bits == 16 && l->K >= kMinK16) ? 16 : 24;
+  const bool bias = (l->options & QTEA_OPT_BIAS) != 0, groups = l->group_size != l->K || bias;
+  a.G = (l->K + l->group_size - 1) / l->group_size;
+  a.gdiv = l->group_size == l->K ? l->n_chunks * 4 : 1;  // 128-column groups per scale group
+  const bool vec = groups && a.gdiv == 1 && a.G % 4 == 0 && aligned(q.row_scale, bias ? 16 : 8);
+  a.gflags = (groups ? kScaleGroups : 0) | (bias ? kScaleBias : 0) | (vec ? kScaleVec : 0);
   a.vec_xv = aligned(q.x, 16) && aligned(q.col_scale, 16);
   a.vec_res = (l->n_salient % kResBlock == 0) && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 2);
   a.unit_begin = g.gp.total_units;
@@ -754,7 +766,7 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
       if (cudaMemsetAsync(q.y, 0, (size_t)M * l->N * sizeof(float), st) != cudaSuccess) rc = QTEA_ERR_CUDA;
       continue;
     }
-    if (M == 1 && l->m1_ok && !is_paper(l)) {
+    if (M == 1 && l->m1_ok && m1_capable(l)) {
       m1_idx[n_m1++] = i;
     } else if (lut_eligible(l, M)) {
       lut_idx[n_lut++] = i;
@@ -814,7 +826,7 @@ int qtea_layout_describe(const qtea_layout* l, qtea_layout_desc* out) {
   out->format = l->format;
   out->packed_bytes = l->packed_bytes;
   out->packed_data = l->packed;
-  out->batch1_kernel = (l->m1_ok && !is_paper(l)) ? 1 : 0;
+  out->batch1_kernel = (l->m1_ok && m1_capable(l)) ? 1 : 0;
   out->options = l->options;
   return QTEA_OK;
 }

@@ -237,6 +237,74 @@ __device__ __forceinline__ void decode_unit(const uint4* row0, const uint4* row1
   }
 }
 
+// Scale groups of 128 columns: the unit's decode finished per group (every 8 words), each group's
+// exact sum of T X scaled by q and its row's alpha, plus beta times the group's sum of x.
+template <int P>
+__device__ __forceinline__ void decode_unit_grouped(const uint4* row0, const uint4* row1, const uint4* pl, int sw,
+                                                    const ChunkMeta* mp, float scale, const uint32_t (&g0)[4],
+                                                    const uint32_t (&g1)[4], float& f0, float& f1) {
+  constexpr int kW = (P == 3) ? 3 : 2;
+  uint4 P0 = pl[0], P1 = pl[1], P2 = kW == 3 ? pl[2] : make_uint4(0, 0, 0, 0);
+  uint4 c0 = row0[0 ^ sw], c1 = row1[0 ^ sw];
+  float e0[4], e1[4];  // exact group sums of T X of both rows
+#pragma unroll 1
+  for (int g = 0; g < 4; ++g) {
+    RowAcc<P> a0, a1;
+#pragma unroll
+    for (int k = 0; k < P; ++k)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) a0.a[k][q] = a1.a[k][q] = 0;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int jj = 2 * g + h;
+      const uint4 n0 = row0[((jj + 1) & 7) ^ sw];
+      const uint4 n1 = row1[((jj + 1) & 7) ^ sw];
+      const uint32_t w0[4] = {c0.x, c0.y, c0.z, c0.w};
+      const uint32_t w1[4] = {c1.x, c1.y, c1.z, c1.w};
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int nw = ((4 * jj + e + 1) & 31) * 3;
+        const uint4 Q0 = pl[nw], Q1 = pl[nw + 1];
+        const uint4 Q2 = kW == 3 ? pl[nw + 2] : make_uint4(0, 0, 0, 0);
+        if constexpr (P == 3) {
+          decode_word3(w0[e], P0, P1, P2, a0);
+          decode_word3(w1[e], P0, P1, P2, a1);
+        } else {
+          decode_word2(w0[e], P0, P1, a0);
+          decode_word2(w1[e], P0, P1, a1);
+        }
+        P0 = Q0;
+        P1 = Q1;
+        P2 = Q2;
+      }
+      c0 = n0;
+      c1 = n1;
+    }
+    const int gsx = mp->gsum_x[g];
+    float d0, d1;
+    if constexpr (P == 2) {
+      d0 = finish_chunk2(a0, gsx);
+      d1 = finish_chunk2(a1, gsx);
+    } else {
+      d0 = finish_chunk3(a0, (long long)gsx);
+      d1 = finish_chunk3(a1, (long long)gsx);
+    }
+    // kept per group (registers selected by index, not an indexed array)
+    if (g == 0) { e0[0] = d0; e1[0] = d1; }
+    else if (g == 1) { e0[1] = d0; e1[1] = d1; }
+    else if (g == 2) { e0[2] = d0; e1[2] = d1; }
+    else { e0[3] = d0; e1[3] = d1; }
+  }
+  // alpha (low half) and beta (high half) of each group, used only now: their loads, issued before
+  // the decode, have had the whole unit to arrive
+#pragma unroll
+  for (int g = 0; g < 4; ++g) {
+    const float sx = mp->gsx[g];
+    f0 = fmaf(h2f((uint16_t)(g0[g] & 0xffffu)) * scale, e0[g], fmaf(h2f((uint16_t)(g0[g] >> 16)), sx, f0));
+    f1 = fmaf(h2f((uint16_t)(g1[g] & 0xffffu)) * scale, e1[g], fmaf(h2f((uint16_t)(g1[g] >> 16)), sx, f1));
+  }
+}
+
 // ---------------------------------------------------------------- staging (helpers)
 
 // x and v of columns 16*lane .. 16*lane+15 of one chunk, as fp16 pairs (zero beyond K).
@@ -376,6 +444,22 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
     dst[0] = make_uint4(reg[0], reg[1], reg[2], reg[3]);
     dst[1] = make_uint4(reg[4], reg[5], reg[6], reg[7]);
     dst[2] = make_uint4(reg[8], reg[9], reg[10], reg[11]);
+  }
+  if (a.gflags & kScaleGroups) {  // per 128-column group (lanes 8k .. 8k+7): sum of X, and sum of x for beta
+    int gs = sx;
+    float xs = 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      xs += h2f((uint16_t)(L.x[i] & 0xffffu)) + h2f((uint16_t)(L.x[i] >> 16));
+#pragma unroll
+    for (int o = 1; o < 8; o <<= 1) {
+      gs += __shfl_xor_sync(0xffffffffu, gs, o);
+      xs += __shfl_xor_sync(0xffffffffu, xs, o);
+    }
+    if ((lane & 7) == 0) {
+      meta->gsum_x[lane >> 3] = gs;
+      meta->gsx[lane >> 3] = xs;
+    }
   }
   // the chunk's sum of X, exact: the lanes' sums split into 16-bit halves, each summed by one warp
   // reduction instruction (|sum| < 2^32 in 24-bit mode)
@@ -664,10 +748,41 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
     const int u = u0 + i;
     const ProblemArgs& a = r.tab[c.p];
     const int n_chunks = a.n_chunks, N = a.N;
+    const bool grouped = (a.gflags & kScaleGroups) != 0;
+    const bool gbias = (a.gflags & kScaleBias) != 0, gvec = (a.gflags & kScaleVec) != 0;
     if (need_alpha) {  // used at the tile's end: unconditional loads (rows clamped), so nothing waits here
-      al0 = __ldg(a.alpha + min(c.t * kTileRows + ra, N - 1));
-      al1 = __ldg(a.alpha + min(c.t * kTileRows + ra + 32, N - 1));
+      if (grouped) {   // alpha is applied per group in the decode
+        al0 = al1 = (uint16_t)0x3C00u;  // 1.0
+      } else {
+        al0 = __ldg(a.alpha + min(c.t * kTileRows + ra, N - 1));
+        al1 = __ldg(a.alpha + min(c.t * kTileRows + ra + 32, N - 1));
+      }
       need_alpha = false;
+    }
+    uint32_t gab0[4], gab1[4];  // scale groups: (alpha, beta) bits of the unit's four groups, both rows
+    if (grouped) {
+      const int r0 = min(c.t * kTileRows + ra, N - 1), r1 = min(c.t * kTileRows + ra + 32, N - 1);
+      const int st_ = gbias ? 2 : 1;
+      if (gvec && gbias) {  // (alpha, beta) of the four groups: one 16-byte load per row
+        const uint4 v0 = __ldg(reinterpret_cast<const uint4*>(a.alpha + ((size_t)r0 * a.G + 4 * c.ch) * 2));
+        const uint4 v1 = __ldg(reinterpret_cast<const uint4*>(a.alpha + ((size_t)r1 * a.G + 4 * c.ch) * 2));
+        gab0[0] = v0.x; gab0[1] = v0.y; gab0[2] = v0.z; gab0[3] = v0.w;
+        gab1[0] = v1.x; gab1[1] = v1.y; gab1[2] = v1.z; gab1[3] = v1.w;
+      } else if (gvec) {         // alpha of the four groups: one 8-byte load per row
+        const uint2 v0 = __ldg(reinterpret_cast<const uint2*>(a.alpha + (size_t)r0 * a.G + 4 * c.ch));
+        const uint2 v1 = __ldg(reinterpret_cast<const uint2*>(a.alpha + (size_t)r1 * a.G + 4 * c.ch));
+        gab0[0] = v0.x & 0xffffu; gab0[1] = v0.x >> 16; gab0[2] = v0.y & 0xffffu; gab0[3] = v0.y >> 16;
+        gab1[0] = v1.x & 0xffffu; gab1[1] = v1.x >> 16; gab1[2] = v1.y & 0xffffu; gab1[3] = v1.y >> 16;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const int g = min((4 * c.ch + k) / a.gdiv, a.G - 1);
+          const uint16_t* s0 = a.alpha + ((size_t)r0 * a.G + g) * st_;
+          const uint16_t* s1 = a.alpha + ((size_t)r1 * a.G + g) * st_;
+          gab0[k] = (uint32_t)__ldg(s0) | (gbias ? (uint32_t)__ldg(s0 + 1) << 16 : 0u);
+          gab1[k] = (uint32_t)__ldg(s1) | (gbias ? (uint32_t)__ldg(s1 + 1) << 16 : 0u);
+        }
+      }
     }
     bool ok = mbar_wait(smem_u32(&r.full_c[st]), ph_c, status);
     ok = ok && mbar_wait(smem_u32(&r.planes_a[slot]), ph_a, status);
@@ -682,8 +797,11 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
         reinterpret_cast<const uint4*>(r.codes + (size_t)st * kStageBytes + (size_t)ra * kChunkRowBytes);
     const uint4* row1 = row0 + 32 * (kChunkRowBytes / 16);
     const uint4* pl = reinterpret_cast<const uint4*>(ax);
-    float d0, d1;
-    if (planes == 2) {
+    float d0 = 0.f, d1 = 0.f;  // ungrouped: sum of T X over the chunk; grouped: the scaled sums
+    if (grouped) {
+      if (planes == 2) decode_unit_grouped<2>(row0, row1, pl, sw, mp, scale, gab0, gab1, d0, d1);
+      else decode_unit_grouped<3>(row0, row1, pl, sw, mp, scale, gab0, gab1, d0, d1);
+    } else if (planes == 2) {
       RowAcc<2> a0, a1;
       decode_unit<2>(row0, row1, pl, sw, a0, a1);
       d0 = finish_chunk2(a0, (int)sum_x);
@@ -706,14 +824,22 @@ __device__ __forceinline__ void consumer_role(const Ring r, const int* cta_u0, l
         const int col = mp->out_col[k];
         const float xv = mp->out_val[k];
         const int off = ((((col >> 6) ^ sw) << 4) | ((col >> 2) & 15)), sh = 2 * (col & 3);
-        o0 = fmaf((float)(int)((cb0[off] >> sh) & 3u) - 1.f, xv, o0);
-        o1 = fmaf((float)(int)((cb1[off] >> sh) & 3u) - 1.f, xv, o1);
+        float t0 = (float)(int)((cb0[off] >> sh) & 3u) - 1.f, t1 = (float)(int)((cb1[off] >> sh) & 3u) - 1.f;
+        if (grouped) {  // scaled by the alpha of the outlier's group
+          const int g = col >> 7;
+          const uint32_t b0 = g == 0 ? gab0[0] : g == 1 ? gab0[1] : g == 2 ? gab0[2] : gab0[3];
+          const uint32_t b1 = g == 0 ? gab1[0] : g == 1 ? gab1[1] : g == 2 ? gab1[2] : gab1[3];
+          t0 *= h2f((uint16_t)(b0 & 0xffffu));
+          t1 *= h2f((uint16_t)(b1 & 0xffffu));
+        }
+        o0 = fmaf(t0, xv, o0);
+        o1 = fmaf(t1, xv, o1);
       }
     }
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_u32(&r.empty_c[st]));  // codes and metadata no longer read
-    yacc0 += fmaf(d0, scale, o0);
-    yacc1 += fmaf(d1, scale, o1);
+    yacc0 += grouped ? d0 + o0 : fmaf(d0, scale, o0);
+    yacc1 += grouped ? d1 + o1 : fmaf(d1, scale, o1);
 
     // the previous unit's residual sums (into the tile they belong to), then its tile's epilogue
     if (pend >= 0) {

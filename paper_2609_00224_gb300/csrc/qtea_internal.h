@@ -44,7 +44,7 @@ constexpr int kResBlock = 8;                                   // salient entrie
 constexpr int kMaxOutliers = 16;
 constexpr int kOutlierRounds = 4;
 
-struct ChunkMeta {  // 128 bytes
+struct ChunkMeta {  // 160 bytes
   float scale;       // q, the fixed-point quantum of v*x in this chunk (a power of two)
   int planes;        // byte planes of the chunk's fixed-point v*x: 3 (24-bit) or 2 (16-bit)
   long long sum_x;   // sum of the chunk's fixed-point v*x values (outliers excluded)
@@ -52,19 +52,21 @@ struct ChunkMeta {  // 128 bytes
   int pad[3];
   uint16_t out_col[kMaxOutliers];  // their columns within the chunk
   float out_val[kMaxOutliers];     // their v*x, exact
+  int gsum_x[4];     // scale groups: the fixed-point v*x summed per 128-column group
+  float gsx[4];      // scale groups with beta: x summed per 128-column group
 };
 
 // Auxiliary slot: planes [32 words][48 bytes], metadata, residual sums [512 rows].
 constexpr int kAuxMeta = kPlaneBytesPerChunk;
 constexpr int kAuxRes = kAuxMeta + (int)sizeof(ChunkMeta);
-constexpr int kAuxBytes = kAuxRes + kTileRows * (int)sizeof(float);  // 3712
+constexpr int kAuxBytes = kAuxRes + kTileRows * (int)sizeof(float);  // 3744
 // Per helper: x at one residual block's 8 entries spread over the 4 positions of a group,
 // T[entry][position] = x * one-hot(position), so that an entry adds with 4 FMAs and no selects.
 constexpr int kOneHotBytes = kResBlock * 4 * 16;               // 512
 
 struct ProblemArgs {
   const uint16_t* x;        // [K] (M = 1)
-  const uint16_t* alpha;    // [N]
+  const uint16_t* alpha;    // [N] alpha, or with scale groups [N][G] alpha or [N][G][2] (alpha, beta)
   const uint16_t* v;        // [K]
   const int32_t* sal;       // [s]
   const uint16_t* rvals;    // [N/4][s]
@@ -76,8 +78,16 @@ struct ProblemArgs {
   int act_bits;             // 24: v*x in 24-bit fixed point; 16: 16-bit where a chunk allows it
   int vec_xv;               // x and v are 16-byte aligned (vector loads)
   int vec_res;              // s % 8 == 0 and rvals 16-byte / ridx 2-byte aligned (vector loads)
+  int gflags;               // kScaleGroups | kScaleBias | kScaleVec (one int: the struct stays 128 bytes,
+                            // which keeps the kernel's copies of it out of local memory)
+  int G, gdiv;              // scale groups per row; 128-column groups per scale group
   long long unit_begin;     // first global unit of this problem
 };
+
+// ProblemArgs::gflags: alpha (and beta) applied per 128-column group inside the decode; beta
+// present; a row's four groups of a chunk are one aligned 16-byte (8 without beta) load.
+constexpr int kScaleGroups = 1, kScaleBias = 2, kScaleVec = 4;
+static_assert(sizeof(ProblemArgs) <= 128, "larger problem records spill the batch-1 kernel's copies");
 
 struct TensorMaps {
   CUtensorMap m[kMaxProblems];

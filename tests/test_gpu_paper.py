@@ -43,8 +43,8 @@ def run_paper(qt, p, fmt, bias, M=None):
     layout = qt.qtea_pack_layout(dev(p.T), n_salient=p.s, group_size=p.group_size or p.K, fmt=fmt)
     opts = (qt.QTEA_OPT_BIAS if bias else 0) | (qt.QTEA_OPT_RESIDUAL_FP8 if p.residual_fp8 else 0)
     layout.set_options(opts)
-    default = fmt == qt.QTEA_FMT_2BIT and not p.group_size and opts == 0  # the library's own storage
-    assert layout.describe()["batch1_kernel"] == int(default) and layout.describe()["options"] == opts
+    batch1 = fmt == qt.QTEA_FMT_2BIT and not p.residual_fp8  # 2-bit codes with fp16 residual values
+    assert layout.describe()["batch1_kernel"] == int(batch1) and layout.describe()["options"] == opts
     x = p.x if M is None else p.x[:M]
     rv = dev(p.residual_vals) if p.residual_fp8 else dev(p.residual_vals.view(np.int16), torch.float16)
     y = qt.qtea_gemv(dev(x.view(np.int16), torch.float16), layout, dev(scales(p, bias).view(np.int16), torch.float16),
@@ -104,13 +104,17 @@ def test_paper_storage_parity_small(qt, fmt, group, bias, fp8):
 
 
 def test_options_switch_a_default_layout_to_the_paper_path(qt):
-    """A 2-bit, one-alpha-per-row layout with QTEA_OPT_BIAS reads (alpha, beta) pairs; clearing the
-    options returns it to the batch-1 kernel."""
+    """A 2-bit, one-alpha-per-row layout with QTEA_OPT_BIAS reads (alpha, beta) pairs (on the batch-1
+    kernel's grouped variant); FP8 residual values move it to the low-batch kernel; clearing the
+    options returns it to the plain batch-1 kernel."""
     N, K = 256, 1024
     p = synth.make_problem("t", N, K, 1, 32, seed=5, beta_std=0.002)
     y, layout = run_paper(qt, p, qt.QTEA_FMT_2BIT, True)
     y_ref, b = reference(p, True)
     assert_within(y, y_ref, b, "2-bit with beta")
+    assert layout.describe()["batch1_kernel"] == 1
+    layout.set_options(qt.QTEA_OPT_RESIDUAL_FP8)
+    assert layout.describe()["batch1_kernel"] == 0
     layout.set_options(0)
     assert layout.describe()["batch1_kernel"] == 1
     layout.set_options(qt.QTEA_OPT_FIXED_POINT)  # a base-3 choice: a 2-bit layout stays on the batch-1 kernel
