@@ -15,8 +15,6 @@ namespace {
 
 constexpr int kGenWarps = 4;
 
-__device__ __forceinline__ float h2f(uint16_t b) { return __half2float(__ushort_as_half(b)); }
-
 template <int MB>
 __global__ void __launch_bounds__(kGenWarps * 32) qtea_gemv_generic_kernel(const GenericParams p) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;

@@ -35,18 +35,6 @@
 namespace qtea {
 namespace {
 
-__device__ __forceinline__ float h2f(uint16_t b) { return __half2float(__ushort_as_half(b)); }
-
-// OFP8 E4M3: bias 7, subnormals m * 2^-9, S.1111.111 is NaN, no infinity.
-__device__ __forceinline__ float e4m3_to_float(uint32_t b) {
-  const uint32_t e = (b >> 3) & 15u, m = b & 7u;
-  float mag;
-  if (e == 15u && m == 7u) mag = __int_as_float(0x7fc00000);
-  else if (e == 0u) mag = (float)m * 0.001953125f;
-  else mag = __int_as_float((int)((e + 120u) << 23 | m << 20));
-  return (b & 0x80u) ? -mag : mag;
-}
-
 // CTA whose range contains unit u.
 __device__ __forceinline__ int unit_owner(long long u, long long total, int grid) {
   return (int)(((u + 1) * grid - 1) / total);

@@ -30,23 +30,6 @@ namespace {
 
 constexpr int kPaperWarps = 4;
 
-__device__ __forceinline__ float h2f(uint16_t b) { return __half2float(__ushort_as_half(b)); }
-
-// FP8 E4M3 (sign bit 7, exponent bits 6-3 with bias 7, mantissa bits 2-0, subnormals at exponent
-// 0, NaN at S.1111.111, no infinity) as fp32, exactly.
-__device__ __forceinline__ float e4m3_to_float(uint32_t b) {
-  const uint32_t e = (b >> 3) & 15u, m = b & 7u;
-  float mag;
-  if (e == 15u && m == 7u) {
-    mag = __int_as_float(0x7fc00000);
-  } else if (e == 0u) {
-    mag = (float)m * 0.001953125f;  // m * 2^-9
-  } else {
-    mag = __int_as_float((int)((e + 120u) << 23 | m << 20));  // (1 + m/8) * 2^(e-7)
-  }
-  return (b & 0x80u) ? -mag : mag;
-}
-
 template <int MB>
 __global__ void __launch_bounds__(kPaperWarps * 32) qtea_gemv_paper_kernel(const PaperParams p) {
   __shared__ uint16_t lut[243];  // base-3 byte -> five 2-bit codes
