@@ -456,6 +456,7 @@ def qtea_arm(args):
             N, K = gm["N"], gm["K"]
             bts = statistics.mean(L[j]["bytes"] for L in layers)
             per_shape[gm["name"]] = {"N": N, "K": K, "s": gm["s"], "us_per_call": round(us, 3),
+                                     "kernel": qt.qtea_gemv_plan([group_args[0][j]])[0],
                                      "gbs": round(bts / (us * 1e-6) / 1e9, 1),
                                      "eff_bits_per_weight": round(8 * (bts - 2 * K - 4 * N) / (N * K), 3)}
 
@@ -480,8 +481,10 @@ def qtea_arm(args):
         ms_s = timed_replay(gs_)
         del gs_
         tok_b = sum(step_bytes)
+        kern = {name: qt.qtea_gemv_plan([group_args[0][j] for j in grp])[0]
+                for name, grp in zip(("q_k_v", "o", "gate_up", "down"), order)}
         stack = {"workload": f"llama3_8b_stack_{len(layers)}_layers_dependency_order", "tokens": n_tok,
-                 "launches_per_token": 4 * len(layers), "us_per_token": round(ms_s * 1e3 / n_tok, 1),
+                 "launches_per_token": 4 * len(layers), "kernels": kern, "us_per_token": round(ms_s * 1e3 / n_tok, 1),
                  "linear_tokens_per_s": round(n_tok / (ms_s * 1e-3), 1),
                  "GBps": round(tok_b * n_tok / (ms_s * 1e-3) / 1e9, 1),
                  "frac_of_measured_hbm": round(tok_b * n_tok / (ms_s * 1e-3) / 1e9 / peak, 3)}
@@ -918,10 +921,11 @@ def qtea_arm(args):
             "data": "synthetic",
             "config": {"workload": WORKLOAD, "M": 1, "shapes": [[g["name"], g["N"], g["K"], g["s"]] for g in layers[0]],
                        "layers_resident": args.layers, "resident_weight_bytes": resident, "l2_bytes": l2,
-                       "linear_tokens_per_s": round(args.steps / args.layers / (total_ms * 1e-3), 1),
                        "l2": "inputs larger than L2: steps rotate over the resident layers",
                        "parallelism": "replicas" if world > 1 else "single"},
             "us_per_call": per_shape,
+            # the 32-layer decode stack, called in a decoder's dependency order (4 calls per layer)
+            "linear_tokens_per_s": None if stack is None else stack["linear_tokens_per_s"],
             "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                          "frac": round(achieved / peak, 4), "peak_source": peak_src, "traffic": traffic,
                          "kernel": "qtea_gemv_m1_kernel", "launches_timed": args.steps,

@@ -62,9 +62,11 @@ typedef enum qtea_option {
   QTEA_OPT_BIAS = 1,         /* row_scale holds (alpha, beta) pairs: fp16 [N][G][2] (Eq. 4's beta) */
   QTEA_OPT_RESIDUAL_FP8 = 2, /* residual_vals holds FP8 E4M3 bytes [N/4][s] (Sec. 4.1), passed
                                 through the same pointer argument */
-  QTEA_OPT_FIXED_POINT = 4   /* base-3 layouts: batch-1 calls decode by the fixed-point
+  QTEA_OPT_FIXED_POINT = 4,  /* base-3 layouts: batch-1 calls decode by the fixed-point
                                 dot-product kernel instead of the paper's sign-symmetric lookup
                                 table (Sec. 3.5, Appendix A), the default */
+  QTEA_OPT_STREAM_K = 8      /* 2-bit layouts: batch-1 calls always take the stream-K kernel, never
+                                the row-resident one (see qtea_gemv_grouped) */
 } qtea_option;
 
 /* Largest batch (rows of x) one qtea_gemv call accepts. */
@@ -92,7 +94,11 @@ typedef enum qtea_option {
  * column in the least significant digit); byte 25 holds three columns and two pad digits; pad
  * digits and columns >= K are digit 1.
  * Which kernel serves a call: the TMA batch-1 kernel takes 2-bit layouts with fp16 residual values
- * at M = 1 (one alpha per row, or alpha and beta per row or per 128-column group); the tensor-core
+ * at M = 1 (one alpha per row, or alpha and beta per row or per 128-column group), in one of two
+ * forms: a row-resident launch, where every CTA holds all the codes of its rows at once (taken when
+ * all of a call's batch-1 problems have one alpha per row, K <= 4096 and at most 256 salient
+ * columns, and fit one such launch: at most 32 rows per CTA with one or two CTAs per SM;
+ * a latency-bound form for small calls), else the persistent stream-K launch; the tensor-core
  * low-batch kernel takes those at M >= 2 and 2-bit layouts with FP8 residual values (groups of 128
  * columns, or beta absent) at any M; base-3 layouts
  * at M = 1 run on the paper's table-lookup decode (Sec. 3.5, Appendix A); base-3 layouts at
@@ -176,6 +182,26 @@ typedef struct qtea_gemv_problem {
  */
 int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, qtea_stream_t stream);
 
+/* The kernels that serve problems (see "Which kernel serves a call" at qtea_pack_layout). */
+typedef enum qtea_kernel {
+  QTEA_KERNEL_NONE = 0,         /* N = 0 (nothing to do) or K = 0 (y is zero-filled) */
+  QTEA_KERNEL_ROWS = 1,         /* batch-1, row-resident launch */
+  QTEA_KERNEL_STREAM_K = 2,     /* batch-1, persistent stream-K launch */
+  QTEA_KERNEL_LUT = 3,          /* the paper's table-lookup decode (base-3 codes, M = 1) */
+  QTEA_KERNEL_LOW_BATCH = 4,    /* tensor-core low-batch kernel (2-bit codes) */
+  QTEA_KERNEL_BASE3_FIXED = 5,  /* base-3 codes, v*x staged once per CTA in fixed point */
+  QTEA_KERNEL_PAPER = 6,        /* general kernel for the paper's storage */
+  QTEA_KERNEL_GENERIC = 7       /* general kernel */
+} qtea_kernel;
+
+/*
+ * The kernel that qtea_gemv_grouped(problems, n_problems, M, ...) would run for each problem:
+ * kernels[i] receives a qtea_kernel value for problems[i]. Host-side only: no device work, no
+ * synchronization. Arguments are validated as qtea_gemv_grouped validates them (same status
+ * codes); kernels is a host array of n_problems ints, unchanged on error.
+ */
+int qtea_gemv_plan(const qtea_gemv_problem* problems, int n_problems, int M, int* kernels);
+
 /* Release a layout and its device memory. NULL is ignored. The caller orders it after the
  * last qtea_gemv that uses the layout has completed; it synchronizes nothing itself. */
 void qtea_free(qtea_layout* layout);
@@ -223,6 +249,10 @@ typedef struct qtea_layout_desc {
   int batch1_kernel;        /* 1 if M = 1 calls run the TMA stream-K batch-1 kernel (2-bit codes,
                                fp16 residual values), 0 otherwise */
   int options;              /* QTEA_OPT_* flags */
+  int rows_kernel;          /* 1 if M = 1 calls may run the row-resident kernel instead (2-bit codes,
+                               one alpha per row, fp16 residual values, K <= 4096, n_salient <= 256,
+                               no QTEA_OPT_STREAM_K): they do when all of a call's batch-1 problems
+                               fit one launch of it */
 } qtea_layout_desc;
 
 int qtea_layout_describe(const qtea_layout* layout, qtea_layout_desc* out);

@@ -28,6 +28,7 @@ QTEA_FMT_BASE3 = 1
 QTEA_OPT_BIAS = 1
 QTEA_OPT_RESIDUAL_FP8 = 2
 QTEA_OPT_FIXED_POINT = 4
+QTEA_OPT_STREAM_K = 8
 QTEA_MAX_M = 16
 
 _lib = None
@@ -48,7 +49,8 @@ class _Problem(ctypes.Structure):
 class _LayoutDesc(ctypes.Structure):
     _fields_ = [("N", ctypes.c_int), ("K", ctypes.c_int), ("K_pad", ctypes.c_int), ("group_size", ctypes.c_int),
                 ("n_salient", ctypes.c_int), ("format", ctypes.c_int), ("packed_bytes", ctypes.c_size_t),
-                ("packed_data", ctypes.c_void_p), ("batch1_kernel", ctypes.c_int), ("options", ctypes.c_int)]
+                ("packed_data", ctypes.c_void_p), ("batch1_kernel", ctypes.c_int), ("options", ctypes.c_int),
+                ("rows_kernel", ctypes.c_int)]
 
 
 def library_path() -> str:
@@ -79,6 +81,8 @@ def load(build_if_missing: bool = True):
     lib.qtea_device_status.argtypes = [P, P]
     lib.qtea_gemv_grouped.restype = i32
     lib.qtea_gemv_grouped.argtypes = [P, i32, i32, P]
+    lib.qtea_gemv_plan.restype = i32
+    lib.qtea_gemv_plan.argtypes = [P, i32, i32, P]
     lib.qtea_set_activation_precision.restype = i32
     lib.qtea_set_activation_precision.argtypes = [P, i32]
     lib.qtea_set_layout_options.restype = i32
@@ -230,12 +234,7 @@ def qtea_gemv(x, layout: Layout, row_scale, col_scale, salient_idx=None, residua
     return y
 
 
-def qtea_gemv_grouped(problems, stream=None):
-    """Several independent GEMVs in as few launches as possible.
-
-    `problems` is a sequence of dicts with keys x, layout, row_scale, col_scale and optionally
-    salient_idx, residual_vals, residual_idx, y. Returns the list of y tensors.
-    """
+def _problem_array(problems):
     ys, arr, M = [], (_Problem * max(len(problems), 1))(), None
     for i, q in enumerate(problems):
         args, y, m = _problem_args(q["x"], q["layout"], q["row_scale"], q["col_scale"], q.get("salient_idx"),
@@ -247,10 +246,34 @@ def qtea_gemv_grouped(problems, stream=None):
         args[1] = args[1].value
         arr[i] = _Problem(*args)
         ys.append(y)
-    rc = load().qtea_gemv_grouped(ctypes.cast(arr, ctypes.c_void_p), len(problems), M or 1, _stream(stream))
+    return arr, ys, M or 1
+
+
+def qtea_gemv_grouped(problems, stream=None):
+    """Several independent GEMVs in as few launches as possible.
+
+    `problems` is a sequence of dicts with keys x, layout, row_scale, col_scale and optionally
+    salient_idx, residual_vals, residual_idx, y. Returns the list of y tensors.
+    """
+    arr, ys, M = _problem_array(problems)
+    rc = load().qtea_gemv_grouped(ctypes.cast(arr, ctypes.c_void_p), len(problems), M, _stream(stream))
     if rc:
         raise QteaError(rc, "qtea_gemv_grouped")
     return ys
+
+
+QTEA_KERNEL_NAMES = {0: "none", 1: "rows", 2: "stream_k", 3: "lut", 4: "low_batch", 5: "base3_fixed", 6: "paper",
+                     7: "generic"}
+
+
+def qtea_gemv_plan(problems) -> list:
+    """The kernel qtea_gemv_grouped(problems) would run for each problem, by name (QTEA_KERNEL_NAMES)."""
+    arr, _, M = _problem_array(problems)
+    out = (ctypes.c_int * max(len(problems), 1))()
+    rc = load().qtea_gemv_plan(ctypes.cast(arr, ctypes.c_void_p), len(problems), M, ctypes.cast(out, ctypes.c_void_p))
+    if rc:
+        raise QteaError(rc, "qtea_gemv_plan")
+    return [QTEA_KERNEL_NAMES[out[i]] for i in range(len(problems))]
 
 
 def qtea_device_status(layout: Layout, stream=None) -> int:

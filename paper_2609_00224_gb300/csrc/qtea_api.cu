@@ -67,6 +67,16 @@ int plan_m1(qtea_layout* l, const cudaDeviceProp& prop) {
                       CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   if (r != CUDA_SUCCESS) return QTEA_OK;
+  {
+    // the row-resident kernel: the same codes in boxes of 8 rows
+    cuuint32_t box8[2] = {(cuuint32_t)kChunkRowBytes, (cuuint32_t)kRowsBoxRows};
+    l->rows_ok = encode(&l->tmap8, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, l->packed, dims, strides, box8, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS &&
+                 rows_configure(prop.sharedMemPerBlockOptin) == cudaSuccess;
+    if (!l->rows_ok) cudaGetLastError();
+    l->rows_smem_optin = prop.sharedMemPerBlockOptin;
+  }
   size_t dyn_max = 0;
   if (m1_configure(prop.sharedMemPerBlockOptin, &dyn_max) != cudaSuccess) {
     cudaGetLastError();
@@ -510,11 +520,11 @@ void group_reset(M1Group& g) {
   g.gp.total_units = 0;
 }
 
-// Add problem q; false if the group is full.
-bool group_add(M1Group& g, const qtea_gemv_problem& q) {
-  if (g.gp.n_problems == kMaxProblems) return false;
+// The batch-1 kernels' record of problem q (the split-tile fields point at the layout's resources).
+ProblemArgs problem_args(const qtea_gemv_problem& q) {
   const qtea_layout* l = q.packed_ternary;
-  ProblemArgs& a = g.gp.prob[g.gp.n_problems];
+  ProblemArgs a;
+  std::memset(&a, 0, sizeof(a));
   a.x = q.x;
   a.alpha = q.row_scale;
   a.v = q.col_scale;
@@ -537,6 +547,15 @@ bool group_add(M1Group& g, const qtea_gemv_problem& q) {
   a.gflags = (groups ? kScaleGroups : 0) | (bias ? kScaleBias : 0) | (vec ? kScaleVec : 0);
   a.vec_xv = aligned(q.x, 16) && aligned(q.col_scale, 16);
   a.vec_res = (l->n_salient % kResBlock == 0) && aligned(q.residual_vals, 16) && aligned(q.residual_idx, 2);
+  return a;
+}
+
+// Add problem q; false if the group is full.
+bool group_add(M1Group& g, const qtea_gemv_problem& q) {
+  if (g.gp.n_problems == kMaxProblems) return false;
+  const qtea_layout* l = q.packed_ternary;
+  ProblemArgs& a = g.gp.prob[g.gp.n_problems];
+  a = problem_args(q);
   a.unit_begin = g.gp.total_units;
   std::memcpy(&g.maps.m[g.gp.n_problems], &l->tmap, sizeof(CUtensorMap));
   if (g.gp.n_problems == 0) g.gp.status = l->status;
@@ -595,6 +614,119 @@ int run_m1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st, 
     i += taken;
   }
   return QTEA_OK;
+}
+
+// ---------------------------------------------------------------- row-resident batch-1 kernel
+// Layouts it may serve: 2-bit codes, one alpha per row, fp16 residual values, one 512-column
+// chunk per warp (K <= 4096), at most kRowsMaxSalient salient columns, not pinned to the
+// stream-K kernel.
+bool rows_capable(const qtea_layout* l) {
+  return l->rows_ok && l->m1_ok && l->format == QTEA_FMT_2BIT && l->group_size == l->K &&
+         (l->options & (QTEA_OPT_BIAS | QTEA_OPT_RESIDUAL_FP8 | QTEA_OPT_STREAM_K)) == 0 &&
+         l->n_chunks <= kRowsWarps && l->n_salient <= kRowsMaxSalient;
+}
+
+struct RowsLaunch {
+  RowsParams rp;
+  TensorMaps maps;
+  int grid = 0;
+  size_t smem = 0;
+};
+
+// CTAs per problem for a grid of at most `ctas`: in proportion to its codes (at least one), then
+// one at a time to the problem with the most codes per CTA. Returns the rows of the largest CTA.
+long long rows_split(const long long* blocks, const int* chunks, int n, int ctas, int* cnt) {
+  long long total = 0;
+  for (int i = 0; i < n; ++i) total += blocks[i] * chunks[i];
+  int used = 0;
+  for (int i = 0; i < n; ++i) {
+    long long c = (long long)ctas * blocks[i] * chunks[i] / total;
+    if (c < 1) c = 1;
+    if (c > blocks[i]) c = blocks[i];
+    cnt[i] = (int)c;
+    used += cnt[i];
+  }
+  auto cost = [&](int i) { return (blocks[i] + cnt[i] - 1) / cnt[i] * chunks[i]; };
+  while (used > ctas) {  // the one-CTA minimums overshot: take from the cheapest per CTA
+    int best = -1;
+    for (int i = 0; i < n; ++i)
+      if (cnt[i] > 1 && (best < 0 || cost(i) < cost(best))) best = i;
+    if (best < 0) return -1;
+    --cnt[best];
+    --used;
+  }
+  while (used < ctas) {
+    int best = -1;
+    for (int i = 0; i < n; ++i)
+      if (cnt[i] < blocks[i] && (best < 0 || cost(i) > cost(best))) best = i;
+    if (best < 0) break;
+    ++cnt[best];
+    ++used;
+  }
+  long long rows = 0;
+  for (int i = 0; i < n; ++i) {
+    const long long r = (blocks[i] + cnt[i] - 1) / cnt[i] * kRowsBoxRows;
+    rows = r > rows ? r : rows;
+  }
+  return rows;
+}
+
+// One row-resident launch for problems idx[0 .. n): one CTA per SM where that leaves every CTA
+// kRowsMaxRows rows or fewer (one per lane), else two CTAs per SM. False if the problems do not
+// fit: more problems than CTAs, more than kRowsMaxRows rows in a CTA, or shared memory beyond the
+// device's limit.
+bool rows_plan(const qtea_gemv_problem* qs, const int* idx, int n, RowsLaunch& L) {
+  if (n < 1 || n > kMaxProblems) return false;
+  const qtea_layout* l0 = qs[idx[0]].packed_ternary;
+  const int sm = l0->sm_count;
+  if (n > sm || 2 * sm > kMaxGrid) return false;
+  long long blocks[kMaxProblems];
+  int chunks[kMaxProblems], cnt[kMaxProblems], nch_max = 0;
+  for (int i = 0; i < n; ++i) {
+    const qtea_layout* l = qs[idx[i]].packed_ternary;
+    if (!rows_capable(l) || l->sm_count != sm || l->device != l0->device) return false;
+    blocks[i] = (l->N + kRowsBoxRows - 1) / kRowsBoxRows;
+    chunks[i] = l->n_chunks;
+    nch_max = chunks[i] > nch_max ? chunks[i] : nch_max;
+  }
+  long long rows_cap = rows_split(blocks, chunks, n, sm, cnt);
+  if (rows_cap > kRowsMaxRows) {
+    int cnt2[kMaxProblems];
+    const long long r2 = rows_split(blocks, chunks, n, 2 * sm, cnt2);
+    if (r2 > 0 && r2 <= kRowsMaxRows) {
+      rows_cap = r2;
+      for (int i = 0; i < n; ++i) cnt[i] = cnt2[i];
+    }
+  }
+  if (rows_cap < 1 || rows_cap > kRowsMaxRows) return false;
+  const RowsSmem so = rows_smem_layout((int)rows_cap, nch_max);
+  if (so.total > l0->rows_smem_optin) return false;
+  std::memset(&L.rp, 0, sizeof(L.rp));
+  int b = 0;
+  for (int i = 0; i < n; ++i) {
+    const qtea_gemv_problem& q = qs[idx[i]];
+    L.rp.prob[i] = problem_args(q);
+    L.rp.cta_begin[i] = b;
+    b += cnt[i];
+    std::memcpy(&L.maps.m[i], &q.packed_ternary->tmap8, sizeof(CUtensorMap));
+  }
+  L.rp.cta_begin[n] = b;
+  L.rp.rows_cap = (int)rows_cap;
+  L.rp.n_chunks_max = nch_max;
+  L.rp.n_problems = n;
+  L.rp.status = l0->status;
+  L.grid = b;
+  L.smem = so.total;
+  return true;
+}
+
+// Batch-1 dispatch of problems idx[0 .. n): one row-resident launch when all of them fit it, else
+// the stream-K kernel.
+int run_batch1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st) {
+  RowsLaunch L;
+  if (rows_plan(qs, idx, n, L))
+    return launch_rows(L.maps, L.rp, L.grid, L.smem, st) == cudaSuccess ? QTEA_OK : QTEA_ERR_CUDA;
+  return run_m1(qs, idx, n, st);
 }
 
 // ---------------------------------------------------------------- allocation-free batch-1 entry
@@ -742,7 +874,23 @@ int qtea_pack_layout(const int8_t* ternary_codes, int N, int K, int group_size, 
   return QTEA_OK;
 }
 
-int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, qtea_stream_t stream) {
+namespace {
+
+// Which path serves problem q at batch M (before the batch-1 choice between the two launch forms).
+enum Route { kRouteNone, kRouteZero, kRouteBatch1, kRouteLut, kRouteMb, kRouteB3, kRoutePaper, kRouteGeneric };
+
+Route route(const qtea_gemv_problem& q, int M) {
+  const qtea_layout* l = q.packed_ternary;
+  if (l->N == 0) return kRouteNone;
+  if (l->K == 0) return kRouteZero;
+  if (M == 1 && l->m1_ok && m1_capable(l)) return kRouteBatch1;
+  if (lut_eligible(l, M)) return kRouteLut;
+  if (mb_capable(l, M)) return kRouteMb;
+  if (is_paper(l)) return b3_eligible(paper_params(q, M)) ? kRouteB3 : kRoutePaper;
+  return kRouteGeneric;
+}
+
+int check_call(const qtea_gemv_problem* problems, int n_problems, int M) {
   if (n_problems < 0 || (n_problems > 0 && !problems)) return QTEA_ERR_INVALID_ARG;
   if (M < 1 || M > QTEA_MAX_M) return QTEA_ERR_INVALID_ARG;
   for (int i = 0; i < n_problems; ++i) {
@@ -751,52 +899,93 @@ int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, 
     for (int j = 0; j < i; ++j)  // a layout's split-K workspace serves one problem per call
       if (problems[j].packed_ternary == problems[i].packed_ternary) return QTEA_ERR_INVALID_ARG;
   }
+  return QTEA_OK;
+}
+
+}  // namespace
+
+int qtea_gemv_grouped(const qtea_gemv_problem* problems, int n_problems, int M, qtea_stream_t stream) {
+  int rc = check_call(problems, n_problems, M);
+  if (rc) return rc;
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   int* m1_idx = n_problems > 0 ? static_cast<int*>(std::malloc(sizeof(int) * 2 * (size_t)n_problems)) : nullptr;
   if (n_problems > 0 && !m1_idx) return QTEA_ERR_ALLOC;
   int* mb_idx = m1_idx + n_problems;
   int b3_idx[8];
-  int n_m1 = 0, n_mb = 0, n_b3 = 0, n_lut = 0, rc = QTEA_OK;
+  int n_m1 = 0, n_mb = 0, n_b3 = 0, n_lut = 0;
   int lut_idx[kMaxProblems];
   for (int i = 0; i < n_problems && rc == QTEA_OK; ++i) {
     const qtea_gemv_problem& q = problems[i];
-    const qtea_layout* l = q.packed_ternary;
-    if (l->N == 0) continue;
-    if (l->K == 0) {
-      if (cudaMemsetAsync(q.y, 0, (size_t)M * l->N * sizeof(float), st) != cudaSuccess) rc = QTEA_ERR_CUDA;
-      continue;
-    }
-    if (M == 1 && l->m1_ok && m1_capable(l)) {
-      m1_idx[n_m1++] = i;
-    } else if (lut_eligible(l, M)) {
-      lut_idx[n_lut++] = i;
-      if (n_lut == kMaxProblems) {
-        rc = run_lut(problems, lut_idx, n_lut, st);
-        n_lut = 0;
-      }
-    } else if (mb_capable(l, M)) {
-      mb_idx[n_mb++] = i;
-    } else if (is_paper(l)) {
-      if (b3_eligible(paper_params(q, M))) {
+    switch (route(q, M)) {
+      case kRouteNone:
+        break;
+      case kRouteZero:
+        if (cudaMemsetAsync(q.y, 0, (size_t)M * q.packed_ternary->N * sizeof(float), st) != cudaSuccess)
+          rc = QTEA_ERR_CUDA;
+        break;
+      case kRouteBatch1:
+        m1_idx[n_m1++] = i;
+        break;
+      case kRouteLut:
+        lut_idx[n_lut++] = i;
+        if (n_lut == kMaxProblems) {
+          rc = run_lut(problems, lut_idx, n_lut, st);
+          n_lut = 0;
+        }
+        break;
+      case kRouteMb:
+        mb_idx[n_mb++] = i;
+        break;
+      case kRouteB3:
         b3_idx[n_b3++] = i;
         if (n_b3 == 8) {
           rc = run_b3(problems, b3_idx, n_b3, M, st);
           n_b3 = 0;
         }
-      } else {
+        break;
+      case kRoutePaper:
         rc = launch_paper_problem(q, M, st);
-      }
-    } else {
-      rc = launch_generic_problem(q, M, st);
+        break;
+      case kRouteGeneric:
+        rc = launch_generic_problem(q, M, st);
+        break;
     }
   }
   if (rc == QTEA_OK && n_b3 > 0) rc = run_b3(problems, b3_idx, n_b3, M, st);
   if (rc == QTEA_OK && n_lut > 0) rc = run_lut(problems, lut_idx, n_lut, st);
-  if (rc == QTEA_OK && n_m1 > 0) rc = run_m1(problems, m1_idx, n_m1, st);
+  if (rc == QTEA_OK && n_m1 > 0) rc = run_batch1(problems, m1_idx, n_m1, st);
   if (rc == QTEA_OK && n_mb > 0) rc = run_mb(problems, mb_idx, n_mb, M, st);
   std::free(m1_idx);
   if (rc != QTEA_OK) cudaGetLastError();
   return rc;
+}
+
+int qtea_gemv_plan(const qtea_gemv_problem* problems, int n_problems, int M, int* kernels) {
+  if (n_problems > 0 && !kernels) return QTEA_ERR_INVALID_ARG;
+  int rc = check_call(problems, n_problems, M);
+  if (rc) return rc;
+  int m1_idx[kMaxProblems], n_m1 = 0;
+  bool m1_many = false;
+  for (int i = 0; i < n_problems; ++i) {
+    switch (route(problems[i], M)) {
+      case kRouteNone:
+      case kRouteZero: kernels[i] = QTEA_KERNEL_NONE; break;
+      case kRouteBatch1:
+        kernels[i] = QTEA_KERNEL_STREAM_K;
+        if (n_m1 < kMaxProblems) m1_idx[n_m1++] = i;
+        else m1_many = true;
+        break;
+      case kRouteLut: kernels[i] = QTEA_KERNEL_LUT; break;
+      case kRouteMb: kernels[i] = QTEA_KERNEL_LOW_BATCH; break;
+      case kRouteB3: kernels[i] = QTEA_KERNEL_BASE3_FIXED; break;
+      case kRoutePaper: kernels[i] = QTEA_KERNEL_PAPER; break;
+      case kRouteGeneric: kernels[i] = QTEA_KERNEL_GENERIC; break;
+    }
+  }
+  RowsLaunch L;
+  if (!m1_many && n_m1 > 0 && rows_plan(problems, m1_idx, n_m1, L))
+    for (int k = 0; k < n_m1; ++k) kernels[m1_idx[k]] = QTEA_KERNEL_ROWS;
+  return QTEA_OK;
 }
 
 int qtea_gemv(const uint16_t* x, const qtea_layout* l, const uint16_t* row_scale, const uint16_t* col_scale,
@@ -827,6 +1016,7 @@ int qtea_layout_describe(const qtea_layout* l, qtea_layout_desc* out) {
   out->packed_bytes = l->packed_bytes;
   out->packed_data = l->packed;
   out->batch1_kernel = (l->m1_ok && m1_capable(l)) ? 1 : 0;
+  out->rows_kernel = rows_capable(l) ? 1 : 0;
   out->options = l->options;
   return QTEA_OK;
 }
@@ -868,7 +1058,8 @@ int qtea_quantize(const float* W, const float* hdiag, int N, int K, int group_si
 }
 
 int qtea_set_layout_options(qtea_layout* l, int options) {
-  if (!l || (options & ~(QTEA_OPT_BIAS | QTEA_OPT_RESIDUAL_FP8 | QTEA_OPT_FIXED_POINT)) != 0) return QTEA_ERR_INVALID_ARG;
+  if (!l || (options & ~(QTEA_OPT_BIAS | QTEA_OPT_RESIDUAL_FP8 | QTEA_OPT_FIXED_POINT | QTEA_OPT_STREAM_K)) != 0)
+    return QTEA_ERR_INVALID_ARG;
   l->options = options;
   return QTEA_OK;
 }

@@ -116,6 +116,47 @@ __host__ __device__ constexpr size_t m1_smem_bytes(int S) {
          (size_t)(2 * S + 3 * kAuxSlots) * sizeof(unsigned long long) + (size_t)kMaxStages * sizeof(int) + 1024;
 }
 
+// ---------------------------------------------------------------- row-resident batch-1 kernel (small groups)
+// For small groups with K <= 4096: every CTA owns whole rows (up to kRowsMaxRows, in 8-row
+// blocks; one or two CTAs per SM) of one problem, so no partial sums cross CTAs. Its codes arrive by TMA before the grid
+// dependency wait, one barrier per 512-column chunk (8-row boxes of 128 bytes, 128-byte swizzle);
+// each of the eight warps stages the planes of one chunk and decodes it for all of the CTA's rows.
+constexpr int kRowsWarps = 8;
+constexpr int kRowsThreads = kRowsWarps * 32;                  // 256
+constexpr int kRowsMaxRows = 32;                               // one row per lane
+constexpr int kRowsBoxRows = 8;
+constexpr int kRowsSlotBytes = 1792;                           // planes + ChunkMeta of one chunk, per warp
+constexpr int kRowsMaxSalient = 256;                           // salient columns (half of them in registers)
+
+struct RowsParams {
+  ProblemArgs prob[kMaxProblems];   // as for the stream-K kernel (ws, counters, n_tiles, unit_begin unused)
+  int cta_begin[kMaxProblems + 1];  // CTAs of problem p: [cta_begin[p], cta_begin[p + 1])
+  int rows_cap;                     // rows of a CTA's buffer per chunk (multiple of 8, at most kRowsMaxRows)
+  int n_chunks_max;                 // over the problems: shared-memory size
+  int n_problems;
+  int* status;                      // device status word (the first layout's)
+};
+
+// Dynamic shared memory of the row-resident kernel (offsets from the 1024-byte aligned base):
+// codes [n_chunks_max][rows_cap][128], the warps' plane slots, their partial row sums, the
+// residual per row, the CTA's problem record, the code barriers, and 1024 bytes of slack.
+struct RowsSmem {
+  size_t slots, dec, res, args, bars, total;
+};
+__host__ __device__ inline RowsSmem rows_smem_layout(int rows_cap, int n_chunks_max) {
+  RowsSmem o;
+  o.slots = (size_t)n_chunks_max * rows_cap * kChunkRowBytes;
+  o.dec = o.slots + (size_t)kRowsWarps * kRowsSlotBytes;
+  o.res = o.dec + (size_t)kRowsWarps * kRowsMaxRows * sizeof(float);
+  o.args = o.res + (size_t)kRowsMaxRows * sizeof(float);
+  o.bars = o.args + sizeof(ProblemArgs);
+  o.total = o.bars + (size_t)n_chunks_max * sizeof(unsigned long long) + 1024;
+  return o;
+}
+
+cudaError_t rows_configure(size_t smem_optin);
+cudaError_t launch_rows(const TensorMaps& maps, const RowsParams& p, int grid, size_t smem, cudaStream_t st);
+
 // ---------------------------------------------------------------- low-batch tensor-core kernel (2 <= M <= 16)
 constexpr int kMaxStagesMb = 6;
 constexpr int kMinStagesMb = 2;
@@ -449,6 +490,9 @@ struct qtea_layout {
   unsigned* counters;    // [n_tiles][kConsumerWarps]
   int* status;
   CUtensorMap tmap;
+  bool rows_ok;          // the row-resident kernel is configured and tmap8 encoded
+  CUtensorMap tmap8;     // the codes in boxes of 8 rows x 128 bytes (row-resident kernel)
+  size_t rows_smem_optin;  // dynamic shared memory the row-resident kernel may use
   // low-batch kernel resources
   bool mb_ok;
   size_t mb_smem_optin;

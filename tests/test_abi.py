@@ -57,6 +57,14 @@ def test_host_side_argument_checks_need_no_gpu():
     assert q(P, P, 4, 256, 64, 0, 0, 2, 2, P, P, P, None, None, None, None) == qt.QTEA_ERR_UNSUPPORTED  # group
     assert q(P, P, 4, 8, 8, 0, 4, 2, 2, P, P, P, None, None, None, None) == qt.QTEA_ERR_INVALID_ARG  # option
     assert q(P, P, 4, 8, 8, 0, 0, -1, 2, P, P, P, None, None, None, None) == qt.QTEA_ERR_INVALID_ARG  # iters
+    out4 = (ctypes.c_int * 4)(9, 9, 9, 9)
+    nul = (ctypes.c_void_p * 8)()  # one problem, every pointer NULL: no layout
+    assert lib.qtea_gemv_plan(None, -1, 1, out4) == qt.QTEA_ERR_INVALID_ARG
+    assert lib.qtea_gemv_plan(nul, 1, 1, None) == qt.QTEA_ERR_INVALID_ARG
+    assert lib.qtea_gemv_plan(nul, 1, 0, out4) == qt.QTEA_ERR_INVALID_ARG  # M < 1
+    assert lib.qtea_gemv_plan(nul, 1, 1, out4) == qt.QTEA_ERR_INVALID_ARG  # no layout
+    assert list(out4) == [9, 9, 9, 9]  # unchanged on error
+    assert lib.qtea_gemv_plan(None, 0, 1, None) == qt.QTEA_OK
     lib.qtea_free(None)
 
 

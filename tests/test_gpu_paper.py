@@ -120,7 +120,7 @@ def test_options_switch_a_default_layout_to_the_paper_path(qt):
     layout.set_options(qt.QTEA_OPT_FIXED_POINT)  # a base-3 choice: a 2-bit layout stays on the batch-1 kernel
     assert layout.describe()["batch1_kernel"] == 1
     with pytest.raises(qt.QteaError):
-        layout.set_options(8)
+        layout.set_options(16)
 
 
 @pytest.mark.parametrize("matrix", range(7))

@@ -63,6 +63,8 @@ def test_static_entry_matches_qtea_gemv(qt, name, make):
     p = make()
     T = _dev(p.T)
     layout = qt.qtea_pack_layout(T, n_salient=p.s)
+    # the static entry runs the stream-K batch-1 kernel: qtea_gemv pinned to the same kernel agrees bitwise
+    layout.set_options(qt.QTEA_OPT_STREAM_K)
     packed = qt.packed_bytes(layout).clone()  # caller-owned copy of the 2-bit layout
     x = _dev(p.x.view(np.int16), torch.float16)
     alpha = _dev(p.alpha.reshape(-1).view(np.int16), torch.float16)
@@ -111,6 +113,7 @@ def test_static_entry_sees_codes_written_just_before_it(qt):
     q = synth.make_problem("other codes", p.N, p.K, 1, p.s, seed=77)
     lay_p = qt_.qtea_pack_layout(_dev(p.T), n_salient=p.s)
     lay_q = qt_.qtea_pack_layout(_dev(q.T), n_salient=p.s)
+    lay_q.set_options(qt_.QTEA_OPT_STREAM_K)  # the static entry's kernel, for a bitwise comparison
     codes_q = qt_.packed_bytes(lay_q).clone()
     packed = qt_.packed_bytes(lay_p).clone()
     x = _dev(p.x.view(np.int16), torch.float16)
