@@ -53,10 +53,10 @@ def profiled_traffic():
     matches the one that was profiled (else None)."""
     import hashlib
     prof = os.path.join(ROOT, "profiles", "qtea_gemv_m1_llama3_8b_layer.md")
-    src = os.path.join(ROOT, "paper_2609_00224_gb300", "csrc", "qtea_gemv_m1.cu")
+    srcs = [os.path.join(ROOT, "paper_2609_00224_gb300", "csrc", f) for f in ("qtea_gemv_m1.cu", "qtea_m1_device.h")]
     try:
         text = open(prof).read()
-        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        sha = hashlib.sha256(b"".join(open(f, "rb").read() for f in srcs)).hexdigest()[:16]
         fields = dict(l.split(":", 1) for l in text.splitlines() if l.startswith(("kernel_source_sha256_16:",
                                                                                    "traffic_bytes_per_launch:")))
         if fields.get("kernel_source_sha256_16", "").strip() != sha:
@@ -947,7 +947,10 @@ def profile_case(args):
 
       qwen3_14b_layer        the Qwen3-14B layer's seven GEMVs at batch --m, grouped (low-batch
                              kernel; batch-1 kernel at --m 1)
-      llama3_8b_layer        the Llama3-8B layer's seven GEMVs at batch 1, grouped (batch-1 kernel)
+      llama3_8b_layer        the Llama3-8B layer's seven GEMVs at batch 1, grouped (batch-1 stream-K
+                             kernel)
+      llama3_8b_qkv          the layer's q, k and v at batch 1, grouped (row-resident batch-1 kernel,
+                             two CTAs per SM), then o alone (one CTA per SM)
       llama3_8b_base3        the same in base-3 codes, one alpha per row (table-lookup kernel;
                              --fixed-point: the fixed-point base-3 kernel)
       llama3_8b_paper        the paper's storage (base-3, alpha and beta per 128 columns, FP8
@@ -993,6 +996,9 @@ def profile_case(args):
         layers = [layer("qwen3_14b_layer", li, work, M_=M) for li in range(n_layers)]
     elif case == "llama3_8b_layer":
         layers = [layer("llama3_8b_layer", li, work) for li in range(n_layers)]
+    elif case == "llama3_8b_qkv":
+        full = [layer("llama3_8b_layer", li, work) for li in range(n_layers)]
+        layers = [g for L in full for g in (L[:3], L[3:4])]
     elif case == "llama3_8b_base3":
         opts = qt.QTEA_OPT_FIXED_POINT if args.fixed_point else 0
         layers = [layer("llama3_8b_layer", li, work, fmt=qt.QTEA_FMT_BASE3, opts=opts) for li in range(n_layers)]
@@ -1067,7 +1073,7 @@ def main():
     ap.add_argument("--no-per-shape", action="store_true")
     ap.add_argument("--act-bits", type=int, choices=[16, 24], default=16,
                     help="activation precision of the timed region (24 = exact default, 16 = fast mode)")
-    ap.add_argument("--profile-case", choices=["qwen3_14b_layer", "llama3_8b_layer", "llama3_8b_base3",
+    ap.add_argument("--profile-case", choices=["qwen3_14b_layer", "llama3_8b_layer", "llama3_8b_qkv", "llama3_8b_base3",
                                                "llama3_8b_paper", "llama3_8b_paper_2bit", "unaligned_residual",
                                                "pack", "quantize"], default=None,
                     help="run a small fixed workload for profilers instead of the benchmark")
