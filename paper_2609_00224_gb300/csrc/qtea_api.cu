@@ -323,7 +323,8 @@ void mb_group_reset(MbGroup& g, int M, size_t prep_smem_optin, size_t smem_optin
   g.grp = false;
   g.gp.M = M;
   g.pg.M = M;
-  g.pg.mt = M <= 8 ? 1 : 2;
+  g.pg.mt = mb_mt(M);
+  g.gp.split = g.pg.split = mb_split(M) ? 1 : 0;
   g.grid = 0;
   g.smem = 0;
   g.prep_smem_optin = prep_smem_optin;
@@ -357,7 +358,7 @@ bool mb_group_add(MbGroup& g, const qtea_gemv_problem& q) {
   g.grp = grp;
   const int n_tiles = (l->N + kMbTileRows - 1) / kMbTileRows;
   const int s = l->n_salient, s16 = round_up(s, 16);
-  const int mt = g.gp.M <= 8 ? 1 : 2;
+  const int mt = mb_mt(g.gp.M);
   uint8_t* res_base = l->mb_ws + (size_t)l->n_chunks * kMbChunkWsBytes;
   float* yres = s > 0 ? reinterpret_cast<float*>(res_base) : nullptr;
   uint16_t* xs = s > 0 ? reinterpret_cast<uint16_t*>(res_base + (size_t)n_tiles * kMbResFloatsPerTile * sizeof(float))
@@ -439,7 +440,7 @@ bool mb_group_plan(MbGroup& g, int sm_count, size_t smem_optin) {
     if (g.gp.prob[k].res_mode == kMbResPrep) g.gp.fused = 0;
   if (g.gp.fused) {
     g.gp.prep = g.pg;
-    const int scratch = 16 * kChunkCols * 2 + kChunkCols * 2;  // prep_chunk's
+    const int scratch = kMbPrepScratch;  // the chunk build's
     if (g.gp.res_stage_bytes < scratch) g.gp.res_stage_bytes = scratch;
   }
   for (int S = kMaxStagesMb; S >= kMinStagesMb; --S) {

@@ -14,6 +14,12 @@
 //    gives (columns i and i + 8 of a word side by side), so v and x of each 512-column chunk are
 //    written once per call in exactly the register order the fragments need ("fragment order"):
 //    one 8-byte shared load per thread and step. Each MMA step stays inside one 128-column group.
+//  * Split encoding, M <= 4: v moves into B, so A = 2T needs only the shift and the mask. B holds
+//    v*x * 2^E (exact in fp32, E per chunk so that every value stays below 2^15) as two fp16
+//    columns per batch row, hi = fp16(v*x 2^E) and lo = fp16(v*x 2^E - hi), whose sum is exact;
+//    the tile's chunks are folded one by one with their 2^(-E-1). Rows whose code is 0 at a column
+//    contribute 0 there, as with 2T*v (an encoding by c = T + 1 would carry a large activation
+//    into every row's accumulator and lose the others' low bits to its alignment).
 //  * The residual of Eq. 11 is an exact contraction too: over "virtual columns", one per salient
 //    column, A holds the residual value (fp16, or FP8 E4M3 converted exactly) of the row's group
 //    where the stored position is the row and 0 elsewhere, and B holds x at the salient column.
@@ -104,17 +110,22 @@ __device__ __forceinline__ uint32_t e4m3_to_f16_bits(uint32_t b) {
 }
 
 // FP8: rv holds one E4M3 byte per entry (row stride rvs bytes), converted to fp16 exactly.
+// With the split encoding (split) B column n of tile j holds batch row 4j + n/2 for even n and zero
+// for odd n, so that the result sits where the decode's (hi, lo) pair of that batch row does.
 template <int NB, bool FP8 = false>
 __device__ __forceinline__ void res_step(const void* rv_, int rvs, const uint8_t* ri, int ris, const uint16_t* xr,
-                                         int xrs, int ne, int step, int tr, int g, int q, int mt, bool quad_loads,
-                                         float (&res)[NB][2][4]) {
+                                         int xrs, int ne, int step, int tr, int g, int q, int mt, bool split,
+                                         bool quad_loads, float (&res)[NB][2][4]) {
   const uint16_t* rv = static_cast<const uint16_t*>(rv_);
   const uint8_t* rv8 = static_cast<const uint8_t*>(rv_);
   const int e0 = step * 16 + 4 * q;
   const uint32_t pos = (uint32_t)(g & 3);  // row & 3 for every row of the thread
   uint2 xb[2];
 #pragma unroll
-  for (int j = 0; j < 2; ++j) xb[j] = *reinterpret_cast<const uint2*>(xr + (8 * j + g) * xrs + e0);
+  for (int j = 0; j < 2; ++j) {
+    if (split) xb[j] = (g & 1) ? make_uint2(0u, 0u) : *reinterpret_cast<const uint2*>(xr + (4 * j + (g >> 1)) * xrs + e0);
+    else xb[j] = *reinterpret_cast<const uint2*>(xr + (8 * j + g) * xrs + e0);
+  }
 #pragma unroll
   for (int b = 0; b < NB; ++b) {
     uint32_t a[4];
@@ -205,6 +216,82 @@ __device__ __forceinline__ void prep_chunk(const MbPrepProblem& p, int M, int mt
     sxv += __shfl_xor_sync(0xffffffffu, sxv, 1);
     sxv += __shfl_xor_sync(0xffffffffu, sxv, 2);
     if (part == 0) reinterpret_cast<float*>(out + kMbVBytes)[16 * k + m] = sxv;
+  }
+}
+
+// Largest of the lanes' non-negative values (their bit patterns order as unsigned integers).
+__device__ __forceinline__ float warp_max_nonneg(float v) {
+  return __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(v)));
+}
+
+// The split encoding's chunk (M <= 8): B = the exact fp16 split hi + lo of v*x * 2^E, with
+// E = 14 - floor(log2(max |v*x|)) over the chunk and all batch rows (every |v*x * 2^E| < 2^15, so
+// hi is finite; v*x is exact in fp32 and hi + lo holds all of its bits); in tile j, B column n is
+// hi (n even) or lo (n odd) of batch row 4j + n/2, zero for batch rows >= M. A is 2T (split_a), so
+// the head holds the fold factor 2^(-E-1) and, as for the other encoding, the sums of x per
+// 128-column group and batch row (the beta term). 256 threads (tid); sm holds kMbPrepScratch bytes;
+// sync() is a barrier over the 256 threads.
+template <typename Sync>
+__device__ __forceinline__ void prep_chunk_split(const MbPrepProblem& p, int M, int mt, int ch, int tid, uint8_t* sm,
+                                                 uint8_t* out, Sync sync) {
+  uint16_t(*xsm)[kChunkCols] = reinterpret_cast<uint16_t(*)[kChunkCols]>(sm);
+  uint16_t* vsm = reinterpret_cast<uint16_t*>(sm + 16 * kChunkCols * 2);
+  float* red = reinterpret_cast<float*>(sm + 16 * kChunkCols * 2 + kChunkCols * 2);  // [8] warp maxima
+  const int col0 = ch * kChunkCols;
+  float lmax = 0.f;
+#pragma unroll 2
+  for (int i = tid; i < kChunkCols; i += 256) {
+    const int col = col0 + i;
+    const bool in = col < p.K;
+    const uint16_t vb = in ? __ldg(p.v + col) : (uint16_t)0;
+    vsm[i] = vb;
+    const float vf = h2f(vb);
+    uint16_t xv[16];
+#pragma unroll
+    for (int m = 0; m < 16; ++m) xv[m] = (in && m < M) ? __ldg(p.x + (size_t)m * p.K + col) : (uint16_t)0;
+#pragma unroll
+    for (int m = 0; m < 16; ++m) {
+      xsm[m][i] = xv[m];
+      lmax = fmaxf(lmax, fabsf(vf * h2f(xv[m])));
+    }
+  }
+  lmax = warp_max_nonneg(lmax);
+  if ((tid & 31) == 0) red[tid >> 5] = lmax;
+  sync();
+  float amax = 0.f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) amax = fmaxf(amax, red[w]);
+  // |v*x| >= 2^-48 when nonzero (products of binary16 values), so amax is an fp32 normal number
+  const int e = amax > 0.f ? (int)((__float_as_uint(amax) >> 23) & 0xffu) - 127 : 0;
+  const float sc = __uint_as_float((uint32_t)(141 - e) << 23);  // 2^E, E = 14 - e
+  auto half_of = [&](const uint16_t* row, int c, int h) -> uint32_t {
+    const float f = (h2f(vsm[c]) * h2f(row[c])) * sc;  // exact: a power-of-two multiple of v*x
+    const __half hi = __float2half_rn(f);
+    if (h == 0) return (uint32_t)__half_as_ushort(hi);
+    return (uint32_t)__half_as_ushort(__float2half_rn(f - __half2float(hi)));
+  };
+  for (int idx = tid; idx < mt * 1024; idx += 256) {
+    const int j = idx >> 10, st = (idx >> 5) & 31, lane = idx & 31, g = lane >> 2, q = lane & 3;
+    const int m = 4 * j + (g >> 1), h = g & 1;
+    const int c0 = 16 * (4 * (st >> 2) + q) + 2 * (st & 3), c1 = c0 + 1;
+    uint2 o = make_uint2(0u, 0u);
+    if (m < M) {
+      o.x = half_of(xsm[m], c0, h) | (half_of(xsm[m], c0 + 8, h) << 16);
+      o.y = half_of(xsm[m], c1, h) | (half_of(xsm[m], c1 + 8, h) << 16);
+    }
+    reinterpret_cast<uint2*>(out + kMbChunkHead)[idx] = o;
+  }
+  {
+    // sum of x over each 128-column group k of the chunk for batch row m (the beta term of Eq. 10):
+    // four lanes per (k, m) add 32 columns each, then a fixed butterfly
+    const int k = tid >> 6, m = (tid >> 2) & 15, part = tid & 3;
+    float sxv = 0.f;
+#pragma unroll 8
+    for (int c = 0; c < 32; ++c) sxv += h2f(xsm[m][128 * k + 32 * part + c]);
+    sxv += __shfl_xor_sync(0xffffffffu, sxv, 1);
+    sxv += __shfl_xor_sync(0xffffffffu, sxv, 2);
+    if (part == 0) reinterpret_cast<float*>(out + kMbVBytes)[16 * k + m] = sxv;
+    if (tid == 0) *reinterpret_cast<float*>(out + kMbHlF) = __uint_as_float((uint32_t)(112 + e) << 23);  // 2^(-E-1)
   }
 }
 
@@ -330,10 +417,10 @@ __global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant
       const bool quad = (rvs & 3) == 0 && (p.native ? (ne & 3) == 0 : true);
       if (quad) {
         for (int step = 0; step * 16 < ne; ++step)
-          res_step<kMbBlocks>(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, true, res);
+          res_step<kMbBlocks>(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, gr.split != 0, true, res);
       } else {
         for (int step = 0; step * 16 < ne; ++step)
-          res_step<kMbBlocks>(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, false, res);
+          res_step<kMbBlocks>(rv, rvs, ri, ris, xr, xrs, ne, step, tr, g, q, gr.mt, gr.split != 0, false, res);
       }
       __syncthreads();
     }
@@ -345,7 +432,10 @@ __global__ void __launch_bounds__(256) qtea_mb_prep_kernel(const __grid_constant
         if (j < gr.mt) dst[b * gr.mt + j] = make_float4(res[b][j][0], res[b][j][1], res[b][j][2], res[b][j][3]);
     return;
   }
-  prep_chunk(p, M, gr.mt, local, tid, sm, p.ws + (size_t)local * kMbChunkWsBytes, [] { __syncthreads(); });
+  if (gr.split)
+    prep_chunk_split(p, M, gr.mt, local, tid, sm, p.ws + (size_t)local * kMbChunkWsBytes, [] { __syncthreads(); });
+  else
+    prep_chunk(p, M, gr.mt, local, tid, sm, p.ws + (size_t)local * kMbChunkWsBytes, [] { __syncthreads(); });
 }
 
 // ---------------------------------------------------------------- decode of one unit
@@ -378,11 +468,57 @@ __device__ __forceinline__ void group_fold(const uint8_t* sb, int tr, int g, int
     }
 }
 
+// Split encoding: the accumulated steps of 128-column group k (or of the whole chunk, k < 0, without
+// scale groups) folded into run: for batch row m = 4j + q, sum_j T v x = (D_hi + D_lo) * 2^(-E-1)
+// (A = 2T, B = v*x 2^E); with scale groups times alpha_k plus beta_k times the group's sum of x
+// (Eq. 10 per group). Only run[.][.][0] (row g) and [2] (row g + 8) carry values. acc = 0 afterwards.
+template <int MT, bool GRP>
+__device__ __forceinline__ void split_fold(const uint8_t* sb, int tr, int g, int q, int k, int ch_odd, bool bias,
+                                           float (&acc)[2][kMbBlocks][MT][4], float (&run)[kMbBlocks][MT][4]) {
+  const uint8_t* head = sb + kMbCodeBytes;
+  const float F = *reinterpret_cast<const float*>(head + kMbHlF);
+  const float* sx = reinterpret_cast<const float*>(head + kMbVBytes);
+  const uint16_t* ab = reinterpret_cast<const uint16_t*>(sb + kMbCodeBytes + kMbChunkHead + MT * kMbXTileBytes);
+#pragma unroll
+  for (int j = 0; j < MT; ++j) {
+    const float bx = GRP ? sx[16 * k + 4 * j + q] : 0.f;
+#pragma unroll
+    for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const float d = (acc[0][b][j][2 * h] + acc[0][b][j][2 * h + 1]) + (acc[1][b][j][2 * h] + acc[1][b][j][2 * h + 1]);
+        if (GRP) {
+          const uint16_t* r = ab + (tr + 16 * b + 8 * h + g) * 8;
+          const float al = __half2float(__ushort_as_half(bias ? r[2 * k] : r[4 * ch_odd + k]));
+          const float be = bias ? __half2float(__ushort_as_half(r[2 * k + 1])) : 0.f;
+          run[b][j][2 * h] += fmaf(al * F, d, be * bx);
+        } else {
+          run[b][j][2 * h] = fmaf(d, F, run[b][j][2 * h]);
+        }
+        acc[0][b][j][2 * h] = acc[1][b][j][2 * h] = 0.f;
+        acc[0][b][j][2 * h + 1] = acc[1][b][j][2 * h + 1] = 0.f;
+      }
+  }
+}
+
+// Split encoding, A = 2T of columns I and I + 8 of code word w: a left shift by 14 - 2I puts their
+// codes c = T + 1 at bits 14-15 and 30-31, and one LOP3 (~w & 0xC000C000) turns each into the fp16
+// value -2, -0 or +2 (sign bit and the top exponent bit). The shift is written as a multiply, which
+// may issue on the multiply pipe beside the masks.
+template <int I>
+__device__ __forceinline__ uint32_t split_a(uint32_t w) {
+  uint32_t t;
+  asm("mul.lo.u32 %0, %1, %2;" : "=r"(t) : "r"(w), "n"(1u << (14 - 2 * I)));
+  return ~t & 0xC000C000u;
+}
+
 // The unit's 32 steps of 16 columns for the warp's 16-row blocks (rows tr + 16b + g and + 8 of the
 // stage); even steps accumulate into acc[0], odd steps into acc[1]. With scale groups (GRP) the
 // steps of each 128-column group k (8k .. 8k + 7) are folded into run after the group's last step:
-// run += alpha_k * acc / 2 + beta_k * sum_k(x), acc = 0 (Eq. 10 per group).
-template <int MT, bool GRP>
+// run += alpha_k * acc / 2 + beta_k * sum_k(x), acc = 0 (Eq. 10 per group). With the split encoding
+// (SPLIT) A is 2T (split_a) and B the chunk's (hi, lo) of v*x; without scale groups the unit's steps
+// are folded into run at its end (split_fold).
+template <int MT, bool GRP, bool SPLIT>
 __device__ __forceinline__ void decode_unit(const uint8_t* sb, int tr, int g, int q, int lane, int ch_odd, bool bias,
                                             float (&acc)[2][kMbBlocks][MT][4], float (&run)[kMbBlocks][MT][4]) {
   const uint8_t* vblk = sb + kMbCodeBytes;
@@ -399,6 +535,42 @@ __device__ __forceinline__ void decode_unit(const uint8_t* sb, int tr, int g, in
 #pragma unroll
       for (int w = 0; w < 8; ++w) wr[b][h][w] = *reinterpret_cast<const uint32_t*>(rp + ((w ^ g) << 4));
     }
+  if constexpr (SPLIT) {
+#pragma unroll
+    for (int w = 0; w < 8; ++w) {
+#pragma unroll
+      for (int tq = 0; tq < 4; ++tq) {
+        const int s = 4 * w + tq;
+        uint32_t a[kMbBlocks][4];
+#pragma unroll
+        for (int b = 0; b < kMbBlocks; ++b) {
+          if (tq == 0) {
+            a[b][0] = split_a<0>(wr[b][0][w]); a[b][1] = split_a<0>(wr[b][1][w]);
+            a[b][2] = split_a<1>(wr[b][0][w]); a[b][3] = split_a<1>(wr[b][1][w]);
+          } else if (tq == 1) {
+            a[b][0] = split_a<2>(wr[b][0][w]); a[b][1] = split_a<2>(wr[b][1][w]);
+            a[b][2] = split_a<3>(wr[b][0][w]); a[b][3] = split_a<3>(wr[b][1][w]);
+          } else if (tq == 2) {
+            a[b][0] = split_a<4>(wr[b][0][w]); a[b][1] = split_a<4>(wr[b][1][w]);
+            a[b][2] = split_a<5>(wr[b][0][w]); a[b][3] = split_a<5>(wr[b][1][w]);
+          } else {
+            a[b][0] = split_a<6>(wr[b][0][w]); a[b][1] = split_a<6>(wr[b][1][w]);
+            a[b][2] = split_a<7>(wr[b][0][w]); a[b][3] = split_a<7>(wr[b][1][w]);
+          }
+        }
+#pragma unroll
+        for (int j = 0; j < MT; ++j) {
+          const uint2 bx = *reinterpret_cast<const uint2*>(xblk + j * kMbXTileBytes + (s * 32 + lane) * 8);
+#pragma unroll
+          for (int b = 0; b < kMbBlocks; ++b)
+            mma_16816(acc[s & 1][b][j], a[b][0], a[b][1], a[b][2], a[b][3], bx.x, bx.y);
+        }
+        if (GRP && (w & 1) && tq == 3) split_fold<MT, GRP>(sb, tr, g, q, w >> 1, ch_odd, bias, acc, run);
+      }
+    }
+    if (!GRP) split_fold<MT, GRP>(sb, tr, g, q, -1, ch_odd, bias, acc, run);
+    return;
+  }
 #pragma unroll
   for (int w = 0; w < 8; ++w) {
 #pragma unroll
@@ -472,7 +644,7 @@ __device__ __forceinline__ void grid_wait(const unsigned long long* bar, unsigne
 // plain loads); then helper warp hw takes 16-row blocks hw, hw + 4, ... of the pass with the same
 // virtual-column MMA as the prep kernel. A wait that times out is recorded in the status word and
 // the helpers carry on, so that every helper reaches every named barrier.
-template <int MT>
+template <int MT, bool SPLIT>
 __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u0, int n_units, float* rslot,
                                          uint8_t* rstage, uint64_t* res_full, uint64_t* res_empty, uint64_t* staged,
                                          const MbGroupParams& gp, int hw, int lane, int* status) {
@@ -536,11 +708,11 @@ __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u
           const int tr = 16 * (rb - G0 / 4);  // first row of the block within the pass
           if (a.fp8) {
             for (int step = 0; step * 16 < s; ++step)
-              res_step<1, true>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, quad, res);
+              res_step<1, true>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, SPLIT, quad, res);
           } else if (quad) {
-            for (int step = 0; step * 16 < s; ++step) res_step<1>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, true, res);
+            for (int step = 0; step * 16 < s; ++step) res_step<1>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, SPLIT, true, res);
           } else {
-            for (int step = 0; step * 16 < s; ++step) res_step<1>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, false, res);
+            for (int step = 0; step * 16 < s; ++step) res_step<1>(rv, s, ri, rs, xr, s16, s, step, tr, g, q, MT, SPLIT, false, res);
           }
           // consumer thread 32 (rb / 2) + lane holds these rows as its block rb % 2
           float4* dst = reinterpret_cast<float4*>(out + (size_t)(32 * (rb >> 1) + lane) * 8 * MT);
@@ -566,9 +738,9 @@ __device__ __noinline__ void helper_role(const MbProblemArgs* tab, int NP, int u
 
 // ---------------------------------------------------------------- main kernel
 
-// MT: n8 tiles of the batch (1 for M <= 8, 2 for M <= 16). GRP: alpha (and beta) per row and
-// 128-column group, loaded per unit by TMA, instead of one alpha per row.
-template <int MT, bool GRP>
+// MT: n8 tiles of the B operand (mb_mt). GRP: alpha (and beta) per row and 128-column group, loaded
+// per unit by TMA, instead of one alpha per row. SPLIT: the split encoding (mb_split), else 2T * v.
+template <int MT, bool GRP, bool SPLIT>
 __global__ void __launch_bounds__(kMbThreads, 1)
     qtea_gemv_mb_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ TensorMaps ab_maps,
                         const __grid_constant__ MbGroupParams gp) {
@@ -643,7 +815,10 @@ __global__ void __launch_bounds__(kMbThreads, 1)
     {
       const UnitPos up = unit_pos(tab, NP, u0);
       const MbPrepProblem pp = gp.prep.prob[up.p];
-      prep_chunk(pp, gp.M, MT, up.ch, (int)threadIdx.x, rstage, stages + kMbCodeBytes, [] { consumers_sync(); });
+      if (SPLIT)
+        prep_chunk_split(pp, gp.M, MT, up.ch, (int)threadIdx.x, rstage, stages + kMbCodeBytes, [] { consumers_sync(); });
+      else
+        prep_chunk(pp, gp.M, MT, up.ch, (int)threadIdx.x, rstage, stages + kMbCodeBytes, [] { consumers_sync(); });
       consumers_sync();
     }
     {
@@ -652,7 +827,10 @@ __global__ void __launch_bounds__(kMbThreads, 1)
         while (pi + 1 < gp.prep.n_problems && item >= gp.prep.prob[pi + 1].block_begin) ++pi;
         const MbPrepProblem pp = gp.prep.prob[pi];
         const int local = item - pp.block_begin;
-        if (local < pp.n_chunks)
+        if (local < pp.n_chunks && SPLIT)
+          prep_chunk_split(pp, gp.M, MT, local, (int)threadIdx.x, rstage, pp.ws + (size_t)local * kMbChunkWsBytes,
+                           [] { consumers_sync(); });
+        else if (local < pp.n_chunks)
           prep_chunk(pp, gp.M, MT, local, (int)threadIdx.x, rstage, pp.ws + (size_t)local * kMbChunkWsBytes,
                      [] { consumers_sync(); });
         else
@@ -664,7 +842,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
   }
 
   if (warp > kMbConsumerWarps) {
-    helper_role<MT>(tab, NP, u0, n_units, rslot, rstage, res_full, res_empty, staged, gp, warp - kMbConsumerWarps - 1,
+    helper_role<MT, SPLIT>(tab, NP, u0, n_units, rslot, rstage, res_full, res_empty, staged, gp, warp - kMbConsumerWarps - 1,
                     lane, gp.status);
   } else if (warp == kMbConsumerWarps) {
     // ---------------------------------------------------------------- producer lane
@@ -756,7 +934,7 @@ __global__ void __launch_bounds__(kMbThreads, 1)
       }
       const bool ok = mbar_wait(smem_u32(&full[st]), (uint32_t)((i / S) & 1), gp.status);
       if (!__all_sync(0xffffffffu, ok)) break;
-      decode_unit<MT, GRP>(stages + (size_t)st * kStage, tr, g, q, lane, c.ch & 1, a.bias != 0, acc, run);
+      decode_unit<MT, GRP, SPLIT>(stages + (size_t)st * kStage, tr, g, q, lane, c.ch & 1, a.bias != 0, acc, run);
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&empty[st]));
 
@@ -797,6 +975,12 @@ __global__ void __launch_bounds__(kMbThreads, 1)
                 part[b][j][e] = run[b][j][e] + res[b][j][e];
                 run[b][j][e] = 0.f;
               }
+            } else if (SPLIT) {  // the folded chunks, then alpha (entries 1 and 3 carry nothing)
+              part[b][j][0] = fmaf(h2f(al[b][0]), run[b][j][0], res[b][j][0]);
+              part[b][j][2] = fmaf(h2f(al[b][1]), run[b][j][2], res[b][j][2]);
+              part[b][j][1] = part[b][j][3] = 0.f;
+#pragma unroll
+              for (int e = 0; e < 4; ++e) run[b][j][e] = 0.f;
             } else {
               part[b][j][0] = fa0 * (acc[0][b][j][0] + acc[1][b][j][0]) + res[b][j][0];
               part[b][j][1] = fa0 * (acc[0][b][j][1] + acc[1][b][j][1]) + res[b][j][1];
@@ -863,8 +1047,14 @@ __global__ void __launch_bounds__(kMbThreads, 1)
           for (int b = 0; b < kMbBlocks; ++b)
 #pragma unroll
             for (int j = 0; j < MT; ++j) {
-              const int n0 = 8 * j + 2 * q;
               const int row0 = c.t * kMbTileRows + tr + 16 * b + g, row1 = row0 + 8;
+              if (SPLIT) {  // batch row 4j + q in entries 0 (row g) and 2 (row g + 8)
+                const int m = 4 * j + q;
+                if (m < M && row0 < a.N) a.y[(size_t)m * a.N + row0] = part[b][j][0];
+                if (m < M && row1 < a.N) a.y[(size_t)m * a.N + row1] = part[b][j][2];
+                continue;
+              }
+              const int n0 = 8 * j + 2 * q;
               if (row0 < a.N) {
                 if (n0 < M) a.y[(size_t)n0 * a.N + row0] = part[b][j][0];
                 if (n0 + 1 < M) a.y[(size_t)(n0 + 1) * a.N + row0] = part[b][j][1];
@@ -909,37 +1099,38 @@ __global__ void __launch_bounds__(kMbThreads, 1)
 }  // namespace
 
 size_t mb_smem_bytes(int S, int M, bool grp, int res_stage_bytes) {
-  return mb_smem_layout(S, M <= 8 ? 1 : 2, grp, res_stage_bytes).total;
+  return mb_smem_layout(S, mb_mt(M), grp, res_stage_bytes).total;
 }
 
+// The six variants of the main kernel: (MT, GRP, SPLIT) in {(1, -, 1), (1, -, 0), (2, -, 0)}.
+#define QTEA_MB_VARIANTS(X)                                                                                 \
+  X(1, false, true) X(1, false, false) X(2, false, false) X(1, true, true) X(1, true, false) X(2, true, false)
+
 cudaError_t mb_configure(size_t smem_optin, size_t* dyn_max) {
-  cudaFuncAttributes a[4];
   cudaError_t e;
-  if ((e = cudaFuncGetAttributes(&a[0], qtea_gemv_mb_kernel<1, false>)) != cudaSuccess) return e;
-  if ((e = cudaFuncGetAttributes(&a[1], qtea_gemv_mb_kernel<2, false>)) != cudaSuccess) return e;
-  if ((e = cudaFuncGetAttributes(&a[2], qtea_gemv_mb_kernel<1, true>)) != cudaSuccess) return e;
-  if ((e = cudaFuncGetAttributes(&a[3], qtea_gemv_mb_kernel<2, true>)) != cudaSuccess) return e;
   size_t st = 0;
-  for (int i = 0; i < 4; ++i) st = a[i].sharedSizeBytes > st ? a[i].sharedSizeBytes : st;
+  cudaFuncAttributes a;
+#define QTEA_MB_ATTR(MT, GRP, SPLIT)                                                                        \
+  if ((e = cudaFuncGetAttributes(&a, qtea_gemv_mb_kernel<MT, GRP, SPLIT>)) != cudaSuccess) return e;      \
+  st = a.sharedSizeBytes > st ? a.sharedSizeBytes : st;
+  QTEA_MB_VARIANTS(QTEA_MB_ATTR)
+#undef QTEA_MB_ATTR
   const size_t dyn = smem_optin > st ? smem_optin - st : 0;
   *dyn_max = dyn;
-  if ((e = cudaFuncSetAttribute(qtea_gemv_mb_kernel<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn)) !=
-      cudaSuccess)
+#define QTEA_MB_SET(MT, GRP, SPLIT)                                                                         \
+  if ((e = cudaFuncSetAttribute(qtea_gemv_mb_kernel<MT, GRP, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize, \
+                                (int)dyn)) != cudaSuccess)                                                  \
     return e;
-  if ((e = cudaFuncSetAttribute(qtea_gemv_mb_kernel<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn)) !=
-      cudaSuccess)
-    return e;
-  if ((e = cudaFuncSetAttribute(qtea_gemv_mb_kernel<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn)) !=
-      cudaSuccess)
-    return e;
-  return cudaFuncSetAttribute(qtea_gemv_mb_kernel<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  QTEA_MB_VARIANTS(QTEA_MB_SET)
+#undef QTEA_MB_SET
+  return cudaSuccess;
 }
 
 size_t mb_prep_smem_bytes(int s, bool native) {
   const size_t E = native ? (size_t)s : (size_t)kMbResEntries;
   const size_t ris = native ? (size_t)((s + 3) / 4) : (size_t)kMbResEntries / 4;
   const size_t res = ((64 * E * 2 + 15) & ~(size_t)15) + ((64 * ris + 15) & ~(size_t)15) + 16 * ((E + 15) & ~(size_t)15) * 2;
-  const size_t chunk = (size_t)16 * kChunkCols * 2 + (size_t)kChunkCols * 2;
+  const size_t chunk = (size_t)kMbPrepScratch;
   return s > 0 && res > chunk ? res : chunk;
 }
 
@@ -977,12 +1168,16 @@ cudaError_t launch_mb(const TensorMaps& maps, const TensorMaps& ab_maps, const M
   attr[1].val.cooperative = 1;
   cfg.attrs = attr;
   cfg.numAttrs = p.fused ? 2 : 1;
+  const int mt = mb_mt(p.M);
+  const bool split = p.split != 0;
   if (grp) {
-    if (p.M <= 8) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, true>, maps, ab_maps, p);
-    return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2, true>, maps, ab_maps, p);
+    if (split) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, true, true>, maps, ab_maps, p);
+    if (mt == 1) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, true, false>, maps, ab_maps, p);
+    return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2, true, false>, maps, ab_maps, p);
   }
-  if (p.M <= 8) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, false>, maps, ab_maps, p);
-  return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2, false>, maps, ab_maps, p);
+  if (split) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, false, true>, maps, ab_maps, p);
+  if (mt == 1) return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<1, false, false>, maps, ab_maps, p);
+  return cudaLaunchKernelEx(&cfg, qtea_gemv_mb_kernel<2, false, false>, maps, ab_maps, p);
 }
 
 }  // namespace qtea

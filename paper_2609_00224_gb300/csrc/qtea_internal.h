@@ -166,6 +166,18 @@ constexpr int kMbSxBytes = 256;                                // sum of x per 1
 constexpr int kMbChunkHead = kMbVBytes + kMbSxBytes;           // the x blocks start here
 constexpr int kMbXTileBytes = 8192;                            // x of a chunk, 8 batch rows, fragment order
 constexpr int kMbChunkWsBytes = kMbChunkHead + 2 * kMbXTileBytes;  // 17664 per 512-column chunk
+// Split encoding (M <= 8): the chunk head holds, instead of v, the chunk's fold factor 2^(-E-1)
+// (fp32) at kMbHlF; the blocks hold B = the exact fp16 (hi, lo) split of v*x * 2^E (see the
+// kernel's header).
+constexpr int kMbHlF = 0;
+// Scratch of the chunk build: x [16][512] and v [512] fp16, then eight warp maxima.
+constexpr int kMbPrepScratch = 16 * kChunkCols * 2 + kChunkCols * 2 + 64;
+// n8 tiles of the B operand and the encoding for batch size M: the split encoding (v*x as fp16 hi
+// and lo in two columns per batch row, one tile) for M <= 4; 2T*v with B = x for 5 <= M <= 16, one
+// tile up to M = 8 and two up to 16. (Measured on the Qwen3-14B layer: the split encoding in two
+// tiles at M = 8 took 50.5 us against 42.8 for 2T*v in one.)
+__host__ __device__ constexpr bool mb_split(int M) { return M <= 4; }
+__host__ __device__ constexpr int mb_mt(int M) { return M <= 8 ? 1 : 2; }
 constexpr int kMbAbBytes = 256 * 16;                           // alpha (and beta) of a unit's rows, 8 fp16 per row
 
 // One shared-memory stage of the low-batch kernel: codes [256 rows][128 bytes], the chunk's v block,
@@ -202,6 +214,7 @@ struct MbPrepProblem {
 struct MbPrepGroup {
   MbPrepProblem prob[kMaxProblems];
   int n_problems, M, mt, n_blocks;
+  int split;                // mb_split(M): the split encoding's chunks
   size_t smem;              // dynamic shared memory of a block
 };
 
@@ -235,6 +248,7 @@ struct MbGroupParams {
   unsigned long long* gbar; // fused: grid barrier counter (monotonic), target below
   unsigned long long gbar_target;
   int n_problems, n_stages, M;
+  int split;                // mb_split(M)
   int res_stage_bytes;      // the helpers' staging buffer (and the fused prep's scratch)
   int* status;              // device status word (the first layout's)
   long long total_units;
