@@ -291,7 +291,9 @@ int qtea_set_layout_options(qtea_layout* layout, int options);
 /*
  * Status written by the kernels of this layout: QTEA_OK, or QTEA_ERR_TIMEOUT if a bounded
  * wait inside a kernel gave up (the kernel then skipped its remaining work and y is
- * unspecified). Synchronizes `stream`, reads the flag and clears it.
+ * unspecified; the layout's split-tile workspace may then hold partial rows that no CTA summed,
+ * so later calls on the layout are unspecified too: free it and pack a new one). Synchronizes
+ * `stream`, reads the flag and clears it.
  */
 int qtea_device_status(const qtea_layout* layout, qtea_stream_t stream);
 
@@ -323,10 +325,11 @@ int qtea_device_status(const qtea_layout* layout, qtea_stream_t stream);
  * Set-up: the first call on each device, with that device current, looks the scratch up with
  * cudaGetSymbolAddress and sets the kernel's shared-memory attribute. Make that first call before
  * any stream capture on the device. Later calls encode a tensor map on the host and launch.
- * Start state: the split-tile counters and the status word in the scratch must be zero when a call
- * starts. Static device memory is zero when the library's module loads, and every completed call
- * leaves them at zero. A call whose kernel gave up a bounded wait (QTEA_ERR_TIMEOUT) can leave
- * counters set: qtea_gemv_m1_static_status reports that and restores the start state.
+ * Start state: the split-tile partial rows, counters and the status word in the scratch must be
+ * zero when a call starts. Static device memory is zero when the library's module loads, and every
+ * completed call leaves them at zero. A call whose kernel gave up a bounded wait (QTEA_ERR_TIMEOUT)
+ * can leave partial rows set: qtea_gemv_m1_static_status reports the timeout and, with clear,
+ * restores the start state.
  * Concurrency: every call on a device shares the one scratch. Calls that may overlap on the
  * device (different streams without ordering, several host threads) race and give wrong results:
  * order them, e.g. on one stream.
@@ -343,14 +346,15 @@ int qtea_gemv_m1_static(const uint16_t* x, const uint8_t* packed, int N, int K, 
  * State of the static scratch of qtea_gemv_m1_static on the current device (no counterpart in the
  * paper; it serves the allocation-free entry point). Synchronizes `stream`, then reads the
  * scratch's status word and split-tile counters:
- *   QTEA_OK           both at zero: the start state every call needs;
- *   QTEA_ERR_TIMEOUT  a kernel of an earlier call gave up a bounded wait (its y is unspecified);
- *   QTEA_ERR_STATE    counters left set without a recorded timeout (e.g. calls that overlapped).
- * With clear != 0, a non-OK state is reset to zero afterwards (cudaMemsetAsync on the static
- * array, then a synchronization of `stream`), so the next call starts correctly. Order this call
- * after the calls it inspects, e.g. on the same stream. It allocates nothing (the counters are
- * copied to an 8 KB array on the calling thread's stack). Returns the state above, or
- * QTEA_ERR_UNSUPPORTED (device ordinal >= 64) or QTEA_ERR_CUDA.
+ *   QTEA_OK           both at zero;
+ *   QTEA_ERR_TIMEOUT  a kernel of an earlier call gave up a bounded wait (its y is unspecified, and
+ *                     partial rows it left in the scratch would corrupt later calls);
+ *   QTEA_ERR_STATE    counters left set without a recorded timeout.
+ * With clear != 0, a non-OK state is reset to zero afterwards (partial rows, counters and status
+ * word: cudaMemsetAsync on the static array, then a synchronization of `stream`), so the next call
+ * starts correctly. Order this call after the calls it inspects, e.g. on the same stream. It
+ * allocates nothing (the counters are copied to an 8 KB array on the calling thread's stack).
+ * Returns the state above, or QTEA_ERR_UNSUPPORTED (device ordinal >= 64) or QTEA_ERR_CUDA.
  */
 int qtea_gemv_m1_static_status(int clear, qtea_stream_t stream);
 

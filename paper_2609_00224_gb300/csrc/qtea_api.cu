@@ -113,6 +113,9 @@ int plan_m1(qtea_layout* l, const cudaDeviceProp& prop) {
   }
   if (cudaMalloc(&l->workspace, (size_t)l->sm_count * 2 * kTileRows * sizeof(float)) != cudaSuccess)
     return QTEA_ERR_ALLOC;
+  // split-tile partial rows: zero reads as "not written yet", and every completed call leaves it zero
+  if (cudaMemset(l->workspace, 0, (size_t)l->sm_count * 2 * kTileRows * sizeof(float)) != cudaSuccess)
+    return QTEA_ERR_CUDA;
   if (cudaMalloc(&l->counters, (size_t)l->n_tiles * kConsumerWarps * sizeof(unsigned)) != cudaSuccess)
     return QTEA_ERR_ALLOC;
   if (cudaMemset(l->counters, 0, (size_t)l->n_tiles * kConsumerWarps * sizeof(unsigned)) != cudaSuccess)
@@ -733,11 +736,12 @@ int run_batch1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t 
 // ---------------------------------------------------------------- allocation-free batch-1 entry
 // qtea_gemv_m1_static serves callers that may not allocate device memory. Its split-tile scratch is
 // this fixed array in static device memory (one copy per device), laid out as
-//   [0, kStaticWsBytes)             partial sums   [kStaticGrid][2][kTileRows] float
-//   [kStaticWsBytes, +kStaticCtrBytes)  counters   [kStaticTiles][kConsumerWarps] unsigned, zero between calls
+//   [0, kStaticWsBytes)             partial sums   [kStaticGrid][2][kTileRows], zero between calls
+//   [kStaticWsBytes, +kStaticCtrBytes)  counters   [kStaticTiles][kConsumerWarps] unsigned, zero
 //   then the status word (int)
-// The counters start at zero because static device memory is zero-initialised when the module
-// is loaded, and every completed call leaves them at zero (the last CTA of a tile resets them).
+// The scratch starts at zero because static device memory is zero-initialised when the module is
+// loaded, and every completed call leaves it at zero (the CTA that sums a split tile zeroes the
+// partial rows it read).
 constexpr int kStaticGrid = 160;                 // CTAs a call may use (>= the 152 SMs of a GB300)
 constexpr int kStaticTiles = 256;                // 512-row tiles: N <= 131072
 constexpr size_t kStaticWsBytes = (size_t)kStaticGrid * 2 * kTileRows * sizeof(float);    // 655,360
@@ -1196,8 +1200,10 @@ int qtea_gemv_m1_static_status(int clear, qtea_stream_t stream) {
   bool dirty = false;
   for (size_t k = 0; k < kStaticCtrBytes / sizeof(unsigned); ++k) dirty = dirty || host_ctr[k] != 0u;
   rc = host_word != 0 ? host_word : dirty ? QTEA_ERR_STATE : QTEA_OK;
-  if (clear && rc != QTEA_OK) {  // counters and status word back to zero: the start state of a call
-    if (cudaMemsetAsync(ctr, 0, kStaticCtrBytes + sizeof(int), st) != cudaSuccess ||
+  // partial rows, counters and status word back to zero: the start state of a call (a call that
+  // timed out may have left partial rows that no CTA summed)
+  if (clear && rc != QTEA_OK) {
+    if (cudaMemsetAsync(d.scratch, 0, kStaticWsBytes + kStaticCtrBytes + sizeof(int), st) != cudaSuccess ||
         cudaStreamSynchronize(st) != cudaSuccess) {
       cudaGetLastError();
       return QTEA_ERR_CUDA;

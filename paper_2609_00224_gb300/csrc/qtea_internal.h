@@ -72,8 +72,8 @@ struct ProblemArgs {
   const uint16_t* rvals;    // [N/4][s]
   const uint8_t* ridx;      // [N/4][ceil(s/4)]
   float* y;                 // [N]
-  float* ws;                // [grid][2][kTileRows] partial sums of split tiles
-  unsigned* counters;       // [n_tiles][kConsumerWarps], zero between calls
+  float* ws;                // [grid][2][kTileRows] partial rows of split tiles (slot 0 used), zero between calls
+  unsigned* counters;       // [n_tiles][kConsumerWarps], zero; not used by the batch-1 kernels
   int N, K, s, n_tiles, n_chunks;
   int act_bits;             // 24: v*x in 24-bit fixed point; 16: 16-bit where a chunk allows it
   int vec_xv;               // x and v are 16-byte aligned (vector loads)

@@ -2,8 +2,9 @@
 
 The file name sorts last so that the GPU tests here also run after every other test has used the
 library in the same process. Each case calls the static entry twice in a row: the second call
-checks that the first left the static scratch's split-tile counters at zero, and
-qtea_gemv_m1_static_status confirms the scratch is back in its start state.
+checks that the first left the static scratch's split-tile partial rows at zero (a row left set
+would be added to the second call's sums), and qtea_gemv_m1_static_status confirms the scratch
+is back in its start state.
 Pass rule: the static entry runs the same kernel on the same grid as qtea_gemv, so its y equals
 qtea_gemv's bit for bit, on both calls; both are within 1e-4 * sum_j |x_j * W^[o][j]| + 1e-6 of the
 oracle's y. The calls allocate nothing: the device's free memory does not change across them.
