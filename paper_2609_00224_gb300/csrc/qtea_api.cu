@@ -106,6 +106,9 @@ int plan_m1(qtea_layout* l, const cudaDeviceProp& prop) {
           cudaMalloc(&l->mb_counters, ctr) != cudaSuccess)
         return QTEA_ERR_ALLOC;
       if (cudaMemset(l->mb_counters, 0, ctr) != cudaSuccess) return QTEA_ERR_CUDA;
+      // partial rows of split tiles: zero reads as "not written yet"; completed calls leave it zero
+      if (cudaMemset(l->mb_part, 0, (size_t)l->sm_count * kMbPartFloatsPerCta * sizeof(float)) != cudaSuccess)
+        return QTEA_ERR_CUDA;
       if (cudaMalloc(&l->mb_gbar, sizeof(unsigned long long)) != cudaSuccess) return QTEA_ERR_ALLOC;
       if (cudaMemset(l->mb_gbar, 0, sizeof(unsigned long long)) != cudaSuccess) return QTEA_ERR_CUDA;
       l->mb_gbar_next = 0;

@@ -333,15 +333,18 @@ struct DoneTile {
 
 // Partial sums of split tiles are stored XOR-ed with this NaN bit pattern, so that zeroed memory
 // reads as "not written yet" and every 4-byte word validates itself (no result has this pattern):
-// a reader needs no flag and no fence, only a load that bypasses L1.
+// a reader needs no flag and no fence, only strong loads of the words (each is single-copy atomic).
 constexpr uint32_t kPartEmpty = 0x7FBADBADu;
 
-__device__ __forceinline__ void part_store(float* p, float v) {
-  __stcg(reinterpret_cast<unsigned*>(p), __float_as_uint(v) ^ kPartEmpty);
+// Loads and stores of those words are strong (relaxed, GPU scope): a weak load may keep returning a
+// stale copy of the line (the two dies' L2 partitions), so it need not ever see another CTA's store.
+__device__ __forceinline__ void part_store_bits(float* p, unsigned w) {
+  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(w) : "memory");
 }
+__device__ __forceinline__ void part_store(float* p, float v) { part_store_bits(p, __float_as_uint(v) ^ kPartEmpty); }
 __device__ __forceinline__ unsigned part_load(const float* p) {
   unsigned w;
-  asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(w) : "l"(p) : "memory");
+  asm volatile("ld.relaxed.gpu.global.u32 %0, [%1];" : "=r"(w) : "l"(p) : "memory");
   return w;
 }
 
@@ -423,8 +426,8 @@ __device__ __forceinline__ void tile_epilogue(const ProblemArgs& a, const DoneTi
       }
       s0 += __uint_as_float(w0 ^ kPartEmpty);
       s1 += __uint_as_float(w1 ^ kPartEmpty);
-      __stcg(reinterpret_cast<unsigned*>(src + ra), 0u);  // empty again for the next call
-      __stcg(reinterpret_cast<unsigned*>(src + ra + 32), 0u);
+      part_store_bits(src + ra, 0u);  // empty again for the next call
+      part_store_bits(src + ra + 32, 0u);
     }
   }
   if (row0g < N) y[row0g] = s0;

@@ -30,9 +30,10 @@
 // group). The consumer threads first build the fragment-order chunks (spread over the CTAs; each
 // CTA's own first chunk straight into its first stage), then decode. Each of eight consumer warps
 // owns two 16-row blocks of a unit, so every B fragment it loads feeds two MMAs; two accumulator
-// sets alternate between steps. A tile whose units span several CTAs is finished by the last of
-// them (per warp, counted with an acq_rel atomic), which adds the partial rows in CTA order, so
-// results do not depend on timing. A producer lane streams the CTA's units through a ring of
+// sets alternate between steps. A tile whose units span several CTAs is finished by the CTA holding
+// its first unit, which reaches it at the end of its range; the others store their partial rows
+// (self-validating words) and carry on without waiting. The sum runs in CTA order, so results do
+// not depend on timing. A producer lane streams the CTA's units through a ring of
 // shared-memory stages: 256 rows x 128 bytes of codes by TMA (128-byte swizzle), the chunk's v and
 // x in fragment order by bulk copy, and with scale groups the unit's alpha (and beta) by TMA.
 // |v| must stay below 32768 (2v is formed in fp16). Every wait is bounded (~2 s, then
@@ -71,6 +72,25 @@ __device__ __forceinline__ uint32_t a_reg(uint32_t w, uint32_t vpair) {
   const uint32_t t2 = ~(w << (14 - 2 * I)) & 0xC000C000u;
   return h2_as_u32(__hmul2(u32_as_h2(t2), u32_as_h2(vpair)));
 }
+
+// Partial rows of split tiles are stored XOR-ed with this NaN bit pattern, so that zeroed memory
+// reads as "not written yet" and every 4-byte word validates itself (no result has this pattern).
+constexpr uint32_t kPartEmpty = 0x7FBADBADu;
+
+// Loads and stores of those words are strong (relaxed, GPU scope): a weak load may keep returning a
+// stale copy of the line (the two dies' L2 partitions), so it need not ever see another CTA's store.
+__device__ __forceinline__ uint4 part_load4(const uint4* p) {
+  uint4 w;
+  asm volatile("ld.relaxed.gpu.global.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(w.x), "=r"(w.y), "=r"(w.z), "=r"(w.w)
+               : "l"(p)
+               : "memory");
+  return w;
+}
+__device__ __forceinline__ void part_store4(uint4* p, uint4 w) {
+  asm volatile("st.relaxed.gpu.global.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
+               : "memory");
+}
+__device__ __forceinline__ bool part_written4(const uint4& w) { return w.x && w.y && w.z && w.w; }
 
 // CTA whose range contains unit u (the inverse of the balanced split cta_u0[b] = b * total / grid).
 __device__ __forceinline__ int unit_owner(long long u, long long total, int grid) {
@@ -897,6 +917,8 @@ __global__ void __launch_bounds__(kMbThreads, 1)
 #pragma unroll
           for (int k = 0; k < 4; ++k) acc[e][b][j][k] = res[b][j][k] = run[b][j][k] = 0.f;
     uint16_t al[kMbBlocks][2] = {};
+    uint4 pw[kMbBlocks];   // MT = 1: the first partner's words of the split tile the range ends in
+    bool pre = false;
     bool need_alpha = true;
     bool own_res = false;  // the helpers compute this tile's residual
     int kc = 0;            // helper result slots taken so far
@@ -930,6 +952,18 @@ __global__ void __launch_bounds__(kMbThreads, 1)
               res[b][j][2] = r4.z;
               res[b][j][3] = r4.w;
             }
+        }
+      }
+      if (MT == 1 && i == n_units - 1) {
+        // the split tile this range ends in, when this CTA sums it: the first partner's partial rows,
+        // loaded now so that they arrive during the decode
+        const long long A = a.unit_begin + (long long)c.t * a.n_chunks, B = A + a.n_chunks;
+        if (A >= u0 && B > u1) {
+          const uint4* src = reinterpret_cast<const uint4*>(
+              a.part + ((size_t)(blockIdx.x + 1) * 2 * kMbConsumerWarps * 32 + tid) * 4 * kMbBlocks * MT);
+#pragma unroll
+          for (int b = 0; b < kMbBlocks; ++b) pw[b] = part_load4(src + b);
+          pre = true;
         }
       }
       const bool ok = mbar_wait(smem_u32(&full[st]), (uint32_t)((i / S) & 1), gp.status);
@@ -992,55 +1026,58 @@ __global__ void __launch_bounds__(kMbThreads, 1)
         const long long A = a.unit_begin + (long long)t * a.n_chunks, B = A + a.n_chunks;
         bool write = true;
         if (!(A >= u0 && B <= u1)) {
-          // partial tile: publish this warp's rows, then the last of the tile's contributors (per
-          // warp: counter t * 8 + warp) adds all partials in CTA order. Slot 0 of a CTA holds the
-          // tile its range starts in, slot 1 the tile its range ends in.
-          const int my_slot = (u0 >= A) ? 0 : 1;
-          float4* mine = reinterpret_cast<float4*>(
-              a.part + (((size_t)blockIdx.x * 2 + my_slot) * kMbConsumerWarps * 32 + tid) * 4 * kMbBlocks * MT);
-#pragma unroll
-          for (int b = 0; b < kMbBlocks; ++b)
-#pragma unroll
-            for (int j = 0; j < MT; ++j)
-              mine[b * MT + j] = make_float4(part[b][j][0], part[b][j][1], part[b][j][2], part[b][j][3]);
-          __syncwarp();
-          const int bf = unit_owner(A, gp.total_units, grid), bl = unit_owner(B - 1, gp.total_units, grid);
-          int last = 0;
-          if (lane == 0) {
-            // acq_rel at gpu scope: the warp's partials (ordered before by __syncwarp) are published
-            // with the increment, and the last arriver sees every other contributor's partials
-            unsigned* ctr = a.counters + (size_t)t * kMbConsumerWarps + warp;
-            unsigned prev;
-            asm volatile("atom.add.acq_rel.gpu.global.u32 %0, [%1], 1;" : "=r"(prev) : "l"(ctr) : "memory");
-            last = (prev == (unsigned)(bl - bf));  // every CTA in [bf, bl] holds units of this tile
-            if (last) *ctr = 0u;                   // self-reset for the next call
-          }
-          last = __shfl_sync(0xffffffffu, last, 0);
-          __syncwarp();
-          write = last != 0;
-          if (write) {
+          // split tile, summed in CTA order by the CTA that holds its first unit (bitwise
+          // reproducible): every other contributor stores its partial rows in slot 0 of its
+          // partial-row slots, each word XOR-ed with kPartEmpty (zero: not written), and carries on;
+          // the first contributor reaches the tile at the end of its range, waits for each partner's
+          // words (bounded), adds them and zeroes them, so every completed call leaves the slots zero
+          const int bl = unit_owner(B - 1, gp.total_units, grid);
+          if (A < u0) {
+            uint4* mine = reinterpret_cast<uint4*>(
+                a.part + ((size_t)blockIdx.x * 2 * kMbConsumerWarps * 32 + tid) * 4 * kMbBlocks * MT);
 #pragma unroll
             for (int b = 0; b < kMbBlocks; ++b)
 #pragma unroll
               for (int j = 0; j < MT; ++j)
+                part_store4(mine + b * MT + j,
+                            make_uint4(__float_as_uint(part[b][j][0]) ^ kPartEmpty, __float_as_uint(part[b][j][1]) ^ kPartEmpty,
+                                       __float_as_uint(part[b][j][2]) ^ kPartEmpty, __float_as_uint(part[b][j][3]) ^ kPartEmpty));
+            write = false;
+          } else {
+            bool timed_out = false;
+            for (int cb = (int)blockIdx.x + 1; cb <= bl; ++cb) {
+              uint4* src = reinterpret_cast<uint4*>(
+                  a.part + ((size_t)cb * 2 * kMbConsumerWarps * 32 + tid) * 4 * kMbBlocks * MT);
+              uint4 w[kMbBlocks][MT];
 #pragma unroll
-                for (int k = 0; k < 4; ++k) part[b][j][k] = 0.f;
-            for (int cb = bf; cb <= bl; ++cb) {
-              const int cslot = (gp.cta_u0[cb] >= A) ? 0 : 1;
-              const float4* src = reinterpret_cast<const float4*>(
-                  a.part + (((size_t)cb * 2 + cslot) * kMbConsumerWarps * 32 + tid) * 4 * kMbBlocks * MT);
+              for (int b = 0; b < kMbBlocks; ++b)
+#pragma unroll
+                for (int j = 0; j < MT; ++j)
+                  w[b][j] = (MT == 1 && pre && cb == (int)blockIdx.x + 1) ? pw[b] : part_load4(src + b * MT + j);
 #pragma unroll
               for (int b = 0; b < kMbBlocks; ++b)
 #pragma unroll
                 for (int j = 0; j < MT; ++j) {
-                  const float4 v4 = __ldcg(src + b * MT + j);
-                  part[b][j][0] += v4.x;
-                  part[b][j][1] += v4.y;
-                  part[b][j][2] += v4.z;
-                  part[b][j][3] += v4.w;
+                  if (!timed_out && !part_written4(w[b][j])) {
+                    const unsigned long long t0 = global_ns();
+                    do {
+                      w[b][j] = part_load4(src + b * MT + j);
+                      if (global_ns() - t0 > kWaitLimitNs) {
+                        atomicExch(gp.status, (int)QTEA_ERR_TIMEOUT);
+                        timed_out = true;
+                        break;
+                      }
+                    } while (!part_written4(w[b][j]));
+                  }
+                  part[b][j][0] += __uint_as_float(w[b][j].x ^ kPartEmpty);
+                  part[b][j][1] += __uint_as_float(w[b][j].y ^ kPartEmpty);
+                  part[b][j][2] += __uint_as_float(w[b][j].z ^ kPartEmpty);
+                  part[b][j][3] += __uint_as_float(w[b][j].w ^ kPartEmpty);
+                  part_store4(src + b * MT + j, make_uint4(0u, 0u, 0u, 0u));  // empty again for the next call
                 }
             }
           }
+          pre = false;
         }
         if (write) {
 #pragma unroll

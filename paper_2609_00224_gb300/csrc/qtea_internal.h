@@ -232,8 +232,8 @@ struct MbProblemArgs {
   const uint8_t* ridx;      // kMbResHelpers: [N/4][ceil(s/4)], 16-byte aligned
   const uint16_t* xs;       // kMbResHelpers: the prep kernel's x at the salient columns [16][s16]
   float* y;                 // [M][N]
-  float* part;              // [grid][2][256 threads][4 kMbBlocks MT] partial rows of split tiles
-  unsigned* counters;       // [n_tiles][kMbConsumerWarps], zero between calls
+  float* part;              // [grid][2][256 threads][4 kMbBlocks MT] partial rows of split tiles (slot 0 used), zero between calls
+  unsigned* counters;       // [n_tiles][kMbConsumerWarps], zero; not used by the kernel
   int N, n_tiles, n_chunks, s, s16, res_mode;
   int res_passes;           // kMbResHelpers: a tile's row groups are staged in 1, 2 or 4 passes
   int bias;                 // scale groups: row_scale holds (alpha, beta) pairs
