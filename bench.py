@@ -1058,6 +1058,24 @@ def profile_case(args):
     return 1 if status else 0
 
 
+def probe_decode():
+    """Issue rates behind the batch-1 decode choice: cycles per instruction per SM sub-partition of
+    mma.sync with constant operands and with A built from a changing word (as a decode builds it), and
+    of dp4a; weights per clock per SM at batch 1 follow from the useful products per instruction."""
+    import torch
+    import paper_2609_00224_gb300 as qt
+    torch.cuda.set_device(0)
+    r = qt.qtea_probe_decode_rates()
+    useful = {"mma_m16n8k16_f16_constant": 256, "mma_m16n8k16_f16_decoded_a": 256, "mma_m16n8k32_e4m3_constant": 512,
+              "mma_m16n8k32_e4m3_decoded_a": 512,
+              "dp4a": 64}  # weights per warp instruction at batch 1 (dp4a: 32 lanes x 4 bytes, 2 planes at 16 bits)
+    per_sm = {k: round(4 * useful[k] / v, 1) for k, v in r.items()}
+    print(json.dumps({"probe": "decode_issue_rates", "cycles_per_instruction_per_smsp": r,
+                      "batch1_weights_per_clock_per_sm_bound": per_sm,
+                      "note": "one instruction stream per chain; the decode adds its own mask and load instructions"}))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -1087,9 +1105,13 @@ def main():
     ap.add_argument("--profile-layers", type=int, default=4, help="resident layers of --profile-case")
     ap.add_argument("--fixed-point", action="store_true", help="--profile-case llama3_8b_base3: fixed-point kernel")
     ap.add_argument("--calls", type=int, default=3, help="grouped calls of --profile-case")
+    ap.add_argument("--probe-decode", action="store_true",
+                    help="print the issue rates behind the batch-1 decode choice (dp4a against mma.sync) and exit")
     args = ap.parse_args()
     if args.profile_case:
         return profile_case(args)
+    if args.probe_decode:
+        return probe_decode()
     if args.impl == "reference":
         return reference_arm(args)
     return qtea_arm(args)

@@ -358,6 +358,22 @@ int qtea_gemv_m1_static(const uint16_t* x, const uint8_t* packed, int N, int K, 
  */
 int qtea_gemv_m1_static_status(int clear, qtea_stream_t stream);
 
+/*
+ * Diagnostic, not a step of the GEMV (the paper has no counterpart): the issue rates that decide
+ * between a dp4a decode and a tensor-core (mma.sync) decode of the 2-bit codes at batch 1, measured
+ * on the current device, in clock cycles per instruction per SM sub-partition (8 warps per SM, 8
+ * independent accumulator chains per warp):
+ *   [0] mma.sync m16n8k16 f16 -> f32, constant operands
+ *   [1] the same with A masked from a word that changes every instruction (as a decode builds it)
+ *   [2] mma.sync m16n8k32 e4m3 -> f32, constant operands
+ *   [3] the same with A masked from a changing word
+ *   [4] dp4a
+ *   cycles_per_instruction  host array of n >= 5 doubles, written
+ * Allocates a few kilobytes of device memory and synchronizes the device. Returns QTEA_OK,
+ * QTEA_ERR_INVALID_ARG (null array or n < 5), QTEA_ERR_ALLOC or QTEA_ERR_CUDA.
+ */
+int qtea_probe_decode_rates(double* cycles_per_instruction, int n);
+
 #ifdef __cplusplus
 }
 #endif

@@ -95,6 +95,8 @@ def load(build_if_missing: bool = True):
     lib.qtea_gemv_m1_static_status.argtypes = [i32, P]
     lib.qtea_quantize.restype = i32
     lib.qtea_quantize.argtypes = [P, P, i32, i32, i32, i32, i32, i32, i32, P, P, P, P, P, P, P]
+    lib.qtea_probe_decode_rates.restype = i32
+    lib.qtea_probe_decode_rates.argtypes = [P, i32]
     _lib = lib
     return lib
 
@@ -278,6 +280,18 @@ def qtea_gemv_plan(problems) -> list:
 
 def qtea_device_status(layout: Layout, stream=None) -> int:
     return load().qtea_device_status(layout.handle, _stream(stream))
+
+
+def qtea_probe_decode_rates() -> dict:
+    """Cycles per instruction per SM sub-partition of the instructions a batch-1 decode could run
+    on (a diagnostic behind the dp4a decode; see include/qtea.h)."""
+    out = (ctypes.c_double * 5)()
+    rc = load().qtea_probe_decode_rates(out, 5)
+    if rc:
+        raise QteaError(rc, "qtea_probe_decode_rates")
+    names = ("mma_m16n8k16_f16_constant", "mma_m16n8k16_f16_decoded_a", "mma_m16n8k32_e4m3_constant",
+             "mma_m16n8k32_e4m3_decoded_a", "dp4a")
+    return {n: round(out[i], 3) for i, n in enumerate(names)}
 
 
 def packed_bytes(layout: Layout):
