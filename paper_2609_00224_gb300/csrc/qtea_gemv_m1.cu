@@ -62,10 +62,12 @@ __device__ __forceinline__ UnitPos unit_pos(const ProblemArgs* tab, int n_proble
 }
 
 // The two TMA boxes of unit (t, ch) into ring stage `dst`, completing on `bar`.
+// The codes are read once per call: their lines are the first L2 evicts.
 __device__ __forceinline__ void issue_unit(const CUtensorMap* map, int t, int ch, uint32_t dst, uint32_t bar) {
+  const uint64_t pol = l2_evict_first_policy();
   mbar_arrive_expect_tx(bar, kStageBytes);
-  tma_load_2d(dst, map, ch * kChunkRowBytes, t * kTileRows, bar);
-  tma_load_2d(dst + kBoxBytes, map, ch * kChunkRowBytes, t * kTileRows + kBoxRows, bar);
+  tma_load_2d_hint(dst, map, ch * kChunkRowBytes, t * kTileRows, bar, pol);
+  tma_load_2d_hint(dst + kBoxBytes, map, ch * kChunkRowBytes, t * kTileRows + kBoxRows, bar, pol);
 }
 
 // ---------------------------------------------------------------- decode (consumers)
