@@ -53,6 +53,10 @@ def load(path: str | None = None):
     lib.qo_packed_bytes_base3.argtypes = [i32, i32]
     lib.qo_lut5.restype = None
     lib.qo_lut5.argtypes = [P, P]
+    lib.qo_salient_from_bitmap.restype = i32
+    lib.qo_salient_from_bitmap.argtypes = [P, i32, P, i32]
+    lib.qo_salient_to_bitmap.restype = i32
+    lib.qo_salient_to_bitmap.argtypes = [P, i32, i32, P]
     lib.qo_asic_latency_us.restype = None
     lib.qo_asic_latency_us.argtypes = [i32, i32, P, P]
     if path is None:
@@ -146,6 +150,31 @@ def unpack(packed, N: int, K: int, fmt: str = "2bit", lib=None) -> np.ndarray:
     if rc != 0:
         raise OracleError(f"unpack returned {rc}")
     return T
+
+
+def salient_from_bitmap(bitmap, K: int, lib=None) -> np.ndarray:
+    """Sec. 3.5's salient bitmap (uint32 words, column j at bit j % 32 of word j // 32) as the
+    ascending index list."""
+    lib = lib or load()
+    bitmap = _c(bitmap, np.uint32)
+    if bitmap.size < (K + 31) // 32:
+        raise ValueError("bitmap shorter than K bits")
+    out = np.zeros(max(K, 1), np.int32)
+    n = lib.qo_salient_from_bitmap(_ptr(bitmap), K, _ptr(out), K)
+    if n < 0:
+        raise OracleError(f"salient_from_bitmap returned {n}")
+    return out[:n].copy()
+
+
+def salient_to_bitmap(idx, K: int, lib=None) -> np.ndarray:
+    """The bitmap of a strictly ascending salient index list (each in [0, K))."""
+    lib = lib or load()
+    idx = _c(idx, np.int32)
+    out = np.zeros(max((K + 31) // 32, 1), np.uint32)
+    rc = lib.qo_salient_to_bitmap(_ptr(idx), idx.size, K, _ptr(out))
+    if rc != 0:
+        raise OracleError(f"salient_to_bitmap returned {rc}")
+    return out[:(K + 31) // 32].copy()
 
 
 def lut5(xs, lib=None) -> np.ndarray:

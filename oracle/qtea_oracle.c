@@ -33,6 +33,10 @@
  *                         least significant digit). Byte 25 covers 3 real columns and 2 pad
  *                         digits; pad digits and columns >= K hold digit 1 (T = 0).
  *   salient_idx           int32 [s], strictly ascending, each < K
+ *   salient bitmap        Sec. 3.5 stores the salient set as a bitmap over the input columns:
+ *                         uint32 words [ceil(K/32)], column j at bit j % 32 of word j / 32 (least
+ *                         significant bit first); bits of columns >= K are ignored on input and
+ *                         zero on output
  *   residual_vals         fp16 [N/4][s]: value of group q (rows 4q..4q+3) in salient column c;
  *                         or, where the paper's storage is used (Sec. 4.1: FP8 residual), one
  *                         byte per value in the FP8 E4M3 format: sign bit 7, exponent bits 6-3
@@ -283,6 +287,31 @@ int qo_unpack_base3(const uint8_t* packed, int N, int K, int8_t* T) {
  * product of the pattern whose base-3 digits are d_0..d_4 (T = d - 1) with the scaled
  * activations xs[0..4] (xs = v * x).
  */
+/* Sec. 3.5: the salient columns marked in the bitmap, ascending; returns their number (-1 for a
+ * negative K) and writes the first max_s of them to out. */
+int qo_salient_from_bitmap(const uint32_t* bitmap, int K, int32_t* out, int max_s) {
+  if (K < 0) return -1;
+  int n = 0;
+  for (int j = 0; j < K; ++j) {
+    if ((bitmap[j / 32] >> (j % 32)) & 1u) {
+      if (n < max_s) out[n] = j;
+      ++n;
+    }
+  }
+  return n;
+}
+
+/* The bitmap of a salient index list (strictly ascending, each in [0, K)). */
+int qo_salient_to_bitmap(const int32_t* idx, int s, int K, uint32_t* bitmap) {
+  if (K < 0 || s < 0) return QO_BAD_ARG;
+  memset(bitmap, 0, sizeof(uint32_t) * (size_t)((K + 31) / 32));
+  for (int i = 0; i < s; ++i) {
+    if (idx[i] < 0 || idx[i] >= K || (i > 0 && idx[i] <= idx[i - 1])) return QO_BAD_DATA;
+    bitmap[idx[i] / 32] |= 1u << (idx[i] % 32);
+  }
+  return QO_OK;
+}
+
 void qo_lut5(const double xs[5], double lut[243]) {
   for (int c = 0; c < 243; ++c) {
     int rest = c;

@@ -445,3 +445,33 @@ def test_generator_is_deterministic_and_thread_independent():
     b = synth.codes(123, 1, (3000, 700), 0.3, 0.4)
     c = synth.codes(123, 1, (10, 700), 0.3, 0.4)    # single thread, same stream prefix
     assert np.array_equal(a, b) and np.array_equal(a[:10], c)
+
+
+# ---------------------------------------------------------------- salient bitmap (Sec. 3.5)
+
+def test_salient_bitmap_known_words():
+    """Sec. 3.5 stores the salient set as a bitmap over input columns. Hand-worked: word 0 =
+    0x80000005 marks columns 0, 2 and 31; word 1 = 0x81 marks columns 32 + 0 and 32 + 7."""
+    words = np.array([0x80000005, 0x81], np.uint32)
+    assert oracle.salient_from_bitmap(words, 40).tolist() == [0, 2, 31, 32, 39]
+    assert oracle.salient_to_bitmap(np.array([0, 2, 31, 32, 39], np.int32), 40).tolist() == [0x80000005, 0x81]
+
+
+def test_salient_bitmap_ignores_bits_past_k():
+    # K = 35: only columns 32, 33, 34 of word 1 exist
+    assert oracle.salient_from_bitmap(np.array([0, 0xFFFFFFFF], np.uint32), 35).tolist() == [32, 33, 34]
+    assert oracle.salient_from_bitmap(np.zeros(0, np.uint32), 0).tolist() == []
+
+
+def test_salient_bitmap_round_trip_and_rejects_bad_lists():
+    rng = np.random.default_rng(5)
+    for K in (1, 31, 32, 33, 1000, 4096):
+        idx = np.sort(rng.choice(K, size=min(K, max(1, K // 10)), replace=False)).astype(np.int32)
+        bm = oracle.salient_to_bitmap(idx, K)
+        assert bm.size == (K + 31) // 32
+        assert np.array_equal(oracle.salient_from_bitmap(bm, K), idx)
+        # popcount equals the list length (no bit set twice, none lost)
+        assert sum(bin(int(w)).count("1") for w in bm) == idx.size
+    for bad in ([3, 3], [5, 2], [-1], [40]):
+        with pytest.raises(oracle.OracleError):
+            oracle.salient_to_bitmap(np.array(bad, np.int32), 40)

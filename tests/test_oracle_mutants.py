@@ -114,6 +114,13 @@ def pin_failures(lib):
     xs = np.array([0.3, -1.25, 2.0, 0.125, -0.5])
     lut = oracle.lut5(xs, lib=lib)
     check("lut", np.array_equal(lut, -lut[::-1]) and all(lut[121 + 3 ** d] == xs[d] for d in range(5)))
+    # the salient bitmap of Sec. 3.5 from hand-written words
+    try:
+        idx = oracle.salient_from_bitmap(np.array([0x80000005, 0x81], np.uint32), 40, lib=lib)
+        bm = oracle.salient_to_bitmap(np.array([0, 2, 31, 32, 39], np.int32), 40, lib=lib)
+        check("bitmap", idx.tolist() == [0, 2, 31, 32, 39] and bm.tolist() == [0x80000005, 0x81])
+    except oracle.OracleError:
+        check("bitmap", False)
     return fails
 
 
@@ -137,6 +144,9 @@ MUTANTS = {
     "lut_digit_offset": [("(double)(rest % 3 - 1) * xs[d]", "(double)(rest % 3) * xs[d]")],
     "residual_position_msb_first": [(">> (2 * (c % 4))) & 3;", ">> (6 - 2 * (c % 4))) & 3;")],
     "residual_position_byte_stride": [("ridx[(size_t)q * residual_stride(s) + c / 4]", "ridx[(size_t)q * (s / 4) + c / 4]")],
+    "bitmap_msb_first": [("if ((bitmap[j / 32] >> (j % 32)) & 1u) {", "if ((bitmap[j / 32] >> (31 - j % 32)) & 1u) {"),
+                         ("bitmap[idx[i] / 32] |= 1u << (idx[i] % 32);", "bitmap[idx[i] / 32] |= 1u << (31 - idx[i] % 32);")],
+    "bitmap_word_stride": [("if ((bitmap[j / 32] >> (j % 32)) & 1u) {", "if ((bitmap[j / 31] >> (j % 32)) & 1u) {")],
 }
 
 
