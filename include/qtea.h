@@ -257,6 +257,25 @@ typedef struct qtea_layout_desc {
 
 int qtea_layout_describe(const qtea_layout* layout, qtea_layout_desc* out);
 
+/*
+ * The salient set as the paper stores it (Sec. 3.5: a binary bitmap over the input columns) and as
+ * qtea_gemv takes it (salient_idx: int32, strictly ascending, each < K).
+ *   bitmap     device uint32 [ceil(K/32)]: column j is bit j % 32 (least significant first) of
+ *              word j / 32; bits of columns >= K are ignored by qtea_salient_from_bitmap and zero
+ *              after qtea_salient_to_bitmap
+ *   salient_idx  device int32 [max_s] (written) / [n_salient] (read)
+ * qtea_salient_from_bitmap writes the marked columns in ascending order and their number to
+ * *n_salient (host memory); more than max_s marked columns: QTEA_ERR_INVALID_ARG, *n_salient = the
+ * number, the first max_s written. qtea_salient_to_bitmap overwrites the whole bitmap; an index
+ * outside [0, K) or not above its predecessor gives QTEA_ERR_INVALID_ARG (the bitmap then holds the
+ * valid ones). Both run on `stream`, synchronize it once, and allocate a 4-byte device word for the
+ * duration of the call (setup-time utilities, not for the decode loop). Null or misaligned pointers,
+ * K < 0 or max_s < 0: QTEA_ERR_INVALID_ARG.
+ */
+int qtea_salient_from_bitmap(const uint32_t* bitmap, int K, int32_t* salient_idx, int max_s, int* n_salient,
+                             qtea_stream_t stream);
+int qtea_salient_to_bitmap(const int32_t* salient_idx, int n_salient, int K, uint32_t* bitmap, qtea_stream_t stream);
+
 /* Copy the layout's packed ternary bytes (qtea_layout_desc.packed_bytes of them) to the
  * caller's device buffer `dst`, asynchronously on `stream`. `bytes` must equal packed_bytes. */
 int qtea_layout_copy_packed(const qtea_layout* layout, void* dst, size_t bytes, qtea_stream_t stream);

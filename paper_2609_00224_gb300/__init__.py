@@ -89,6 +89,10 @@ def load(build_if_missing: bool = True):
     lib.qtea_set_layout_options.argtypes = [P, i32]
     lib.qtea_layout_copy_packed.restype = i32
     lib.qtea_layout_copy_packed.argtypes = [P, P, ctypes.c_size_t, P]
+    lib.qtea_salient_from_bitmap.restype = i32
+    lib.qtea_salient_from_bitmap.argtypes = [P, i32, P, i32, ctypes.POINTER(i32), P]
+    lib.qtea_salient_to_bitmap.restype = i32
+    lib.qtea_salient_to_bitmap.argtypes = [P, i32, i32, P, P]
     lib.qtea_gemv_m1_static.restype = i32
     lib.qtea_gemv_m1_static.argtypes = [P, P, i32, i32, i32, P, P, P, P, P, P, P]
     lib.qtea_gemv_m1_static_status.restype = i32
@@ -336,3 +340,32 @@ def qtea_quantize(W, hdiag, group_size: Optional[int] = None, n_salient: int = 0
     if rc:
         raise QteaError(rc, "qtea_quantize")
     return out
+
+
+def qtea_salient_from_bitmap(bitmap, K: int, max_s: Optional[int] = None, stream=None):
+    """Sec. 3.5's salient bitmap (int32 or uint32 CUDA tensor of ceil(K/32) words, column j at bit
+    j % 32 of word j // 32) as the ascending int32 index list qtea_gemv takes."""
+    import torch
+    words = (K + 31) // 32
+    ptr = _ptr(bitmap, (torch.int32,) + ((torch.uint32,) if hasattr(torch, "uint32") else ()), "bitmap", (words,))
+    max_s = K if max_s is None else int(max_s)
+    out = torch.empty(max(max_s, 1), dtype=torch.int32, device=bitmap.device)
+    n = ctypes.c_int32(0)
+    rc = load().qtea_salient_from_bitmap(ptr, int(K), out.data_ptr(), max_s, ctypes.byref(n), _stream(stream))
+    if rc != QTEA_OK:
+        raise QteaError(rc, "qtea_salient_from_bitmap")
+    return out[:n.value]
+
+
+def qtea_salient_to_bitmap(salient_idx, K: int, stream=None):
+    """The bitmap (int32 CUDA tensor of ceil(K/32) words holding the uint32 bits) of a strictly
+    ascending int32 salient index list."""
+    import torch
+    s = 0 if salient_idx is None else int(salient_idx.numel())
+    ptr = _ptr(salient_idx, (torch.int32,), "salient_idx") if s else None
+    dev = salient_idx.device if salient_idx is not None else torch.device("cuda")
+    out = torch.empty(max((K + 31) // 32, 1), dtype=torch.int32, device=dev)
+    rc = load().qtea_salient_to_bitmap(ptr, s, int(K), out.data_ptr(), _stream(stream))
+    if rc != QTEA_OK:
+        raise QteaError(rc, "qtea_salient_to_bitmap")
+    return out[:(K + 31) // 32]

@@ -1078,6 +1078,57 @@ int qtea_set_activation_precision(qtea_layout* l, int bits) {
   return QTEA_OK;
 }
 
+int qtea_salient_from_bitmap(const uint32_t* bitmap, int K, int32_t* salient_idx, int max_s, int* n_salient,
+                             qtea_stream_t stream) {
+  if (K < 0 || max_s < 0 || !n_salient || (K > 0 && (!bitmap || !aligned(bitmap, 4))) ||
+      (max_s > 0 && (!salient_idx || !aligned(salient_idx, 4))))
+    return QTEA_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int* count = nullptr;
+  if (cudaMalloc(&count, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_ERR_ALLOC;
+  }
+  int host = 0;
+  int rc = QTEA_OK;
+  if (launch_bitmap_to_index(bitmap, K, salient_idx, max_s, count, st) != cudaSuccess ||
+      cudaMemcpyAsync(&host, count, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    rc = QTEA_ERR_CUDA;
+  cudaFree(count);
+  if (rc != QTEA_OK) {
+    cudaGetLastError();
+    return rc;
+  }
+  *n_salient = host;
+  return host > max_s ? QTEA_ERR_INVALID_ARG : QTEA_OK;
+}
+
+int qtea_salient_to_bitmap(const int32_t* salient_idx, int n_salient, int K, uint32_t* bitmap, qtea_stream_t stream) {
+  if (K < 0 || n_salient < 0 || n_salient > K || (n_salient > 0 && (!salient_idx || !aligned(salient_idx, 4))) ||
+      (K > 0 && (!bitmap || !aligned(bitmap, 4))))
+    return QTEA_ERR_INVALID_ARG;
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  int* bad = nullptr;
+  if (cudaMalloc(&bad, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    return QTEA_ERR_ALLOC;
+  }
+  int host = 0;
+  int rc = QTEA_OK;
+  if (cudaMemsetAsync(bad, 0, sizeof(int), st) != cudaSuccess ||
+      launch_index_to_bitmap(salient_idx, n_salient, K, bitmap, bad, st) != cudaSuccess ||
+      cudaMemcpyAsync(&host, bad, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    rc = QTEA_ERR_CUDA;
+  cudaFree(bad);
+  if (rc != QTEA_OK) {
+    cudaGetLastError();
+    return rc;
+  }
+  return host ? QTEA_ERR_INVALID_ARG : QTEA_OK;
+}
+
 int qtea_layout_copy_packed(const qtea_layout* l, void* dst, size_t bytes, qtea_stream_t stream) {
   if (!l || bytes != l->packed_bytes || (bytes > 0 && !dst)) return QTEA_ERR_INVALID_ARG;
   if (bytes == 0) return QTEA_OK;

@@ -398,6 +398,10 @@ bool b3_eligible(const PaperParams& p);
 cudaError_t paper_configure(size_t smem_optin);
 cudaError_t launch_pack_base3(const int8_t* codes, int N, int K, uint8_t* packed, int* bad_flag, cudaStream_t st);
 cudaError_t launch_m1(const TensorMaps& maps, const GroupParams& p, int grid, size_t smem, cudaStream_t st);
+// Sec. 3.5's salient bitmap (column j at bit j % 32 of word j / 32) and the ascending index list.
+cudaError_t launch_bitmap_to_index(const uint32_t* bitmap, int K, int32_t* idx, int max_s, int* count,
+                                   cudaStream_t st);
+cudaError_t launch_index_to_bitmap(const int32_t* idx, int s, int K, uint32_t* bitmap, int* bad, cudaStream_t st);
 cudaError_t m1_configure(size_t smem_optin, size_t* dyn_max);
 cudaError_t launch_generic(const GenericParams& p, cudaStream_t st);
 cudaError_t launch_pack(const int8_t* codes, int N, int K, int K_pad, uint32_t* packed, int* bad_flag,
