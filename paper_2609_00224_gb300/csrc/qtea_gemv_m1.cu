@@ -440,6 +440,7 @@ __device__ __forceinline__ void tile_epilogue(const ProblemArgs& a, const DoneTi
 // the tile's epilogue, wait until the next unit has been decoded, so the helpers' residual work is
 // not waited for right after each decode; the sums are still added in unit order, so results stay
 // bitwise reproducible.
+template <bool GRP>
 __device__ __forceinline__ void consumer_role(const Ring r, long long total, int u0, int u1,
                                            int warp, int lane, int* status) {
   const int n_units = u1 - u0;
@@ -461,7 +462,7 @@ __device__ __forceinline__ void consumer_role(const Ring r, long long total, int
     const int u = u0 + i;
     const ProblemArgs& a = r.tab[c.p];
     const int n_chunks = a.n_chunks, N = a.N;
-    const bool grouped = (a.gflags & kScaleGroups) != 0;
+    const bool grouped = GRP && (a.gflags & kScaleGroups) != 0;
     const bool gbias = (a.gflags & kScaleBias) != 0, gvec = (a.gflags & kScaleVec) != 0;
     if (need_alpha) {  // used at the tile's end: unconditional loads (rows clamped), so nothing waits here
       if (grouped) {   // alpha is applied per group in the decode
@@ -622,6 +623,7 @@ __device__ __forceinline__ void consumer_role(const Ring r, long long total, int
   }
 }
 
+template <bool GRP>
 __global__ void __launch_bounds__(kThreads, 1)
     qtea_gemv_m1_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ GroupParams gp) {
   extern __shared__ uint8_t smem_raw[];
@@ -698,7 +700,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   if (!pre_fill && warp == kProducerWarp && lane == 0) first_fills(maps, r, u0, n_units);
 
-  if (warp < kConsumerWarps) consumer_role(r, gp.total_units, u0, u1, warp, lane, gp.status);
+  if (warp < kConsumerWarps) consumer_role<GRP>(r, gp.total_units, u0, u1, warp, lane, gp.status);
   else if (warp < kProducerWarp) helper_role(r, u0, n_units, warp - kConsumerWarps, lane, gp.status);
   else if (lane == 0) producer_role(maps, r, u0, n_units, gp.status);
 
@@ -719,11 +721,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 // shared memory; *dyn_max receives that size.
 cudaError_t m1_configure(size_t smem_optin, size_t* dyn_max) {
   cudaFuncAttributes attr;
-  cudaError_t e = cudaFuncGetAttributes(&attr, qtea_gemv_m1_kernel);
+  cudaError_t e = cudaFuncGetAttributes(&attr, qtea_gemv_m1_kernel<true>);
   if (e != cudaSuccess) return e;
   const size_t dyn = smem_optin > attr.sharedSizeBytes ? smem_optin - attr.sharedSizeBytes : 0;
   *dyn_max = dyn;
-  return cudaFuncSetAttribute(qtea_gemv_m1_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  e = cudaFuncSetAttribute(qtea_gemv_m1_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(qtea_gemv_m1_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
 }
 
 // Programmatic stream serialisation lets this launch start while the previous kernel on the
@@ -739,7 +743,10 @@ cudaError_t launch_m1(const TensorMaps& maps, const GroupParams& p, int grid, si
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel, maps, p);
+  // the variant without the scale groups' decode when no problem of the launch has them: a smaller
+  // kernel, whose code stays in the instruction caches
+  return p.grp ? cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel<true>, maps, p)
+               : cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel<false>, maps, p);
 }
 
 }  // namespace qtea
