@@ -564,7 +564,7 @@ bool group_add(M1Group& g, const qtea_gemv_problem& q) {
   ProblemArgs& a = g.gp.prob[g.gp.n_problems];
   a = problem_args(q);
   a.unit_begin = g.gp.total_units;
-  if (a.gflags & kScaleGroups) g.gp.grp = 1;
+  if (a.gflags & kScaleGroups) g.gp.n_grp += 1;
   std::memcpy(&g.maps.m[g.gp.n_problems], &l->tmap, sizeof(CUtensorMap));
   if (g.gp.n_problems == 0) g.gp.status = l->status;
   g.gp.total_units += (long long)l->n_tiles * l->n_chunks;

@@ -440,7 +440,7 @@ __device__ __forceinline__ void tile_epilogue(const ProblemArgs& a, const DoneTi
 // the tile's epilogue, wait until the next unit has been decoded, so the helpers' residual work is
 // not waited for right after each decode; the sums are still added in unit order, so results stay
 // bitwise reproducible.
-template <bool GRP>
+template <int GM>
 __device__ __forceinline__ void consumer_role(const Ring r, long long total, int u0, int u1,
                                            int warp, int lane, int* status) {
   const int n_units = u1 - u0;
@@ -462,7 +462,8 @@ __device__ __forceinline__ void consumer_role(const Ring r, long long total, int
     const int u = u0 + i;
     const ProblemArgs& a = r.tab[c.p];
     const int n_chunks = a.n_chunks, N = a.N;
-    const bool grouped = GRP && (a.gflags & kScaleGroups) != 0;
+    // GM: 0 no problem of the launch has scale groups, 2 every one has, 1 some have
+    const bool grouped = GM == 2 || (GM == 1 && (a.gflags & kScaleGroups) != 0);
     const bool gbias = (a.gflags & kScaleBias) != 0, gvec = (a.gflags & kScaleVec) != 0;
     if (need_alpha) {  // used at the tile's end: unconditional loads (rows clamped), so nothing waits here
       if (grouped) {   // alpha is applied per group in the decode
@@ -623,7 +624,7 @@ __device__ __forceinline__ void consumer_role(const Ring r, long long total, int
   }
 }
 
-template <bool GRP>
+template <int GM>
 __global__ void __launch_bounds__(kThreads, 1)
     qtea_gemv_m1_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ GroupParams gp) {
   extern __shared__ uint8_t smem_raw[];
@@ -700,7 +701,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   if (!pre_fill && warp == kProducerWarp && lane == 0) first_fills(maps, r, u0, n_units);
 
-  if (warp < kConsumerWarps) consumer_role<GRP>(r, gp.total_units, u0, u1, warp, lane, gp.status);
+  if (warp < kConsumerWarps) consumer_role<GM>(r, gp.total_units, u0, u1, warp, lane, gp.status);
   else if (warp < kProducerWarp) helper_role(r, u0, n_units, warp - kConsumerWarps, lane, gp.status);
   else if (lane == 0) producer_role(maps, r, u0, n_units, gp.status);
 
@@ -721,13 +722,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 // shared memory; *dyn_max receives that size.
 cudaError_t m1_configure(size_t smem_optin, size_t* dyn_max) {
   cudaFuncAttributes attr;
-  cudaError_t e = cudaFuncGetAttributes(&attr, qtea_gemv_m1_kernel<true>);
+  cudaError_t e = cudaFuncGetAttributes(&attr, qtea_gemv_m1_kernel<1>);
   if (e != cudaSuccess) return e;
   const size_t dyn = smem_optin > attr.sharedSizeBytes ? smem_optin - attr.sharedSizeBytes : 0;
   *dyn_max = dyn;
-  e = cudaFuncSetAttribute(qtea_gemv_m1_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(qtea_gemv_m1_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+  for (auto k : {qtea_gemv_m1_kernel<0>, qtea_gemv_m1_kernel<1>, qtea_gemv_m1_kernel<2>}) {
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dyn);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 // Programmatic stream serialisation lets this launch start while the previous kernel on the
@@ -743,10 +746,12 @@ cudaError_t launch_m1(const TensorMaps& maps, const GroupParams& p, int grid, si
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  // the variant without the scale groups' decode when no problem of the launch has them: a smaller
-  // kernel, whose code stays in the instruction caches
-  return p.grp ? cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel<true>, maps, p)
-               : cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel<false>, maps, p);
+  // the variant holding only the decodes the launch's problems need (with or without scale groups,
+  // or both): a smaller kernel, whose code stays in the instruction caches
+  const int gm = p.n_grp == 0 ? 0 : p.n_grp == p.n_problems ? 2 : 1;
+  return gm == 0 ? cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel<0>, maps, p)
+                 : gm == 2 ? cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel<2>, maps, p)
+                           : cudaLaunchKernelEx(&cfg, qtea_gemv_m1_kernel<1>, maps, p);
 }
 
 }  // namespace qtea

@@ -96,7 +96,7 @@ struct TensorMaps {
 struct GroupParams {
   ProblemArgs prob[kMaxProblems];
   int n_problems, n_stages;
-  int grp;                  // some problem has scale groups (the kernel variant that decodes them)
+  int n_grp;                // problems with scale groups (the kernel variants: none, some, all)
   int codes_after_wait;     // the codes belong to the caller: no code fill before the grid dependency wait
   int* status;              // device status word (the first layout's)
   long long total_units;
