@@ -719,6 +719,19 @@ bool rows_plan(const qtea_gemv_problem* qs, const int* idx, int n, RowsLaunch& L
     std::memcpy(&L.maps.m[i], &q.packed_ternary->tmap8, sizeof(CUtensorMap));
   }
   L.rp.cta_begin[n] = b;
+  // lanes per row (4 for up to 8 rows, 2 for 16, 1 for more): one value for every CTA, or 0
+  int kp = -1;
+  for (int i = 0; i < n && kp != 0; ++i) {
+    const int N = qs[idx[i]].packed_ternary->N;
+    for (int j = 0; j < cnt[i]; ++j) {
+      const long long r0 = blocks[i] * j / cnt[i] * kRowsBoxRows, r1 = blocks[i] * (j + 1) / cnt[i] * kRowsBoxRows;
+      const long long R = (r1 < N ? r1 : N) - r0;
+      const int k = R <= 8 ? 4 : R <= 16 ? 2 : 1;
+      if (kp < 0) kp = k;
+      else if (kp != k) kp = 0;
+    }
+  }
+  L.rp.kparts = kp < 0 ? 0 : kp;
   L.rp.rows_cap = (int)rows_cap;
   L.rp.n_chunks_max = nch_max;
   L.rp.n_problems = n;

@@ -100,8 +100,8 @@ __device__ __forceinline__ void decode_part(const uint8_t* row, const uint8_t* s
 
 // Chunk ch of the CTA's rows, with kparts lanes per row (row lane / kparts, part lane % kparts): the
 // row's sum of T X scaled by q plus the outliers, added to part on every lane of the row.
-__device__ __forceinline__ void decode_chunk(const uint8_t* region, const uint8_t* slot, int lane, int kparts,
-                                             float& part) {
+template <int kparts>
+__device__ __forceinline__ void decode_chunk(const uint8_t* region, const uint8_t* slot, int lane, float& part) {
   const ChunkMeta* mp = reinterpret_cast<const ChunkMeta*>(slot + kAuxMeta);
   const float scale = mp->scale;
   const int planes = mp->planes, n_out = mp->n_out;
@@ -110,7 +110,7 @@ __device__ __forceinline__ void decode_chunk(const uint8_t* region, const uint8_
   const int sw = row & 7;  // 128-byte swizzle phase of the row
   const uint8_t* rb = region + (size_t)row * kChunkRowBytes;
   float d0;
-  if (kparts == 1) {
+  if constexpr (kparts == 1) {
     const uint4* pl = reinterpret_cast<const uint4*>(slot);
     if (planes == 2) {
       RowAcc<2> a0;
@@ -148,6 +148,7 @@ __device__ __forceinline__ void prefetch_range(const void* p, size_t n, int t, i
     asm volatile("prefetch.global.L2 [%0];" ::"l"(l) : "memory");
 }
 
+template <int KP>
 __global__ void __launch_bounds__(kRowsThreads, 2)
     qtea_gemv_rows_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ RowsParams rp) {
   extern __shared__ uint8_t smem_raw[];
@@ -210,7 +211,9 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
 
   const ProblemArgs& a = *args;
   const int s = a.s;
-  const int kparts = R <= 8 ? 4 : R <= 16 ? 2 : 1;  // lanes per row
+  // lanes per row: 4 for up to 8 rows, 2 for 16, 1 for up to 32; KP > 0 when every CTA of the launch
+  // takes the same (the variant then holds only that decode)
+  const int kparts = KP ? KP : (R <= 8 ? 4 : R <= 16 ? 2 : 1);
   // the first chunk's x and v go out before everything else
   ChunkLoads L0;
   if (warp < n_chunks) load_chunk(a, warp, lane, L0);
@@ -261,7 +264,10 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
       ok = false;
       break;
     }
-    decode_chunk(codes + (size_t)c * rp.rows_cap * kChunkRowBytes, slot, lane, kparts, part);
+    const uint8_t* region = codes + (size_t)c * rp.rows_cap * kChunkRowBytes;
+    if (KP == 1 || (KP == 0 && kparts == 1)) decode_chunk<1>(region, slot, lane, part);
+    else if (KP == 2 || (KP == 0 && kparts == 2)) decode_chunk<2>(region, slot, lane, part);
+    else decode_chunk<4>(region, slot, lane, part);
     __syncwarp();  // the slot is rewritten by the warp's next chunk
   }
   if (!gathered) gather();
@@ -322,7 +328,11 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
 }  // namespace
 
 cudaError_t rows_configure(size_t smem_optin) {
-  return cudaFuncSetAttribute(qtea_gemv_rows_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_optin);
+  for (auto k : {qtea_gemv_rows_kernel<0>, qtea_gemv_rows_kernel<1>, qtea_gemv_rows_kernel<2>, qtea_gemv_rows_kernel<4>}) {
+    const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_optin);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 // Programmatic stream serialisation lets the launch start while the previous kernel on the
@@ -338,7 +348,11 @@ cudaError_t launch_rows(const TensorMaps& maps, const RowsParams& p, int grid, s
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel, maps, p);
+  // lanes per row: a variant holding only that decode when every CTA takes the same
+  return p.kparts == 4   ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<4>, maps, p)
+         : p.kparts == 2 ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<2>, maps, p)
+         : p.kparts == 1 ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<1>, maps, p)
+                         : cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<0>, maps, p);
 }
 
 }  // namespace qtea

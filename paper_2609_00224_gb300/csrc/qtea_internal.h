@@ -135,6 +135,7 @@ struct RowsParams {
   int rows_cap;                     // rows of a CTA's buffer per chunk (multiple of 8, at most kRowsMaxRows)
   int n_chunks_max;                 // over the problems: shared-memory size
   int n_problems;
+  int kparts;                       // lanes per row of every CTA (1, 2 or 4), or 0: each CTA by its rows
   int* status;                      // device status word (the first layout's)
 };
 
