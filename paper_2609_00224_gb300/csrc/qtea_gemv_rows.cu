@@ -99,13 +99,15 @@ __device__ __forceinline__ void decode_part(const uint8_t* row, const uint8_t* s
 }
 
 // Chunk ch of the CTA's rows, with kparts lanes per row (row lane / kparts, part lane % kparts): the
-// row's sum of T X scaled by q plus the outliers, added to part on every lane of the row.
+// row's sum of T X scaled by q plus the outliers, added to part on every lane of the row. cs holds
+// the chunk's fixed-point parameters as this warp staged them; the outlier list is in the slot.
 template <int kparts>
-__device__ __forceinline__ void decode_chunk(const uint8_t* region, const uint8_t* slot, int lane, float& part) {
+__device__ __forceinline__ void decode_chunk(const uint8_t* region, const uint8_t* slot, int lane,
+                                             const ChunkStage& cs, float& part) {
   const ChunkMeta* mp = reinterpret_cast<const ChunkMeta*>(slot + kAuxMeta);
-  const float scale = mp->scale;
-  const int planes = mp->planes, n_out = mp->n_out;
-  const long long sum_x = mp->sum_x;
+  const float scale = cs.scale;
+  const int planes = cs.planes, n_out = cs.n_out;
+  const long long sum_x = cs.sum_x;
   const int row = kparts == 1 ? lane : lane / kparts, k = lane - row * kparts;
   const int sw = row & 7;  // 128-byte swizzle phase of the row
   const uint8_t* rb = region + (size_t)row * kChunkRowBytes;
@@ -250,12 +252,13 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
   float part = 0.f;
   bool ok = true;
   for (int c = warp; c < n_chunks; c += kRowsWarps) {
+    ChunkStage cs;
     if (c == warp) {
-      write_planes(a, L0, slot, lane);
+      cs = write_planes<false>(a, L0, slot, lane);
     } else {
       ChunkLoads L;
       load_chunk(a, c, lane, L);
-      write_planes(a, L, slot, lane);
+      cs = write_planes<false>(a, L, slot, lane);
     }
     if (!gathered) gather();
     __syncwarp();
@@ -265,9 +268,9 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
       break;
     }
     const uint8_t* region = codes + (size_t)c * rp.rows_cap * kChunkRowBytes;
-    if (KP == 1 || (KP == 0 && kparts == 1)) decode_chunk<1>(region, slot, lane, part);
-    else if (KP == 2 || (KP == 0 && kparts == 2)) decode_chunk<2>(region, slot, lane, part);
-    else decode_chunk<4>(region, slot, lane, part);
+    if (KP == 1 || (KP == 0 && kparts == 1)) decode_chunk<1>(region, slot, lane, cs, part);
+    else if (KP == 2 || (KP == 0 && kparts == 2)) decode_chunk<2>(region, slot, lane, cs, part);
+    else decode_chunk<4>(region, slot, lane, cs, part);
     __syncwarp();  // the slot is rewritten by the warp's next chunk
   }
   if (!gathered) gather();

@@ -153,6 +153,51 @@ __device__ __forceinline__ float warp_max(float v) {
   return __uint_as_float(__reduce_max_sync(0xffffffffu, __float_as_uint(v)));
 }
 
+// Largest |xt[i]| of the lane's values whose bit in skip is clear, as a tree (a short chain).
+__device__ __forceinline__ float lane_max(const float (&xt)[16], uint32_t skip) {
+  float m[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+    m[i] = fmaxf(((skip >> (2 * i)) & 1u) ? 0.f : fabsf(xt[2 * i]), ((skip >> (2 * i + 1)) & 1u) ? 0.f : fabsf(xt[2 * i + 1]));
+#pragma unroll
+  for (int w = 4; w; w >>= 1)
+#pragma unroll
+    for (int i = 0; i < w; ++i) m[i] = fmaxf(m[i], m[i + w]);
+  return m[0];
+}
+
+// 2^-(e+1) for amax in [2^e, 2^(e+1)) (2^126 for amax = 0): values up to amax scale into (-1, 1).
+__device__ __forceinline__ float binade_scale(float amax) {
+  return __uint_as_float((uint32_t)(253 - (int)((__float_as_uint(amax) >> 23) & 0xff)) << 23);
+}
+
+// Sum over the warp of the squares of the values whose bit in skip is clear, scaled by
+// binade_scale(amax)^2 and then by 2^20, in integer units: a lane's share is below 16 * 2^20, so the
+// warp's sum fits 32 bits and one warp reduction instruction serves. Truncation costs at most one
+// unit per lane against a sum of at least 2^18 (the largest value alone): this feeds only the choice
+// between 16- and 24-bit planes.
+__device__ __forceinline__ unsigned warp_sq_units(const float (&xt)[16], uint32_t skip, float amax) {
+  const float sc = binade_scale(amax);
+  float q0 = 0.f, q1 = 0.f, q2 = 0.f, q3 = 0.f;  // four partial sums per lane (short chains)
+#pragma unroll
+  for (int i = 0; i < 16; i += 4) {
+    const float z0 = xt[i] * sc, z1 = xt[i + 1] * sc, z2 = xt[i + 2] * sc, z3 = xt[i + 3] * sc;
+    q0 = ((skip >> i) & 1u) ? q0 : fmaf(z0, z0, q0);
+    q1 = ((skip >> (i + 1)) & 1u) ? q1 : fmaf(z1, z1, q1);
+    q2 = ((skip >> (i + 2)) & 1u) ? q2 : fmaf(z2, z2, q2);
+    q3 = ((skip >> (i + 3)) & 1u) ? q3 : fmaf(z3, z3, q3);
+  }
+  return __reduce_add_sync(0xffffffffu, __float2uint_rz(((q0 + q1) + (q2 + q3)) * 1048576.f));
+}
+
+// The fixed-point parameters of a staged chunk, the same on every lane of the staging warp.
+struct ChunkStage {
+  float scale;      // q
+  int planes;       // 2 or 3
+  int n_out;        // outliers taken out
+  long long sum_x;  // sum of the fixed-point values
+};
+
 // The chunk's v*x as fixed point: byte planes of this lane's word, and the metadata.
 //  * Outliers: in up to kOutlierRounds rounds, the elements above 1/16 of the largest |v*x| not yet
 //    taken are taken, as long as at most kMaxOutliers are taken in all. A round of ordinary values
@@ -163,17 +208,21 @@ __device__ __forceinline__ float warp_max(float v) {
 //    q = 2^(e-22) for 24 bits (|X| < 2^23) or q = 2^(e-14) for 16 bits (|X| < 2^15). 16 bits are
 //    taken where the caller allows it and amax is within 8 times the root mean square of the
 //    remaining values (no heavy tail that would coarsen the quantum of the others).
-__device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLoads& L, uint8_t* ax, int lane) {
+// kMeta: lane 0 also stores q, the plane count, the outlier count and the sum of X in the metadata
+// (for consumers in other warps); the outlier list and the scale groups' sums are always stored.
+// The returned values let a warp that decodes the chunk itself skip the shared-memory round trip.
+template <bool kMeta = true>
+__device__ __forceinline__ ChunkStage write_planes(const ProblemArgs& a, const ChunkLoads& L, uint8_t* ax,
+                                                   int lane) {
   float xt[16];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {  // exact: fp16 x fp16 fits fp32
     xt[2 * i] = h2f((uint16_t)(L.v[i] & 0xffffu)) * h2f((uint16_t)(L.x[i] & 0xffffu));
     xt[2 * i + 1] = h2f((uint16_t)(L.v[i] >> 16)) * h2f((uint16_t)(L.x[i] >> 16));
   }
-  float lmax = 0.f;
-#pragma unroll
-  for (int i = 0; i < 16; ++i) lmax = fmaxf(lmax, fabsf(xt[i]));
-  float amax = warp_max(lmax);
+  float amax = warp_max(lane_max(xt, 0u));
+  // the sum of squares for the usual case, no outliers, goes out beside the first round's count
+  unsigned sq = warp_sq_units(xt, 0u, amax);
   uint32_t outm = 0;  // bit i: xt[i] is an outlier
   int n_out = 0;
 #pragma unroll 1
@@ -187,11 +236,9 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
     if (c > kMaxOutliers - n_out) break;
     outm |= m;
     n_out += c;
-    lmax = 0.f;
-#pragma unroll
-    for (int i = 0; i < 16; ++i) lmax = fmaxf(lmax, ((outm >> i) & 1u) ? 0.f : fabsf(xt[i]));
-    amax = warp_max(lmax);
+    amax = warp_max(lane_max(xt, outm));
   }
+  if (n_out > 0) sq = warp_sq_units(xt, outm, amax);  // the remaining values, against their amax
   ChunkMeta* meta = reinterpret_cast<ChunkMeta*>(ax + kAuxMeta);
   if (n_out > 0) {  // list them: lane order, then element order
     const int mine = __popc(outm);
@@ -210,19 +257,10 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
         ++off;
       }
   }
-  // sum of squares of the other values: four partial sums per lane (short dependency chains)
-  float sq0 = 0.f, sq1 = 0.f, sq2 = 0.f, sq3 = 0.f;
-#pragma unroll
-  for (int i = 0; i < 16; i += 4) {
-    sq0 = ((outm >> i) & 1u) ? sq0 : fmaf(xt[i], xt[i], sq0);
-    sq1 = ((outm >> (i + 1)) & 1u) ? sq1 : fmaf(xt[i + 1], xt[i + 1], sq1);
-    sq2 = ((outm >> (i + 2)) & 1u) ? sq2 : fmaf(xt[i + 2], xt[i + 2], sq2);
-    sq3 = ((outm >> (i + 3)) & 1u) ? sq3 : fmaf(xt[i + 3], xt[i + 3], sq3);
-  }
-  float ssq = (sq0 + sq1) + (sq2 + sq3);
-#pragma unroll
-  for (int o = 16; o; o >>= 1) ssq += __shfl_xor_sync(0xffffffffu, ssq, o);
-  const bool two = a.act_bits == 16 && amax * amax <= 64.f * (ssq / (float)(kChunkCols - n_out));
+  // amax^2 <= 64 * (sum of squares) / (values), both sides scaled by binade_scale(amax)^2:
+  // 64 / 2^20 = 2^-14 turns the integer units back
+  const float an = amax * binade_scale(amax);
+  const bool two = a.act_bits == 16 && an * an * (float)(kChunkCols - n_out) <= (float)sq * 6.103515625e-05f;
   const int e = amax > 0.f ? (int)((__float_as_uint(amax) >> 23) & 0xff) - 127 : 0;
   const int qsh = two ? 14 : 22;
   const int xmax = two ? 32767 : 8388607;  // a value of amax rounds to at most 2^(qsh+1): clamp
@@ -280,12 +318,18 @@ __device__ __forceinline__ void write_planes(const ProblemArgs& a, const ChunkLo
   // reduction instruction (|sum| < 2^32 in 24-bit mode)
   const unsigned s_lo = __reduce_add_sync(0xffffffffu, (unsigned)sx & 0xFFFFu);
   const int s_hi = (int)__reduce_add_sync(0xffffffffu, (unsigned)(sx >> 16));
-  if (lane == 0) {
-    meta->scale = __uint_as_float((uint32_t)(127 + e - qsh) << 23);  // q
-    meta->planes = two ? 2 : 3;
-    meta->sum_x = (long long)s_hi * 65536 + (long long)s_lo;
-    meta->n_out = n_out;
+  ChunkStage cs;
+  cs.scale = __uint_as_float((uint32_t)(127 + e - qsh) << 23);  // q
+  cs.planes = two ? 2 : 3;
+  cs.n_out = n_out;
+  cs.sum_x = (long long)s_hi * 65536 + (long long)s_lo;
+  if (kMeta && lane == 0) {
+    meta->scale = cs.scale;
+    meta->planes = cs.planes;
+    meta->sum_x = cs.sum_x;
+    meta->n_out = cs.n_out;
   }
+  return cs;
 }
 
 // x at the salient columns of entries e0 .. e0+31 (lane j holds entry e0 + j, zero past e_end).
