@@ -80,21 +80,37 @@ __device__ __forceinline__ float outlier_sum(const ChunkMeta* mp, int n_out, con
 
 // Part k of kparts of one row's chunk (words k * W .. k * W + W - 1, W = 32 / kparts), taken in an
 // order rotated by k so that the parts' plane reads fall in different banks. Each word is read with
-// one 32-bit load from its 128-byte-swizzled granule.
-template <int P>
-__device__ __forceinline__ void decode_part(const uint8_t* row, const uint8_t* slot, int sw, int k, int W,
-                                            RowAcc<P>& a0) {
+// one 32-bit load from its 128-byte-swizzled granule; all W code words are loaded first, and each
+// word's planes while the word before it decodes.
+template <int P, int W>
+__device__ __forceinline__ void decode_part(const uint8_t* row, const uint8_t* slot, int sw, int k, RowAcc<P>& a0) {
 #pragma unroll
   for (int kk = 0; kk < P; ++kk)
 #pragma unroll
     for (int g = 0; g < 4; ++g) a0.a[kk][g] = 0;
-#pragma unroll 4
+  auto word = [&](int t) { return k * W + ((t + k) & (W - 1)); };
+  uint32_t code[W];
+#pragma unroll
   for (int t = 0; t < W; ++t) {
-    const int w = k * W + ((t + k) & (W - 1));
-    const uint32_t code = *reinterpret_cast<const uint32_t*>(row + ((((w >> 2) ^ sw) << 4) | ((w & 3) << 2)));
-    const uint4* pw = reinterpret_cast<const uint4*>(slot + w * kPlaneBytesPerWord);
-    if constexpr (P == 3) decode_word3(code, pw[0], pw[1], pw[2], a0);
-    else decode_word2(code, pw[0], pw[1], a0);
+    const int w = word(t);
+    code[t] = *reinterpret_cast<const uint32_t*>(row + ((((w >> 2) ^ sw) << 4) | ((w & 3) << 2)));
+  }
+  const uint4* pw = reinterpret_cast<const uint4*>(slot + word(0) * kPlaneBytesPerWord);
+  uint4 P0 = pw[0], P1 = pw[1], P2 = P == 3 ? pw[2] : make_uint4(0, 0, 0, 0);
+#pragma unroll
+  for (int t = 0; t < W; ++t) {
+    uint4 Q0 = P0, Q1 = P1, Q2 = P2;
+    if (t + 1 < W) {
+      const uint4* qw = reinterpret_cast<const uint4*>(slot + word(t + 1) * kPlaneBytesPerWord);
+      Q0 = qw[0];
+      Q1 = qw[1];
+      if constexpr (P == 3) Q2 = qw[2];
+    }
+    if constexpr (P == 3) decode_word3(code[t], P0, P1, P2, a0);
+    else decode_word2(code[t], P0, P1, a0);
+    P0 = Q0;
+    P1 = Q1;
+    P2 = Q2;
   }
 }
 
@@ -124,14 +140,14 @@ __device__ __forceinline__ void decode_chunk(const uint8_t* region, const uint8_
       d0 = finish_chunk3(a0, sum_x);
     }
   } else {
-    const int W = 32 / kparts;
+    constexpr int W = 32 / kparts;
     if (planes == 2) {
       RowAcc<2> a0;
-      decode_part<2>(rb, slot, sw, k, W, a0);
+      decode_part<2, W>(rb, slot, sw, k, a0);
       d0 = finish_chunk2(a0, k == 0 ? (int)sum_x : 0);  // the chunk's sum of X once per row
     } else {
       RowAcc<3> a0;
-      decode_part<3>(rb, slot, sw, k, W, a0);
+      decode_part<3, W>(rb, slot, sw, k, a0);
       d0 = finish_chunk3(a0, k == 0 ? sum_x : 0ll);
     }
   }
@@ -229,7 +245,7 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
   const bool has_group = s > 0 && warp < R / 4;
   uint32_t rv[kResRegs], pb[kResRegs];
   int col[kResRegs];
-  float xsv[kResRegs];
+  uint32_t xsb[kResRegs];  // x at the salient columns, fp16 bits: converted only when the residual is formed
 #pragma unroll
   for (int i = 0; i < kResRegs; ++i) {
     const int e = lane + 32 * i;
@@ -239,12 +255,15 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
     pb[i] = in ? __ldg(a.ridx + (size_t)q * rs + (e >> 2)) : 0u;
   }
   bool gathered = false;
-  auto gather = [&]() {  // x at the salient columns, in flight until the residual is formed
+  // x at the salient columns, in flight until the residual is formed (no instruction reads the
+  // loaded registers before then, so the decode does not wait for them)
+  auto gather = [&]() {
 #pragma unroll
     for (int i = 0; i < kResRegs; ++i) {
       const int e = lane + 32 * i;
       const int cc = col[i] < 0 ? 0 : (col[i] >= a.K ? a.K - 1 : col[i]);
-      xsv[i] = has_group && e < s ? h2f(__ldg(a.x + cc)) : 0.f;
+      xsb[i] = 0u;
+      if (has_group && e < s) xsb[i] = __ldg(a.x + cc);
     }
     gathered = true;
   };
@@ -284,7 +303,7 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
 #pragma unroll
     for (int i = 0; i < kResRegs; ++i) {
       const int e = lane + 32 * i;
-      const float pr = h2f((uint16_t)rv[i]) * xsv[i];  // zero past s
+      const float pr = h2f((uint16_t)rv[i]) * h2f((uint16_t)xsb[i]);  // zero past s
       const int pos = (pb[i] >> (2 * (e & 3))) & 3;
       acc0 += pos == 0 ? pr : 0.f;
       acc1 += pos == 1 ? pr : 0.f;
