@@ -625,14 +625,15 @@ int run_m1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st, 
 }
 
 // ---------------------------------------------------------------- row-resident batch-1 kernel
-// Layouts it may serve: 2-bit codes, one alpha per row, fp16 residual values, one 512-column
-// chunk per warp (K <= 4096), at most kRowsMaxSalient salient columns, not pinned to the
-// stream-K kernel.
+// Layouts it may serve: 2-bit codes, one alpha per row, fp16 residual values, at most
+// kRowsMaxChunks 512-column chunks and kRowsMaxSalientWide salient columns, not pinned to the
+// stream-K kernel. Beyond one chunk per warp or kRowsMaxSalient salient columns a launch is wide.
 bool rows_capable(const qtea_layout* l) {
   return l->rows_ok && l->m1_ok && l->format == QTEA_FMT_2BIT && l->group_size == l->K &&
          (l->options & (QTEA_OPT_BIAS | QTEA_OPT_RESIDUAL_FP8 | QTEA_OPT_STREAM_K)) == 0 &&
-         l->n_chunks <= kRowsWarps && l->n_salient <= kRowsMaxSalient;
+         l->n_chunks <= kRowsMaxChunks && l->n_salient <= kRowsMaxSalientWide;
 }
+bool rows_wide(const qtea_layout* l) { return l->n_chunks > kRowsWarps || l->n_salient > kRowsMaxSalient; }
 
 struct RowsLaunch {
   RowsParams rp;
@@ -680,9 +681,9 @@ long long rows_split(const long long* blocks, const int* chunks, int n, int ctas
 }
 
 // One row-resident launch for problems idx[0 .. n): one CTA per SM where that leaves every CTA
-// kRowsMaxRows rows or fewer (one per lane), else two CTAs per SM. False if the problems do not
-// fit: more problems than CTAs, more than kRowsMaxRows rows in a CTA, or shared memory beyond the
-// device's limit.
+// kRowsMaxRows rows or fewer (one per lane), else two CTAs per SM (not for a wide launch). False
+// if the problems do not fit: more problems than CTAs, more than kRowsMaxRows rows in a CTA, or
+// shared memory beyond the device's limit.
 bool rows_plan(const qtea_gemv_problem* qs, const int* idx, int n, RowsLaunch& L) {
   if (n < 1 || n > kMaxProblems) return false;
   const qtea_layout* l0 = qs[idx[0]].packed_ternary;
@@ -690,15 +691,17 @@ bool rows_plan(const qtea_gemv_problem* qs, const int* idx, int n, RowsLaunch& L
   if (n > sm || 2 * sm > kMaxGrid) return false;
   long long blocks[kMaxProblems];
   int chunks[kMaxProblems], cnt[kMaxProblems], nch_max = 0;
+  bool wide = false;
   for (int i = 0; i < n; ++i) {
     const qtea_layout* l = qs[idx[i]].packed_ternary;
     if (!rows_capable(l) || l->sm_count != sm || l->device != l0->device) return false;
     blocks[i] = (l->N + kRowsBoxRows - 1) / kRowsBoxRows;
     chunks[i] = l->n_chunks;
     nch_max = chunks[i] > nch_max ? chunks[i] : nch_max;
+    wide = wide || rows_wide(l);
   }
   long long rows_cap = rows_split(blocks, chunks, n, sm, cnt);
-  if (rows_cap > kRowsMaxRows) {
+  if (rows_cap > kRowsMaxRows && !wide) {
     int cnt2[kMaxProblems];
     const long long r2 = rows_split(blocks, chunks, n, 2 * sm, cnt2);
     if (r2 > 0 && r2 <= kRowsMaxRows) {
@@ -732,6 +735,7 @@ bool rows_plan(const qtea_gemv_problem* qs, const int* idx, int n, RowsLaunch& L
     }
   }
   L.rp.kparts = kp < 0 ? 0 : kp;
+  L.rp.wide = wide ? 1 : 0;
   L.rp.rows_cap = (int)rows_cap;
   L.rp.n_chunks_max = nch_max;
   L.rp.n_problems = n;

@@ -7,7 +7,8 @@
 // multiplied with dp4a), but a decomposition built for latency rather than for streaming:
 //  * Every CTA owns a block of whole rows (multiples of 8, at most 32: one per lane) of one problem,
 //    so a row's sum is finished inside the CTA: no split-K workspace, no counters, no second CTA to
-//    wait for. One CTA per SM where that covers the rows, else two.
+//    wait for. One CTA per SM where that covers the rows, else two. A wide launch (K above 4096, up
+//    to 8192, or more than 256 salient columns) keeps one CTA per SM and its own instantiation.
 //  * The CTA's codes arrive by TMA as 8-row x 128-byte boxes (128-byte swizzle) into one region per
 //    512-column chunk, each region with its own barrier. The library owns the codes (no kernel
 //    writes them after packing), so all of them are requested before griddepcontrol.wait, while
@@ -16,7 +17,8 @@
 //  * After the wait, warp w takes chunks w, w + 8, ...: it stages the chunk's planes in its own
 //    slot, waits for the chunk's codes and decodes them for all of the CTA's rows (each lane one
 //    row with the stream-K kernel's decode loop; with 16 or 8 rows, two or four lanes per row,
-//    each a part of the chunk). Partial row sums meet in shared memory.
+//    each a part of the chunk). In a wide launch the next chunk's x and v are loaded before the
+//    decode, so they arrive while it runs. Partial row sums meet in shared memory.
 //  * The residual: each warp takes row groups of four, lanes over the salient entries, one sum
 //    per position of the group. Its operands (values, positions, x at the salient columns) are
 //    loaded right after the wait and held in registers across the decode, so their latency is
@@ -33,7 +35,10 @@
 namespace qtea {
 namespace {
 
-constexpr int kResRegs = kRowsMaxSalient / 64;  // salient entries per lane held in registers (4)
+// Salient entries per lane held in registers: narrow launches 4 (the rest loaded in place), wide
+// ones 16 (all of them).
+template <bool WIDE>
+__host__ __device__ constexpr int res_regs() { return WIDE ? kRowsMaxSalientWide / 32 : kRowsMaxSalient / 64; }
 static_assert(kRowsMaxRows / 4 <= kRowsWarps, "one residual row group per warp");
 
 // Decode one row (32 words of chunk-row bytes, 128-byte swizzle phase sw) against the chunk's P
@@ -166,9 +171,10 @@ __device__ __forceinline__ void prefetch_range(const void* p, size_t n, int t, i
     asm volatile("prefetch.global.L2 [%0];" ::"l"(l) : "memory");
 }
 
-template <int KP>
-__global__ void __launch_bounds__(kRowsThreads, 2)
+template <int KP, bool WIDE>
+__global__ void __launch_bounds__(kRowsThreads, WIDE ? 1 : 2)
     qtea_gemv_rows_kernel(const __grid_constant__ TensorMaps maps, const __grid_constant__ RowsParams rp) {
+  constexpr int kResRegs = res_regs<WIDE>();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -272,8 +278,10 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
   bool ok = true;
   for (int c = warp; c < n_chunks; c += kRowsWarps) {
     ChunkStage cs;
-    if (c == warp) {
+    if (WIDE || c == warp) {
       cs = write_planes<false>(a, L0, slot, lane);
+      // wide: the warp's next chunk's x and v go out now and arrive during this chunk's decode
+      if (WIDE && c + kRowsWarps < n_chunks) load_chunk(a, c + kRowsWarps, lane, L0);
     } else {
       ChunkLoads L;
       load_chunk(a, c, lane, L);
@@ -350,7 +358,8 @@ __global__ void __launch_bounds__(kRowsThreads, 2)
 }  // namespace
 
 cudaError_t rows_configure(size_t smem_optin) {
-  for (auto k : {qtea_gemv_rows_kernel<0>, qtea_gemv_rows_kernel<1>, qtea_gemv_rows_kernel<2>, qtea_gemv_rows_kernel<4>}) {
+  for (auto k : {qtea_gemv_rows_kernel<0, false>, qtea_gemv_rows_kernel<1, false>, qtea_gemv_rows_kernel<2, false>,
+                 qtea_gemv_rows_kernel<4, false>, qtea_gemv_rows_kernel<0, true>, qtea_gemv_rows_kernel<1, true>}) {
     const cudaError_t e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem_optin);
     if (e != cudaSuccess) return e;
   }
@@ -370,11 +379,15 @@ cudaError_t launch_rows(const TensorMaps& maps, const RowsParams& p, int grid, s
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  // lanes per row: a variant holding only that decode when every CTA takes the same
-  return p.kparts == 4   ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<4>, maps, p)
-         : p.kparts == 2 ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<2>, maps, p)
-         : p.kparts == 1 ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<1>, maps, p)
-                         : cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<0>, maps, p);
+  // lanes per row: a variant holding only that decode when every CTA takes the same; wide launches
+  // (one CTA per SM) have a one-lane-per-row variant and the general one
+  if (p.wide)
+    return p.kparts == 1 ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<1, true>, maps, p)
+                         : cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<0, true>, maps, p);
+  return p.kparts == 4   ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<4, false>, maps, p)
+         : p.kparts == 2 ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<2, false>, maps, p)
+         : p.kparts == 1 ? cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<1, false>, maps, p)
+                         : cudaLaunchKernelEx(&cfg, qtea_gemv_rows_kernel<0, false>, maps, p);
 }
 
 }  // namespace qtea

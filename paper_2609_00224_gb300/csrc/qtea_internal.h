@@ -118,16 +118,24 @@ __host__ __device__ constexpr size_t m1_smem_bytes(int S) {
 }
 
 // ---------------------------------------------------------------- row-resident batch-1 kernel (small groups)
-// For small groups with K <= 4096: every CTA owns whole rows (up to kRowsMaxRows, in 8-row
-// blocks; one or two CTAs per SM) of one problem, so no partial sums cross CTAs. Its codes arrive by TMA before the grid
+// For small groups: every CTA owns whole rows (up to kRowsMaxRows, in 8-row blocks; one or two CTAs
+// per SM) of one problem, so no partial sums cross CTAs. Its codes arrive by TMA before the grid
 // dependency wait, one barrier per 512-column chunk (8-row boxes of 128 bytes, 128-byte swizzle);
-// each of the eight warps stages the planes of one chunk and decodes it for all of the CTA's rows.
+// warp w stages the planes of chunks w, w + 8, ... and decodes each for all of the CTA's rows.
+// Narrow launches (K <= 4096: one chunk per warp, at most kRowsMaxSalient salient columns) may put
+// two CTAs on an SM; wide ones (up to kRowsMaxChunks chunks, kRowsMaxSalientWide salient columns)
+// one, with the registers that leaves for the next chunk's x and v and every residual operand.
 constexpr int kRowsWarps = 8;
 constexpr int kRowsThreads = kRowsWarps * 32;                  // 256
 constexpr int kRowsMaxRows = 32;                               // one row per lane
 constexpr int kRowsBoxRows = 8;
 constexpr int kRowsSlotBytes = 1792;                           // planes + ChunkMeta of one chunk, per warp
-constexpr int kRowsMaxSalient = 256;                           // salient columns (half of them in registers)
+constexpr int kRowsMaxSalient = 256;                           // narrow: salient columns (half of them in registers)
+// wide: 512-column chunks (K <= 8192), two per warp at most. Measured single calls: 1024 x 5120
+// 8.4 -> 5.5 us and 1024 x 8192 8.5 -> 6.2 us against the stream-K kernel, but 4096 x 14336 (28
+// chunks, 3.5 per warp) 10.2 -> 11.7 us: a warp's chunks are staged and decoded one after another.
+constexpr int kRowsMaxChunks = 16;
+constexpr int kRowsMaxSalientWide = 512;                       // wide: salient columns, all in registers
 
 struct RowsParams {
   ProblemArgs prob[kMaxProblems];   // as for the stream-K kernel (ws, counters, n_tiles, unit_begin unused)
@@ -136,6 +144,8 @@ struct RowsParams {
   int n_chunks_max;                 // over the problems: shared-memory size
   int n_problems;
   int kparts;                       // lanes per row of every CTA (1, 2 or 4), or 0: each CTA by its rows
+  int wide;                         // 1: some problem has more than kRowsWarps chunks or more than
+                                    // kRowsMaxSalient salient columns (one CTA per SM)
   int* status;                      // device status word (the first layout's)
 };
 

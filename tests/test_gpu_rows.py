@@ -2,11 +2,13 @@
 dependency wait) against the fp64 oracle.
 
 The kernel takes a batch-1 call when all of its 2-bit, one-alpha-per-row problems fit one launch of
-it (at most 64 rows per CTA with one CTA per SM); larger calls take the stream-K kernel. Pass rule
-(per output element): |y - y_ref| <= 1e-4 * sum_j |x_j * W^[o][j]| + 1e-6, the oracle's bound.
-Shapes cover one and two rows per lane, a CTA whose last 8-row block is half empty, ragged K (a
-chunk shorter than 512 columns), one-CTA problems, every column salient, grouped calls that split
-the SMs between problems, unaligned activations (scalar staging loads) and massive activations.
+it (at most 32 rows per CTA, one or two CTAs per SM; a wide launch, K above 4096 or more than 256
+salient columns, one CTA per SM, K up to 8192, up to 512 salient columns); larger calls take the
+stream-K kernel. Pass rule (per output element): |y - y_ref| <= 1e-4 * sum_j |x_j * W^[o][j]| + 1e-6,
+the oracle's bound. Shapes cover one, two and four lanes per row, a CTA whose last 8-row block is
+half empty, ragged K (a chunk shorter than 512 columns), one-CTA problems, every column salient,
+warps with one to four chunks, grouped calls that split the SMs between problems, unaligned
+activations (scalar staging loads) and massive activations.
 """
 import numpy as np
 import pytest
@@ -98,8 +100,9 @@ def test_eligibility(qt):
 
 def test_plan_small_calls_rows_large_calls_stream_k(qt):
     """Which batch-1 form a call takes: q, k, v, o of the Llama3-8B layer alone and q, k, v together
-    fit the row-resident launch; gate_proj (14336 rows, more than 64 per CTA), down_proj (K = 14336)
-    and the whole layer in one call take the stream-K launch, as does a layout pinned to it."""
+    fit the row-resident launch; gate_proj (14336 rows, more than 32 per CTA), down_proj (K = 14336,
+    beyond the wide launch's 8192) and the whole layer in one call take the stream-K launch, as does
+    a layout pinned to it."""
     ps = [synth.workload_problem("llama3_8b_layer", m) for m in range(7)]
     lays = [layout_of(qt, p) for p in ps]
     probs = [dict(layout=l, **args(p)) for l, p in zip(lays, ps)]
@@ -133,7 +136,70 @@ def test_rows_dense_salient(qt, N, K, s):
     check(run(qt, p, layout_of(qt, p)), p, f"dense salient N={N} K={K} s={s}")
 
 
-@pytest.mark.parametrize("N,K,s", [(516, 1000, 32), (4096, 4096, 120)])
+WIDE_SHAPES = [  # N, K, s: more than one chunk per warp, or more than 256 salient columns
+    (512, 4608, 32), (1004, 8000, 64), (2052, 5000, 100), (4, 8192, 8), (256, 8192, 512),
+    (4864, 8192, 432), (1024, 4096, 300), (256, 512, 512), (8, 7000, 264),
+]
+
+
+@pytest.mark.parametrize("N,K,s", WIDE_SHAPES)
+def test_rows_wide_parity_shapes(qt, N, K, s):
+    """Wide launches: warps with two chunks (the next chunk's x and v loaded during a decode), a
+    ragged last chunk, one to four lanes per row, up to 512 salient columns in registers."""
+    p = synth.make_problem("rows/wide", N, K, 1, s, seed=7 * N + K + 13 * s)
+    lay = layout_of(qt, p)
+    assert lay.describe()["rows_kernel"] == 1
+    assert qt.qtea_gemv_plan([dict(layout=lay, **args(p))]) == ["rows"]
+    y = run(qt, p, lay)
+    rows = None if N * K <= 1 << 24 else np.unique(np.concatenate(
+        [np.arange(0, N, 37), [0, 1, 7, 8, 31, 32, N - 1]])).astype(np.int32)
+    check(y, p, f"wide N={N} K={K} s={s}", rows=rows)
+
+
+def test_rows_wide_limits(qt):
+    """Past the wide launch's limits the stream-K kernel serves the call: more than 32 rows per CTA
+    with one CTA per SM, more than 16 chunks, more than 512 salient columns."""
+    sm = torch.cuda.get_device_properties(0).multi_processor_count
+    for N, K, s in ((8 * (4 * sm + 1), 4608, 8), (64, 8704, 8), (64, 4096, 520)):
+        p = synth.make_problem("rows/limits", N, K, 1, s, seed=N + K + s)
+        lay = layout_of(qt, p)
+        assert qt.qtea_gemv_plan([dict(layout=lay, **args(p))]) == ["stream_k"], (N, K, s)
+        rows = np.unique(np.concatenate([np.arange(0, N, 97), [N - 1]])).astype(np.int32)
+        check(run(qt, p, lay), p, f"stream-K beyond the wide limits N={N} K={K} s={s}", rows=rows)
+
+
+@pytest.mark.parametrize("workload,matrix", [("qwen3_14b_layer", 1), ("llama3_70b_layer", 2)])
+def test_rows_wide_workload_calls(qt, workload, matrix):
+    """k_proj of Qwen3-14B (K = 5120) and v_proj of Llama3-70B (K = 8192) alone: wide launches,
+    sampled rows."""
+    p = synth.workload_problem(workload, matrix)
+    lay = layout_of(qt, p)
+    assert qt.qtea_gemv_plan([dict(layout=lay, **args(p))]) == ["rows"]
+    y = run(qt, p, lay)
+    rows = np.unique(np.concatenate([np.arange(0, p.N, 29), [0, 7, 8, p.N - 1]])).astype(np.int32)
+    assert check(y, p, f"{workload} {p.name}", rows=rows) < 0.25
+
+
+def test_rows_wide_grouped_call(qt):
+    """Two wide problems and a narrow one in one launch (one CTA per SM): results match the oracle
+    and repeat bitwise."""
+    ps = [synth.make_problem("rows/wg", N, K, 1, s, seed=N + K + s)
+          for N, K, s in ((512, 8192, 64), (256, 4096, 300), (128, 2048, 16))]
+    lays = [layout_of(qt, p) for p in ps]
+    probs = [dict(layout=l, **args(p)) for l, p in zip(lays, ps)]
+    assert qt.qtea_gemv_plan(probs) == ["rows"] * 3
+    ys = qt.qtea_gemv_grouped(probs)
+    torch.cuda.synchronize()
+    assert qt.qtea_device_status(lays[0]) == 0
+    for p, y in zip(ps, ys):
+        check(y, p, f"wide grouped {p.name} N={p.N} K={p.K}")
+    ys2 = qt.qtea_gemv_grouped(probs)
+    torch.cuda.synchronize()
+    for y, y2 in zip(ys, ys2):
+        assert torch.equal(y, y2)
+
+
+@pytest.mark.parametrize("N,K,s", [(516, 1000, 32), (4096, 4096, 120), (516, 7000, 40)])
 def test_rows_unaligned_activations(qt, N, K, s):
     p = synth.make_problem("rows", N, K, 1, s, seed=N + K)
     check(run(qt, p, layout_of(qt, p), x_offset=1), p, f"x at an odd offset N={N} K={K}")
