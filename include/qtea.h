@@ -96,8 +96,9 @@ typedef enum qtea_option {
  * Which kernel serves a call: the TMA batch-1 kernel takes 2-bit layouts with fp16 residual values
  * at M = 1 (one alpha per row, or alpha and beta per row or per 128-column group), in one of two
  * forms: a row-resident launch, where every CTA holds all the codes of its rows at once (taken when
- * all of a call's batch-1 problems have one alpha per row, K <= 4096 and at most 256 salient
- * columns, and fit one such launch: at most 32 rows per CTA with one or two CTAs per SM;
+ * all of a call's batch-1 problems have one alpha per row, K <= 8192 and at most 512 salient
+ * columns, and fit one such launch: at most 32 rows per CTA with one or two CTAs per SM, one when
+ * some problem has K > 4096 or more than 256 salient columns;
  * a latency-bound form for small calls), else the persistent stream-K launch; the tensor-core
  * low-batch kernel takes those at M >= 2 and 2-bit layouts with FP8 residual values (groups of 128
  * columns, or beta absent) at any M; base-3 layouts
@@ -250,7 +251,7 @@ typedef struct qtea_layout_desc {
                                fp16 residual values), 0 otherwise */
   int options;              /* QTEA_OPT_* flags */
   int rows_kernel;          /* 1 if M = 1 calls may run the row-resident kernel instead (2-bit codes,
-                               one alpha per row, fp16 residual values, K <= 4096, n_salient <= 256,
+                               one alpha per row, fp16 residual values, K <= 8192, n_salient <= 512,
                                no QTEA_OPT_STREAM_K): they do when all of a call's batch-1 problems
                                fit one launch of it */
 } qtea_layout_desc;
