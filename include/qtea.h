@@ -203,6 +203,25 @@ typedef enum qtea_kernel {
  */
 int qtea_gemv_plan(const qtea_gemv_problem* problems, int n_problems, int M, int* kernels);
 
+/*
+ * The row-resident launch that qtea_gemv_grouped would plan for n batch-1 problems (2-bit codes,
+ * one alpha per row, fp16 residual values) from their shapes alone (no counterpart in the paper:
+ * it exposes the batch-1 dispatch rule so that it can be checked without a device). Problem i has
+ * N[i] rows, K[i] columns and n_salient[i] salient columns; the device has sm_count SMs and
+ * smem_optin bytes of opt-in shared memory per block (cudaDeviceProp::sharedMemPerBlockOptin).
+ *   QTEA_OK               the problems fit one row-resident launch: plan[0..3] receive the grid
+ *                         (CTAs), the most rows of a CTA, wide (1: K above 4096 or more than 256
+ *                         salient columns somewhere, one CTA per SM) and the lanes per row of every
+ *                         CTA (4, 2 or 1; 0 when the CTAs differ); ctas[i], when ctas is not NULL,
+ *                         problem i's CTAs;
+ *   QTEA_ERR_UNSUPPORTED  they take the stream-K launch (plan and ctas unchanged);
+ *   QTEA_ERR_INVALID_ARG  a NULL array, n outside 1..8, sm_count < 1, N or K zero (such problems
+ *                         launch nothing) or a shape qtea_pack_layout rejects.
+ * Host only: touches no device.
+ */
+int qtea_rows_plan_shapes(const int* N, const int* K, const int* n_salient, int n, int sm_count,
+                          size_t smem_optin, int* ctas, int* plan);
+
 /* Release a layout and its device memory. NULL is ignored. The caller orders it after the
  * last qtea_gemv that uses the layout has completed; it synchronizes nothing itself. */
 void qtea_free(qtea_layout* layout);

@@ -83,6 +83,8 @@ def load(build_if_missing: bool = True):
     lib.qtea_gemv_grouped.argtypes = [P, i32, i32, P]
     lib.qtea_gemv_plan.restype = i32
     lib.qtea_gemv_plan.argtypes = [P, i32, i32, P]
+    lib.qtea_rows_plan_shapes.restype = i32
+    lib.qtea_rows_plan_shapes.argtypes = [P, P, P, i32, i32, ctypes.c_size_t, P, P]
     lib.qtea_set_activation_precision.restype = i32
     lib.qtea_set_activation_precision.argtypes = [P, i32]
     lib.qtea_set_layout_options.restype = i32
@@ -280,6 +282,24 @@ def qtea_gemv_plan(problems) -> list:
     if rc:
         raise QteaError(rc, "qtea_gemv_plan")
     return [QTEA_KERNEL_NAMES[out[i]] for i in range(len(problems))]
+
+
+def qtea_rows_plan_shapes(shapes, sm_count: int, smem_optin: int):
+    """The row-resident launch qtea_gemv_grouped would plan for batch-1 problems of these (N, K,
+    n_salient) shapes on a device of sm_count SMs (host only): a dict with grid, rows_cap, wide,
+    kparts and ctas (per problem), or None when they take the stream-K launch."""
+    n = len(shapes)
+    arr = lambda vals: (ctypes.c_int * max(n, 1))(*vals)
+    N, K, S = arr([int(a) for a, _, _ in shapes]), arr([int(b) for _, b, _ in shapes]), arr([int(c) for _, _, c in shapes])
+    ctas, plan = (ctypes.c_int * max(n, 1))(), (ctypes.c_int * 4)()
+    rc = load().qtea_rows_plan_shapes(ctypes.cast(N, ctypes.c_void_p), ctypes.cast(K, ctypes.c_void_p),
+                                      ctypes.cast(S, ctypes.c_void_p), n, int(sm_count), int(smem_optin),
+                                      ctypes.cast(ctas, ctypes.c_void_p), ctypes.cast(plan, ctypes.c_void_p))
+    if rc == QTEA_ERR_UNSUPPORTED:
+        return None
+    if rc:
+        raise QteaError(rc, "qtea_rows_plan_shapes")
+    return dict(grid=plan[0], rows_cap=plan[1], wide=plan[2], kparts=plan[3], ctas=[ctas[i] for i in range(n)])
 
 
 def qtea_device_status(layout: Layout, stream=None) -> int:

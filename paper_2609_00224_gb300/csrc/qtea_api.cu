@@ -628,12 +628,13 @@ int run_m1(const qtea_gemv_problem* qs, const int* idx, int n, cudaStream_t st, 
 // Layouts it may serve: 2-bit codes, one alpha per row, fp16 residual values, at most
 // kRowsMaxChunks 512-column chunks and kRowsMaxSalientWide salient columns, not pinned to the
 // stream-K kernel. Beyond one chunk per warp or kRowsMaxSalient salient columns a launch is wide.
+bool rows_shape_ok(int n_chunks, int s) { return n_chunks <= kRowsMaxChunks && s <= kRowsMaxSalientWide; }
+bool rows_shape_wide(int n_chunks, int s) { return n_chunks > kRowsWarps || s > kRowsMaxSalient; }
 bool rows_capable(const qtea_layout* l) {
   return l->rows_ok && l->m1_ok && l->format == QTEA_FMT_2BIT && l->group_size == l->K &&
          (l->options & (QTEA_OPT_BIAS | QTEA_OPT_RESIDUAL_FP8 | QTEA_OPT_STREAM_K)) == 0 &&
-         l->n_chunks <= kRowsMaxChunks && l->n_salient <= kRowsMaxSalientWide;
+         rows_shape_ok(l->n_chunks, l->n_salient);
 }
-bool rows_wide(const qtea_layout* l) { return l->n_chunks > kRowsWarps || l->n_salient > kRowsMaxSalient; }
 
 struct RowsLaunch {
   RowsParams rp;
@@ -680,68 +681,94 @@ long long rows_split(const long long* blocks, const int* chunks, int n, int ctas
   return rows;
 }
 
-// One row-resident launch for problems idx[0 .. n): one CTA per SM where that leaves every CTA
-// kRowsMaxRows rows or fewer (one per lane), else two CTAs per SM (not for a wide launch). False
-// if the problems do not fit: more problems than CTAs, more than kRowsMaxRows rows in a CTA, or
-// shared memory beyond the device's limit.
-bool rows_plan(const qtea_gemv_problem* qs, const int* idx, int n, RowsLaunch& L) {
-  if (n < 1 || n > kMaxProblems) return false;
-  const qtea_layout* l0 = qs[idx[0]].packed_ternary;
-  const int sm = l0->sm_count;
-  if (n > sm || 2 * sm > kMaxGrid) return false;
+// The shape of a row-resident launch for n problems (rows N[i], chunks nch[i], salient columns s[i])
+// on a device of sm SMs with smem_optin bytes of shared memory per CTA: one CTA per SM where that
+// leaves every CTA kRowsMaxRows rows or fewer (one per lane), else two CTAs per SM (not for a wide
+// launch). False if the problems do not fit: a shape beyond the kernel's limits, more problems than
+// CTAs, more than kRowsMaxRows rows in a CTA, or shared memory beyond the device's limit.
+struct RowsShapePlan {
+  int cnt[kMaxProblems];  // CTAs of each problem
+  int grid, rows_cap, nch_max, kparts;
+  bool wide;
+  size_t smem;
+};
+bool rows_plan_shapes(const long long* N, const int* nch, const int* s, int n, int sm, size_t smem_optin,
+                      RowsShapePlan& P) {
+  if (n < 1 || n > kMaxProblems || sm < 1 || n > sm || 2 * sm > kMaxGrid) return false;
   long long blocks[kMaxProblems];
-  int chunks[kMaxProblems], cnt[kMaxProblems], nch_max = 0;
-  bool wide = false;
+  P.nch_max = 0;
+  P.wide = false;
   for (int i = 0; i < n; ++i) {
-    const qtea_layout* l = qs[idx[i]].packed_ternary;
-    if (!rows_capable(l) || l->sm_count != sm || l->device != l0->device) return false;
-    blocks[i] = (l->N + kRowsBoxRows - 1) / kRowsBoxRows;
-    chunks[i] = l->n_chunks;
-    nch_max = chunks[i] > nch_max ? chunks[i] : nch_max;
-    wide = wide || rows_wide(l);
+    if (N[i] < 1 || nch[i] < 1 || s[i] < 0 || !rows_shape_ok(nch[i], s[i])) return false;
+    blocks[i] = (N[i] + kRowsBoxRows - 1) / kRowsBoxRows;
+    P.nch_max = nch[i] > P.nch_max ? nch[i] : P.nch_max;
+    P.wide = P.wide || rows_shape_wide(nch[i], s[i]);
   }
-  long long rows_cap = rows_split(blocks, chunks, n, sm, cnt);
-  if (rows_cap > kRowsMaxRows && !wide) {
+  long long rows_cap = rows_split(blocks, nch, n, sm, P.cnt);
+  if (rows_cap > kRowsMaxRows && !P.wide) {
     int cnt2[kMaxProblems];
-    const long long r2 = rows_split(blocks, chunks, n, 2 * sm, cnt2);
+    const long long r2 = rows_split(blocks, nch, n, 2 * sm, cnt2);
     if (r2 > 0 && r2 <= kRowsMaxRows) {
       rows_cap = r2;
-      for (int i = 0; i < n; ++i) cnt[i] = cnt2[i];
+      for (int i = 0; i < n; ++i) P.cnt[i] = cnt2[i];
     }
   }
   if (rows_cap < 1 || rows_cap > kRowsMaxRows) return false;
-  const RowsSmem so = rows_smem_layout((int)rows_cap, nch_max);
-  if (so.total > l0->rows_smem_optin) return false;
+  const RowsSmem so = rows_smem_layout((int)rows_cap, P.nch_max);
+  if (so.total > smem_optin) return false;
+  // lanes per row (4 for up to 8 rows, 2 for 16, 1 for more): one value for every CTA, or 0
+  int kp = -1;
+  P.grid = 0;
+  for (int i = 0; i < n; ++i) {
+    P.grid += P.cnt[i];
+    for (int j = 0; j < P.cnt[i] && kp != 0; ++j) {
+      const long long r0 = blocks[i] * j / P.cnt[i] * kRowsBoxRows, r1 = blocks[i] * (j + 1) / P.cnt[i] * kRowsBoxRows;
+      const long long R = (r1 < N[i] ? r1 : N[i]) - r0;
+      const int k = R <= 8 ? 4 : R <= 16 ? 2 : 1;
+      if (kp < 0) kp = k;
+      else if (kp != k) kp = 0;
+    }
+  }
+  P.kparts = kp < 0 ? 0 : kp;
+  P.rows_cap = (int)rows_cap;
+  P.smem = so.total;
+  return true;
+}
+
+// One row-resident launch for problems idx[0 .. n), planned by rows_plan_shapes; false if a layout
+// cannot take the kernel or the problems do not fit one launch.
+bool rows_plan(const qtea_gemv_problem* qs, const int* idx, int n, RowsLaunch& L) {
+  if (n < 1 || n > kMaxProblems) return false;
+  const qtea_layout* l0 = qs[idx[0]].packed_ternary;
+  long long N[kMaxProblems];
+  int nch[kMaxProblems], sal[kMaxProblems];
+  for (int i = 0; i < n; ++i) {
+    const qtea_layout* l = qs[idx[i]].packed_ternary;
+    if (!rows_capable(l) || l->sm_count != l0->sm_count || l->device != l0->device) return false;
+    N[i] = l->N;
+    nch[i] = l->n_chunks;
+    sal[i] = l->n_salient;
+  }
+  RowsShapePlan P;
+  if (!rows_plan_shapes(N, nch, sal, n, l0->sm_count, l0->rows_smem_optin, P)) return false;
   std::memset(&L.rp, 0, sizeof(L.rp));
   int b = 0;
   for (int i = 0; i < n; ++i) {
     const qtea_gemv_problem& q = qs[idx[i]];
     L.rp.prob[i] = problem_args(q);
     L.rp.cta_begin[i] = b;
-    b += cnt[i];
+    b += P.cnt[i];
     std::memcpy(&L.maps.m[i], &q.packed_ternary->tmap8, sizeof(CUtensorMap));
   }
   L.rp.cta_begin[n] = b;
-  // lanes per row (4 for up to 8 rows, 2 for 16, 1 for more): one value for every CTA, or 0
-  int kp = -1;
-  for (int i = 0; i < n && kp != 0; ++i) {
-    const int N = qs[idx[i]].packed_ternary->N;
-    for (int j = 0; j < cnt[i]; ++j) {
-      const long long r0 = blocks[i] * j / cnt[i] * kRowsBoxRows, r1 = blocks[i] * (j + 1) / cnt[i] * kRowsBoxRows;
-      const long long R = (r1 < N ? r1 : N) - r0;
-      const int k = R <= 8 ? 4 : R <= 16 ? 2 : 1;
-      if (kp < 0) kp = k;
-      else if (kp != k) kp = 0;
-    }
-  }
-  L.rp.kparts = kp < 0 ? 0 : kp;
-  L.rp.wide = wide ? 1 : 0;
-  L.rp.rows_cap = (int)rows_cap;
-  L.rp.n_chunks_max = nch_max;
+  L.rp.kparts = P.kparts;
+  L.rp.wide = P.wide ? 1 : 0;
+  L.rp.rows_cap = P.rows_cap;
+  L.rp.n_chunks_max = P.nch_max;
   L.rp.n_problems = n;
   L.rp.status = l0->status;
   L.grid = b;
-  L.smem = so.total;
+  L.smem = P.smem;
   return true;
 }
 
@@ -1011,6 +1038,30 @@ int qtea_gemv_plan(const qtea_gemv_problem* problems, int n_problems, int M, int
   RowsLaunch L;
   if (!m1_many && n_m1 > 0 && rows_plan(problems, m1_idx, n_m1, L))
     for (int k = 0; k < n_m1; ++k) kernels[m1_idx[k]] = QTEA_KERNEL_ROWS;
+  return QTEA_OK;
+}
+
+int qtea_rows_plan_shapes(const int* N, const int* K, const int* n_salient, int n, int sm_count, size_t smem_optin,
+                          int* ctas, int* plan) {
+  if (!N || !K || !n_salient || !plan || n < 1 || n > kMaxProblems || sm_count < 1) return QTEA_ERR_INVALID_ARG;
+  long long NN[kMaxProblems];
+  int nch[kMaxProblems], sal[kMaxProblems];
+  for (int i = 0; i < n; ++i) {
+    if (N[i] < 1 || K[i] < 1 || N[i] > (1 << 20) || K[i] > 65536 || n_salient[i] < 0 || n_salient[i] > K[i] ||
+        (n_salient[i] > 0 && N[i] % 4))
+      return QTEA_ERR_INVALID_ARG;
+    NN[i] = N[i];
+    nch[i] = (K[i] + kChunkCols - 1) / kChunkCols;  // a 2-bit layout's chunks (K padded to 64 columns)
+    sal[i] = n_salient[i];
+  }
+  RowsShapePlan P;
+  if (!rows_plan_shapes(NN, nch, sal, n, sm_count, smem_optin, P)) return QTEA_ERR_UNSUPPORTED;
+  plan[0] = P.grid;
+  plan[1] = P.rows_cap;
+  plan[2] = P.wide ? 1 : 0;
+  plan[3] = P.kparts;
+  if (ctas)
+    for (int i = 0; i < n; ++i) ctas[i] = P.cnt[i];
   return QTEA_OK;
 }
 
